@@ -1,0 +1,370 @@
+"""Pins for the fp64 oracle: closed forms, hand cases, brute force, library
+routines and finite differences -- none of them re-types the oracle's own
+formula.  CPU only."""
+
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import spo_oracle as O
+
+
+def _golden(golden_dir, name):
+    with open(os.path.join(golden_dir, name)) as f:
+        return json.load(f)
+
+
+def _rand_hw(T, d, V, seed, scale_w=0.5):
+    rng = np.random.default_rng(seed)
+    return rng.standard_normal((T, d)), scale_w * rng.standard_normal((V, d))
+
+
+# ---------------------------------------------------------------- bf16 widening
+def test_bf16_widening_exact():
+    x = torch.tensor([1.0, -2.5, 3.140625, 1e-3, -65504.0, 0.0], dtype=torch.bfloat16)
+    bits = x.view(torch.int16).numpy().view(np.uint16)
+    np.testing.assert_array_equal(O.bf16_bits_to_f64(bits), x.double().numpy())
+
+
+# ---------------------------------------------------------------- log-probs
+def test_uniform_logits_closed_form(golden_dir):
+    for case in _golden(golden_dir, "uniform_logits.json")["cases"]:
+        V = case["V"]
+        d = 8
+        H = np.zeros((3, d))
+        W = np.random.default_rng(0).standard_normal((V, d))
+        lp, ent, lse = O.logprobs(H, W, np.array([0, V // 2, V - 1]))
+        np.testing.assert_allclose(lp, case["logp"], rtol=0, atol=1e-12)
+        np.testing.assert_allclose(ent, case["entropy"], rtol=0, atol=1e-12)
+        np.testing.assert_allclose(lse, -np.asarray(case["logp"]), atol=1e-12)
+
+
+def test_logprobs_normalise_over_vocab():
+    # exp(logp) summed over every possible target is 1 for each token
+    T, d, V = 4, 6, 37
+    H, W = _rand_hw(T, d, V, 1)
+    Hrep = np.repeat(H, V, axis=0)
+    tgt = np.tile(np.arange(V), T)
+    lp, _, _ = O.logprobs(Hrep, W, tgt)
+    sums = np.exp(lp).reshape(T, V).sum(axis=1)
+    np.testing.assert_allclose(sums, 1.0, atol=1e-13)
+    assert (lp <= 0).all()
+
+
+def test_logprobs_brute_force_tiny():
+    T, d, V = 3, 4, 5
+    H, W = _rand_hw(T, d, V, 2)
+    tgt = np.array([4, 0, 2])
+    tau_inv = 0.7
+    lp, ent, lse = O.logprobs(H, W, tgt, inv_temp=tau_inv)
+    for t in range(T):
+        z = []
+        for v in range(V):
+            acc = 0.0
+            for k in range(d):
+                acc += H[t][k] * W[v][k]
+            z.append(tau_inv * acc)
+        norm = sum(math.exp(x) for x in z)
+        probs = [math.exp(x) / norm for x in z]
+        assert abs(lp[t] - math.log(probs[tgt[t]])) < 1e-12
+        assert abs(ent[t] - (-sum(p * math.log(p) for p in probs))) < 1e-12
+        assert abs(lse[t] - math.log(norm)) < 1e-12
+
+
+def test_logprobs_vs_torch_fp64():
+    T, d, V = 17, 32, 301
+    H, W = _rand_hw(T, d, V, 3)
+    tgt = np.random.default_rng(4).integers(0, V, T)
+    lp, ent, lse = O.logprobs(H, W, tgt, inv_temp=1.3)
+    z = 1.3 * (torch.from_numpy(H) @ torch.from_numpy(W).T)
+    ref_lp = torch.log_softmax(z, dim=-1)[torch.arange(T), torch.from_numpy(tgt)]
+    ref_ent = torch.distributions.Categorical(logits=z).entropy()
+    np.testing.assert_allclose(lp, ref_lp.numpy(), atol=1e-12)
+    np.testing.assert_allclose(ent, ref_ent.numpy(), atol=1e-12)
+    np.testing.assert_allclose(lse, torch.logsumexp(z, -1).numpy(), atol=1e-12)
+
+
+def test_logprobs_dominant_logit_and_shift():
+    d, V = 4, 50
+    W = np.zeros((V, d))
+    W[7, 0] = 1.0
+    H = np.array([[60.0, 0, 0, 0]])
+    lp, ent, _ = O.logprobs(H, W, np.array([7]))
+    assert abs(lp[0]) < 1e-20
+    assert ent[0] < 1e-20
+    # a bias shared by every vocab entry leaves log-probs unchanged
+    H2, W2 = _rand_hw(5, 3, 11, 5)
+    tgt = np.arange(5)
+    a, ea, _ = O.logprobs(H2, W2, tgt)
+    Hb = np.concatenate([H2, np.full((5, 1), 3.7)], axis=1)
+    Wb = np.concatenate([W2, np.ones((11, 1))], axis=1)
+    b, eb, lb = O.logprobs(Hb, Wb, tgt)
+    np.testing.assert_allclose(a, b, atol=1e-12)
+    np.testing.assert_allclose(ea, eb, atol=1e-12)
+
+
+def test_logprobs_mask_and_ignore_index():
+    H, W = _rand_hw(6, 4, 9, 6)
+    tgt = np.array([1, -100, 3, 4, 5, 6])
+    mask = np.array([1, 1, 0, 1, 1, 1], dtype=np.uint8)
+    lp, ent, lse = O.logprobs(H, W, tgt, mask=mask)
+    assert lp[1] == 0 and lp[2] == 0 and ent[2] == 0 and lse[1] == 0
+    full, _, _ = O.logprobs(H, W, np.array([1, 2, 3, 4, 5, 6]))
+    np.testing.assert_allclose(lp[[0, 3, 4, 5]], full[[0, 3, 4, 5]], atol=1e-14)
+
+
+# ---------------------------------------------------------------- token select
+def test_token_select_hand_case():
+    cu = [0, 6, 10]
+    mask = np.array([0, 1, 1, 1, 1, 1, 1, 0, 1, 1], dtype=np.uint8)
+    tgt = np.array([5, 5, -100, 5, 5, 5, 5, 5, 5, 5])
+    lm, n = O.token_select(cu, mask, tgt, window=3)
+    assert lm.tolist() == [0, 1, 0, 1, 1, 0, 1, 0, 1, 1]
+    assert n.tolist() == [3, 3]
+    lm2, n2 = O.token_select(cu, mask, tgt, window=0)
+    assert lm2.tolist() == [0, 1, 0, 1, 1, 1, 1, 0, 1, 1]
+    assert n2.tolist() == [4, 3]
+
+
+# ---------------------------------------------------------------- advantages
+def test_advantage_worked_example(golden_dir):
+    gold = _golden(golden_dir, "advantage_worked_example.json")
+    r = gold["rewards"]
+    a = O.group_advantages(r, [0, 0, 0, 0], 1, O.STD_UNBIASED, eps=0.0)
+    np.testing.assert_allclose(a, gold["unbiased"], atol=1e-15)
+    a = O.group_advantages(r, [0, 0, 0, 0], 1, O.STD_POPULATION, eps=0.0)
+    np.testing.assert_allclose(a, gold["population"], atol=1e-15)
+    a32 = O.group_advantages_f32(r, [0, 0, 0, 0], 1, O.STD_UNBIASED, eps=0.0)
+    np.testing.assert_allclose(a32, gold["unbiased"], atol=1e-6)
+
+
+def test_advantage_invariants():
+    rng = np.random.default_rng(7)
+    n_groups, per = 6, 16
+    r = rng.uniform(0, 3, n_groups * per)
+    gid = np.repeat(np.arange(n_groups), per)
+    perm = rng.permutation(r.size)          # members need not be contiguous
+    r, gid = r[perm], gid[perm]
+    a = O.group_advantages(r, gid, n_groups, O.STD_UNBIASED, eps=0.0)
+    for g in range(n_groups):
+        ag = a[gid == g]
+        assert abs(ag.sum()) < 1e-12
+        assert abs((ag ** 2).sum() - (per - 1)) < 1e-10
+    # affine invariance for a positive scale
+    b = O.group_advantages(2.5 * r - 7.0, gid, n_groups, O.STD_UNBIASED, eps=0.0)
+    np.testing.assert_allclose(a, b, atol=1e-12)
+
+
+def test_advantage_degenerate_groups():
+    r = np.array([1.5, 1.5, 1.5, 0.3, 7.0, 2.0])
+    gid = np.array([0, 0, 0, 1, 2, 2])
+    for fn in (O.group_advantages, O.group_advantages_f32):
+        a = fn(r, gid, 4, O.STD_UNBIASED, 1e-6)
+        assert a[0] == 0 and a[1] == 0 and a[2] == 0      # zero variance
+        assert a[3] == 0                                   # singleton group
+        assert a[4] > 0 > a[5]
+
+
+def test_advantage_f32_matches_f64():
+    rng = np.random.default_rng(8)
+    r = rng.normal(0.3, 1.0, 4096).astype(np.float32)
+    gid = rng.integers(0, 256, r.size)
+    a64 = O.group_advantages(r.astype(np.float64), gid, 256)
+    a32 = O.group_advantages_f32(r, gid, 256)
+    np.testing.assert_allclose(a32, a64, atol=2e-6, rtol=0)
+
+
+# ---------------------------------------------------------------- loss
+def _single_token(rho, adv, beta, logp=None, ref=None, eps=0.2):
+    lp = np.log(rho) if logp is None else logp
+    old = lp - np.log(rho)
+    loss, g, st = O.policy_loss(np.array([lp]), np.array([old]),
+                                None if ref is None else np.array([ref]), np.array([adv]),
+                                [0, 1], [0], 1, np.array([1], np.uint8), eps, beta)
+    return loss, g[0], st
+
+
+def test_surrogate_hand_cases(golden_dir):
+    gold = _golden(golden_dir, "surrogate_hand_cases.json")
+    for c in gold["cases"]:
+        loss, g, _ = _single_token(c["rho"], c["adv"], c["beta"], c.get("logp"), c.get("ref"),
+                                   gold["clip_eps"])
+        assert abs(loss - c["loss"]) < 1e-12, c
+        assert abs(g - c["g"]) < 1e-12, c
+
+
+def test_ratio_one_no_kl_is_minus_mean_advantage():
+    # with pi_theta == pi_old and beta = 0 the objective is the weighted mean advantage
+    rng = np.random.default_rng(9)
+    lens = [5, 9, 3, 7, 4, 6]
+    cu = np.concatenate([[0], np.cumsum(lens)])
+    gid = np.array([0, 0, 1, 1, 1, 2])
+    adv = rng.standard_normal(len(lens))          # arbitrary, not group-normalised
+    T = cu[-1]
+    lp = -rng.uniform(0.1, 5, T)
+    lm = np.ones(T, np.uint8)
+    loss, g, st = O.policy_loss(lp, lp, None, adv, cu, gid, 3, lm, 0.2, 0.0, O.AGG_SEQ_GROUP)
+    # SEQ_GROUP: mean over groups of mean over outputs of A_i
+    want = -np.mean([adv[gid == k].mean() for k in range(3)])
+    assert abs(loss - want) < 1e-12
+    loss_t, _, _ = O.policy_loss(lp, lp, None, adv, cu, gid, 3, lm, 0.2, 0.0, O.AGG_TOKEN)
+    want_t = -(np.repeat(adv, lens)).mean()
+    assert abs(loss_t - want_t) < 1e-12
+    assert st["clip_frac"] == 0 and abs(st["mean_ratio"] - 1) < 1e-15
+
+
+def test_kl_properties():
+    rng = np.random.default_rng(10)
+    T = 50
+    lp = -rng.uniform(0.1, 5, T)
+    cu = [0, 20, 50]
+    lm = np.ones(T, np.uint8)
+    _, g0, st0 = O.policy_loss(lp, lp, lp, np.zeros(2), cu, [0, 0], 1, lm, 0.2, 0.3)
+    assert st0["mean_kl"] == 0 and np.all(g0 == 0)
+    ref = lp + rng.normal(0, 0.5, T)
+    _, _, st = O.policy_loss(lp, lp, ref, np.zeros(2), cu, [0, 0], 1, lm, 0.2, 0.3)
+    assert st["mean_kl"] > 0
+
+
+def test_aggregations_agree_on_uniform_layout():
+    rng = np.random.default_rng(11)
+    lens = [8] * 8
+    cu = np.concatenate([[0], np.cumsum(lens)])
+    gid = np.repeat(np.arange(2), 4)
+    T = cu[-1]
+    lp = -rng.uniform(0.1, 3, T)
+    old = lp + rng.normal(0, 0.3, T)
+    ref = lp + rng.normal(0, 0.1, T)
+    adv = rng.standard_normal(8)
+    lm = np.ones(T, np.uint8)
+    a = O.policy_loss(lp, old, ref, adv, cu, gid, 2, lm, 0.2, 0.04, O.AGG_SEQ_GROUP)
+    b = O.policy_loss(lp, old, ref, adv, cu, gid, 2, lm, 0.2, 0.04, O.AGG_TOKEN)
+    assert abs(a[0] - b[0]) < 1e-13
+    np.testing.assert_allclose(a[1], b[1], atol=1e-15)
+
+
+def test_dloss_dlogp_finite_difference():
+    rng = np.random.default_rng(12)
+    lens = [6, 4, 9, 5]
+    cu = np.concatenate([[0], np.cumsum(lens)])
+    gid = np.array([0, 0, 1, 1])
+    T = cu[-1]
+    lp = -rng.uniform(0.1, 3, T)
+    old = lp + rng.normal(0, 0.4, T)
+    ref = lp + rng.normal(0, 0.2, T)
+    adv = rng.standard_normal(4)
+    lm = np.ones(T, np.uint8)
+    lm[3] = 0
+    eps = 0.2
+    rho = np.exp(lp - old)
+    for agg in (O.AGG_SEQ_GROUP, O.AGG_TOKEN):
+        _, g, _ = O.policy_loss(lp, old, ref, adv, cu, gid, 2, lm, eps, 0.07, agg)
+        h = 1e-6
+        for t in range(T):
+            if min(abs(rho[t] - 1 - eps), abs(rho[t] - 1 + eps)) < 1e-4:
+                continue
+            lp_p, lp_m = lp.copy(), lp.copy()
+            lp_p[t] += h
+            lp_m[t] -= h
+            fp = O.policy_loss(lp_p, old, ref, adv, cu, gid, 2, lm, eps, 0.07, agg)[0]
+            fm = O.policy_loss(lp_m, old, ref, adv, cu, gid, 2, lm, eps, 0.07, agg)[0]
+            assert abs((fp - fm) / (2 * h) - g[t]) < 1e-8, (agg, t)
+        assert g[3] == 0
+
+
+# ---------------------------------------------------------------- backward
+def _loss_of_hw(H, W, tgt, cu, gid, n_groups, lm, old, ref, adv, eps, beta, tau):
+    lp, _, _ = O.logprobs(H, W, tgt, tau, lm)
+    return O.policy_loss(lp, old, ref, adv, cu, gid, n_groups, lm, eps, beta)
+
+
+def test_backward_finite_difference():
+    rng = np.random.default_rng(13)
+    T, d, V = 7, 5, 11
+    H, W = _rand_hw(T, d, V, 14)
+    tgt = rng.integers(0, V, T)
+    cu = [0, 3, 7]
+    gid = [0, 0]
+    lm = np.array([1, 1, 0, 1, 1, 1, 1], np.uint8)
+    tau = 0.8
+    lp0, _, _ = O.logprobs(H, W, tgt, tau, lm)
+    old = lp0 + rng.normal(0, 0.05, T)
+    ref = lp0 + rng.normal(0, 0.05, T)
+    adv = np.array([0.7, -1.3])
+    args = (tgt, cu, gid, 1, lm, old, ref, adv, 0.2, 0.05, tau)
+    _, g, _ = _loss_of_hw(H, W, *args)
+    dH, dW = O.policy_loss_bwd(H, W, tgt, g, tau)
+    h = 1e-6
+    for (t, k) in [(0, 0), (1, 4), (2, 2), (4, 1), (6, 3)]:
+        Hp, Hm = H.copy(), H.copy()
+        Hp[t, k] += h
+        Hm[t, k] -= h
+        fd = (_loss_of_hw(Hp, W, *args)[0] - _loss_of_hw(Hm, W, *args)[0]) / (2 * h)
+        assert abs(fd - dH[t, k]) < 1e-8, (t, k, fd, dH[t, k])
+    for (v, k) in [(0, 0), (int(tgt[0]), 2), (5, 4), (10, 1), (int(tgt[6]), 3)]:
+        Wp, Wm = W.copy(), W.copy()
+        Wp[v, k] += h
+        Wm[v, k] -= h
+        fd = (_loss_of_hw(H, Wp, *args)[0] - _loss_of_hw(H, Wm, *args)[0]) / (2 * h)
+        assert abs(fd - dW[v, k]) < 1e-8, (v, k, fd, dW[v, k])
+    assert np.all(dH[2] == 0)
+
+
+def test_backward_vs_torch_cross_entropy_autograd():
+    # rho = 1, beta = 0: L = sum_t c_t A_i * CE(z_t, y_t) + const, so torch's
+    # fp64 cross_entropy autograd gives the same dH and dW.
+    rng = np.random.default_rng(15)
+    T, d, V = 12, 9, 23
+    H, W = _rand_hw(T, d, V, 16)
+    tgt = rng.integers(0, V, T)
+    cu = np.array([0, 5, 12])
+    gid = [0, 1]
+    lm = np.ones(T, np.uint8)
+    adv = np.array([0.9, -0.4])
+    lp, _, _ = O.logprobs(H, W, tgt, 1.0, lm)
+    _, g, _ = O.policy_loss(lp, lp, None, adv, cu, gid, 2, lm, 0.2, 0.0)
+    dH, dW = O.policy_loss_bwd(H, W, tgt, g, 1.0)
+    Ht = torch.tensor(H, requires_grad=True)
+    Wt = torch.tensor(W, requires_grad=True)
+    ce = torch.nn.functional.cross_entropy(Ht @ Wt.T, torch.tensor(tgt), reduction="none")
+    c = torch.tensor(np.concatenate([np.full(5, adv[0] / (2 * 5)), np.full(7, adv[1] / (2 * 7))]))
+    (c * ce).sum().backward()
+    np.testing.assert_allclose(dH, Ht.grad.numpy(), atol=1e-13)
+    np.testing.assert_allclose(dW, Wt.grad.numpy(), atol=1e-13)
+
+
+def test_backward_invariants():
+    rng = np.random.default_rng(17)
+    T, d, V = 9, 6, 14
+    H, W = _rand_hw(T, d, V, 18)
+    tgt = rng.integers(0, V, T)
+    g = rng.standard_normal(T)
+    g[4] = 0.0
+    _, dW = O.policy_loss_bwd(H, W, tgt, g)
+    # each row of G sums to zero over the vocabulary
+    np.testing.assert_allclose(dW.sum(axis=0), 0.0, atol=1e-12)
+    Wsame = np.tile(W[:1], (V, 1))
+    dH, _ = O.policy_loss_bwd(H, Wsame, tgt, g)
+    np.testing.assert_allclose(dH, 0.0, atol=1e-12)
+    dH, _ = O.policy_loss_bwd(H, W, tgt, g)
+    assert np.all(dH[4] == 0)
+
+
+def test_grpo_step_runs_on_tiny_workload():
+    from paper_2607_20908_gb300 import inputs
+    case = inputs.tiny_case()
+    H = O.bf16_bits_to_f64(inputs.bf16_bits(case["H"]))
+    W = O.bf16_bits_to_f64(inputs.bf16_bits(case["W"]))
+    tgt = case["tgt"].numpy()
+    lp, _, _ = O.logprobs(H, W, tgt)
+    old = lp + case["old_noise"].double().numpy()
+    ref = lp + case["ref_noise"].double().numpy()
+    out = O.grpo_step(H, W, tgt, case["mask"].numpy(), case["cu_seqlens"].numpy(),
+                      case["group_id"].numpy(), case["n_groups"], case["rewards"].numpy(),
+                      old, ref, case["clip_eps"], case["kl_beta"])
+    assert np.isfinite(out["loss"]) and out["stats"]["n_loss_tokens"] == case["T"]
+    assert np.all(out["logp"] <= 0)
