@@ -1,0 +1,233 @@
+/*
+ * spo.h -- C ABI of libspo: the GRPO policy log-prob / policy-loss hot path of
+ * CUDAPerf (arxiv 2607.20908) on NVIDIA GB300 (sm_103a).
+ *
+ * The paper's online RL phase (section 3, "Multi-turn RL Training") maximises
+ * the GRPO objective of Eq. 3: for every rollout token it needs the policy's
+ * log-probability of the sampled token over the full vocabulary, the ratio
+ * against the old policy, group-normalised advantages of the composite reward,
+ * the clipped surrogate with a KL term, and the gradient of all of it back to
+ * the final hidden states H and the LM-head weight W.  This header is that
+ * path, one call per step:
+ *
+ *   spo_token_select       loss tokens: mask, ignore index, 1024-token window
+ *   spo_logprobs_fwd       logits H W^T tile by tile + online logsumexp
+ *                          (logits never reach memory) -> logp, entropy, lse
+ *   spo_group_advantages   A_hat_i = (r_i - mean_g) / (std_g + eps)
+ *   spo_policy_loss_fwd    ratio, clip, KL, aggregation -> loss, dL/dlogp
+ *   spo_policy_loss_bwd    dH = G W, dW = G^T H with
+ *                          G = tau^-1 g (onehot - softmax), logits recomputed
+ *
+ * Conventions shared by every call
+ *   - Every array argument is a DEVICE pointer owned by the caller unless the
+ *     comment says otherwise.  The library never allocates device memory,
+ *     never frees, and never synchronises the stream (except
+ *     spo_device_error, which says so).  Scratch memory comes only from the
+ *     caller's `ws` buffer, sized by the matching *_workspace_size call.
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream).  Work is
+ *     enqueued asynchronously in stream order.  Calls on distinct workspaces
+ *     may run concurrently on different streams.
+ *   - Layouts are row-major and dense.  bf16 matrices (H, W, dH) must start on
+ *     a 16-byte boundary (the tensor-memory-accelerator loads require it).
+ *   - Argument errors are detected on the host before anything is enqueued
+ *     and have no side effects; the status says which class of error, and
+ *     spo_last_error() returns a one-line description (per host thread).
+ *   - A launch failure returns SPO_ERR_CUDA.  Every device-side wait in the
+ *     tensor-core kernels is bounded; a wait that expires records a code that
+ *     spo_device_error() returns (SPO_ERR_TIMEOUT) instead of hanging.
+ *   - The sign convention is that of an optimiser: `loss` = -J_GRPO, to be
+ *     minimised.
+ *
+ * Symbols: the precision of every result is stated per call.  Token ids are
+ * already shifted (tgt[t] is the token whose probability row t predicts);
+ * tgt[t] < 0 marks an ignored token (e.g. -100).
+ */
+#ifndef SPO_H_
+#define SPO_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define SPO_API __attribute__((visibility("default")))
+#else
+#define SPO_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum spo_status {
+    SPO_OK = 0,
+    SPO_ERR_INVALID_ARG = 1, /* null pointer, bad enum, non-finite scalar */
+    SPO_ERR_SHAPE = 2,       /* sizes out of range or inconsistent         */
+    SPO_ERR_ALIGNMENT = 3,   /* pointer or leading dimension misaligned    */
+    SPO_ERR_WORKSPACE = 4,   /* ws NULL or smaller than *_workspace_size   */
+    SPO_ERR_UNSUPPORTED = 5, /* device is not sm_103 / sm_100 class        */
+    SPO_ERR_CUDA = 6,        /* a CUDA runtime call or launch failed       */
+    SPO_ERR_TIMEOUT = 7      /* a bounded device wait expired              */
+} spo_status;
+
+/* Aggregation of per-token terms into the scalar objective (Eq. 3). */
+typedef enum spo_agg {
+    SPO_AGG_SEQ_GROUP = 0, /* Eq. 3: mean over groups of (1/G) sum_i (1/|o_i|) sum_t */
+    SPO_AGG_TOKEN = 1      /* one mean over every loss token of the batch          */
+} spo_agg;
+
+/* Standard deviation used by the group-normalised advantage. */
+typedef enum spo_std {
+    SPO_STD_UNBIASED = 0,  /* divide the sum of squares by n - 1 */
+    SPO_STD_POPULATION = 1 /* divide by n                        */
+} spo_std;
+
+/* Library version, (major << 16) | minor. */
+SPO_API int spo_version(void);
+
+/* Static text for a status code (never NULL). */
+SPO_API const char* spo_status_string(int status);
+
+/* Copies the calling host thread's description of its last failed call into
+ * buf (NUL-terminated, truncated to n bytes).  Returns the status of that
+ * call (SPO_OK if none failed). */
+SPO_API int spo_last_error(char* buf, size_t n);
+
+/* Reads and clears the device-side error word that bounded waits set on
+ * timeout.  SYNCHRONISES `stream`.  *code receives 0 or the kernel's code.
+ * Returns SPO_ERR_TIMEOUT if a wait expired, else SPO_OK / SPO_ERR_CUDA. */
+SPO_API spo_status spo_device_error(int* code, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * a1. Loss-token selection (section 3, "Multi-turn RL Training": masked
+ * log-probabilities over a truncated window of 1024 tokens).
+ *
+ * Sequence i (one generated output o_i, or one turn of it) spans tokens
+ * [cu_seqlens[i], cu_seqlens[i+1]).  Token t of sequence i is a loss token
+ * when mask[t] == 1, tgt[t] >= 0, and fewer than `window` earlier tokens of the
+ * same sequence are loss tokens (window <= 0: no cap).
+ *
+ *   cu_seqlens int32[n_seq+1]  non-decreasing, cu[0] = 0, cu[n_seq] = T
+ *   mask       uint8[T]        1 = generated token, 0 = prompt/feedback; NULL = all 1
+ *   tgt        int32[T]
+ *   loss_mask  uint8[T]  out   1 for loss tokens, else 0
+ *   n_tok      int32[n_seq] out number of loss tokens of each sequence (|o_i|)
+ * Bit-exact (integer work).  cu_seqlens monotonicity is the caller's contract
+ * (device data is not inspected on the host).
+ * ------------------------------------------------------------------------- */
+SPO_API spo_status spo_token_select(const int32_t* cu_seqlens, const uint8_t* mask,
+                                    const int32_t* tgt, int32_t n_seq, int64_t T, int32_t window,
+                                    uint8_t* loss_mask, int32_t* n_tok, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * a2 + a3. Per-token policy log-probabilities over the full vocabulary: the
+ * pi_theta(o_{i,t} | q, o_{i,<t}) in the ratio of Eq. 3.
+ *
+ *   z_t      = inv_temp * H[t] . W^T           (bf16 inputs, fp32 accumulate)
+ *   lse_t    = log sum_v exp(z_t[v])
+ *   logp[t]  = z_t[tgt[t]] - lse_t             (<= 0)
+ *   entropy[t] = lse_t - sum_v softmax(z_t)[v] z_t[v]   (natural log)
+ *
+ * The T x V logits are produced tile by tile in tensor memory and reduced by
+ * an online max / sum-exp epilogue; only per-(token, vocab-tile) partials and
+ * the three per-token results reach device memory.
+ *
+ *   H        bf16[T, d]  row-major, 16-byte aligned
+ *   W        bf16[V, d]  row-major (LM-head layout), 16-byte aligned
+ *   tgt      int32[T]    values in [0, V) for kept tokens (not range-checked)
+ *   mask     uint8[T]    tokens with mask[t] == 0 are skipped; NULL = keep all
+ *   sizes    1 <= T <= 2^24, 64 <= d <= 65536 with d % 64 == 0,
+ *            256 <= V <= 2^24 with V % 8 == 0
+ *   logp, entropy, lse  fp32[T] out; skipped tokens (mask 0 or tgt < 0) get 0.
+ *            entropy and lse may be NULL.  lse feeds spo_policy_loss_bwd.
+ *   ws       device scratch of at least spo_logprobs_workspace_size bytes,
+ *            256-byte aligned
+ * Accuracy vs an fp64 evaluation on the same bf16 inputs: |d logp| and
+ * |d entropy| are O(1e-5) for d ~ 5e3 (fp32 accumulation and exp2).
+ * ------------------------------------------------------------------------- */
+SPO_API spo_status spo_logprobs_workspace_size(int64_t T, int64_t d, int64_t V, size_t* bytes);
+SPO_API spo_status spo_logprobs_fwd(const void* H, const void* W, const int32_t* tgt,
+                                    const uint8_t* mask, int64_t T, int64_t d, int64_t V,
+                                    float inv_temp, float* logp, float* entropy, float* lse,
+                                    void* ws, size_t ws_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * a4. Group-normalised advantage (definition under Eq. 3):
+ *   A_hat_i = (r_i - mean(r_g)) / (std(r_g) + eps), g = group_id[i].
+ * Members of a group are taken in ascending i; the arithmetic is IEEE fp32
+ * in one fixed order (sum, divide, sum of rounded squared deviations,
+ * divide, sqrt, add eps, divide; no fused multiply-add), so results are
+ * reproducible bit for bit.  Groups of size <= 1 or with all rewards equal
+ * give exactly 0.
+ *
+ *   rewards  fp32[n_seq]   composite reward r_i = R_ver(i) + R_str(i)
+ *   group_id int32[n_seq]  values in [0, n_groups); members need not be contiguous
+ *   adv      fp32[n_seq] out
+ * ------------------------------------------------------------------------- */
+SPO_API spo_status spo_group_advantages(const float* rewards, const int32_t* group_id,
+                                        int32_t n_seq, int32_t n_groups, int std_mode, float eps,
+                                        float* adv, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * a5. Clipped surrogate, KL and aggregation of Eq. 3, forward, plus
+ * g[t] = dL/dlogp[t] for the backward.  Per loss token t of sequence i:
+ *   rho  = exp(logp - old_logp)
+ *   surr = min(rho A_i, clip(rho, 1 - clip_eps, 1 + clip_eps) A_i)
+ *   kl   = exp(ref - logp) - (ref - logp) - 1       (k3 estimator)
+ *   l_t  = -(surr - kl_beta * kl)
+ *   loss = sum_t c_t l_t,  c_t = 1/(N_g |S_g| n_i) (SEQ_GROUP: N_g non-empty
+ *          groups, |S_g| sequences in i's group, n_i loss tokens of i) or
+ *          1/sum_i n_i (TOKEN).
+ *   g[t] = c_t (-A_i rho [clip not binding] + kl_beta (1 - exp(ref - logp)));
+ *          the clip binds when A_i > 0 and rho > 1 + eps, or A_i < 0 and
+ *          rho < 1 - eps (the bound itself counts as not binding).
+ *
+ *   logp, old_logp fp32[T]; ref_logp fp32[T] or NULL (NULL or kl_beta == 0: no KL)
+ *   adv        fp32[n_seq]  per-sequence advantage (broadcast to its tokens)
+ *   cu_seqlens int32[n_seq+1], group_id int32[n_seq] in [0, n_groups)
+ *   loss_mask  uint8[T]  (spo_token_select output)
+ *   loss       fp32[1] out;  g fp32[T] out (0 off the loss set)
+ *   stats      fp32[4] out or NULL: {clip fraction, mean ratio, mean kl,
+ *              number of loss tokens} over loss tokens
+ *   ws         >= spo_policy_loss_workspace_size bytes
+ * The reduction order is fixed (per-sequence sums in fp64, then a
+ * fixed-order sum), so results are run-to-run deterministic.
+ * ------------------------------------------------------------------------- */
+SPO_API spo_status spo_policy_loss_workspace_size(int32_t n_seq, int32_t n_groups, size_t* bytes);
+SPO_API spo_status spo_policy_loss_fwd(const float* logp, const float* old_logp,
+                                       const float* ref_logp, const float* adv,
+                                       const int32_t* cu_seqlens, const int32_t* group_id,
+                                       int32_t n_seq, int32_t n_groups, const uint8_t* loss_mask,
+                                       int64_t T, float clip_eps, float kl_beta, int agg,
+                                       float* loss, float* g, float* stats, void* ws,
+                                       size_t ws_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * a6 - a8. Backward of the loss through the log-probabilities to H and W (the
+ * policy update that maximises Eq. 3):
+ *   G[t, v] = inv_temp * g[t] * (1[v == tgt[t]] - exp(z_t[v] - lse[t]))
+ *   dH      = G W        (bf16 out, fp32 accumulate)
+ *   dW      = G^T H      (fp32 out, fp32 accumulate; += if accumulate_dW)
+ * z is recomputed tile by tile with the tensor cores; G is staged in bf16
+ * scratch (chunks of at most 32768 rows).  Rows with g[t] == 0 contribute
+ * nothing and are skipped; their dH rows are written as 0.
+ *
+ *   H, W, tgt, T, d, V, inv_temp  as in spo_logprobs_fwd
+ *   lse      fp32[T]   from spo_logprobs_fwd
+ *   g        fp32[T]   from spo_policy_loss_fwd
+ *   dH       bf16[T, d] out (may be NULL to skip it)
+ *   dW       fp32[V, d] out (may be NULL to skip it)
+ *   ws       >= spo_policy_loss_bwd_workspace_size bytes
+ * Accuracy vs fp64 on the same inputs: relative L2 error O(1e-3) (bf16 G).
+ * ------------------------------------------------------------------------- */
+SPO_API spo_status spo_policy_loss_bwd_workspace_size(int64_t T, int64_t d, int64_t V,
+                                                      size_t* bytes);
+SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32_t* tgt,
+                                       const float* lse, const float* g, int64_t T, int64_t d,
+                                       int64_t V, float inv_temp, void* dH, float* dW,
+                                       int accumulate_dW, void* ws, size_t ws_bytes, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SPO_H_ */

@@ -1,0 +1,448 @@
+// api.cu -- the C ABI declared in include/spo.h: argument validation on the
+// host, workspace carving, and the launch sequence of each call.
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include "../../include/spo.h"
+#include "internal.h"
+
+namespace {
+
+thread_local char g_err_text[512] = "";
+thread_local int g_err_status = SPO_OK;
+
+// Device error word written by bounded waits that expire.
+__device__ int g_dev_error = 0;
+
+spo_status fail(spo_status st, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err_text, sizeof(g_err_text), fmt, ap);
+  va_end(ap);
+  g_err_status = st;
+  return st;
+}
+
+spo_status ok() {
+  g_err_status = SPO_OK;
+  g_err_text[0] = '\0';
+  return SPO_OK;
+}
+
+spo_status cuda_fail(cudaError_t e, const char* what) {
+  return fail(SPO_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+#define SPO_CUDA(call, what)                       \
+  do {                                             \
+    cudaError_t e_ = (call);                       \
+    if (e_ != cudaSuccess) return cuda_fail(e_, what); \
+  } while (0)
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+long long round_up(long long x, long long m) { return (x + m - 1) / m * m; }
+
+struct DevInfo {
+  int dev = -1;
+  int sms = 0;
+  int major = 0;
+  int* err = nullptr;
+};
+
+spo_status device_info(DevInfo* info) {
+  int dev = 0;
+  SPO_CUDA(cudaGetDevice(&dev), "cudaGetDevice");
+  static DevInfo cache[64];
+  if (dev < 0 || dev >= 64) return fail(SPO_ERR_UNSUPPORTED, "device ordinal %d out of range", dev);
+  DevInfo& c = cache[dev];
+  if (c.dev != dev) {
+    DevInfo n;
+    n.dev = dev;
+    SPO_CUDA(cudaDeviceGetAttribute(&n.sms, cudaDevAttrMultiProcessorCount, dev), "attribute");
+    SPO_CUDA(cudaDeviceGetAttribute(&n.major, cudaDevAttrComputeCapabilityMajor, dev), "attribute");
+    if (n.major != 10)
+      return fail(SPO_ERR_UNSUPPORTED, "device %d has compute capability %d.x; libspo needs sm_103a",
+                  dev, n.major);
+    SPO_CUDA(cudaGetSymbolAddress(reinterpret_cast<void**>(&n.err), g_dev_error),
+             "cudaGetSymbolAddress(error word)");
+    c = n;
+  }
+  *info = c;
+  return SPO_OK;
+}
+
+// Host-side shape checks shared by the forward and backward.
+spo_status check_hwv(const void* H, const void* W, const int32_t* tgt, int64_t T, int64_t d,
+                     int64_t V, float inv_temp) {
+  if (!H || !W || !tgt) return fail(SPO_ERR_INVALID_ARG, "H, W and tgt must be non-NULL");
+  if (T < 1 || T > (1ll << 24)) return fail(SPO_ERR_SHAPE, "T = %lld outside [1, 2^24]", (long long)T);
+  if (d < 64 || d > 65536 || d % 64 != 0)
+    return fail(SPO_ERR_SHAPE, "d = %lld must be a multiple of 64 in [64, 65536]", (long long)d);
+  if (V < 256 || V > (1ll << 24) || V % 8 != 0)
+    return fail(SPO_ERR_SHAPE, "V = %lld must be a multiple of 8 in [256, 2^24]", (long long)V);
+  if (!aligned16(H) || !aligned16(W)) return fail(SPO_ERR_ALIGNMENT, "H and W must be 16-byte aligned");
+  if (!(inv_temp > 0.f) || !isfinite(inv_temp))
+    return fail(SPO_ERR_INVALID_ARG, "inv_temp must be finite and > 0");
+  return SPO_OK;
+}
+
+// ------------------------------------------------------------ workspaces
+struct FwdWs {
+  int* idx;
+  int* count;
+  int* scratch;
+  int* tgt_c;
+  float* ztgt;
+  __nv_bfloat16* Hc;
+  float4* partials;
+  long long T_pad;
+  int nsplit;
+  size_t bytes;
+};
+
+FwdWs carve_fwd(void* base, long long T, long long d, long long V) {
+  FwdWs w{};
+  w.T_pad = round_up(T, spo::BM);
+  w.nsplit = static_cast<int>((V + spo::BN - 1) / spo::BN);
+  const int nb = spo::compact_blocks(T);
+  char* p = static_cast<char*>(base);
+  size_t off = 0;
+  auto take = [&](size_t n) {
+    char* q = p ? p + off : nullptr;
+    off += align256(n);
+    return q;
+  };
+  w.idx = reinterpret_cast<int*>(take(sizeof(int) * w.T_pad));
+  w.count = reinterpret_cast<int*>(take(sizeof(int)));
+  w.scratch = reinterpret_cast<int*>(take(sizeof(int) * 2 * nb));
+  w.tgt_c = reinterpret_cast<int*>(take(sizeof(int) * w.T_pad));
+  w.ztgt = reinterpret_cast<float*>(take(sizeof(float) * w.T_pad));
+  w.Hc = reinterpret_cast<__nv_bfloat16*>(take(sizeof(__nv_bfloat16) * w.T_pad * d));
+  w.partials = reinterpret_cast<float4*>(take(sizeof(float4) * w.nsplit * w.T_pad));
+  w.bytes = off;
+  return w;
+}
+
+constexpr long long kBwdChunkRows = 32768;  // G scratch rows per chunk (multiple of 128)
+
+struct BwdWs {
+  int* idx;
+  int* count;
+  int* scratch;
+  int* tgt_c;
+  float* lse_c;
+  float* g_c;
+  __nv_bfloat16* Hc;
+  __nv_bfloat16* G;
+  long long T_pad;
+  long long chunk;
+  size_t bytes;
+};
+
+BwdWs carve_bwd(void* base, long long T, long long d, long long V) {
+  BwdWs w{};
+  w.T_pad = round_up(T, spo::BM);
+  w.chunk = w.T_pad < kBwdChunkRows ? w.T_pad : kBwdChunkRows;
+  const int nb = spo::compact_blocks(T);
+  char* p = static_cast<char*>(base);
+  size_t off = 0;
+  auto take = [&](size_t n) {
+    char* q = p ? p + off : nullptr;
+    off += align256(n);
+    return q;
+  };
+  w.idx = reinterpret_cast<int*>(take(sizeof(int) * w.T_pad));
+  w.count = reinterpret_cast<int*>(take(sizeof(int)));
+  w.scratch = reinterpret_cast<int*>(take(sizeof(int) * 2 * nb));
+  w.tgt_c = reinterpret_cast<int*>(take(sizeof(int) * w.T_pad));
+  w.lse_c = reinterpret_cast<float*>(take(sizeof(float) * w.T_pad));
+  w.g_c = reinterpret_cast<float*>(take(sizeof(float) * w.T_pad));
+  w.Hc = reinterpret_cast<__nv_bfloat16*>(take(sizeof(__nv_bfloat16) * w.T_pad * d));
+  w.G = reinterpret_cast<__nv_bfloat16*>(take(sizeof(__nv_bfloat16) * w.chunk * V));
+  w.bytes = off;
+  return w;
+}
+
+spo::GemmArgs base_args(const DevInfo& di) {
+  spo::GemmArgs a;
+  memset(&a, 0, sizeof(a));
+  a.group_m = 16;
+  a.scale = 1.f;
+  a.err = di.err;
+  return a;
+}
+
+int grid_for(const DevInfo& di, long long max_m, long long n) {
+  const long long tiles = ((max_m + spo::BM - 1) / spo::BM) * ((n + spo::BN - 1) / spo::BN);
+  long long g = tiles < di.sms ? tiles : di.sms;
+  return static_cast<int>(g < 1 ? 1 : g);
+}
+
+}  // namespace
+
+extern "C" {
+
+SPO_API int spo_version(void) { return (0 << 16) | 1; }
+
+SPO_API const char* spo_status_string(int status) {
+  switch (status) {
+    case SPO_OK: return "SPO_OK";
+    case SPO_ERR_INVALID_ARG: return "SPO_ERR_INVALID_ARG";
+    case SPO_ERR_SHAPE: return "SPO_ERR_SHAPE";
+    case SPO_ERR_ALIGNMENT: return "SPO_ERR_ALIGNMENT";
+    case SPO_ERR_WORKSPACE: return "SPO_ERR_WORKSPACE";
+    case SPO_ERR_UNSUPPORTED: return "SPO_ERR_UNSUPPORTED";
+    case SPO_ERR_CUDA: return "SPO_ERR_CUDA";
+    case SPO_ERR_TIMEOUT: return "SPO_ERR_TIMEOUT";
+    default: return "SPO_ERR_UNKNOWN";
+  }
+}
+
+SPO_API int spo_last_error(char* buf, size_t n) {
+  if (buf && n) {
+    strncpy(buf, g_err_text, n - 1);
+    buf[n - 1] = '\0';
+  }
+  return g_err_status;
+}
+
+SPO_API spo_status spo_device_error(int* code, void* stream) {
+  if (!code) return fail(SPO_ERR_INVALID_ARG, "code must be non-NULL");
+  DevInfo di;
+  spo_status st = device_info(&di);
+  if (st != SPO_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int v = 0;
+  SPO_CUDA(cudaMemcpyAsync(&v, di.err, sizeof(int), cudaMemcpyDeviceToHost, s), "read error word");
+  SPO_CUDA(cudaMemsetAsync(di.err, 0, sizeof(int), s), "clear error word");
+  SPO_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
+  *code = v;
+  if (v != 0) return fail(SPO_ERR_TIMEOUT, "device wait expired (code 0x%x)", v);
+  return ok();
+}
+
+SPO_API spo_status spo_token_select(const int32_t* cu_seqlens, const uint8_t* mask,
+                                    const int32_t* tgt, int32_t n_seq, int64_t T, int32_t window,
+                                    uint8_t* loss_mask, int32_t* n_tok, void* stream) {
+  if (!cu_seqlens || !tgt || !loss_mask || !n_tok)
+    return fail(SPO_ERR_INVALID_ARG, "cu_seqlens, tgt, loss_mask and n_tok must be non-NULL");
+  if (n_seq < 1 || n_seq > (1 << 24)) return fail(SPO_ERR_SHAPE, "n_seq = %d outside [1, 2^24]", n_seq);
+  if (T < 1 || T > (1ll << 31) - 1) return fail(SPO_ERR_SHAPE, "T = %lld out of range", (long long)T);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  SPO_CUDA(spo::launch_token_select(cu_seqlens, mask, tgt, n_seq, window, loss_mask, n_tok, s),
+           "token_select launch");
+  return ok();
+}
+
+SPO_API spo_status spo_logprobs_workspace_size(int64_t T, int64_t d, int64_t V, size_t* bytes) {
+  if (!bytes) return fail(SPO_ERR_INVALID_ARG, "bytes must be non-NULL");
+  if (T < 1 || d < 1 || V < 1) return fail(SPO_ERR_SHAPE, "sizes must be positive");
+  *bytes = carve_fwd(nullptr, T, d, V).bytes;
+  return ok();
+}
+
+SPO_API spo_status spo_logprobs_fwd(const void* H, const void* W, const int32_t* tgt,
+                                    const uint8_t* mask, int64_t T, int64_t d, int64_t V,
+                                    float inv_temp, float* logp, float* entropy, float* lse,
+                                    void* ws, size_t ws_bytes, void* stream) {
+  spo_status st = check_hwv(H, W, tgt, T, d, V, inv_temp);
+  if (st != SPO_OK) return st;
+  if (!logp) return fail(SPO_ERR_INVALID_ARG, "logp must be non-NULL");
+  const FwdWs need = carve_fwd(nullptr, T, d, V);
+  if (!ws || ws_bytes < need.bytes)
+    return fail(SPO_ERR_WORKSPACE, "workspace needs %zu bytes, got %zu", need.bytes, ws_bytes);
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
+    return fail(SPO_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
+  DevInfo di;
+  if ((st = device_info(&di)) != SPO_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const FwdWs w = carve_fwd(ws, T, d, V);
+
+  // a1 (row selection) + gather of the kept rows into a dense bf16 block
+  SPO_CUDA(spo::launch_compact(0, mask, tgt, nullptr, T, w.scratch, w.idx, w.count, s), "compact");
+  SPO_CUDA(spo::launch_gather(static_cast<const __nv_bfloat16*>(H), static_cast<int>(d), w.idx,
+                              w.count, static_cast<int>(w.T_pad), w.Hc, tgt, w.tgt_c, nullptr,
+                              nullptr, nullptr, nullptr, s),
+           "gather");
+  // a2: logits tile by tile + online logsumexp partials
+  CUtensorMap ta, tb;
+  SPO_CUDA(spo::make_tmap_bf16(&ta, w.Hc, d, w.T_pad, d * 2, spo::BK, spo::BM), "tensor map H");
+  SPO_CUDA(spo::make_tmap_bf16(&tb, W, d, V, d * 2, spo::BK, spo::BN), "tensor map W");
+  spo::GemmArgs a = base_args(di);
+  a.m_count = w.count;
+  a.m_offset = 0;
+  a.m_cap = static_cast<int>(w.T_pad);
+  a.n = static_cast<int>(V);
+  a.k_static = static_cast<int>(d);
+  a.scale = inv_temp;
+  a.tgt = w.tgt_c;
+  a.partials = w.partials;
+  a.ld_part = static_cast<int>(w.T_pad);
+  a.ztgt = w.ztgt;
+  SPO_CUDA(spo::launch_gemm(spo::EPI_LSE, false, false, ta, tb, a, grid_for(di, w.T_pad, V), s),
+           "lse gemm launch");
+  // a3: split-vocab combine, scattered back to token positions (skipped tokens read 0)
+  SPO_CUDA(cudaMemsetAsync(logp, 0, sizeof(float) * T, s), "memset logp");
+  if (entropy) SPO_CUDA(cudaMemsetAsync(entropy, 0, sizeof(float) * T, s), "memset entropy");
+  if (lse) SPO_CUDA(cudaMemsetAsync(lse, 0, sizeof(float) * T, s), "memset lse");
+  SPO_CUDA(spo::launch_lse_combine(w.partials, static_cast<int>(w.T_pad), w.nsplit, w.ztgt, w.idx,
+                                   w.count, static_cast<int>(w.T_pad), logp, entropy, lse, s),
+           "combine launch");
+  return ok();
+}
+
+SPO_API spo_status spo_group_advantages(const float* rewards, const int32_t* group_id,
+                                        int32_t n_seq, int32_t n_groups, int std_mode, float eps,
+                                        float* adv, void* stream) {
+  if (!rewards || !group_id || !adv)
+    return fail(SPO_ERR_INVALID_ARG, "rewards, group_id and adv must be non-NULL");
+  if (n_seq < 1 || n_groups < 1 || n_seq > (1 << 26) || n_groups > (1 << 26))
+    return fail(SPO_ERR_SHAPE, "n_seq = %d, n_groups = %d out of range", n_seq, n_groups);
+  if (std_mode != SPO_STD_UNBIASED && std_mode != SPO_STD_POPULATION)
+    return fail(SPO_ERR_INVALID_ARG, "std_mode %d unknown", std_mode);
+  if (!(eps >= 0.f) || !isfinite(eps)) return fail(SPO_ERR_INVALID_ARG, "eps must be finite and >= 0");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  SPO_CUDA(spo::launch_group_advantages(rewards, group_id, n_seq, n_groups, std_mode, eps, adv, s),
+           "advantage launch");
+  return ok();
+}
+
+SPO_API spo_status spo_policy_loss_workspace_size(int32_t n_seq, int32_t n_groups, size_t* bytes) {
+  if (!bytes) return fail(SPO_ERR_INVALID_ARG, "bytes must be non-NULL");
+  if (n_seq < 1 || n_groups < 1) return fail(SPO_ERR_SHAPE, "n_seq and n_groups must be >= 1");
+  *bytes = spo::loss_ws_bytes(n_seq, n_groups);
+  return ok();
+}
+
+SPO_API spo_status spo_policy_loss_fwd(const float* logp, const float* old_logp,
+                                       const float* ref_logp, const float* adv,
+                                       const int32_t* cu_seqlens, const int32_t* group_id,
+                                       int32_t n_seq, int32_t n_groups, const uint8_t* loss_mask,
+                                       int64_t T, float clip_eps, float kl_beta, int agg,
+                                       float* loss, float* g, float* stats, void* ws,
+                                       size_t ws_bytes, void* stream) {
+  if (!logp || !old_logp || !adv || !cu_seqlens || !group_id || !loss_mask || !loss || !g)
+    return fail(SPO_ERR_INVALID_ARG, "a required pointer is NULL");
+  if (n_seq < 1 || n_groups < 1 || n_seq > (1 << 24) || n_groups > (1 << 24))
+    return fail(SPO_ERR_SHAPE, "n_seq = %d, n_groups = %d out of range", n_seq, n_groups);
+  if (T < 1 || T > (1ll << 31) - 1) return fail(SPO_ERR_SHAPE, "T = %lld out of range", (long long)T);
+  if (agg != SPO_AGG_SEQ_GROUP && agg != SPO_AGG_TOKEN)
+    return fail(SPO_ERR_INVALID_ARG, "agg %d unknown", agg);
+  if (!(clip_eps >= 0.f && clip_eps < 1.f)) return fail(SPO_ERR_INVALID_ARG, "clip_eps must be in [0, 1)");
+  if (!isfinite(kl_beta)) return fail(SPO_ERR_INVALID_ARG, "kl_beta must be finite");
+  const size_t need = spo::loss_ws_bytes(n_seq, n_groups);
+  if (!ws || ws_bytes < need)
+    return fail(SPO_ERR_WORKSPACE, "workspace needs %zu bytes, got %zu", need, ws_bytes);
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
+    return fail(SPO_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const spo::LossWs w = spo::carve_loss_ws(ws, n_seq, n_groups);
+  SPO_CUDA(spo::launch_policy_loss(logp, old_logp, ref_logp, adv, cu_seqlens, group_id, n_seq,
+                                   n_groups, loss_mask, T, clip_eps, kl_beta, agg, loss, g, stats,
+                                   w, s),
+           "policy loss launch");
+  return ok();
+}
+
+SPO_API spo_status spo_policy_loss_bwd_workspace_size(int64_t T, int64_t d, int64_t V,
+                                                      size_t* bytes) {
+  if (!bytes) return fail(SPO_ERR_INVALID_ARG, "bytes must be non-NULL");
+  if (T < 1 || d < 1 || V < 1) return fail(SPO_ERR_SHAPE, "sizes must be positive");
+  *bytes = carve_bwd(nullptr, T, d, V).bytes;
+  return ok();
+}
+
+SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32_t* tgt,
+                                       const float* lse, const float* g, int64_t T, int64_t d,
+                                       int64_t V, float inv_temp, void* dH, float* dW,
+                                       int accumulate_dW, void* ws, size_t ws_bytes, void* stream) {
+  spo_status st = check_hwv(H, W, tgt, T, d, V, inv_temp);
+  if (st != SPO_OK) return st;
+  if (!lse || !g) return fail(SPO_ERR_INVALID_ARG, "lse and g must be non-NULL");
+  if (dH && !aligned16(dH)) return fail(SPO_ERR_ALIGNMENT, "dH must be 16-byte aligned");
+  if (dW && !aligned16(dW)) return fail(SPO_ERR_ALIGNMENT, "dW must be 16-byte aligned");
+  const BwdWs need = carve_bwd(nullptr, T, d, V);
+  if (!ws || ws_bytes < need.bytes)
+    return fail(SPO_ERR_WORKSPACE, "workspace needs %zu bytes, got %zu", need.bytes, ws_bytes);
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
+    return fail(SPO_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
+  DevInfo di;
+  if ((st = device_info(&di)) != SPO_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const BwdWs w = carve_bwd(ws, T, d, V);
+  if (!dH && !dW) return ok();
+
+  // rows with g != 0 are the only ones with a non-zero gradient row
+  SPO_CUDA(spo::launch_compact(1, nullptr, nullptr, g, T, w.scratch, w.idx, w.count, s), "compact");
+  SPO_CUDA(spo::launch_gather(static_cast<const __nv_bfloat16*>(H), static_cast<int>(d), w.idx,
+                              w.count, static_cast<int>(w.T_pad), w.Hc, tgt, w.tgt_c, lse, w.lse_c,
+                              g, w.g_c, s),
+           "gather");
+  if (dH) SPO_CUDA(cudaMemsetAsync(dH, 0, sizeof(uint16_t) * T * d, s), "memset dH");
+
+  CUtensorMap tW_k, tW_mn, tG_k, tG_mn;
+  SPO_CUDA(spo::make_tmap_bf16(&tW_k, W, d, V, d * 2, spo::BK, spo::BN), "tensor map W");
+  SPO_CUDA(spo::make_tmap_bf16(&tW_mn, W, d, V, d * 2, 64, spo::BK), "tensor map W (MN)");
+  SPO_CUDA(spo::make_tmap_bf16(&tG_k, w.G, V, w.chunk, V * 2, spo::BK, spo::BM), "tensor map G");
+  SPO_CUDA(spo::make_tmap_bf16(&tG_mn, w.G, V, w.chunk, V * 2, 64, spo::BK), "tensor map G (MN)");
+
+  const long long n_chunks = (w.T_pad + w.chunk - 1) / w.chunk;
+  for (long long c = 0; c < n_chunks; ++c) {
+    const long long r0 = c * w.chunk;
+    const long long rows = (w.T_pad - r0) < w.chunk ? (w.T_pad - r0) : w.chunk;
+    const __nv_bfloat16* Hc0 = w.Hc + r0 * d;
+    CUtensorMap tH_k, tH_mn;
+    SPO_CUDA(spo::make_tmap_bf16(&tH_k, Hc0, d, rows, d * 2, spo::BK, spo::BM), "tensor map Hc");
+    SPO_CUDA(spo::make_tmap_bf16(&tH_mn, Hc0, d, rows, d * 2, 64, spo::BK), "tensor map Hc (MN)");
+
+    // a6: G = inv_temp * g * (onehot - softmax), logits recomputed
+    spo::GemmArgs a = base_args(di);
+    a.m_count = w.count;
+    a.m_offset = static_cast<int>(r0);
+    a.m_cap = static_cast<int>(w.chunk);
+    a.n = static_cast<int>(V);
+    a.k_static = static_cast<int>(d);
+    a.scale = inv_temp;
+    a.tgt = w.tgt_c + r0;
+    a.lse = w.lse_c + r0;
+    a.gvec = w.g_c + r0;
+    a.G = w.G;
+    a.ldG = V;
+    SPO_CUDA(spo::launch_gemm(spo::EPI_GRAD, false, false, tH_k, tW_k, a, grid_for(di, rows, V), s),
+             "grad gemm launch");
+    // a7: dH rows = G W, scattered to token rows
+    if (dH) {
+      spo::GemmArgs b = base_args(di);
+      b.m_count = w.count;
+      b.m_offset = static_cast<int>(r0);
+      b.m_cap = static_cast<int>(w.chunk);
+      b.n = static_cast<int>(d);
+      b.k_static = static_cast<int>(V);
+      b.row_idx = w.idx + r0;
+      b.out_bf16 = static_cast<__nv_bfloat16*>(dH);
+      b.ld_out = d;
+      SPO_CUDA(spo::launch_gemm(spo::EPI_DH, false, true, tG_k, tW_mn, b, grid_for(di, rows, d), s),
+               "dH gemm launch");
+    }
+    // a8: dW (+)= G^T Hc over this chunk's rows
+    if (dW) {
+      spo::GemmArgs b = base_args(di);
+      b.m_static = static_cast<int>(V);
+      b.n = static_cast<int>(d);
+      b.k_count = w.count;
+      b.k_offset = static_cast<int>(r0);
+      b.k_cap = static_cast<int>(w.chunk);
+      b.out_f32 = dW;
+      b.ld_out = d;
+      b.accumulate = (c == 0) ? (accumulate_dW ? 1 : 0) : 1;
+      SPO_CUDA(spo::launch_gemm(spo::EPI_DW, true, true, tG_mn, tH_mn, b, grid_for(di, V, d), s),
+               "dW gemm launch");
+    }
+  }
+  return ok();
+}
+
+}  // extern "C"

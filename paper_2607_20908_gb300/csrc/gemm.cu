@@ -1,0 +1,456 @@
+// gemm.cu -- persistent, warp-specialised tcgen05 GEMM for sm_103a with the
+// fused epilogues of the GRPO log-prob path.
+//
+//   C[M, N] = A[M, K] * B[N, K]^T    (bf16 in, fp32 accumulate in TMEM)
+//
+// One CTA per SM walks output tiles of 128 x 256.  Warp 0 issues TMA loads
+// into a 4-stage shared-memory ring, warp 1 issues tcgen05.mma (one thread)
+// into one of two TMEM accumulators (2 x 256 columns), warps 2-5 drain the
+// other accumulator through the epilogue, so MMA and epilogue overlap.
+// Operands may be K-major (rows of K contiguous) or MN-major (rows of M or N
+// contiguous); both are staged with the 128-byte swizzle.
+//
+// The epilogues are the four places where the path touches the logits:
+//   EPI_LSE  : forward. Online max / sum-exp / sum-exp*z of each row over the
+//              tile plus the target logit; writes one partial per
+//              (vocab tile, row).  The logits themselves never leave TMEM.
+//   EPI_GRAD : backward. G = inv_temp * g_t * (onehot - exp(z - lse_t)) in bf16.
+//   EPI_DH   : dH = G W rows, bf16, scattered back to token rows.
+//   EPI_DW   : dW = G^T H rows, fp32, overwrite or accumulate.
+#include <math.h>
+
+#include "internal.h"
+#include "tc.cuh"
+
+namespace spo {
+
+namespace {
+
+constexpr uint32_t A_BYTES = BM * BK * 2;          // 16 KB
+constexpr uint32_t B_BYTES = BN * BK * 2;          // 32 KB
+constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr uint32_t MN_BLOCK_BYTES = 64 * BK * 2;   // [BK rows][64 MN] block, 8 KB
+constexpr int NUM_THREADS = 192;
+constexpr float kLog2e = 1.4426950408889634f;
+
+__device__ __forceinline__ int clampi(int v, int lo, int hi) { return v < lo ? lo : (v > hi ? hi : v); }
+
+// Grouped raster: `gm` tile rows are walked together across all tile columns,
+// so the A rows of a group stay in L2 while B streams past them.
+__device__ __forceinline__ void tile_coords(int tile, int mt, int nt, int gm, int& mb, int& nb) {
+  const int per_group = gm * nt;
+  const int group = tile / per_group;
+  const int first = group * gm;
+  const int size = min(gm, mt - first);
+  const int in = tile - group * per_group;
+  mb = first + in % size;
+  nb = in / size;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+// ------------------------------------------------------------ epilogues
+// Each thread owns one accumulator row (TMEM lane) and walks its 256 columns
+// in 8 chunks of 32.
+
+__device__ __forceinline__ void epi_lse(const GemmArgs& p, uint32_t taddr, int row, int M, int nb) {
+  const bool row_ok = row < M;
+  const int y = row_ok ? p.tgt[row] : -1;
+  const float sc2 = p.scale * kLog2e;  // logits in log2 units: t = z * log2(e)
+  const int col_base = nb * BN;
+  const bool full = col_base + BN <= p.n;
+  float run_m = -INFINITY, run_s = 0.f, run_e = 0.f, zt = 0.f;
+  bool hit = false;
+#pragma unroll 1
+  for (int c = 0; c < BN / 32; ++c) {
+    float v[32];
+    tmem_ld32(taddr + c * 32, v);
+    const int c0 = col_base + c * 32;
+    if (y >= c0 && y < c0 + 32) {
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (c0 + j == y) zt = v[j] * p.scale;
+      hit = true;
+    }
+    float cm = -INFINITY;
+    if (full) {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) cm = fmaxf(cm, v[j]);
+    } else {
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (c0 + j < p.n) cm = fmaxf(cm, v[j]);
+    }
+    if (c0 >= p.n) continue;  // chunk entirely past the vocabulary (warp-uniform)
+    const float nm = fmaxf(run_m, cm * sc2);
+    const float r = exp2f(run_m - nm);
+    run_s *= r;
+    run_e *= r;
+    if (full) {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) {
+        const float t = v[j] * sc2;
+        const float e = exp2f(t - nm);
+        run_s += e;
+        run_e = fmaf(e, t, run_e);
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) {
+        if (c0 + j < p.n) {
+          const float t = v[j] * sc2;
+          const float e = exp2f(t - nm);
+          run_s += e;
+          run_e = fmaf(e, t, run_e);
+        }
+      }
+    }
+    run_m = nm;
+  }
+  if (row_ok) {
+    p.partials[static_cast<size_t>(nb) * p.ld_part + row] = make_float4(run_m, run_s, run_e, 0.f);
+    if (hit) p.ztgt[row] = zt;
+  }
+}
+
+__device__ __forceinline__ void epi_grad(const GemmArgs& p, uint32_t taddr, int row, int M, int nb) {
+  const bool row_ok = row < M;
+  const float gl = row_ok ? p.gvec[row] : 0.f;
+  const float l2 = row_ok ? p.lse[row] * kLog2e : 0.f;
+  const int y = row_ok ? p.tgt[row] : -1;
+  const float coef = p.scale * gl;
+  const float sc2 = p.scale * kLog2e;
+  const int col_base = nb * BN;
+  __nv_bfloat16* grow = p.G + static_cast<size_t>(row) * p.ldG;
+#pragma unroll 1
+  for (int c = 0; c < BN / 32; ++c) {
+    const int c0 = col_base + c * 32;
+    if (c0 >= p.n) break;  // warp-uniform
+    float v[32];
+    tmem_ld32(taddr + c * 32, v);
+    uint32_t pk[16];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      const int ca = c0 + 2 * j;
+      const float pa = exp2f(fmaf(v[2 * j], sc2, -l2));
+      const float pb = exp2f(fmaf(v[2 * j + 1], sc2, -l2));
+      const float ga = coef * ((ca == y ? 1.f : 0.f) - pa);
+      const float gb = coef * ((ca + 1 == y ? 1.f : 0.f) - pb);
+      pk[j] = pack_bf16x2(ga, gb);
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      if (c0 + 8 * q < p.n)
+        *reinterpret_cast<uint4*>(grow + c0 + 8 * q) =
+            make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+  }
+}
+
+__device__ __forceinline__ void epi_dh(const GemmArgs& p, uint32_t taddr, int row, int M, int nb) {
+  const bool row_ok = row < M;
+  const int out_row = row_ok ? (p.row_idx ? p.row_idx[row] : row) : 0;
+  __nv_bfloat16* dst = p.out_bf16 + static_cast<size_t>(out_row) * p.ld_out;
+  const int col_base = nb * BN;
+#pragma unroll 1
+  for (int c = 0; c < BN / 32; ++c) {
+    const int c0 = col_base + c * 32;
+    if (c0 >= p.n) break;
+    float v[32];
+    tmem_ld32(taddr + c * 32, v);
+    if (!row_ok) continue;
+    uint32_t pk[16];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) pk[j] = pack_bf16x2(v[2 * j], v[2 * j + 1]);
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      if (c0 + 8 * q < p.n)
+        *reinterpret_cast<uint4*>(dst + c0 + 8 * q) =
+            make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+  }
+}
+
+__device__ __forceinline__ void epi_dw(const GemmArgs& p, uint32_t taddr, int row, int M, int nb,
+                                       bool kzero) {
+  const bool row_ok = row < M;
+  float* dst = p.out_f32 + static_cast<size_t>(row_ok ? row : 0) * p.ld_out;
+  const int col_base = nb * BN;
+#pragma unroll 1
+  for (int c = 0; c < BN / 32; ++c) {
+    const int c0 = col_base + c * 32;
+    if (c0 >= p.n) break;
+    float v[32];
+    if (kzero) {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) v[j] = 0.f;
+    } else {
+      tmem_ld32(taddr + c * 32, v);
+    }
+    if (!row_ok) continue;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      if (c0 + 4 * q < p.n) {
+        float4* d4 = reinterpret_cast<float4*>(dst + c0 + 4 * q);
+        float4 o = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+        if (p.accumulate) {
+          const float4 a = *d4;
+          o.x += a.x; o.y += a.y; o.z += a.z; o.w += a.w;
+        }
+        *d4 = o;
+      }
+    }
+  }
+}
+
+// ------------------------------------------------------------ the kernel
+template <int EPI, bool A_MN, bool B_MN>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                const GemmArgs p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + STAGES * A_BYTES;
+  uint64_t* full_bar = reinterpret_cast<uint64_t*>(sB + STAGES * B_BYTES);
+  uint64_t* empty_bar = full_bar + STAGES;
+  uint64_t* tfull_bar = empty_bar + STAGES;
+  uint64_t* tempty_bar = tfull_bar + 2;
+  uint64_t* drain_bar = tempty_bar + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  const int M = p.m_count ? clampi(*p.m_count - p.m_offset, 0, p.m_cap) : p.m_static;
+  const int K = p.k_count ? clampi(*p.k_count - p.k_offset, 0, p.k_cap) : p.k_static;
+  const int mt = (M + BM - 1) / BM;
+  const int nt = (p.n + BN - 1) / BN;
+  const int num_tiles = mt * nt;
+  const int num_kb = (K + BK - 1) / BK;
+  const int gm = max(1, p.group_m);
+  // dW += (empty chunk): nothing to add.  Uniform across the CTA, before any setup.
+  if (EPI == EPI_DW && num_kb == 0 && p.accumulate) return;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full_bar[s], 1);
+      mbar_init(&empty_bar[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull_bar[a], 1);
+      mbar_init(&tempty_bar[a], 4);  // one arrival per epilogue warp
+    }
+    mbar_init(drain_bar, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, 2 * BN);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    // ------------------------------------------------ TMA producer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int issued = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+        int mb, nb;
+        tile_coords(tile, mt, nt, gm, mb, nb);
+        for (int kb = 0; kb < num_kb; ++kb) {
+          if (!mbar_wait(&empty_bar[stage], phase ^ 1u, abort_flag, p.err, kErrWaitProducer)) {
+            ok = false;
+            break;
+          }
+          uint8_t* a_dst = sA + stage * A_BYTES;
+          uint8_t* b_dst = sB + stage * B_BYTES;
+          mbar_arrive_expect_tx(&full_bar[stage], STAGE_BYTES);
+          if (A_MN) {
+#pragma unroll
+            for (int j = 0; j < BM / 64; ++j)
+              tma_load_2d(a_dst + j * MN_BLOCK_BYTES, &tmA, &full_bar[stage], mb * BM + j * 64, kb * BK);
+          } else {
+            tma_load_2d(a_dst, &tmA, &full_bar[stage], kb * BK, mb * BM);
+          }
+          if (B_MN) {
+#pragma unroll
+            for (int j = 0; j < BN / 64; ++j)
+              tma_load_2d(b_dst + j * MN_BLOCK_BYTES, &tmB, &full_bar[stage], nb * BN + j * 64, kb * BK);
+          } else {
+            tma_load_2d(b_dst, &tmB, &full_bar[stage], kb * BK, nb * BN);
+          }
+          ++issued;
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      if (!ok) {
+        // Aborted: let the copies already in flight land before the CTA exits.
+        int s = stage;
+        uint32_t ph = phase;
+        for (int i = 0; i < STAGES && i < issued; ++i) {
+          if (--s < 0) {
+            s = STAGES - 1;
+            ph ^= 1u;
+          }
+          mbar_wait_drain(&full_bar[s], ph);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t kIdesc = idesc_bf16_f32(BM, BN, A_MN, B_MN);
+      int stage = 0;
+      uint32_t phase = 0;
+      int local = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++local) {
+        const int acc = local & 1;
+        const uint32_t acc_phase = (local >> 1) & 1;
+        if (!mbar_wait(&tempty_bar[acc], acc_phase ^ 1u, abort_flag, p.err, kErrWaitMma)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
+        for (int kb = 0; kb < num_kb; ++kb) {
+          if (!mbar_wait(&full_bar[stage], phase, abort_flag, p.err, kErrWaitMma)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(sA + stage * A_BYTES);
+          const uint32_t b0 = smem_u32(sB + stage * B_BYTES);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k) {
+            const uint64_t ad = A_MN ? sdesc_sw128(a0 + k * 2048, MN_BLOCK_BYTES, 1024)
+                                     : sdesc_sw128(a0 + k * 32, 16, 1024);
+            const uint64_t bd = B_MN ? sdesc_sw128(b0 + k * 2048, MN_BLOCK_BYTES, 1024)
+                                     : sdesc_sw128(b0 + k * 32, 16, 1024);
+            umma_bf16(d_tmem, ad, bd, kIdesc, (kb | k) != 0 ? 1u : 0u);
+          }
+          umma_commit(&empty_bar[stage]);  // frees the stage when these MMAs finish
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        if (num_kb > 0)
+          umma_commit(&tfull_bar[acc]);  // accumulator complete
+        else
+          mbar_arrive(&tfull_bar[acc]);  // K == 0: nothing to wait for
+      }
+      // Every MMA this thread issued must finish before TMEM is released.
+      umma_commit(drain_bar);
+      if (!mbar_wait_drain(drain_bar, 0) && p.err) atomicCAS(p.err, 0, kErrWaitDrain);
+    }
+  } else {
+    // ------------------------------------------------ epilogue warps 2..5
+    const int q = warp & 3;  // TMEM lanes [32q, 32q+32) are reachable from this warp
+    int local = 0;
+    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++local) {
+      const int acc = local & 1;
+      const uint32_t acc_phase = (local >> 1) & 1;
+      int mb, nb;
+      tile_coords(tile, mt, nt, gm, mb, nb);
+      const bool ok = mbar_wait(&tfull_bar[acc], acc_phase, abort_flag, p.err, kErrWaitEpilogue);
+      if (!__all_sync(0xffffffffu, ok)) break;
+      tc_fence_after();
+      const int row = mb * BM + q * 32 + lane;
+      const uint32_t taddr =
+          tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN);
+      if (EPI == EPI_LSE) epi_lse(p, taddr, row, M, nb);
+      if (EPI == EPI_GRAD) epi_grad(p, taddr, row, M, nb);
+      if (EPI == EPI_DH) epi_dh(p, taddr, row, M, nb);
+      if (EPI == EPI_DW) epi_dw(p, taddr, row, M, nb, num_kb == 0);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty_bar[acc]);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem_base, 2 * BN);
+  }
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  }
+  return fn;
+}
+
+template <int EPI, bool A_MN, bool B_MN>
+cudaError_t launch_one(const CUtensorMap& ta, const CUtensorMap& tb, const GemmArgs& args, int grid,
+                       cudaStream_t s) {
+  auto k = gemm_kernel<EPI, A_MN, B_MN>;
+  const size_t smem = gemm_smem_bytes();
+  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  k<<<grid, NUM_THREADS, smem, s>>>(ta, tb, args);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+size_t gemm_smem_bytes() { return 1024 + STAGES * STAGE_BYTES + 128; }
+
+cudaError_t make_tmap_bf16(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer,
+                           uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return cudaErrorNotSupported;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {row_bytes};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+cudaError_t launch_gemm(int epi, bool a_mn, bool b_mn, const CUtensorMap& ta, const CUtensorMap& tb,
+                        const GemmArgs& args, int grid, cudaStream_t s) {
+  if (epi == EPI_LSE && !a_mn && !b_mn) return launch_one<EPI_LSE, false, false>(ta, tb, args, grid, s);
+  if (epi == EPI_GRAD && !a_mn && !b_mn) return launch_one<EPI_GRAD, false, false>(ta, tb, args, grid, s);
+  if (epi == EPI_DH && !a_mn && b_mn) return launch_one<EPI_DH, false, true>(ta, tb, args, grid, s);
+  if (epi == EPI_DW && a_mn && b_mn) return launch_one<EPI_DW, true, true>(ta, tb, args, grid, s);
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace spo

@@ -1,0 +1,117 @@
+// internal.h -- interface between the C-ABI layer (api.cu) and the kernels.
+// Not part of the public ABI.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace spo {
+
+// Tensor-core tile: 128 rows x 256 columns per CTA, K staged 64 at a time
+// (one 128-byte swizzle atom of bf16), 4-deep shared-memory ring.
+constexpr int BM = 128;
+constexpr int BN = 256;
+constexpr int BK = 64;
+constexpr int STAGES = 4;
+
+// What the epilogue does with a finished 128 x 256 fp32 accumulator tile.
+enum EpiKind : int {
+  EPI_LSE = 0,   // online max / sum-exp / sum-exp*z per row + target logit -> partials
+  EPI_GRAD = 1,  // G = scale * g_row * (onehot - exp(scale*acc - lse_row)) -> bf16
+  EPI_DH = 2,    // bf16 rows scattered to row_idx[row]
+  EPI_DW = 3,    // fp32 rows, overwrite or accumulate
+};
+
+struct GemmArgs {
+  // rows M: m_static, or clamp(*m_count - m_offset, 0, m_cap) read on the device
+  int m_static;
+  const int* m_count;
+  int m_offset;
+  int m_cap;
+  int n;  // columns N
+  // reduction length K: k_static, or clamp(*k_count - k_offset, 0, k_cap) on the device
+  int k_static;
+  const int* k_count;
+  int k_offset;
+  int k_cap;
+  int group_m;  // rows of tiles walked together (L2 reuse of the B operand)
+  float scale;  // inv_temp for EPI_LSE / EPI_GRAD
+  // EPI_LSE
+  const int* tgt;     // target id of each row
+  float4* partials;   // [ceil(n / BN)][ld_part]: (max*log2e, sum 2^(t-max), sum 2^(t-max) t, 0)
+  int ld_part;
+  float* ztgt;        // target logit (natural units) of each row
+  // EPI_GRAD
+  const float* lse;   // natural-log lse of each row
+  const float* gvec;  // dL/dlogp of each row
+  __nv_bfloat16* G;   // [rows][ldG]
+  long long ldG;
+  // EPI_DH
+  const int* row_idx;         // output row of each row (NULL: identity)
+  __nv_bfloat16* out_bf16;
+  long long ld_out;
+  // EPI_DW
+  float* out_f32;
+  int accumulate;
+  int* err;  // device error word
+};
+
+size_t gemm_smem_bytes();
+
+// Encodes a 2-D bf16 tensor map with 128-byte swizzle.  inner/outer are the
+// extents in elements / rows, row_bytes the pitch, box the staged tile.
+cudaError_t make_tmap_bf16(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer,
+                           uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer);
+
+// Supported (epi, a_mn, b_mn): (LSE,0,0) (GRAD,0,0) (DH,0,1) (DW,1,1).
+cudaError_t launch_gemm(int epi, bool a_mn, bool b_mn, const CUtensorMap& ta,
+                        const CUtensorMap& tb, const GemmArgs& args, int grid,
+                        cudaStream_t s);
+
+// ---------------------------------------------------------------- small kernels
+// Compaction of selected rows: kind 0 selects (mask == NULL || mask[t]) &&
+// tgt[t] >= 0, kind 1 selects g[t] != 0.  Writes idx[0..count) ascending and
+// *count.  scratch holds 2 * compact_blocks(T) ints.
+int compact_blocks(long long T);
+cudaError_t launch_compact(int kind, const uint8_t* mask, const int* tgt, const float* g,
+                           long long T, int* scratch, int* idx, int* count, cudaStream_t s);
+
+// Hc[r] = H[idx[r]] for r < count and 0 for count <= r < round_up(count, 128)
+// (r < rows_cap); also gathers up to three per-row vectors (NULL to skip).
+cudaError_t launch_gather(const __nv_bfloat16* H, int d, const int* idx, const int* count,
+                          int rows_cap, __nv_bfloat16* Hc, const int* tgt, int* tgt_c,
+                          const float* a, float* a_c, const float* b, float* b_c,
+                          cudaStream_t s);
+
+cudaError_t launch_lse_combine(const float4* partials, int ld_part, int nsplit,
+                               const float* ztgt, const int* idx, const int* count,
+                               int rows_cap, float* logp, float* entropy, float* lse,
+                               cudaStream_t s);
+
+cudaError_t launch_token_select(const int* cu_seqlens, const uint8_t* mask, const int* tgt,
+                                int n_seq, int window, uint8_t* loss_mask, int* n_tok,
+                                cudaStream_t s);
+
+cudaError_t launch_group_advantages(const float* rewards, const int* group_id, int n_seq,
+                                    int n_groups, int std_mode, float eps, float* adv,
+                                    cudaStream_t s);
+
+struct LossWs {
+  int* gsize;        // [n_groups]
+  int* n_tok;        // [n_seq]
+  long long* scal;   // [2]: non-empty groups, total loss tokens
+  double* part;      // [n_seq][3]: sum c*l, sum rho, sum kl
+  int* part_clip;    // [n_seq]
+};
+size_t loss_ws_bytes(int n_seq, int n_groups);
+LossWs carve_loss_ws(void* ws, int n_seq, int n_groups);
+
+cudaError_t launch_policy_loss(const float* logp, const float* old_logp, const float* ref_logp,
+                               const float* adv, const int* cu_seqlens, const int* group_id,
+                               int n_seq, int n_groups, const uint8_t* loss_mask, long long T,
+                               float clip_eps, float kl_beta, int agg, float* loss, float* g,
+                               float* stats, const LossWs& w, cudaStream_t s);
+
+}  // namespace spo

@@ -1,0 +1,487 @@
+// small.cu -- the bandwidth- and latency-bound steps of the path: loss-token
+// selection, row compaction and gather, the split-vocabulary logsumexp
+// combine, group-normalised advantages and the policy-loss forward.
+#include <math.h>
+
+#include "internal.h"
+
+namespace spo {
+
+namespace {
+
+constexpr int kCompactThreads = 256;
+constexpr int kCompactItems = 4;
+constexpr int kCompactTile = kCompactThreads * kCompactItems;  // tokens per block
+constexpr float kLn2 = 0.69314718055994531f;
+
+__device__ __forceinline__ bool selected(int kind, const uint8_t* mask, const int* tgt,
+                                         const float* g, long long t) {
+  if (kind == 0) return (mask == nullptr || mask[t] != 0) && tgt[t] >= 0;
+  return g[t] != 0.f;
+}
+
+// Exclusive block-wide prefix sum of one int per thread (blockDim = 256).
+__device__ __forceinline__ int block_exclusive_scan(int v, int* total) {
+  __shared__ int warp_sums[kCompactThreads / 32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) warp_sums[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    int w = lane < kCompactThreads / 32 ? warp_sums[lane] : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += y;
+    }
+    if (lane < kCompactThreads / 32) warp_sums[lane] = w;
+  }
+  __syncthreads();
+  const int before = (warp > 0 ? warp_sums[warp - 1] : 0) + x - v;
+  if (total) *total = warp_sums[kCompactThreads / 32 - 1];
+  __syncthreads();
+  return before;
+}
+
+__global__ void compact_count_kernel(int kind, const uint8_t* mask, const int* tgt, const float* g,
+                                     long long T, int* block_counts) {
+  const long long base = static_cast<long long>(blockIdx.x) * kCompactTile;
+  int c = 0;
+#pragma unroll
+  for (int i = 0; i < kCompactItems; ++i) {
+    const long long t = base + static_cast<long long>(threadIdx.x) * kCompactItems + i;
+    if (t < T && selected(kind, mask, tgt, g, t)) ++c;
+  }
+  int total;
+  block_exclusive_scan(c, &total);
+  if (threadIdx.x == 0) block_counts[blockIdx.x] = total;
+}
+
+// Single block: exclusive scan of the per-block counts, total -> *count.
+__global__ void compact_scan_kernel(const int* block_counts, int nblocks, int* block_offsets,
+                                    int* count) {
+  __shared__ int carry;
+  if (threadIdx.x == 0) carry = 0;
+  __syncthreads();
+  for (int base = 0; base < nblocks; base += kCompactThreads) {
+    const int i = base + threadIdx.x;
+    const int v = i < nblocks ? block_counts[i] : 0;
+    int total;
+    const int ex = block_exclusive_scan(v, &total);
+    if (i < nblocks) block_offsets[i] = carry + ex;
+    __syncthreads();
+    if (threadIdx.x == 0) carry += total;
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) *count = carry;
+}
+
+__global__ void compact_write_kernel(int kind, const uint8_t* mask, const int* tgt, const float* g,
+                                     long long T, const int* block_offsets, int* idx) {
+  const long long base = static_cast<long long>(blockIdx.x) * kCompactTile;
+  bool f[kCompactItems];
+  int c = 0;
+#pragma unroll
+  for (int i = 0; i < kCompactItems; ++i) {
+    const long long t = base + static_cast<long long>(threadIdx.x) * kCompactItems + i;
+    f[i] = t < T && selected(kind, mask, tgt, g, t);
+    c += f[i];
+  }
+  int pos = block_offsets[blockIdx.x] + block_exclusive_scan(c, nullptr);
+#pragma unroll
+  for (int i = 0; i < kCompactItems; ++i) {
+    if (f[i]) idx[pos++] = static_cast<int>(base + static_cast<long long>(threadIdx.x) * kCompactItems + i);
+  }
+}
+
+// One warp per compacted row: copy the bf16 row in 16-byte pieces.
+__global__ void gather_kernel(const uint4* H, int row_vecs, const int* idx, const int* count,
+                              int rows_cap, uint4* Hc, const int* tgt, int* tgt_c, const float* a,
+                              float* a_c, const float* b, float* b_c) {
+  const int n = *count;
+  const int zero_end = min(rows_cap, (n + 127) / 128 * 128);
+  const int warps_per_block = blockDim.x >> 5;
+  const int lane = threadIdx.x & 31;
+  for (int r = blockIdx.x * warps_per_block + (threadIdx.x >> 5); r < zero_end;
+       r += gridDim.x * warps_per_block) {
+    uint4* dst = Hc + static_cast<size_t>(r) * row_vecs;
+    if (r < n) {
+      const int src_row = idx[r];
+      const uint4* src = H + static_cast<size_t>(src_row) * row_vecs;
+      for (int i = lane; i < row_vecs; i += 32) dst[i] = src[i];
+      if (lane == 0) {
+        if (tgt_c) tgt_c[r] = tgt[src_row];
+        if (a_c) a_c[r] = a[src_row];
+        if (b_c) b_c[r] = b[src_row];
+      }
+    } else {
+      for (int i = lane; i < row_vecs; i += 32) dst[i] = make_uint4(0, 0, 0, 0);
+      if (lane == 0) {
+        if (tgt_c) tgt_c[r] = 0;
+        if (a_c) a_c[r] = 0.f;
+        if (b_c) b_c[r] = 0.f;
+      }
+    }
+  }
+}
+
+// Merge (m2, s2, e2) into (m, s, e); m in log2 units, s = sum 2^(t-m), e = sum 2^(t-m) t.
+__device__ __forceinline__ void lse_merge(float& m, float& s, float& e, float m2, float s2, float e2) {
+  if (m2 == -INFINITY) return;
+  if (m == -INFINITY) {
+    m = m2; s = s2; e = e2;
+    return;
+  }
+  const float nm = fmaxf(m, m2);
+  const float r1 = exp2f(m - nm), r2 = exp2f(m2 - nm);
+  s = s * r1 + s2 * r2;
+  e = e * r1 + e2 * r2;
+  m = nm;
+}
+
+// Split-vocabulary combine: 32 rows per block, warp w merges vocab tiles
+// w, w+8, ...; the 8 per-warp results are merged through shared memory.
+__global__ void __launch_bounds__(256) lse_combine_kernel(const float4* partials, int ld_part,
+                                                          int nsplit, const float* ztgt,
+                                                          const int* idx, const int* count,
+                                                          float* logp, float* entropy,
+                                                          float* lse_out) {
+  __shared__ float sm[8][32][3];
+  const int n = *count;
+  const int row0 = blockIdx.x * 32;
+  if (row0 >= n) return;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int row = row0 + lane;
+  float m = -INFINITY, s = 0.f, e = 0.f;
+  if (row < n) {
+#pragma unroll 4
+    for (int j = warp; j < nsplit; j += 8) {
+      const float4 pr = partials[static_cast<size_t>(j) * ld_part + row];
+      lse_merge(m, s, e, pr.x, pr.y, pr.z);
+    }
+  }
+  sm[warp][lane][0] = m;
+  sm[warp][lane][1] = s;
+  sm[warp][lane][2] = e;
+  __syncthreads();
+  if (warp == 0 && row < n) {
+    for (int w = 1; w < 8; ++w) lse_merge(m, s, e, sm[w][lane][0], sm[w][lane][1], sm[w][lane][2]);
+    const float lse2 = m + log2f(s);
+    const float lse_nat = lse2 * kLn2;
+    const int t = idx[row];
+    logp[t] = ztgt[row] - lse_nat;
+    if (entropy) entropy[t] = (lse2 - e / s) * kLn2;
+    if (lse_out) lse_out[t] = lse_nat;
+  }
+}
+
+// One warp per sequence: ballot + popcount prefix over its tokens.
+__global__ void token_select_kernel(const int* cu, const uint8_t* mask, const int* tgt, int n_seq,
+                                    int window, uint8_t* loss_mask, int* n_tok) {
+  const int warps = blockDim.x >> 5;
+  const int seq = blockIdx.x * warps + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (seq >= n_seq) return;
+  const int b = cu[seq], e = cu[seq + 1];
+  int kept = 0;
+  for (int base = b; base < e; base += 32) {
+    const int t = base + lane;
+    const bool in = t < e;
+    const bool elig = in && (mask == nullptr || mask[t] != 0) && tgt[t] >= 0;
+    const unsigned bal = __ballot_sync(0xffffffffu, elig);
+    const int rank = kept + __popc(bal & ((1u << lane) - 1u));
+    if (in) loss_mask[t] = (elig && (window <= 0 || rank < window)) ? 1 : 0;
+    kept += __popc(bal);
+  }
+  if (lane == 0) n_tok[seq] = (window > 0 && kept > window) ? window : kept;
+}
+
+// One warp per group.  Members are visited in ascending sequence index and
+// every operation is a single IEEE fp32 operation in a fixed order, so the
+// result is reproducible bit for bit (the _rn intrinsics also keep the
+// compiler from contracting into fused multiply-adds).
+__global__ void group_adv_kernel(const float* rewards, const int* gid, int n_seq, int n_groups,
+                                 int std_mode, float eps, float* adv) {
+  const int warps = blockDim.x >> 5;
+  const int g = blockIdx.x * warps + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (g >= n_groups) return;
+  float acc = 0.f, lo = INFINITY, hi = -INFINITY;
+  int n = 0;
+  for (int base = 0; base < n_seq; base += 32) {
+    const int i = base + lane;
+    const bool mem = i < n_seq && gid[i] == g;
+    const float r = mem ? rewards[i] : 0.f;
+    unsigned bal = __ballot_sync(0xffffffffu, mem);
+    while (bal) {
+      const int l = __ffs(bal) - 1;
+      const float rl = __shfl_sync(0xffffffffu, r, l);
+      acc = __fadd_rn(acc, rl);
+      lo = fminf(lo, rl);
+      hi = fmaxf(hi, rl);
+      ++n;
+      bal &= bal - 1u;
+    }
+  }
+  const bool zero = n <= 1 || lo == hi;
+  float mu = 0.f, den = 1.f;
+  if (!zero) {
+    mu = __fdiv_rn(acc, static_cast<float>(n));
+    float ss = 0.f;
+    for (int base = 0; base < n_seq; base += 32) {
+      const int i = base + lane;
+      const bool mem = i < n_seq && gid[i] == g;
+      const float dv = mem ? __fsub_rn(rewards[i], mu) : 0.f;
+      unsigned bal = __ballot_sync(0xffffffffu, mem);
+      while (bal) {
+        const int l = __ffs(bal) - 1;
+        const float dl = __shfl_sync(0xffffffffu, dv, l);
+        ss = __fadd_rn(ss, __fmul_rn(dl, dl));
+        bal &= bal - 1u;
+      }
+    }
+    const float var = __fdiv_rn(ss, static_cast<float>(std_mode == 0 ? n - 1 : n));
+    den = __fadd_rn(__fsqrt_rn(var), eps);
+  }
+  for (int base = 0; base < n_seq; base += 32) {
+    const int i = base + lane;
+    if (i < n_seq && gid[i] == g) adv[i] = zero ? 0.f : __fdiv_rn(__fsub_rn(rewards[i], mu), den);
+  }
+}
+
+// ---------------------------------------------------------------- policy loss
+constexpr int kLossThreads = 256;
+
+__device__ __forceinline__ double block_sum_d(double v, double* sh) {
+  // fixed-order tree over the block (deterministic for a fixed blockDim)
+  sh[threadIdx.x] = v;
+  __syncthreads();
+  for (int s = kLossThreads / 2; s > 0; s >>= 1) {
+    if (threadIdx.x < s) sh[threadIdx.x] += sh[threadIdx.x + s];
+    __syncthreads();
+  }
+  const double r = sh[0];
+  __syncthreads();
+  return r;
+}
+
+// (a) loss tokens per sequence and sequences per group.
+__global__ void loss_count_kernel(const int* cu, const int* gid, const uint8_t* lm, int* n_tok,
+                                  int* gsize) {
+  __shared__ double sh[kLossThreads];
+  const int i = blockIdx.x;
+  const int b = cu[i], e = cu[i + 1];
+  double c = 0;
+  for (int t = b + threadIdx.x; t < e; t += kLossThreads) c += lm[t] ? 1.0 : 0.0;
+  const double tot = block_sum_d(c, sh);
+  if (threadIdx.x == 0) {
+    n_tok[i] = static_cast<int>(tot);
+    atomicAdd(&gsize[gid[i]], 1);
+  }
+}
+
+// (b) number of non-empty groups and of loss tokens.
+__global__ void loss_scalars_kernel(const int* gsize, int n_groups, const int* n_tok, int n_seq,
+                                    long long* scal) {
+  __shared__ double sh[kLossThreads];
+  double ng = 0, nt = 0;
+  for (int g = threadIdx.x; g < n_groups; g += kLossThreads) ng += gsize[g] > 0 ? 1.0 : 0.0;
+  for (int i = threadIdx.x; i < n_seq; i += kLossThreads) nt += n_tok[i];
+  ng = block_sum_d(ng, sh);
+  nt = block_sum_d(nt, sh);
+  if (threadIdx.x == 0) {
+    scal[0] = static_cast<long long>(ng);
+    scal[1] = static_cast<long long>(nt);
+  }
+}
+
+// (c) per-token surrogate, KL, dL/dlogp; per-sequence fp64 partial sums.
+__global__ void loss_token_kernel(const float* logp, const float* old_logp, const float* ref_logp,
+                                  const float* adv, const int* cu, const int* gid,
+                                  const uint8_t* lm, float clip_eps, float kl_beta, int agg,
+                                  const int* n_tok, const int* gsize, const long long* scal,
+                                  float* g, double* part, int* part_clip) {
+  __shared__ double sh[kLossThreads];
+  const int i = blockIdx.x;
+  const int b = cu[i], e = cu[i + 1];
+  const int ni = n_tok[i];
+  float c = 0.f;
+  if (agg == 0) {
+    const long long ng = scal[0];
+    if (ni > 0 && ng > 0)
+      c = static_cast<float>(1.0 / (static_cast<double>(ng) * gsize[gid[i]] * ni));
+  } else {
+    const long long nt = scal[1];
+    if (nt > 0) c = static_cast<float>(1.0 / static_cast<double>(nt));
+  }
+  const float A = adv[i];
+  const bool use_kl = ref_logp != nullptr && kl_beta != 0.f;
+  const float lo = 1.f - clip_eps, hi = 1.f + clip_eps;
+  double s_l = 0, s_rho = 0, s_kl = 0, s_clip = 0;
+  for (int t = b + threadIdx.x; t < e; t += kLossThreads) {
+    if (!lm[t]) {
+      g[t] = 0.f;
+      continue;
+    }
+    const float lp = logp[t];
+    const float rho = expf(lp - old_logp[t]);
+    const float clipped = fminf(fmaxf(rho, lo), hi);
+    const float surr = fminf(rho * A, clipped * A);
+    const bool binds = (A > 0.f && rho > hi) || (A < 0.f && rho < lo);
+    float kl = 0.f, dkl = 0.f;
+    if (use_kl) {
+      const float delta = ref_logp[t] - lp;
+      const float em1 = expm1f(delta);
+      kl = em1 - delta;  // exp(delta) - delta - 1
+      dkl = -em1;        // 1 - exp(delta)
+    }
+    const float ell = -(surr - kl_beta * kl);
+    g[t] = c * ((binds ? 0.f : -A * rho) + (use_kl ? kl_beta * dkl : 0.f));
+    s_l += static_cast<double>(c) * ell;
+    s_rho += rho;
+    s_kl += kl;
+    s_clip += binds ? 1.0 : 0.0;
+  }
+  s_l = block_sum_d(s_l, sh);
+  s_rho = block_sum_d(s_rho, sh);
+  s_kl = block_sum_d(s_kl, sh);
+  s_clip = block_sum_d(s_clip, sh);
+  if (threadIdx.x == 0) {
+    part[3 * i + 0] = s_l;
+    part[3 * i + 1] = s_rho;
+    part[3 * i + 2] = s_kl;
+    part_clip[i] = static_cast<int>(s_clip);
+  }
+}
+
+// (d) fixed-order sum over sequences -> loss and stats.
+__global__ void loss_final_kernel(const double* part, const int* part_clip, int n_seq,
+                                  const long long* scal, float* loss, float* stats) {
+  __shared__ double sh[kLossThreads];
+  double l = 0, r = 0, k = 0, c = 0;
+  for (int i = threadIdx.x; i < n_seq; i += kLossThreads) {
+    l += part[3 * i];
+    r += part[3 * i + 1];
+    k += part[3 * i + 2];
+    c += part_clip[i];
+  }
+  l = block_sum_d(l, sh);
+  r = block_sum_d(r, sh);
+  k = block_sum_d(k, sh);
+  c = block_sum_d(c, sh);
+  if (threadIdx.x == 0) {
+    *loss = static_cast<float>(l);
+    if (stats) {
+      const double n = static_cast<double>(scal[1]);
+      stats[0] = n > 0 ? static_cast<float>(c / n) : 0.f;
+      stats[1] = n > 0 ? static_cast<float>(r / n) : 0.f;
+      stats[2] = n > 0 ? static_cast<float>(k / n) : 0.f;
+      stats[3] = static_cast<float>(n);
+    }
+  }
+}
+
+size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+}  // namespace
+
+int compact_blocks(long long T) { return static_cast<int>((T + kCompactTile - 1) / kCompactTile); }
+
+cudaError_t launch_compact(int kind, const uint8_t* mask, const int* tgt, const float* g,
+                           long long T, int* scratch, int* idx, int* count, cudaStream_t s) {
+  const int nb = compact_blocks(T);
+  int* counts = scratch;
+  int* offsets = scratch + nb;
+  compact_count_kernel<<<nb, kCompactThreads, 0, s>>>(kind, mask, tgt, g, T, counts);
+  compact_scan_kernel<<<1, kCompactThreads, 0, s>>>(counts, nb, offsets, count);
+  compact_write_kernel<<<nb, kCompactThreads, 0, s>>>(kind, mask, tgt, g, T, offsets, idx);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather(const __nv_bfloat16* H, int d, const int* idx, const int* count,
+                          int rows_cap, __nv_bfloat16* Hc, const int* tgt, int* tgt_c,
+                          const float* a, float* a_c, const float* b, float* b_c, cudaStream_t s) {
+  const int row_vecs = d / 8;  // 16-byte pieces per row
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int blocks = max(1, min((rows_cap + 7) / 8, sms * 8));
+  gather_kernel<<<blocks, 256, 0, s>>>(reinterpret_cast<const uint4*>(H), row_vecs, idx, count,
+                                       rows_cap, reinterpret_cast<uint4*>(Hc), tgt, tgt_c, a, a_c,
+                                       b, b_c);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_lse_combine(const float4* partials, int ld_part, int nsplit, const float* ztgt,
+                               const int* idx, const int* count, int rows_cap, float* logp,
+                               float* entropy, float* lse, cudaStream_t s) {
+  const int blocks = (rows_cap + 31) / 32;
+  lse_combine_kernel<<<blocks, 256, 0, s>>>(partials, ld_part, nsplit, ztgt, idx, count, logp,
+                                            entropy, lse);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_token_select(const int* cu_seqlens, const uint8_t* mask, const int* tgt,
+                                int n_seq, int window, uint8_t* loss_mask, int* n_tok,
+                                cudaStream_t s) {
+  const int warps = 8;
+  token_select_kernel<<<(n_seq + warps - 1) / warps, warps * 32, 0, s>>>(
+      cu_seqlens, mask, tgt, n_seq, window, loss_mask, n_tok);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_group_advantages(const float* rewards, const int* group_id, int n_seq,
+                                    int n_groups, int std_mode, float eps, float* adv,
+                                    cudaStream_t s) {
+  const int warps = 4;
+  group_adv_kernel<<<(n_groups + warps - 1) / warps, warps * 32, 0, s>>>(
+      rewards, group_id, n_seq, n_groups, std_mode, eps, adv);
+  return cudaGetLastError();
+}
+
+size_t loss_ws_bytes(int n_seq, int n_groups) {
+  return align256(sizeof(int) * n_groups) + align256(sizeof(int) * n_seq) +
+         align256(2 * sizeof(long long)) + align256(3 * sizeof(double) * n_seq) +
+         align256(sizeof(int) * n_seq);
+}
+
+LossWs carve_loss_ws(void* ws, int n_seq, int n_groups) {
+  char* p = static_cast<char*>(ws);
+  LossWs w;
+  w.gsize = reinterpret_cast<int*>(p);
+  p += align256(sizeof(int) * n_groups);
+  w.n_tok = reinterpret_cast<int*>(p);
+  p += align256(sizeof(int) * n_seq);
+  w.scal = reinterpret_cast<long long*>(p);
+  p += align256(2 * sizeof(long long));
+  w.part = reinterpret_cast<double*>(p);
+  p += align256(3 * sizeof(double) * n_seq);
+  w.part_clip = reinterpret_cast<int*>(p);
+  return w;
+}
+
+cudaError_t launch_policy_loss(const float* logp, const float* old_logp, const float* ref_logp,
+                               const float* adv, const int* cu_seqlens, const int* group_id,
+                               int n_seq, int n_groups, const uint8_t* loss_mask, long long T,
+                               float clip_eps, float kl_beta, int agg, float* loss, float* g,
+                               float* stats, const LossWs& w, cudaStream_t s) {
+  (void)T;
+  cudaError_t e = cudaMemsetAsync(w.gsize, 0, sizeof(int) * n_groups, s);
+  if (e != cudaSuccess) return e;
+  loss_count_kernel<<<n_seq, kLossThreads, 0, s>>>(cu_seqlens, group_id, loss_mask, w.n_tok,
+                                                   w.gsize);
+  loss_scalars_kernel<<<1, kLossThreads, 0, s>>>(w.gsize, n_groups, w.n_tok, n_seq, w.scal);
+  loss_token_kernel<<<n_seq, kLossThreads, 0, s>>>(logp, old_logp, ref_logp, adv, cu_seqlens,
+                                                   group_id, loss_mask, clip_eps, kl_beta, agg,
+                                                   w.n_tok, w.gsize, w.scal, g, w.part,
+                                                   w.part_clip);
+  loss_final_kernel<<<1, kLossThreads, 0, s>>>(w.part, w.part_clip, n_seq, w.scal, loss, stats);
+  return cudaGetLastError();
+}
+
+}  // namespace spo

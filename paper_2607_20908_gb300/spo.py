@@ -1,0 +1,255 @@
+"""Thin Python binding of libspo (include/spo.h) over PyTorch tensors.
+
+Argument marshalling only: every function checks dtypes / devices /
+contiguity, allocates the outputs and the workspace with torch (the library
+itself never allocates), and forwards raw device pointers plus the current
+CUDA stream to the C entry point of the same name.  All computation happens
+in libspo's CUDA kernels; there is no fallback path.  If the shared library
+is not built, every call raises.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "lib", "libspo.so")
+
+SPO_AGG_SEQ_GROUP = 0
+SPO_AGG_TOKEN = 1
+SPO_STD_UNBIASED = 0
+SPO_STD_POPULATION = 1
+
+_lib = None
+
+_c_size = ctypes.c_size_t
+_vp = ctypes.c_void_p
+_i32 = ctypes.c_int32
+_i64 = ctypes.c_int64
+_f32 = ctypes.c_float
+
+_SIGS = {
+    "spo_version": ([], ctypes.c_int),
+    "spo_status_string": ([ctypes.c_int], ctypes.c_char_p),
+    "spo_last_error": ([ctypes.c_char_p, _c_size], ctypes.c_int),
+    "spo_device_error": ([ctypes.POINTER(ctypes.c_int), _vp], ctypes.c_int),
+    "spo_token_select": ([_vp, _vp, _vp, _i32, _i64, _i32, _vp, _vp, _vp], ctypes.c_int),
+    "spo_logprobs_workspace_size": ([_i64, _i64, _i64, ctypes.POINTER(_c_size)], ctypes.c_int),
+    "spo_logprobs_fwd": ([_vp, _vp, _vp, _vp, _i64, _i64, _i64, _f32, _vp, _vp, _vp, _vp, _c_size,
+                          _vp], ctypes.c_int),
+    "spo_group_advantages": ([_vp, _vp, _i32, _i32, ctypes.c_int, _f32, _vp, _vp], ctypes.c_int),
+    "spo_policy_loss_workspace_size": ([_i32, _i32, ctypes.POINTER(_c_size)], ctypes.c_int),
+    "spo_policy_loss_fwd": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, _i32, _vp, _i64, _f32, _f32,
+                             ctypes.c_int, _vp, _vp, _vp, _vp, _c_size, _vp], ctypes.c_int),
+    "spo_policy_loss_bwd_workspace_size": ([_i64, _i64, _i64, ctypes.POINTER(_c_size)],
+                                           ctypes.c_int),
+    "spo_policy_loss_bwd": ([_vp, _vp, _vp, _vp, _vp, _i64, _i64, _i64, _f32, _vp, _vp,
+                             ctypes.c_int, _vp, _c_size, _vp], ctypes.c_int),
+}
+
+
+class SpoError(RuntimeError):
+    def __init__(self, status: int, text: str):
+        super().__init__(f"{status_string(status)}: {text}")
+        self.status = status
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded libspo.so (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(
+                f"libspo.so not found at {LIB_PATH}: build it with "
+                "`python -m paper_2607_20908_gb300.build` (the CUDA path has no fallback)")
+        handle = ctypes.CDLL(LIB_PATH)
+        for name, (args, res) in _SIGS.items():
+            fn = getattr(handle, name)
+            fn.argtypes = args
+            fn.restype = res
+        _lib = handle
+    return _lib
+
+
+def exported_symbols():
+    return list(_SIGS)
+
+
+def status_string(status: int) -> str:
+    return lib().spo_status_string(int(status)).decode()
+
+
+def _check(status: int):
+    if status != 0:
+        buf = ctypes.create_string_buffer(512)
+        lib().spo_last_error(buf, 512)
+        raise SpoError(status, buf.value.decode())
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(device) -> ctypes.c_void_p:
+    return ctypes.c_void_p(torch.cuda.current_stream(device).cuda_stream)
+
+
+def _need(t, name, dtype, numel=None, device=None):
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be on a CUDA device")
+    if device is not None and t.device != device:
+        raise ValueError(f"{name} is on {t.device}, expected {device}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if numel is not None and t.numel() != numel:
+        raise ValueError(f"{name} has {t.numel()} elements, expected {numel}")
+    return t
+
+
+def _workspace(nbytes: int, device, ws=None):
+    if ws is not None:
+        if ws.numel() < nbytes or ws.dtype != torch.uint8:
+            raise ValueError(f"workspace needs {nbytes} uint8 bytes")
+        return ws
+    return torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=device)
+
+
+def spo_device_error(device=None) -> int:
+    """Reads and clears the device error word (synchronises the current stream)."""
+    device = torch.device(device or torch.cuda.current_device())
+    code = ctypes.c_int(0)
+    st = lib().spo_device_error(ctypes.byref(code), _stream(device))
+    if st not in (0, 7):
+        _check(st)
+    return code.value
+
+
+def spo_token_select(cu_seqlens, mask, tgt, window: int = 1024):
+    """a1: loss-token mask and per-sequence loss-token counts."""
+    dev = tgt.device
+    T = tgt.numel()
+    n_seq = cu_seqlens.numel() - 1
+    _need(cu_seqlens, "cu_seqlens", torch.int32, device=dev)
+    _need(tgt, "tgt", torch.int32)
+    if mask is not None:
+        _need(mask, "mask", torch.uint8, T, dev)
+    loss_mask = torch.empty(T, dtype=torch.uint8, device=dev)
+    n_tok = torch.empty(n_seq, dtype=torch.int32, device=dev)
+    _check(lib().spo_token_select(_ptr(cu_seqlens), _ptr(mask), _ptr(tgt), n_seq, T, int(window),
+                                  _ptr(loss_mask), _ptr(n_tok), _stream(dev)))
+    return loss_mask, n_tok
+
+
+def logprobs_workspace_size(T: int, d: int, V: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().spo_logprobs_workspace_size(T, d, V, ctypes.byref(n)))
+    return n.value
+
+
+def spo_logprobs_fwd(H, W, tgt, mask=None, inv_temp: float = 1.0, ws=None, want_entropy=True):
+    """a2+a3: returns (logp, entropy or None, lse), fp32[T]."""
+    dev = H.device
+    T, d = H.shape
+    V = W.shape[0]
+    _need(H, "H", torch.bfloat16, device=dev)
+    _need(W, "W", torch.bfloat16, device=dev)
+    if W.shape[1] != d:
+        raise ValueError(f"W has {W.shape[1]} columns, H has {d}")
+    _need(tgt, "tgt", torch.int32, T, dev)
+    if mask is not None:
+        _need(mask, "mask", torch.uint8, T, dev)
+    logp = torch.empty(T, dtype=torch.float32, device=dev)
+    ent = torch.empty(T, dtype=torch.float32, device=dev) if want_entropy else None
+    lse = torch.empty(T, dtype=torch.float32, device=dev)
+    nbytes = logprobs_workspace_size(T, d, V)
+    w = _workspace(nbytes, dev, ws)
+    _check(lib().spo_logprobs_fwd(_ptr(H), _ptr(W), _ptr(tgt), _ptr(mask), T, d, V,
+                                  float(inv_temp), _ptr(logp), _ptr(ent), _ptr(lse), _ptr(w),
+                                  w.numel(), _stream(dev)))
+    return logp, ent, lse
+
+
+def spo_group_advantages(rewards, group_id, n_groups: int, std_mode: int = SPO_STD_UNBIASED,
+                         eps: float = 1e-6):
+    """a4: per-sequence group-normalised advantages, fp32[n_seq]."""
+    dev = rewards.device
+    n = rewards.numel()
+    _need(rewards, "rewards", torch.float32, device=dev)
+    _need(group_id, "group_id", torch.int32, n, dev)
+    adv = torch.empty(n, dtype=torch.float32, device=dev)
+    _check(lib().spo_group_advantages(_ptr(rewards), _ptr(group_id), n, int(n_groups),
+                                      int(std_mode), float(eps), _ptr(adv), _stream(dev)))
+    return adv
+
+
+def policy_loss_workspace_size(n_seq: int, n_groups: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().spo_policy_loss_workspace_size(n_seq, n_groups, ctypes.byref(n)))
+    return n.value
+
+
+def spo_policy_loss_fwd(logp, old_logp, ref_logp, adv, cu_seqlens, group_id, n_groups: int,
+                        loss_mask, clip_eps: float = 0.2, kl_beta: float = 0.0,
+                        agg: int = SPO_AGG_SEQ_GROUP, ws=None):
+    """a5: returns (loss fp32[1], g fp32[T], stats fp32[4])."""
+    dev = logp.device
+    T = logp.numel()
+    n_seq = adv.numel()
+    _need(logp, "logp", torch.float32, device=dev)
+    _need(old_logp, "old_logp", torch.float32, T, dev)
+    if ref_logp is not None:
+        _need(ref_logp, "ref_logp", torch.float32, T, dev)
+    _need(adv, "adv", torch.float32, device=dev)
+    _need(cu_seqlens, "cu_seqlens", torch.int32, n_seq + 1, dev)
+    _need(group_id, "group_id", torch.int32, n_seq, dev)
+    _need(loss_mask, "loss_mask", torch.uint8, T, dev)
+    loss = torch.empty(1, dtype=torch.float32, device=dev)
+    g = torch.empty(T, dtype=torch.float32, device=dev)
+    stats = torch.empty(4, dtype=torch.float32, device=dev)
+    w = _workspace(policy_loss_workspace_size(n_seq, n_groups), dev, ws)
+    _check(lib().spo_policy_loss_fwd(_ptr(logp), _ptr(old_logp), _ptr(ref_logp), _ptr(adv),
+                                     _ptr(cu_seqlens), _ptr(group_id), n_seq, int(n_groups),
+                                     _ptr(loss_mask), T, float(clip_eps), float(kl_beta), int(agg),
+                                     _ptr(loss), _ptr(g), _ptr(stats), _ptr(w), w.numel(),
+                                     _stream(dev)))
+    return loss, g, stats
+
+
+def policy_loss_bwd_workspace_size(T: int, d: int, V: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().spo_policy_loss_bwd_workspace_size(T, d, V, ctypes.byref(n)))
+    return n.value
+
+
+def spo_policy_loss_bwd(H, W, tgt, lse, g, inv_temp: float = 1.0, dH=None, dW=None,
+                        accumulate_dW: bool = False, want_dH=True, want_dW=True, ws=None):
+    """a6-a8: returns (dH bf16[T, d] or None, dW fp32[V, d] or None)."""
+    dev = H.device
+    T, d = H.shape
+    V = W.shape[0]
+    _need(H, "H", torch.bfloat16, device=dev)
+    _need(W, "W", torch.bfloat16, device=dev)
+    _need(tgt, "tgt", torch.int32, T, dev)
+    _need(lse, "lse", torch.float32, T, dev)
+    _need(g, "g", torch.float32, T, dev)
+    if want_dH and dH is None:
+        dH = torch.empty((T, d), dtype=torch.bfloat16, device=dev)
+    if want_dW and dW is None:
+        dW = (torch.zeros if accumulate_dW else torch.empty)((V, d), dtype=torch.float32,
+                                                             device=dev)
+    if dH is not None:
+        _need(dH, "dH", torch.bfloat16, T * d, dev)
+    if dW is not None:
+        _need(dW, "dW", torch.float32, V * d, dev)
+    w = _workspace(policy_loss_bwd_workspace_size(T, d, V), dev, ws)
+    _check(lib().spo_policy_loss_bwd(_ptr(H), _ptr(W), _ptr(tgt), _ptr(lse), _ptr(g), T, d, V,
+                                     float(inv_temp), _ptr(dH), _ptr(dW), int(bool(accumulate_dW)),
+                                     _ptr(w), w.numel(), _stream(dev)))
+    return dH, dW

@@ -1,0 +1,89 @@
+"""The C-ABI library loads, exports every symbol include/spo.h declares, and
+rejects bad arguments on the host before touching a GPU.  CPU only: no call
+here reaches a kernel."""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2607_20908_gb300 import build as B
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    B.build()
+    from paper_2607_20908_gb300 import spo
+    return spo.lib()
+
+
+def _declared():
+    text = open(os.path.join(ROOT, "include", "spo.h")).read()
+    return sorted(set(re.findall(r"SPO_API\s+[^;(]*?\b(spo_\w+)\s*\(", text)))
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = _declared()
+    assert len(names) >= 12
+    from paper_2607_20908_gb300 import spo
+    for n in names:
+        assert hasattr(lib, n), n
+        assert n in spo.exported_symbols(), f"binding misses {n}"
+
+
+def test_status_strings(lib):
+    from paper_2607_20908_gb300 import spo
+    assert spo.status_string(0) == "SPO_OK"
+    assert spo.status_string(4) == "SPO_ERR_WORKSPACE"
+    assert spo.status_string(99) == "SPO_ERR_UNKNOWN"
+    assert lib.spo_version() >= 1
+
+
+def test_workspace_sizes_are_host_only(lib):
+    from paper_2607_20908_gb300 import spo
+    small = spo.logprobs_workspace_size(256, 256, 4096)
+    big = spo.logprobs_workspace_size(16384, 5120, 151936)
+    assert 0 < small < big
+    # partials (ceil(V/256) x T_pad x 16 B) dominate at the full vocabulary
+    assert big >= 594 * 16384 * 16
+    bwd = spo.policy_loss_bwd_workspace_size(16384, 5120, 151936)
+    assert bwd >= 16384 * 151936 * 2          # one bf16 G chunk
+    assert spo.policy_loss_bwd_workspace_size(131072, 5120, 151936) < 131072 * 151936 * 2
+    assert spo.policy_loss_workspace_size(128, 16) > 0
+
+
+def _err(lib):
+    buf = ctypes.create_string_buffer(256)
+    st = lib.spo_last_error(buf, 256)
+    return st, buf.value.decode()
+
+
+def test_host_validation_without_gpu(lib):
+    p = ctypes.c_void_p(4096)  # never dereferenced: validation fails first
+    nul = ctypes.c_void_p(0)
+    f = lib.spo_logprobs_fwd
+    st = f(nul, p, p, nul, 256, 256, 4096, 1.0, p, nul, nul, p, 1 << 30, nul)
+    assert st == 1 and "non-NULL" in _err(lib)[1]
+    st = f(p, p, p, nul, 256, 100, 4096, 1.0, p, nul, nul, p, 1 << 30, nul)
+    assert st == 2 and "multiple of 64" in _err(lib)[1]
+    st = f(p, p, p, nul, 256, 256, 4100, 1.0, p, nul, nul, p, 1 << 30, nul)
+    assert st == 2
+    st = f(ctypes.c_void_p(4097), p, p, nul, 256, 256, 4096, 1.0, p, nul, nul, p, 1 << 30, nul)
+    assert st == 3
+    st = f(p, p, p, nul, 256, 256, 4096, -1.0, p, nul, nul, p, 1 << 30, nul)
+    assert st == 1
+    st = f(p, p, p, nul, 256, 256, 4096, 1.0, p, nul, nul, p, 16, nul)
+    assert st == 4 and "workspace" in _err(lib)[1]
+    g = lib.spo_group_advantages
+    assert g(p, p, 16, 4, 7, 1e-6, p, nul) == 1
+    assert g(p, p, 0, 4, 0, 1e-6, p, nul) == 2
+    lf = lib.spo_policy_loss_fwd
+    assert lf(p, p, nul, p, p, p, 4, 2, p, 64, 0.2, 0.0, 5, p, p, nul, p, 1 << 20, nul) == 1
+    assert lf(p, p, nul, p, p, p, 4, 2, p, 64, 1.5, 0.0, 0, p, p, nul, p, 1 << 20, nul) == 1
+    assert lf(p, p, nul, p, p, p, 4, 2, p, 64, 0.2, 0.0, 0, p, p, nul, p, 8, nul) == 4
+    bw = lib.spo_policy_loss_bwd
+    assert bw(p, p, p, nul, p, 256, 256, 4096, 1.0, p, p, 0, p, 1 << 40, nul) == 1
+    assert bw(p, p, p, p, p, 256, 256, 4096, 1.0, ctypes.c_void_p(4098), p, 0, p, 1 << 40, nul) == 3

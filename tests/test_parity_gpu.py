@@ -1,0 +1,132 @@
+"""GPU parity: the CUDA path (through the C ABI) against the fp64 oracle on
+identical seeded inputs, element by element, at sizes the oracle finishes in
+seconds that still span several tiles and a ragged tail."""
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import spo_oracle as O
+from paper_2607_20908_gb300 import inputs
+from tests import pipeline as P
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    from paper_2607_20908_gb300 import build
+    build.build()
+
+
+def _compare(case, agg=0, std_mode=0):
+    o = P.run_oracle(case, agg=agg, std_mode=std_mode)
+    g = P.run_gpu(case, o["old"], o["ref"], agg=agg, std_mode=std_mode)
+    lm = o["loss_mask"].astype(bool)
+    np.testing.assert_array_equal(g["loss_mask"], o["loss_mask"])
+    np.testing.assert_array_equal(g["n_tok"], o["n_tok"])
+    err_lp = np.abs(g["logp"] - o["logp"]).max()
+    err_ent = np.abs(g["entropy"] - o["entropy"]).max()
+    err_lse = np.abs(g["lse"] - o["lse"]).max()
+    assert err_lp <= P.TOL_LOGP, err_lp
+    assert err_ent <= P.TOL_LOGP, err_ent
+    assert err_lse <= P.TOL_LOGP, err_lse
+    assert np.all(g["logp"][~lm] == 0) and np.all(g["lse"][~lm] == 0)
+    np.testing.assert_allclose(g["adv"], o["adv"], atol=1e-6, rtol=0)
+    rel_loss = abs(g["loss"] - o["loss"]) / max(abs(o["loss"]), 1e-12)
+    assert rel_loss <= P.TOL_LOSS_REL, (g["loss"], o["loss"])
+    assert P.rel_l2(g["g"], o["g"]) <= P.TOL_GRAD_REL
+    assert np.all(g["g"][~lm] == 0)
+    e_dH = P.rel_l2(g["dH"], o["dH"])
+    e_dW = P.rel_l2(g["dW"], o["dW"])
+    assert e_dH <= P.TOL_GRAD_REL, e_dH
+    assert e_dW <= P.TOL_GRAD_REL, e_dW
+    assert abs(g["stats"][3] - o["stats"]["n_loss_tokens"]) == 0
+    assert abs(g["stats"][0] - o["stats"]["clip_frac"]) <= 1e-6
+    assert abs(g["stats"][1] - o["stats"]["mean_ratio"]) <= 1e-4
+    print(f"\n[{case['name']}] |dlogp|={err_lp:.2e} |dent|={err_ent:.2e} "
+          f"loss rel={rel_loss:.2e} dH rel={e_dH:.2e} dW rel={e_dW:.2e}")
+    return o, g
+
+
+def test_tiny_workload_fwd_bwd():
+    """4 groups x 4 rollouts x 16 tokens, d=256, V=4096 (2 x 16 output tiles)."""
+    _compare(inputs.tiny_case())
+
+
+def test_tiny_workload_clipping_active():
+    """Old-policy noise 0.3: a large share of tokens sit on the clipped branch."""
+    case = inputs.tiny_case(seed=1011, old_noise_std=0.3)
+    o, g = _compare(case)
+    assert o["stats"]["clip_frac"] > 0.05
+
+
+def test_ragged_tails_and_window():
+    """T, d and V that are not multiples of the tile (T=1000, d=320, V=5000),
+    prompt masks, ignored targets and a window that truncates sequences."""
+    case = inputs.tiny_case(seed=1021, T_per_seq=125, n_groups=2, rollouts=4, d=320, V=5000)
+    T = case["T"]
+    g = torch.Generator().manual_seed(5)
+    mask = (torch.rand(T, generator=g) > 0.3).to(torch.uint8)
+    tgt = case["tgt"].clone()
+    tgt[torch.rand(T, generator=g) < 0.05] = -100
+    case.update(mask=mask, tgt=tgt, window=64)
+    for agg in (O.AGG_SEQ_GROUP, O.AGG_TOKEN):
+        _compare(case, agg=agg)
+
+
+def test_population_std_and_temperature():
+    case = inputs.tiny_case(seed=1031)
+    case["inv_temp"] = 1.0 / 0.7
+    _compare(case, std_mode=O.STD_POPULATION)
+
+
+def test_advantages_bit_exact_fp32_order():
+    from paper_2607_20908_gb300 import spo
+    rng = np.random.default_rng(3)
+    n, ng = 3000, 200
+    r = rng.normal(0.3, 1.0, n).astype(np.float32)
+    gid = rng.integers(0, ng, n).astype(np.int32)
+    gid[:16] = 7          # one group gets a burst of members
+    r[gid == 11] = 1.25   # zero-variance group
+    want = O.group_advantages_f32(r, gid, ng)
+    got = spo.spo_group_advantages(torch.from_numpy(r).cuda(), torch.from_numpy(gid).cuda(), ng)
+    got = got.cpu().numpy()
+    np.testing.assert_array_equal(got.view(np.uint32), want.view(np.uint32))
+    assert np.all(got[gid == 11] == 0)
+
+
+def test_no_loss_tokens():
+    """Every token masked: log-probs, loss, g, dH and dW are exactly zero."""
+    case = inputs.tiny_case(seed=1041)
+    case["mask"] = torch.zeros(case["T"], dtype=torch.uint8)
+    o = P.run_oracle(case)
+    g = P.run_gpu(case, o["old"], o["ref"])
+    for k in ("logp", "lse", "entropy", "g", "dH", "dW"):
+        assert np.all(g[k] == 0), k
+    assert g["loss"] == 0.0
+
+
+def test_single_loss_token():
+    case = inputs.tiny_case(seed=1051)
+    m = torch.zeros(case["T"], dtype=torch.uint8)
+    m[37] = 1
+    case["mask"] = m
+    _compare(case)
+
+
+def test_dw_accumulate_and_skip_outputs():
+    from paper_2607_20908_gb300 import spo
+    case = inputs.tiny_case(seed=1061)
+    H, W, tgt = case["H"].cuda(), case["W"].cuda(), case["tgt"].cuda()
+    _, _, lse = spo.spo_logprobs_fwd(H, W, tgt)
+    g = torch.randn(case["T"], device="cuda") * 1e-2
+    _, dW1 = spo.spo_policy_loss_bwd(H, W, tgt, lse, g, want_dH=False)
+    base = torch.randn_like(dW1)
+    _, dW2 = spo.spo_policy_loss_bwd(H, W, tgt, lse, g, dW=base.clone(), accumulate_dW=True,
+                                     want_dH=False)
+    torch.testing.assert_close(dW2, base + dW1, rtol=1e-5, atol=1e-6)
+    dH, dWn = spo.spo_policy_loss_bwd(H, W, tgt, lse, g, want_dW=False)
+    assert dWn is None and dH is not None
