@@ -1,0 +1,464 @@
+#!/usr/bin/env python
+"""Throughput of the GRPO log-prob + policy-loss path (fwd + bwd) on GB300.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+One step = one pass of the whole path over one batch held in HBM:
+token selection -> log-probs over the full vocabulary (tensor-core logits +
+online logsumexp) -> group advantages -> clipped surrogate + KL loss ->
+backward (logit recompute, dH = G W, dW = G^T H).  Workload: 16 groups x 8
+rollouts x 128 tokens = 16384 tokens, d = 5120, V = 151936, bf16.
+
+Prints one JSON line (rank 0).  `value` is loss tokens per second over all
+GPUs; `e2e` is the same metric with host<->device copies of every input and
+output inside the timed region; `roofline` is the dominant kernel's
+algorithmic TFLOP/s (from CUDA events recorded around each launch on its
+stream) against the measured bf16 peak; `cpu_baseline` is the fp64 oracle on
+a bounded sample of the same workload on this machine's host cores.
+
+--impl reference times the fp64 oracle itself (host cores) on bounded
+samples of the same workload and prints the same line with impl=reference.
+Under torchrun each rank runs its own batch (weak scaling, no collective on
+the data path); only the timing uses a barrier and a max over ranks.
+"""
+
+from __future__ import annotations
+
+import os
+
+_CORES = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else (os.cpu_count() or 1)
+os.environ.setdefault("OPENBLAS_NUM_THREADS", str(_CORES))
+os.environ.setdefault("OMP_NUM_THREADS", str(_CORES))
+
+import argparse  # noqa: E402
+import ctypes  # noqa: E402
+import json  # noqa: E402
+import statistics  # noqa: E402
+import subprocess  # noqa: E402
+import sys  # noqa: E402
+import threading  # noqa: E402
+import time  # noqa: E402
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2607_20908_gb300 import inputs  # noqa: E402
+
+METRIC = "tokens/s fused logprob+PG loss fwd+bwd (d=5120,V=151936); % BF16 tensor peak"
+UNIT = "tokens/s"
+WORKLOAD = ("full loss fwd+bwd: T=16384 tokens (16 groups x 8 rollouts x 128 tokens), d=5120, "
+            "V=151936, bf16 H/W, fp32 accumulate, rewards correctness+log-speedup+structural, "
+            "clip eps=0.2, KL beta=0.04, window 1024, SEQ_GROUP aggregation")
+KERNEL_NAMES = {0: "logits_lse_fwd", 1: "logits_grad_recompute", 2: "gemm_dH", 3: "gemm_dW"}
+SAMPLE_SEQS, SAMPLE_TOKENS = 8, 8   # CPU sample: one group of 8 rollouts, first 8 tokens each
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            j = json.load(f)
+        return dict(bf16_burst=float(j["bf16_tflops"]), bf16_sustained=float(j["bf16_tflops_sustained"]),
+                    hbm=float(j["hbm_gbs"]), source="measured (MEASURED_PEAKS.json)")
+    return dict(bf16_burst=1900.0, bf16_sustained=1700.0, hbm=6800.0,
+                source="fallback (no MEASURED_PEAKS.json)")
+
+
+# ----------------------------------------------------------------- distributed
+class Dist:
+    def __init__(self):
+        self.world = int(os.environ.get("WORLD_SIZE", "1"))
+        self.rank = int(os.environ.get("RANK", "0"))
+        self.local = int(os.environ.get("LOCAL_RANK", "0"))
+        self.pg = None
+
+    def init(self, backend):
+        if self.world > 1:
+            import torch.distributed as dist
+            dist.init_process_group(backend)
+            self.pg = dist
+
+    def barrier(self):
+        if self.pg:
+            self.pg.barrier()
+
+    def max(self, x: float, device) -> float:
+        if not self.pg:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device=device)
+        self.pg.all_reduce(t, op=self.pg.ReduceOp.MAX)
+        return float(t.item())
+
+    def close(self):
+        if self.pg:
+            self.pg.destroy_process_group()
+
+
+# ----------------------------------------------------------------- clocks
+class ClockSampler:
+    """Samples nvidia-smi clocks / throttle reasons in the background."""
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+    NAMES = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+
+    def __init__(self, device):
+        self.samples = []
+        self.proc = None
+        try:
+            uuid = str(torch.cuda.get_device_properties(device).uuid)
+            sel = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+        except Exception:
+            sel = str(device.index or 0)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", sel, f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            threading.Thread(target=self._read, daemon=True).start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) >= 7:
+                self.samples.append((time.time(), parts))
+
+    def stop(self):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self, t0, t1):
+        win = [p for (t, p) in self.samples if t0 <= t <= t1]
+        scope = "timed region"
+        if len(win) < 3:
+            win = [p for (_, p) in self.samples]
+            scope = "warm-up + timed region"
+        if not win:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+        sm = [num(p[0]) for p in win if num(p[0]) is not None]
+        reasons = sorted({self.NAMES[i] for p in win for i in range(4) if p[3 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": num(win[0][1]), "power_w_max": max((num(p[2]) or 0) for p in win),
+                "reasons": reasons, "samples": len(win), "scope": scope}
+
+
+# ----------------------------------------------------------------- the GPU step
+class Step:
+    """Device buffers + workspaces for one batch, driven through the C ABI."""
+
+    def __init__(self, case, dev):
+        from paper_2607_20908_gb300 import spo
+        self.spo = spo
+        self.L = spo.lib()
+        self.dev = dev
+        self.case = case
+        T, d, V = case["T"], case["d"], case["V"]
+        self.T, self.d, self.V = T, d, V
+        self.n_seq = case["cu_seqlens"].numel() - 1
+        self.n_groups = case["n_groups"]
+        to = lambda t: t.to(dev).contiguous()
+        self.H, self.W = to(case["H"]), to(case["W"])
+        self.tgt, self.mask = to(case["tgt"]), to(case["mask"])
+        self.cu, self.gid = to(case["cu_seqlens"]), to(case["group_id"])
+        self.rewards = to(case["rewards"])
+        f32 = dict(dtype=torch.float32, device=dev)
+        self.loss_mask = torch.empty(T, dtype=torch.uint8, device=dev)
+        self.n_tok = torch.empty(self.n_seq, dtype=torch.int32, device=dev)
+        self.logp, self.ent, self.lse = (torch.empty(T, **f32) for _ in range(3))
+        self.adv = torch.empty(self.n_seq, **f32)
+        self.loss, self.stats = torch.empty(1, **f32), torch.empty(4, **f32)
+        self.g = torch.empty(T, **f32)
+        self.dH = torch.empty((T, d), dtype=torch.bfloat16, device=dev)
+        self.dW = torch.empty((V, d), **f32)
+        self.ws_f = torch.empty(spo.logprobs_workspace_size(T, d, V), dtype=torch.uint8, device=dev)
+        self.ws_l = torch.empty(max(256, spo.policy_loss_workspace_size(self.n_seq, self.n_groups)),
+                                dtype=torch.uint8, device=dev)
+        self.ws_b = torch.empty(spo.policy_loss_bwd_workspace_size(T, d, V), dtype=torch.uint8, device=dev)
+        self.old = torch.empty(T, **f32)
+        self.ref = torch.empty(T, **f32)
+        self.stream = torch.cuda.current_stream(dev)
+
+    def prepare_old_ref(self):
+        """Old / reference log-probs = current log-probs + noise (one forward, untimed)."""
+        self.run(stop_after_fwd=True)
+        torch.cuda.synchronize(self.dev)
+        self.old.copy_(self.logp + self.case["old_noise"].to(self.dev))
+        self.ref.copy_(self.logp + self.case["ref_noise"].to(self.dev))
+
+    def run(self, stop_after_fwd=False):
+        L, p, c = self.L, lambda t: ctypes.c_void_p(t.data_ptr()), self.case
+        s = ctypes.c_void_p(self.stream.cuda_stream)
+        chk = self.spo._check
+        chk(L.spo_token_select(p(self.cu), p(self.mask), p(self.tgt), self.n_seq, self.T, c["window"],
+                               p(self.loss_mask), p(self.n_tok), s))
+        chk(L.spo_logprobs_fwd(p(self.H), p(self.W), p(self.tgt), p(self.loss_mask), self.T, self.d,
+                               self.V, c["inv_temp"], p(self.logp), p(self.ent), p(self.lse),
+                               p(self.ws_f), self.ws_f.numel(), s))
+        if stop_after_fwd:
+            return
+        chk(L.spo_group_advantages(p(self.rewards), p(self.gid), self.n_seq, self.n_groups, 0, 1e-6,
+                                   p(self.adv), s))
+        chk(L.spo_policy_loss_fwd(p(self.logp), p(self.old), p(self.ref), p(self.adv), p(self.cu),
+                                  p(self.gid), self.n_seq, self.n_groups, p(self.loss_mask), self.T,
+                                  c["clip_eps"], c["kl_beta"], 0, p(self.loss), p(self.g),
+                                  p(self.stats), p(self.ws_l), self.ws_l.numel(), s))
+        chk(L.spo_policy_loss_bwd(p(self.H), p(self.W), p(self.tgt), p(self.lse), p(self.g), self.T,
+                                  self.d, self.V, c["inv_temp"], p(self.dH), p(self.dW), 0,
+                                  p(self.ws_b), self.ws_b.numel(), s))
+
+
+class HostIO:
+    """Pinned host copies of every input and output of a step (for e2e)."""
+
+    def __init__(self, st: Step):
+        self.st = st
+        pinned = lambda t: torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+        self.ins = [(dev_t, pinned(dev_t).copy_(dev_t))
+                    for dev_t in (st.H, st.W, st.tgt, st.mask, st.cu, st.gid, st.rewards, st.old, st.ref)]
+        self.outs = [(dev_t, pinned(dev_t)) for dev_t in (st.loss, st.stats, st.logp, st.ent, st.dH, st.dW)]
+        self.h2d = sum(t.numel() * t.element_size() for t, _ in self.ins)
+        self.d2h = sum(t.numel() * t.element_size() for t, _ in self.outs)
+
+    def step(self):
+        for dev_t, host_t in self.ins:
+            dev_t.copy_(host_t, non_blocking=True)
+        self.st.run()
+        for dev_t, host_t in self.outs:
+            host_t.copy_(dev_t, non_blocking=True)
+
+
+def timed(fn, K, dist, dev, stream):
+    dist.barrier()
+    torch.cuda.synchronize(dev)
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0 = time.time()
+    a.record(stream)
+    for _ in range(K):
+        fn()
+    b.record(stream)
+    torch.cuda.synchronize(dev)
+    t1 = time.time()
+    dist.barrier()
+    return dist.max(a.elapsed_time(b), dev), t0, t1
+
+
+# ----------------------------------------------------------------- CPU sample (oracle)
+def cpu_sample(H, W, tgt, cu, rewards, old, ref, case):
+    """One group of SAMPLE_SEQS rollouts, the first SAMPLE_TOKENS tokens of each (full d, V)."""
+    rows = np.concatenate([np.arange(int(cu[i]), int(cu[i]) + SAMPLE_TOKENS) for i in range(SAMPLE_SEQS)])
+    n = rows.size
+    return dict(
+        H=H[rows], W=W, tgt=tgt[rows], mask=np.ones(n, np.uint8),
+        cu=np.arange(0, n + 1, SAMPLE_TOKENS, dtype=np.int64), gid=np.zeros(SAMPLE_SEQS, np.int64),
+        rewards=rewards[:SAMPLE_SEQS], old=old[rows], ref=ref[rows],
+        eps=case["clip_eps"], beta=case["kl_beta"], tau=case["inv_temp"], n=n)
+
+
+def oracle_step(O, s):
+    return O.grpo_step(s["H"], s["W"], s["tgt"], s["mask"], s["cu"], s["gid"], 1, s["rewards"],
+                       s["old"], s["ref"], s["eps"], s["beta"], s["tau"], 1024)
+
+
+def sample_description(n):
+    return (f"one group of {SAMPLE_SEQS} rollouts x first {SAMPLE_TOKENS} tokens = {n} loss tokens of "
+            f"the same workload, full d=5120 and V=151936, whole path (a1-a8) in fp64 numpy/BLAS; "
+            f"tokens/s extrapolated linearly in tokens")
+
+
+def host_inputs_from_device(st: Step):
+    """fp64 host copies of the step's inputs (exact bf16 widening done by torch)."""
+    return (st.H.double().cpu().numpy(), st.W.double().cpu().numpy(), st.tgt.cpu().numpy(),
+            st.cu.cpu().numpy(), st.rewards.double().cpu().numpy(), st.old.double().cpu().numpy(),
+            st.ref.double().cpu().numpy())
+
+
+def run_cpu_baseline(st: Step, budget_s: float = 12.0):
+    from oracle import spo_oracle as O
+    H, W, tgt, cu, rew, old, ref = host_inputs_from_device(st)
+    s = cpu_sample(H, W, tgt, cu, rew, old, ref, st.case)
+    oracle_step(O, s)  # warm (page-in, BLAS threads)
+    reps, t0 = 0, time.perf_counter()
+    while True:
+        oracle_step(O, s)
+        reps += 1
+        el = time.perf_counter() - t0
+        if el >= budget_s or reps >= 20:
+            break
+    return {"value": s["n"] * reps / el, "unit": UNIT, "cores": int(os.environ["OPENBLAS_NUM_THREADS"]),
+            "kind": "oracle", "sample": sample_description(s["n"]) + f"; {reps} reps in {el:.1f} s"}
+
+
+# ----------------------------------------------------------------- arms
+def config_block(case, T_L, world):
+    return {"workload": WORKLOAD, "T": case["T"], "loss_tokens": T_L, "d": case["d"], "V": case["V"],
+            "groups": case["n_groups"], "rollouts_per_group": 8, "tokens_per_rollout": 128,
+            "clip_eps": case["clip_eps"], "kl_beta": case["kl_beta"], "window": case["window"],
+            "l2": "inputs larger than L2 (W alone is 1.56 GB; each step also streams a 5 GB bf16 G buffer)",
+            "parallelism": f"{world} replica(s), independent batch per GPU" if world > 1 else "1 GPU"}
+
+
+def ours(args):
+    dist = Dist()
+    dist.init("nccl")
+    dev = torch.device("cuda", dist.local)
+    torch.cuda.set_device(dev)
+    from paper_2607_20908_gb300 import build, spo
+    if dist.rank == 0 and not os.path.exists(spo.LIB_PATH):
+        build.build()
+    dist.barrier()
+    case = inputs.full_case(seed=1003 + dist.rank, device=str(dev))
+    st = Step(case, dev)
+    st.prepare_old_ref()
+    torch.cuda.synchronize(dev)
+    T_L = int(st.loss_mask.sum().item())
+    flop_gemm = 2.0 * T_L * st.d * st.V          # one GEMM-equivalent (algorithmic)
+    flop_metric = 3.0 * flop_gemm                 # fwd + dH + dW (the recompute is not counted)
+    pk = peaks()
+
+    for _ in range(args.warmup):
+        st.run()
+    torch.cuda.synchronize(dev)
+    assert spo.spo_device_error(dev) == 0, "device wait expired during warm-up"
+
+    clocks = ClockSampler(dev)
+    time.sleep(0.3)
+    for _ in range(2):             # keep the GPU loaded while the sampler starts
+        st.run()
+    spo.spo_trace_enable(True)
+    n0 = spo.spo_launch_count()
+    ms, t0, t1 = timed(st.run, args.steps, dist, dev, st.stream)
+    n_launch = spo.spo_launch_count() - n0
+    spo.spo_trace_enable(False)
+    clocks.stop()
+    trace = spo.spo_trace_read()
+    err = spo.spo_device_error(dev)
+    assert err == 0, f"device wait expired (code {err:#x})"
+
+    tokens_s = dist.world * T_L * args.steps / (ms / 1e3)
+    kern = {}
+    for kind, t in trace:
+        k = kern.setdefault(KERNEL_NAMES.get(kind, str(kind)), {"launches": 0, "total_ms": 0.0})
+        k["launches"] += 1
+        k["total_ms"] += t
+    for k in kern.values():
+        k["avg_ms"] = k["total_ms"] / k["launches"]
+        k["share_of_step"] = k["total_ms"] / ms
+        k["tflops"] = flop_gemm / (k["avg_ms"] / 1e3) / 1e12
+    dom_name, dom = max(kern.items(), key=lambda kv: kv[1]["total_ms"])
+    achieved = dom["tflops"]
+    roofline = {"bound": "tensor", "kernel": dom_name, "achieved": achieved,
+                "peak": pk["bf16_sustained"], "unit": "TFLOP/s", "frac": achieved / pk["bf16_sustained"],
+                "peak_kind": f"bf16 dense sustained, {pk['source']}",
+                "frac_of_burst": achieved / pk["bf16_burst"],
+                "flop_per_launch": flop_gemm, "traffic": None,
+                "traffic_note": "ncu dram bytes: see profiles/ (null here until captured for this build)"}
+
+    # e2e: host buffers, H2D + step + D2H inside the timed region
+    hio = HostIO(st)
+    for _ in range(2):
+        hio.step()
+    ms_e2e, _, _ = timed(hio.step, args.steps, dist, dev, st.stream)
+    e2e = {"value": dist.world * T_L * args.steps / (ms_e2e / 1e3), "unit": UNIT,
+           "h2d_bytes_per_step": hio.h2d, "d2h_bytes_per_step": hio.d2h,
+           "ms_per_step": ms_e2e / args.steps,
+           "path": "pinned host -> device copies of every input, the C-ABI calls, device -> host copies "
+                   "of loss, stats, logp, entropy, dH, dW"}
+
+    line = {
+        "metric": METRIC, "value": tokens_s, "unit": UNIT, "n_gpus": dist.world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded; H~N(0,1), W~N(0,0.02^2) rounded to bf16: random-init stand-in for "
+                "the policy's final hidden states and LM head)",
+        "config": config_block(case, T_L, dist.world),
+        "tensor_peak_frac": {"metric_tflops": flop_metric * args.steps / (ms / 1e3) / 1e12,
+                             "of_burst": flop_metric * args.steps / (ms / 1e3) / 1e12 / pk["bf16_burst"],
+                             "of_sustained": flop_metric * args.steps / (ms / 1e3) / 1e12 / pk["bf16_sustained"],
+                             "flop_per_step": flop_metric,
+                             "note": "algorithmic 3 x 2*T*d*V per step; the backward's logit recompute "
+                                     "is done but not counted"},
+        "roofline": roofline,
+        "kernels": kern,
+        "e2e": e2e,
+        "gpu_launches": n_launch,
+        "launches_per_step": n_launch / args.steps,
+        "clocks": clocks.summary(t0, t1),
+    }
+    if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = run_cpu_baseline(st)
+    if dist.rank == 0:
+        print(json.dumps(line), flush=True)
+    dist.close()
+
+
+def reference(args):
+    dist = Dist()
+    if dist.rank != 0:
+        return
+    from oracle import spo_oracle as O
+    dev = torch.device("cuda", dist.local) if torch.cuda.is_available() else torch.device("cpu")
+    case = inputs.full_case(seed=1003, device=str(dev))
+    # inputs (H, W on the device when there is one, else on the host); old/ref = noise around a
+    # reference log-prob level, since the sample never sees the GPU path
+    H = case["H"].double().cpu().numpy()
+    W = case["W"].double().cpu().numpy()
+    del case["H"], case["W"]
+    tgt, cu = case["tgt"].numpy(), case["cu_seqlens"].numpy()
+    s0 = cpu_sample(H, W, tgt, cu, case["rewards"].double().numpy(), np.zeros(case["T"]),
+                    np.zeros(case["T"]), case)
+    lp, _, _ = O.logprobs(s0["H"], s0["W"], s0["tgt"], s0["tau"])
+    rows_noise_old = case["old_noise"].double().numpy()[:s0["n"]]
+    rows_noise_ref = case["ref_noise"].double().numpy()[:s0["n"]]
+    s0["old"], s0["ref"] = lp + rows_noise_old, lp + rows_noise_ref
+    for _ in range(args.warmup):
+        oracle_step(O, s0)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle_step(O, s0)
+    el = time.perf_counter() - t0
+    val = s0["n"] * args.steps / el
+    line = {
+        "metric": METRIC, "value": val, "unit": UNIT, "n_gpus": dist.world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": el * 1e3 / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "impl": "reference",
+        "data": "synthetic (same seeded workload as the GPU arm)",
+        "config": config_block(case, case["T"], 1),
+        "cpu_baseline": {"value": val, "unit": UNIT, "cores": int(os.environ["OPENBLAS_NUM_THREADS"]),
+                         "kind": "oracle", "sample": sample_description(s0["n"]) + " per step"},
+        "e2e": {"value": val, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle timing")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        reference(args)
+    else:
+        ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -226,6 +226,25 @@ SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32
                                        int64_t V, float inv_temp, void* dH, float* dW,
                                        int accumulate_dW, void* ws, size_t ws_bytes, void* stream);
 
+/* ---------------------------------------------------------------------------
+ * Measurement hooks (no counterpart in the paper; used to report per-kernel
+ * device time against the tensor-core roofline).
+ *
+ * spo_trace_enable(1): from now on every tensor-core GEMM launch of this
+ *   library is bracketed by a start/stop CUDA event pair recorded on the
+ *   launch stream.  Host-global; costs two event records per GEMM.
+ * spo_trace_read: waits for every recorded pair, writes up to max_records
+ *   (kind, milliseconds) in launch order, returns the number recorded in
+ *   *n_records (may exceed max_records) and clears the record list.  kind:
+ *   0 = logits + online logsumexp (a2), 1 = logits recompute -> G (a6),
+ *   2 = dH = G W (a7), 3 = dW = G^T H (a8).
+ * spo_launch_count: kernels launched by this library since it was loaded
+ *   (host-side counter; every kernel launch adds one).
+ * ------------------------------------------------------------------------- */
+SPO_API spo_status spo_trace_enable(int on);
+SPO_API spo_status spo_trace_read(int* kinds, float* ms, int max_records, int* n_records);
+SPO_API long long spo_launch_count(void);
+
 #ifdef __cplusplus
 }
 #endif

@@ -5,6 +5,9 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <mutex>
+#include <vector>
+
 #include "../../include/spo.h"
 #include "internal.h"
 
@@ -166,6 +169,51 @@ BwdWs carve_bwd(void* base, long long T, long long d, long long V) {
   return w;
 }
 
+// ------------------------------------------------------------ tracing
+// When enabled, a start/stop CUDA event pair is recorded on the launch stream
+// around every tensor-core GEMM launch; spo_trace_read returns the durations.
+struct TraceRec {
+  int kind;
+  int dev;
+  cudaEvent_t start, stop;
+};
+std::mutex g_trace_mu;
+bool g_trace_on = false;
+std::vector<TraceRec> g_trace;
+std::vector<TraceRec> g_trace_pool;  // event pairs ready for reuse
+
+spo_status traced_gemm(int kind, bool a_mn, bool b_mn, const CUtensorMap& ta, const CUtensorMap& tb,
+                       const spo::GemmArgs& args, int grid, cudaStream_t s, const DevInfo& di) {
+  TraceRec rec{kind, di.dev, nullptr, nullptr};
+  bool tracing;
+  {
+    std::lock_guard<std::mutex> lk(g_trace_mu);
+    tracing = g_trace_on;
+    if (tracing) {
+      for (size_t i = 0; i < g_trace_pool.size(); ++i) {
+        if (g_trace_pool[i].dev == di.dev) {
+          rec.start = g_trace_pool[i].start;
+          rec.stop = g_trace_pool[i].stop;
+          g_trace_pool.erase(g_trace_pool.begin() + i);
+          break;
+        }
+      }
+    }
+  }
+  if (tracing && !rec.start) {
+    SPO_CUDA(cudaEventCreate(&rec.start), "cudaEventCreate");
+    SPO_CUDA(cudaEventCreate(&rec.stop), "cudaEventCreate");
+  }
+  if (tracing) SPO_CUDA(cudaEventRecord(rec.start, s), "cudaEventRecord");
+  SPO_CUDA(spo::launch_gemm(kind, a_mn, b_mn, ta, tb, args, grid, s), "gemm launch");
+  if (tracing) {
+    SPO_CUDA(cudaEventRecord(rec.stop, s), "cudaEventRecord");
+    std::lock_guard<std::mutex> lk(g_trace_mu);
+    g_trace.push_back(rec);
+  }
+  return SPO_OK;
+}
+
 spo::GemmArgs base_args(const DevInfo& di) {
   spo::GemmArgs a;
   memset(&a, 0, sizeof(a));
@@ -282,8 +330,9 @@ SPO_API spo_status spo_logprobs_fwd(const void* H, const void* W, const int32_t*
   a.partials = w.partials;
   a.ld_part = static_cast<int>(w.T_pad);
   a.ztgt = w.ztgt;
-  SPO_CUDA(spo::launch_gemm(spo::EPI_LSE, false, false, ta, tb, a, grid_for(di, w.T_pad, V), s),
-           "lse gemm launch");
+  if ((st = traced_gemm(spo::EPI_LSE, false, false, ta, tb, a, grid_for(di, w.T_pad, V), s, di)) !=
+      SPO_OK)
+    return st;
   // a3: split-vocab combine, scattered back to token positions (skipped tokens read 0)
   SPO_CUDA(cudaMemsetAsync(logp, 0, sizeof(float) * T, s), "memset logp");
   if (entropy) SPO_CUDA(cudaMemsetAsync(entropy, 0, sizeof(float) * T, s), "memset entropy");
@@ -411,8 +460,9 @@ SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32
     a.gvec = w.g_c + r0;
     a.G = w.G;
     a.ldG = V;
-    SPO_CUDA(spo::launch_gemm(spo::EPI_GRAD, false, false, tH_k, tW_k, a, grid_for(di, rows, V), s),
-             "grad gemm launch");
+    if ((st = traced_gemm(spo::EPI_GRAD, false, false, tH_k, tW_k, a, grid_for(di, rows, V), s,
+                          di)) != SPO_OK)
+      return st;
     // a7: dH rows = G W, scattered to token rows
     if (dH) {
       spo::GemmArgs b = base_args(di);
@@ -424,8 +474,9 @@ SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32
       b.row_idx = w.idx + r0;
       b.out_bf16 = static_cast<__nv_bfloat16*>(dH);
       b.ld_out = d;
-      SPO_CUDA(spo::launch_gemm(spo::EPI_DH, false, true, tG_k, tW_mn, b, grid_for(di, rows, d), s),
-               "dH gemm launch");
+      if ((st = traced_gemm(spo::EPI_DH, false, true, tG_k, tW_mn, b, grid_for(di, rows, d), s,
+                            di)) != SPO_OK)
+        return st;
     }
     // a8: dW (+)= G^T Hc over this chunk's rows
     if (dW) {
@@ -438,11 +489,49 @@ SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32
       b.out_f32 = dW;
       b.ld_out = d;
       b.accumulate = (c == 0) ? (accumulate_dW ? 1 : 0) : 1;
-      SPO_CUDA(spo::launch_gemm(spo::EPI_DW, true, true, tG_mn, tH_mn, b, grid_for(di, V, d), s),
-               "dW gemm launch");
+      if ((st = traced_gemm(spo::EPI_DW, true, true, tG_mn, tH_mn, b, grid_for(di, V, d), s, di)) !=
+          SPO_OK)
+        return st;
     }
   }
   return ok();
 }
+
+SPO_API spo_status spo_trace_enable(int on) {
+  std::lock_guard<std::mutex> lk(g_trace_mu);
+  g_trace_on = on != 0;
+  return ok();
+}
+
+SPO_API spo_status spo_trace_read(int* kinds, float* ms, int max_records, int* n_records) {
+  if (!n_records || max_records < 0 || (max_records > 0 && (!kinds || !ms)))
+    return fail(SPO_ERR_INVALID_ARG, "kinds/ms/n_records invalid");
+  std::vector<TraceRec> recs;
+  {
+    std::lock_guard<std::mutex> lk(g_trace_mu);
+    recs.swap(g_trace);
+  }
+  int n = 0;
+  spo_status st = SPO_OK;
+  for (const TraceRec& r : recs) {
+    float t = 0.f;
+    cudaError_t e = cudaEventSynchronize(r.stop);
+    if (e == cudaSuccess) e = cudaEventElapsedTime(&t, r.start, r.stop);
+    if (e != cudaSuccess && st == SPO_OK) st = cuda_fail(e, "trace event");
+    if (n < max_records) {
+      kinds[n] = r.kind;
+      ms[n] = t;
+    }
+    ++n;
+  }
+  {
+    std::lock_guard<std::mutex> lk(g_trace_mu);
+    for (const TraceRec& r : recs) g_trace_pool.push_back(r);
+  }
+  *n_records = n;
+  return st == SPO_OK ? ok() : st;
+}
+
+SPO_API long long spo_launch_count(void) { return spo::launches(); }
 
 }  // extern "C"

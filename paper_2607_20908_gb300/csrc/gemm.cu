@@ -423,6 +423,7 @@ cudaError_t launch_one(const CUtensorMap& ta, const CUtensorMap& tb, const GemmA
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   k<<<grid, NUM_THREADS, smem, s>>>(ta, tb, args);
+  note_launches(1);
   return cudaGetLastError();
 }
 

@@ -60,6 +60,10 @@ struct GemmArgs {
 
 size_t gemm_smem_bytes();
 
+// Host-side count of kernels this library has launched (for launch accounting).
+void note_launches(int n);
+long long launches();
+
 // Encodes a 2-D bf16 tensor map with 128-byte swizzle.  inner/outer are the
 // extents in elements / rows, row_bytes the pitch, box the staged tile.
 cudaError_t make_tmap_bf16(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer,

@@ -3,6 +3,8 @@
 // combine, group-normalised advantages and the policy-loss forward.
 #include <math.h>
 
+#include <atomic>
+
 #include "internal.h"
 
 namespace spo {
@@ -388,7 +390,12 @@ __global__ void loss_final_kernel(const double* part, const int* part_clip, int 
 
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
+std::atomic<long long> g_launches{0};
+
 }  // namespace
+
+void note_launches(int n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+long long launches() { return g_launches.load(std::memory_order_relaxed); }
 
 int compact_blocks(long long T) { return static_cast<int>((T + kCompactTile - 1) / kCompactTile); }
 
@@ -400,6 +407,7 @@ cudaError_t launch_compact(int kind, const uint8_t* mask, const int* tgt, const 
   compact_count_kernel<<<nb, kCompactThreads, 0, s>>>(kind, mask, tgt, g, T, counts);
   compact_scan_kernel<<<1, kCompactThreads, 0, s>>>(counts, nb, offsets, count);
   compact_write_kernel<<<nb, kCompactThreads, 0, s>>>(kind, mask, tgt, g, T, offsets, idx);
+  note_launches(3);
   return cudaGetLastError();
 }
 
@@ -414,6 +422,7 @@ cudaError_t launch_gather(const __nv_bfloat16* H, int d, const int* idx, const i
   gather_kernel<<<blocks, 256, 0, s>>>(reinterpret_cast<const uint4*>(H), row_vecs, idx, count,
                                        rows_cap, reinterpret_cast<uint4*>(Hc), tgt, tgt_c, a, a_c,
                                        b, b_c);
+  note_launches(1);
   return cudaGetLastError();
 }
 
@@ -423,6 +432,7 @@ cudaError_t launch_lse_combine(const float4* partials, int ld_part, int nsplit, 
   const int blocks = (rows_cap + 31) / 32;
   lse_combine_kernel<<<blocks, 256, 0, s>>>(partials, ld_part, nsplit, ztgt, idx, count, logp,
                                             entropy, lse);
+  note_launches(1);
   return cudaGetLastError();
 }
 
@@ -432,6 +442,7 @@ cudaError_t launch_token_select(const int* cu_seqlens, const uint8_t* mask, cons
   const int warps = 8;
   token_select_kernel<<<(n_seq + warps - 1) / warps, warps * 32, 0, s>>>(
       cu_seqlens, mask, tgt, n_seq, window, loss_mask, n_tok);
+  note_launches(1);
   return cudaGetLastError();
 }
 
@@ -441,6 +452,7 @@ cudaError_t launch_group_advantages(const float* rewards, const int* group_id, i
   const int warps = 4;
   group_adv_kernel<<<(n_groups + warps - 1) / warps, warps * 32, 0, s>>>(
       rewards, group_id, n_seq, n_groups, std_mode, eps, adv);
+  note_launches(1);
   return cudaGetLastError();
 }
 
@@ -481,6 +493,7 @@ cudaError_t launch_policy_loss(const float* logp, const float* old_logp, const f
                                                    w.n_tok, w.gsize, w.scal, g, w.part,
                                                    w.part_clip);
   loss_final_kernel<<<1, kLossThreads, 0, s>>>(w.part, w.part_clip, n_seq, w.scal, loss, stats);
+  note_launches(4);
   return cudaGetLastError();
 }
 

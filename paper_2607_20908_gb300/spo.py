@@ -48,7 +48,13 @@ _SIGS = {
                                            ctypes.c_int),
     "spo_policy_loss_bwd": ([_vp, _vp, _vp, _vp, _vp, _i64, _i64, _i64, _f32, _vp, _vp,
                              ctypes.c_int, _vp, _c_size, _vp], ctypes.c_int),
+    "spo_trace_enable": ([ctypes.c_int], ctypes.c_int),
+    "spo_trace_read": ([ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_float), ctypes.c_int,
+                        ctypes.POINTER(ctypes.c_int)], ctypes.c_int),
+    "spo_launch_count": ([], ctypes.c_longlong),
 }
+
+TRACE_KINDS = {0: "logits_lse_fwd", 1: "logits_grad_recompute", 2: "gemm_dH", 3: "gemm_dW"}
 
 
 class SpoError(RuntimeError):
@@ -253,3 +259,20 @@ def spo_policy_loss_bwd(H, W, tgt, lse, g, inv_temp: float = 1.0, dH=None, dW=No
                                      float(inv_temp), _ptr(dH), _ptr(dW), int(bool(accumulate_dW)),
                                      _ptr(w), w.numel(), _stream(dev)))
     return dH, dW
+
+
+def spo_trace_enable(on: bool = True):
+    _check(lib().spo_trace_enable(1 if on else 0))
+
+
+def spo_trace_read(max_records: int = 65536):
+    """[(kind, ms)] for every traced GEMM launch since the last read (synchronises)."""
+    kinds = (ctypes.c_int * max_records)()
+    ms = (ctypes.c_float * max_records)()
+    n = ctypes.c_int(0)
+    _check(lib().spo_trace_read(kinds, ms, max_records, ctypes.byref(n)))
+    return [(int(kinds[i]), float(ms[i])) for i in range(min(n.value, max_records))]
+
+
+def spo_launch_count() -> int:
+    return int(lib().spo_launch_count())
