@@ -1,11 +1,13 @@
 """Runs the whole path a few times on a reduced, profiler-friendly case.
 
-    python -m paper_2607_20908_gb300.profile_case --T 2048 --d 5120 --V 32768 --iters 3
+    python -m paper_2607_20908_gb300.profile_case --T 16384 --d 5120 --V 8192 --iters 3
 
-Used as the target of ncu captures: the same kernels as the full workload,
-sized so that one launch is well under a millisecond and the device holds a
-few GB at most, while every operand is still larger than the 129 MB L2
-(W = V x d bf16).  Prints per-GEMM CUDA-event times of the last iteration.
+Used as the target of ncu captures: the same kernels as the full workload
+with the same reduction lengths (K = d = 5120 for the logits and their
+recompute, K = T = 16384 tokens for dW), but a vocabulary cut to 8192 so one
+launch takes about a millisecond and the device holds about 1 GB.  The
+streamed operands of dW (G = 268 MB, H = 168 MB) stay larger than the
+129 MB L2.  Prints per-GEMM CUDA-event times of the last iteration.
 """
 
 import argparse
@@ -22,9 +24,9 @@ if ROOT not in sys.path:
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--T", type=int, default=2048)
+    ap.add_argument("--T", type=int, default=16384)
     ap.add_argument("--d", type=int, default=5120)
-    ap.add_argument("--V", type=int, default=32768)
+    ap.add_argument("--V", type=int, default=8192)
     ap.add_argument("--iters", type=int, default=3)
     a = ap.parse_args()
     from paper_2607_20908_gb300 import spo
