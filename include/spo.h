@@ -227,6 +227,35 @@ SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32
                                        int accumulate_dW, void* ws, size_t ws_bytes, void* stream);
 
 /* ---------------------------------------------------------------------------
+ * spo_policy_loss_fwd without a caller workspace.  The paper has no
+ * counterpart: this is a convenience for callers that cannot hand out device
+ * scratch memory -- for example code running under a framework whose memory
+ * pool already owns all device memory, or a host that must not call
+ * cudaMalloc on this path because it would synchronise the device.  It
+ * allocates nothing: its scratch is a 1 MiB array in the library's own device
+ * image (present on every GPU that loads libspo, until the process exits).
+ *
+ * Arguments, results and accuracy are those of spo_policy_loss_fwd minus
+ * ws / ws_bytes; inputs and outputs are still the caller's device buffers.
+ * Limit: spo_policy_loss_workspace_size(n_seq, n_groups) must be at most
+ * 1 MiB (roughly n_seq <= 32000 for a few thousand groups); larger sizes are
+ * rejected with SPO_ERR_WORKSPACE before anything is enqueued.
+ * The first call on a device looks up the array's device address (with that
+ * device current); make that first call before any stream capture.
+ * Every call shares the one array, and what is left in it is overwritten or
+ * cleared on the stream by the next call: calls that can overlap on the GPU
+ * (different streams, or several host threads) race on it and must be
+ * serialised by the caller.
+ * ------------------------------------------------------------------------- */
+SPO_API spo_status spo_policy_loss_fwd_noalloc(const float* logp, const float* old_logp,
+                                               const float* ref_logp, const float* adv,
+                                               const int32_t* cu_seqlens, const int32_t* group_id,
+                                               int32_t n_seq, int32_t n_groups,
+                                               const uint8_t* loss_mask, int64_t T, float clip_eps,
+                                               float kl_beta, int agg, float* loss, float* g,
+                                               float* stats, void* stream);
+
+/* ---------------------------------------------------------------------------
  * Measurement hooks (no counterpart in the paper; used to report per-kernel
  * device time against the tensor-core roofline).
  *

@@ -535,3 +535,73 @@ SPO_API spo_status spo_trace_read(int* kinds, float* ms, int max_records, int* n
 SPO_API long long spo_launch_count(void) { return spo::launches(); }
 
 }  // extern "C"
+
+// ------------------------------------------------------------ no-allocation loss forward
+// Scratch of spo_policy_loss_fwd_noalloc.  It is part of the library's device
+// image: every GPU that loads libspo holds these bytes until the process exits.
+namespace {
+
+constexpr size_t kNoAllocLossScratchBytes = static_cast<size_t>(1) << 20;  // 1 MiB
+
+static __device__ __align__(256) unsigned char g_noalloc_loss_scratch[kNoAllocLossScratchBytes];
+
+std::mutex g_noalloc_mu;
+void* g_noalloc_scratch_ptr[64] = {};
+
+// The array's name is only a host-side handle; its device address is looked
+// up once per device (with that device current) and cached.
+spo_status noalloc_scratch(int dev, void** out) {
+  std::lock_guard<std::mutex> lk(g_noalloc_mu);
+  if (!g_noalloc_scratch_ptr[dev]) {
+    void* p = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_loss_scratch);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(no-alloc loss scratch)");
+    g_noalloc_scratch_ptr[dev] = p;
+  }
+  *out = g_noalloc_scratch_ptr[dev];
+  return SPO_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+SPO_API spo_status spo_policy_loss_fwd_noalloc(const float* logp, const float* old_logp,
+                                               const float* ref_logp, const float* adv,
+                                               const int32_t* cu_seqlens, const int32_t* group_id,
+                                               int32_t n_seq, int32_t n_groups,
+                                               const uint8_t* loss_mask, int64_t T, float clip_eps,
+                                               float kl_beta, int agg, float* loss, float* g,
+                                               float* stats, void* stream) {
+  if (!logp || !old_logp || !adv || !cu_seqlens || !group_id || !loss_mask || !loss || !g)
+    return fail(SPO_ERR_INVALID_ARG, "a required pointer is NULL");
+  if (n_seq < 1 || n_groups < 1 || n_seq > (1 << 24) || n_groups > (1 << 24))
+    return fail(SPO_ERR_SHAPE, "n_seq = %d, n_groups = %d out of range", n_seq, n_groups);
+  if (T < 1 || T > (1ll << 31) - 1) return fail(SPO_ERR_SHAPE, "T = %lld out of range", (long long)T);
+  if (agg != SPO_AGG_SEQ_GROUP && agg != SPO_AGG_TOKEN)
+    return fail(SPO_ERR_INVALID_ARG, "agg %d unknown", agg);
+  if (!(clip_eps >= 0.f && clip_eps < 1.f)) return fail(SPO_ERR_INVALID_ARG, "clip_eps must be in [0, 1)");
+  if (!isfinite(kl_beta)) return fail(SPO_ERR_INVALID_ARG, "kl_beta must be finite");
+  const size_t need = spo::loss_ws_bytes(n_seq, n_groups);
+  if (need > kNoAllocLossScratchBytes)
+    return fail(SPO_ERR_WORKSPACE,
+                "n_seq = %d, n_groups = %d need %zu scratch bytes but the static scratch of "
+                "spo_policy_loss_fwd_noalloc holds %zu; use spo_policy_loss_fwd with a workspace",
+                n_seq, n_groups, need, kNoAllocLossScratchBytes);
+  DevInfo di;
+  spo_status st = device_info(&di);
+  if (st != SPO_OK) return st;
+  void* scratch = nullptr;
+  if ((st = noalloc_scratch(di.dev, &scratch)) != SPO_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // carve_loss_ws lays out the same buffers as the workspace entry point; the
+  // group-size counters are cleared on the stream by launch_policy_loss.
+  const spo::LossWs w = spo::carve_loss_ws(scratch, n_seq, n_groups);
+  SPO_CUDA(spo::launch_policy_loss(logp, old_logp, ref_logp, adv, cu_seqlens, group_id, n_seq,
+                                   n_groups, loss_mask, T, clip_eps, kl_beta, agg, loss, g, stats,
+                                   w, s),
+           "policy loss launch");
+  return ok();
+}
+
+}  // extern "C"

@@ -52,6 +52,8 @@ _SIGS = {
     "spo_trace_read": ([ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_float), ctypes.c_int,
                         ctypes.POINTER(ctypes.c_int)], ctypes.c_int),
     "spo_launch_count": ([], ctypes.c_longlong),
+    "spo_policy_loss_fwd_noalloc": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, _i32, _vp, _i64, _f32,
+                                     _f32, ctypes.c_int, _vp, _vp, _vp, _vp], ctypes.c_int),
 }
 
 TRACE_KINDS = {0: "logits_lse_fwd", 1: "logits_grad_recompute", 2: "gemm_dH", 3: "gemm_dW"}
@@ -276,3 +278,30 @@ def spo_trace_read(max_records: int = 65536):
 
 def spo_launch_count() -> int:
     return int(lib().spo_launch_count())
+
+
+def spo_policy_loss_fwd_noalloc(logp, old_logp, ref_logp, adv, cu_seqlens, group_id,
+                                n_groups: int, loss_mask, loss, g, stats=None,
+                                clip_eps: float = 0.2, kl_beta: float = 0.0,
+                                agg: int = SPO_AGG_SEQ_GROUP):
+    """a5 without a workspace: writes into the caller's loss / g / stats tensors and
+    allocates nothing (scratch is the library's static 1 MiB device array)."""
+    dev = logp.device
+    T = logp.numel()
+    n_seq = adv.numel()
+    _need(logp, "logp", torch.float32, device=dev)
+    _need(old_logp, "old_logp", torch.float32, T, dev)
+    if ref_logp is not None:
+        _need(ref_logp, "ref_logp", torch.float32, T, dev)
+    _need(adv, "adv", torch.float32, device=dev)
+    _need(cu_seqlens, "cu_seqlens", torch.int32, n_seq + 1, dev)
+    _need(group_id, "group_id", torch.int32, n_seq, dev)
+    _need(loss_mask, "loss_mask", torch.uint8, T, dev)
+    _need(loss, "loss", torch.float32, 1, dev)
+    _need(g, "g", torch.float32, T, dev)
+    if stats is not None:
+        _need(stats, "stats", torch.float32, 4, dev)
+    _check(lib().spo_policy_loss_fwd_noalloc(
+        _ptr(logp), _ptr(old_logp), _ptr(ref_logp), _ptr(adv), _ptr(cu_seqlens), _ptr(group_id),
+        n_seq, int(n_groups), _ptr(loss_mask), T, float(clip_eps), float(kl_beta), int(agg),
+        _ptr(loss), _ptr(g), _ptr(stats), _stream(dev)))
