@@ -98,8 +98,8 @@ SPO_API int spo_last_error(char* buf, size_t n);
 SPO_API spo_status spo_device_error(int* code, void* stream);
 
 /* ---------------------------------------------------------------------------
- * a1. Loss-token selection (section 3, "Multi-turn RL Training": masked
- * log-probabilities over a truncated window of 1024 tokens).
+ * a1. Loss-token selection (section 3, "Multi-turn RL Training": the loss uses
+ * only unmasked tokens within a 1024-token window of each generation).
  *
  * Sequence i (one generated output o_i, or one turn of it) spans tokens
  * [cu_seqlens[i], cu_seqlens[i+1]).  Token t of sequence i is a loss token

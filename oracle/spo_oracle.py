@@ -58,8 +58,8 @@ def bf16_bits_to_f64(bits) -> np.ndarray:
 
 
 # --------------------------------------------------------------------------
-# a1: loss-token selection (§3 "Multi-turn RL Training": masked log-probs
-#     over a truncated window of 1024 tokens)
+# a1: loss-token selection (§3 "Multi-turn RL Training": only unmasked tokens
+#     within a 1024-token window of each generation enter the loss)
 # --------------------------------------------------------------------------
 def token_select(cu_seqlens, mask, tgt, window: int):
     """Loss tokens of every sequence.
