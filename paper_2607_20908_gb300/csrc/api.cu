@@ -108,7 +108,7 @@ struct FwdWs {
 
 FwdWs carve_fwd(void* base, long long T, long long d, long long V) {
   FwdWs w{};
-  w.T_pad = round_up(T, spo::BM);
+  w.T_pad = round_up(T, spo::kRowPad);
   w.nsplit = static_cast<int>((V + spo::BN - 1) / spo::BN);
   const int nb = spo::compact_blocks(T);
   char* p = static_cast<char*>(base);
@@ -129,7 +129,7 @@ FwdWs carve_fwd(void* base, long long T, long long d, long long V) {
   return w;
 }
 
-constexpr long long kBwdChunkRows = 32768;  // G scratch rows per chunk (multiple of 128)
+constexpr long long kBwdChunkRows = 32768;  // G scratch rows per chunk (multiple of kRowPad)
 
 struct BwdWs {
   int* idx;
@@ -147,7 +147,7 @@ struct BwdWs {
 
 BwdWs carve_bwd(void* base, long long T, long long d, long long V) {
   BwdWs w{};
-  w.T_pad = round_up(T, spo::BM);
+  w.T_pad = round_up(T, spo::kRowPad);
   w.chunk = w.T_pad < kBwdChunkRows ? w.T_pad : kBwdChunkRows;
   const int nb = spo::compact_blocks(T);
   char* p = static_cast<char*>(base);
@@ -168,6 +168,12 @@ BwdWs carve_bwd(void* base, long long T, long long d, long long V) {
   w.bytes = off;
   return w;
 }
+
+// ------------------------------------------------------------ tuning
+// Host-global launch choices (spo_set_tuning): CTA-pair MMA on/off and the
+// number of tile rows walked together by the raster.
+int g_tune_pair = 1;
+int g_tune_group_m = 16;
 
 // ------------------------------------------------------------ tracing
 // When enabled, a start/stop CUDA event pair is recorded on the launch stream
@@ -205,7 +211,8 @@ spo_status traced_gemm(int kind, bool a_mn, bool b_mn, const CUtensorMap& ta, co
     SPO_CUDA(cudaEventCreate(&rec.stop), "cudaEventCreate");
   }
   if (tracing) SPO_CUDA(cudaEventRecord(rec.start, s), "cudaEventRecord");
-  SPO_CUDA(spo::launch_gemm(kind, a_mn, b_mn, ta, tb, args, grid, s), "gemm launch");
+  SPO_CUDA(spo::launch_gemm(kind, a_mn, b_mn, g_tune_pair != 0, ta, tb, args, grid, s),
+           "gemm launch");
   if (tracing) {
     SPO_CUDA(cudaEventRecord(rec.stop, s), "cudaEventRecord");
     std::lock_guard<std::mutex> lk(g_trace_mu);
@@ -217,17 +224,24 @@ spo_status traced_gemm(int kind, bool a_mn, bool b_mn, const CUtensorMap& ta, co
 spo::GemmArgs base_args(const DevInfo& di) {
   spo::GemmArgs a;
   memset(&a, 0, sizeof(a));
-  a.group_m = 16;
+  a.group_m = g_tune_group_m;
   a.scale = 1.f;
   a.err = di.err;
   return a;
 }
 
+// Persistent grid: one CTA per SM (pairs in pair mode), never more than tiles.
 int grid_for(const DevInfo& di, long long max_m, long long n) {
-  const long long tiles = ((max_m + spo::BM - 1) / spo::BM) * ((n + spo::BN - 1) / spo::BN);
-  long long g = tiles < di.sms ? tiles : di.sms;
-  return static_cast<int>(g < 1 ? 1 : g);
+  const bool pair = g_tune_pair != 0;
+  const long long tm = spo::gemm_tile_m(pair);
+  const long long tiles = ((max_m + tm - 1) / tm) * ((n + spo::BN - 1) / spo::BN);
+  const long long units = pair ? di.sms / 2 : di.sms;
+  long long g = tiles < units ? tiles : units;
+  if (g < 1) g = 1;
+  return static_cast<int>(pair ? 2 * g : g);
 }
+
+uint32_t b_box_rows() { return static_cast<uint32_t>(spo::gemm_b_box_rows(g_tune_pair != 0)); }
 
 }  // namespace
 
@@ -318,7 +332,7 @@ SPO_API spo_status spo_logprobs_fwd(const void* H, const void* W, const int32_t*
   // a2: logits tile by tile + online logsumexp partials
   CUtensorMap ta, tb;
   SPO_CUDA(spo::make_tmap_bf16(&ta, w.Hc, d, w.T_pad, d * 2, spo::BK, spo::BM), "tensor map H");
-  SPO_CUDA(spo::make_tmap_bf16(&tb, W, d, V, d * 2, spo::BK, spo::BN), "tensor map W");
+  SPO_CUDA(spo::make_tmap_bf16(&tb, W, d, V, d * 2, spo::BK, b_box_rows()), "tensor map W");
   spo::GemmArgs a = base_args(di);
   a.m_count = w.count;
   a.m_offset = 0;
@@ -433,7 +447,7 @@ SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32
   if (dH) SPO_CUDA(cudaMemsetAsync(dH, 0, sizeof(uint16_t) * T * d, s), "memset dH");
 
   CUtensorMap tW_k, tW_mn, tG_k, tG_mn;
-  SPO_CUDA(spo::make_tmap_bf16(&tW_k, W, d, V, d * 2, spo::BK, spo::BN), "tensor map W");
+  SPO_CUDA(spo::make_tmap_bf16(&tW_k, W, d, V, d * 2, spo::BK, b_box_rows()), "tensor map W");
   SPO_CUDA(spo::make_tmap_bf16(&tW_mn, W, d, V, d * 2, 64, spo::BK), "tensor map W (MN)");
   SPO_CUDA(spo::make_tmap_bf16(&tG_k, w.G, V, w.chunk, V * 2, spo::BK, spo::BM), "tensor map G");
   SPO_CUDA(spo::make_tmap_bf16(&tG_mn, w.G, V, w.chunk, V * 2, 64, spo::BK), "tensor map G (MN)");
@@ -533,6 +547,21 @@ SPO_API spo_status spo_trace_read(int* kinds, float* ms, int max_records, int* n
 }
 
 SPO_API long long spo_launch_count(void) { return spo::launches(); }
+
+SPO_API spo_status spo_set_tuning(int key, int64_t value) {
+  switch (key) {
+    case SPO_TUNE_PAIR_MMA:
+      if (value != 0 && value != 1) return fail(SPO_ERR_INVALID_ARG, "pair must be 0 or 1");
+      g_tune_pair = static_cast<int>(value);
+      return ok();
+    case SPO_TUNE_GROUP_M:
+      if (value < 1 || value > 4096) return fail(SPO_ERR_INVALID_ARG, "group_m must be in [1, 4096]");
+      g_tune_group_m = static_cast<int>(value);
+      return ok();
+    default:
+      return fail(SPO_ERR_INVALID_ARG, "unknown tuning key %d", key);
+  }
+}
 
 }  // extern "C"
 

@@ -26,9 +26,6 @@ namespace spo {
 
 namespace {
 
-constexpr uint32_t A_BYTES = BM * BK * 2;          // 16 KB
-constexpr uint32_t B_BYTES = BN * BK * 2;          // 32 KB
-constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr uint32_t MN_BLOCK_BYTES = 64 * BK * 2;   // [BK rows][64 MN] block, 8 KB
 constexpr int NUM_THREADS = 192;
 constexpr float kLog2e = 1.4426950408889634f;
@@ -205,18 +202,36 @@ __device__ __forceinline__ void epi_dw(const GemmArgs& p, uint32_t taddr, int ro
 }
 
 // ------------------------------------------------------------ the kernel
-template <int EPI, bool A_MN, bool B_MN>
+// Stage geometry.  Solo: one CTA stages A (128 x 64) and B (256 x 64).  Pair:
+// the two CTAs of a cluster compute one 256 x 256 tile with a shared
+// cta_group::2 MMA; each stages its own 128 rows of A and 128 of the 256 B
+// rows, so a stage is 32 KB and six fit in shared memory.
+template <bool PAIR>
+struct Geo {
+  static constexpr int kStages = PAIR ? 6 : 4;
+  static constexpr int kBRows = PAIR ? BN / 2 : BN;        // B rows staged per CTA
+  static constexpr uint32_t kABytes = BM * BK * 2;         // 16 KB
+  static constexpr uint32_t kBBytes = kBRows * BK * 2;     // 16 or 32 KB
+  static constexpr uint32_t kStageBytes = kABytes + kBBytes;
+  static constexpr int kTileM = PAIR ? 2 * BM : BM;         // output rows per tile
+  static constexpr uint32_t kTxBytes = PAIR ? 2 * kStageBytes : kStageBytes;  // per full barrier
+  static constexpr size_t kSmem = 1024 + kStages * kStageBytes + 256;
+};
+
+template <int EPI, bool A_MN, bool B_MN, bool PAIR>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                 const GemmArgs p) {
+  using G = Geo<PAIR>;
+  constexpr int S = G::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* sA = smem;
-  uint8_t* sB = smem + STAGES * A_BYTES;
-  uint64_t* full_bar = reinterpret_cast<uint64_t*>(sB + STAGES * B_BYTES);
-  uint64_t* empty_bar = full_bar + STAGES;
-  uint64_t* tfull_bar = empty_bar + STAGES;
+  uint8_t* sB = smem + S * G::kABytes;
+  uint64_t* full_bar = reinterpret_cast<uint64_t*>(sB + S * G::kBBytes);
+  uint64_t* empty_bar = full_bar + S;
+  uint64_t* tfull_bar = empty_bar + S;
   uint64_t* tempty_bar = tfull_bar + 2;
   uint64_t* drain_bar = tempty_bar + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
@@ -224,25 +239,28 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  const uint32_t rank = PAIR ? cluster_ctarank() : 0u;          // 0 = leader of the pair
+  const int unit = PAIR ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
+  const int n_units = PAIR ? static_cast<int>(gridDim.x >> 1) : static_cast<int>(gridDim.x);
 
   const int M = p.m_count ? clampi(*p.m_count - p.m_offset, 0, p.m_cap) : p.m_static;
   const int K = p.k_count ? clampi(*p.k_count - p.k_offset, 0, p.k_cap) : p.k_static;
-  const int mt = (M + BM - 1) / BM;
+  const int mt = (M + G::kTileM - 1) / G::kTileM;
   const int nt = (p.n + BN - 1) / BN;
   const int num_tiles = mt * nt;
   const int num_kb = (K + BK - 1) / BK;
   const int gm = max(1, p.group_m);
-  // dW += (empty chunk): nothing to add.  Uniform across the CTA, before any setup.
+  // dW += (empty chunk): nothing to add.  Uniform across the cluster, before any setup.
   if (EPI == EPI_DW && num_kb == 0 && p.accumulate) return;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) {
+    for (int s = 0; s < S; ++s) {
       mbar_init(&full_bar[s], 1);
       mbar_init(&empty_bar[s], 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull_bar[a], 1);
-      mbar_init(&tempty_bar[a], 4);  // one arrival per epilogue warp
+      mbar_init(&tempty_bar[a], PAIR ? 8 : 4);  // one arrival per epilogue warp of the pair
     }
     mbar_init(drain_bar, 1);
     *abort_flag = 0;
@@ -253,60 +271,71 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     tma_prefetch_desc(&tmB);
   }
   if (warp == 1) {
-    tmem_alloc(tmem_slot, 2 * BN);
-    tmem_relinquish();
+    tmem_alloc<PAIR>(tmem_slot, 2 * BN);
+    tmem_relinquish<PAIR>();
   }
   tc_fence_before();
-  __syncthreads();
+  if (PAIR)
+    cluster_sync();  // peer barriers initialised before any remote arrive / TMA signal
+  else
+    __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
   if (warp == 0) {
-    // ------------------------------------------------ TMA producer
+    // ------------------------------------------------ TMA producer (both CTAs)
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
       int issued = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+      for (int tile = unit; tile < num_tiles && ok; tile += n_units) {
         int mb, nb;
         tile_coords(tile, mt, nt, gm, mb, nb);
+        const int a_row = mb * G::kTileM + static_cast<int>(rank) * BM;
+        const int b_row = nb * BN + static_cast<int>(rank) * G::kBRows;
         for (int kb = 0; kb < num_kb; ++kb) {
           if (!mbar_wait(&empty_bar[stage], phase ^ 1u, abort_flag, p.err, kErrWaitProducer)) {
             ok = false;
             break;
           }
-          uint8_t* a_dst = sA + stage * A_BYTES;
-          uint8_t* b_dst = sB + stage * B_BYTES;
-          mbar_arrive_expect_tx(&full_bar[stage], STAGE_BYTES);
+          uint8_t* a_dst = sA + stage * G::kABytes;
+          uint8_t* b_dst = sB + stage * G::kBBytes;
+          if (!PAIR || rank == 0) mbar_arrive_expect_tx(&full_bar[stage], G::kTxBytes);
+          const uint32_t bar = PAIR ? mapa_shared(smem_u32(&full_bar[stage]), 0) : 0u;
+          auto load = [&](uint8_t* dst, const CUtensorMap* tm, int x, int y) {
+            if (PAIR)
+              tma_load_2d_pair(dst, tm, bar, x, y);
+            else
+              tma_load_2d(dst, tm, &full_bar[stage], x, y);
+          };
           if (A_MN) {
 #pragma unroll
-            for (int j = 0; j < BM / 64; ++j)
-              tma_load_2d(a_dst + j * MN_BLOCK_BYTES, &tmA, &full_bar[stage], mb * BM + j * 64, kb * BK);
+            for (int j = 0; j < BM / 64; ++j) load(a_dst + j * MN_BLOCK_BYTES, &tmA, a_row + j * 64, kb * BK);
           } else {
-            tma_load_2d(a_dst, &tmA, &full_bar[stage], kb * BK, mb * BM);
+            load(a_dst, &tmA, kb * BK, a_row);
           }
           if (B_MN) {
 #pragma unroll
-            for (int j = 0; j < BN / 64; ++j)
-              tma_load_2d(b_dst + j * MN_BLOCK_BYTES, &tmB, &full_bar[stage], nb * BN + j * 64, kb * BK);
+            for (int j = 0; j < G::kBRows / 64; ++j)
+              load(b_dst + j * MN_BLOCK_BYTES, &tmB, b_row + j * 64, kb * BK);
           } else {
-            tma_load_2d(b_dst, &tmB, &full_bar[stage], kb * BK, nb * BN);
+            load(b_dst, &tmB, kb * BK, b_row);
           }
           ++issued;
-          if (++stage == STAGES) {
+          if (++stage == S) {
             stage = 0;
             phase ^= 1u;
           }
         }
       }
-      if (!ok) {
+      if (!ok && (!PAIR || rank == 0)) {
         // Aborted: let the copies already in flight land before the CTA exits.
         int s = stage;
         uint32_t ph = phase;
-        for (int i = 0; i < STAGES && i < issued; ++i) {
+        for (int i = 0; i < S && i < issued; ++i) {
           if (--s < 0) {
-            s = STAGES - 1;
+            s = S - 1;
             ph ^= 1u;
           }
           mbar_wait_drain(&full_bar[s], ph);
@@ -314,14 +343,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       }
     }
   } else if (warp == 1) {
-    // ------------------------------------------------ MMA issuer
-    if (lane == 0) {
-      constexpr uint32_t kIdesc = idesc_bf16_f32(BM, BN, A_MN, B_MN);
+    // ------------------------------------------------ MMA issuer (leader CTA only)
+    if (lane == 0 && rank == 0) {
+      constexpr uint32_t kIdesc = idesc_bf16_f32(G::kTileM, BN, A_MN, B_MN);
       int stage = 0;
       uint32_t phase = 0;
       int local = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++local) {
+      for (int tile = unit; tile < num_tiles; tile += n_units, ++local) {
         const int acc = local & 1;
         const uint32_t acc_phase = (local >> 1) & 1;
         if (!mbar_wait(&tempty_bar[acc], acc_phase ^ 1u, abort_flag, p.err, kErrWaitMma)) {
@@ -336,37 +365,39 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             break;
           }
           tc_fence_after();
-          const uint32_t a0 = smem_u32(sA + stage * A_BYTES);
-          const uint32_t b0 = smem_u32(sB + stage * B_BYTES);
+          const uint32_t a0 = smem_u32(sA + stage * G::kABytes);
+          const uint32_t b0 = smem_u32(sB + stage * G::kBBytes);
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k) {
             const uint64_t ad = A_MN ? sdesc_sw128(a0 + k * 2048, MN_BLOCK_BYTES, 1024)
                                      : sdesc_sw128(a0 + k * 32, 16, 1024);
             const uint64_t bd = B_MN ? sdesc_sw128(b0 + k * 2048, MN_BLOCK_BYTES, 1024)
                                      : sdesc_sw128(b0 + k * 32, 16, 1024);
-            umma_bf16(d_tmem, ad, bd, kIdesc, (kb | k) != 0 ? 1u : 0u);
+            umma_bf16<PAIR>(d_tmem, ad, bd, kIdesc, (kb | k) != 0 ? 1u : 0u);
           }
-          umma_commit(&empty_bar[stage]);  // frees the stage when these MMAs finish
-          if (++stage == STAGES) {
+          umma_commit<PAIR>(&empty_bar[stage]);  // frees the stage (in both CTAs) when done
+          if (++stage == S) {
             stage = 0;
             phase ^= 1u;
           }
         }
         if (!ok) break;
-        if (num_kb > 0)
-          umma_commit(&tfull_bar[acc]);  // accumulator complete
-        else
-          mbar_arrive(&tfull_bar[acc]);  // K == 0: nothing to wait for
+        if (num_kb > 0) {
+          umma_commit<PAIR>(&tfull_bar[acc]);  // accumulator complete (both CTAs)
+        } else {                               // K == 0: nothing to wait for
+          mbar_arrive(&tfull_bar[acc]);
+          if (PAIR) mbar_arrive_cluster(mapa_shared(smem_u32(&tfull_bar[acc]), 1));
+        }
       }
       // Every MMA this thread issued must finish before TMEM is released.
-      umma_commit(drain_bar);
+      umma_commit_local<PAIR>(drain_bar);
       if (!mbar_wait_drain(drain_bar, 0) && p.err) atomicCAS(p.err, 0, kErrWaitDrain);
     }
   } else {
-    // ------------------------------------------------ epilogue warps 2..5
+    // ------------------------------------------------ epilogue warps 2..5 (both CTAs)
     const int q = warp & 3;  // TMEM lanes [32q, 32q+32) are reachable from this warp
     int local = 0;
-    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++local) {
+    for (int tile = unit; tile < num_tiles; tile += n_units, ++local) {
       const int acc = local & 1;
       const uint32_t acc_phase = (local >> 1) & 1;
       int mb, nb;
@@ -374,7 +405,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const bool ok = mbar_wait(&tfull_bar[acc], acc_phase, abort_flag, p.err, kErrWaitEpilogue);
       if (!__all_sync(0xffffffffu, ok)) break;
       tc_fence_after();
-      const int row = mb * BM + q * 32 + lane;
+      const int row = mb * G::kTileM + static_cast<int>(rank) * BM + q * 32 + lane;
       const uint32_t taddr =
           tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN);
       if (EPI == EPI_LSE) epi_lse(p, taddr, row, M, nb);
@@ -383,16 +414,25 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       if (EPI == EPI_DW) epi_dw(p, taddr, row, M, nb, num_kb == 0);
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&tempty_bar[acc]);
+      if (lane == 0) {
+        if (PAIR)
+          mbar_arrive_cluster(mapa_shared(smem_u32(&tempty_bar[acc]), 0));  // leader's barrier
+        else
+          mbar_arrive(&tempty_bar[acc]);
+      }
     }
   }
 
   tc_fence_before();
-  __syncthreads();
+  __syncwarp();
+  if (PAIR)
+    cluster_sync();  // no CTA leaves while its pair may still touch its smem or TMEM
+  else
+    __syncthreads();
   if (warp == 1) {
     __syncwarp();
     tc_fence_after();
-    tmem_dealloc(tmem_base, 2 * BN);
+    tmem_dealloc<PAIR>(tmem_base, 2 * BN);
   }
 }
 
@@ -414,22 +454,39 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-template <int EPI, bool A_MN, bool B_MN>
+template <int EPI, bool A_MN, bool B_MN, bool PAIR>
 cudaError_t launch_one(const CUtensorMap& ta, const CUtensorMap& tb, const GemmArgs& args, int grid,
                        cudaStream_t s) {
-  auto k = gemm_kernel<EPI, A_MN, B_MN>;
-  const size_t smem = gemm_smem_bytes();
+  auto k = gemm_kernel<EPI, A_MN, B_MN, PAIR>;
+  const size_t smem = Geo<PAIR>::kSmem;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  k<<<grid, NUM_THREADS, smem, s>>>(ta, tb, args);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(grid), 1, 1);
+  cfg.blockDim = dim3(NUM_THREADS, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = PAIR ? 2 : 1;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, k, ta, tb, args);
   note_launches(1);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
 }  // namespace
 
-size_t gemm_smem_bytes() { return 1024 + STAGES * STAGE_BYTES + 128; }
+size_t gemm_smem_bytes(bool pair) { return pair ? Geo<true>::kSmem : Geo<false>::kSmem; }
+
+int gemm_tile_m(bool pair) { return pair ? Geo<true>::kTileM : Geo<false>::kTileM; }
+
+int gemm_b_box_rows(bool pair) { return pair ? Geo<true>::kBRows : Geo<false>::kBRows; }
 
 cudaError_t make_tmap_bf16(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer,
                            uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer) {
@@ -445,12 +502,17 @@ cudaError_t make_tmap_bf16(CUtensorMap* tm, const void* base, uint64_t inner, ui
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-cudaError_t launch_gemm(int epi, bool a_mn, bool b_mn, const CUtensorMap& ta, const CUtensorMap& tb,
-                        const GemmArgs& args, int grid, cudaStream_t s) {
-  if (epi == EPI_LSE && !a_mn && !b_mn) return launch_one<EPI_LSE, false, false>(ta, tb, args, grid, s);
-  if (epi == EPI_GRAD && !a_mn && !b_mn) return launch_one<EPI_GRAD, false, false>(ta, tb, args, grid, s);
-  if (epi == EPI_DH && !a_mn && b_mn) return launch_one<EPI_DH, false, true>(ta, tb, args, grid, s);
-  if (epi == EPI_DW && a_mn && b_mn) return launch_one<EPI_DW, true, true>(ta, tb, args, grid, s);
+cudaError_t launch_gemm(int epi, bool a_mn, bool b_mn, bool pair, const CUtensorMap& ta,
+                        const CUtensorMap& tb, const GemmArgs& args, int grid, cudaStream_t s) {
+#define SPO_GEMM_CASE(E, AM, BMN)                                                        \
+  if (epi == E && a_mn == AM && b_mn == BMN)                                             \
+    return pair ? launch_one<E, AM, BMN, true>(ta, tb, args, grid, s)                    \
+                : launch_one<E, AM, BMN, false>(ta, tb, args, grid, s);
+  SPO_GEMM_CASE(EPI_LSE, false, false)
+  SPO_GEMM_CASE(EPI_GRAD, false, false)
+  SPO_GEMM_CASE(EPI_DH, false, true)
+  SPO_GEMM_CASE(EPI_DW, true, true)
+#undef SPO_GEMM_CASE
   return cudaErrorInvalidValue;
 }
 

@@ -9,12 +9,15 @@
 
 namespace spo {
 
-// Tensor-core tile: 128 rows x 256 columns per CTA, K staged 64 at a time
-// (one 128-byte swizzle atom of bf16), 4-deep shared-memory ring.
+// Tensor-core tile: 128 accumulator rows x 256 columns per CTA, K staged 64
+// at a time (one 128-byte swizzle atom of bf16).  In pair mode two CTAs share
+// one 256 x 256 tile.
 constexpr int BM = 128;
 constexpr int BN = 256;
 constexpr int BK = 64;
-constexpr int STAGES = 4;
+// Compacted row buffers are padded (and zero-filled) to this many rows so a
+// pair tile never reads rows past the buffer.
+constexpr int kRowPad = 256;
 
 // What the epilogue does with a finished 128 x 256 fp32 accumulator tile.
 enum EpiKind : int {
@@ -58,7 +61,9 @@ struct GemmArgs {
   int* err;  // device error word
 };
 
-size_t gemm_smem_bytes();
+size_t gemm_smem_bytes(bool pair);
+int gemm_tile_m(bool pair);        // output rows per tile (128 solo, 256 pair)
+int gemm_b_box_rows(bool pair);    // rows of a K-major B operand staged per CTA
 
 // Host-side count of kernels this library has launched (for launch accounting).
 void note_launches(int n);
@@ -69,8 +74,9 @@ long long launches();
 cudaError_t make_tmap_bf16(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer,
                            uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer);
 
-// Supported (epi, a_mn, b_mn): (LSE,0,0) (GRAD,0,0) (DH,0,1) (DW,1,1).
-cudaError_t launch_gemm(int epi, bool a_mn, bool b_mn, const CUtensorMap& ta,
+// Supported (epi, a_mn, b_mn): (LSE,0,0) (GRAD,0,0) (DH,0,1) (DW,1,1).  With
+// `pair` the grid must be even (clusters of two CTAs).
+cudaError_t launch_gemm(int epi, bool a_mn, bool b_mn, bool pair, const CUtensorMap& ta,
                         const CUtensorMap& tb, const GemmArgs& args, int grid,
                         cudaStream_t s);
 
@@ -82,7 +88,7 @@ int compact_blocks(long long T);
 cudaError_t launch_compact(int kind, const uint8_t* mask, const int* tgt, const float* g,
                            long long T, int* scratch, int* idx, int* count, cudaStream_t s);
 
-// Hc[r] = H[idx[r]] for r < count and 0 for count <= r < round_up(count, 128)
+// Hc[r] = H[idx[r]] for r < count and 0 for count <= r < round_up(count, kRowPad)
 // (r < rows_cap); also gathers up to three per-row vectors (NULL to skip).
 cudaError_t launch_gather(const __nv_bfloat16* H, int d, const int* idx, const int* count,
                           int rows_cap, __nv_bfloat16* Hc, const int* tgt, int* tgt_c,

@@ -106,7 +106,7 @@ __global__ void gather_kernel(const uint4* H, int row_vecs, const int* idx, cons
                               int rows_cap, uint4* Hc, const int* tgt, int* tgt_c, const float* a,
                               float* a_c, const float* b, float* b_c) {
   const int n = *count;
-  const int zero_end = min(rows_cap, (n + 127) / 128 * 128);
+  const int zero_end = min(rows_cap, (n + kRowPad - 1) / kRowPad * kRowPad);
   const int warps_per_block = blockDim.x >> 5;
   const int lane = threadIdx.x & 31;
   for (int r = blockIdx.x * warps_per_block + (threadIdx.x >> 5); r < zero_end;

@@ -52,6 +52,7 @@ _SIGS = {
     "spo_trace_read": ([ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_float), ctypes.c_int,
                         ctypes.POINTER(ctypes.c_int)], ctypes.c_int),
     "spo_launch_count": ([], ctypes.c_longlong),
+    "spo_set_tuning": ([ctypes.c_int, ctypes.c_int64], ctypes.c_int),
     "spo_policy_loss_fwd_noalloc": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, _i32, _vp, _i64, _f32,
                                      _f32, ctypes.c_int, _vp, _vp, _vp, _vp], ctypes.c_int),
 }
@@ -305,3 +306,12 @@ def spo_policy_loss_fwd_noalloc(logp, old_logp, ref_logp, adv, cu_seqlens, group
         _ptr(logp), _ptr(old_logp), _ptr(ref_logp), _ptr(adv), _ptr(cu_seqlens), _ptr(group_id),
         n_seq, int(n_groups), _ptr(loss_mask), T, float(clip_eps), float(kl_beta), int(agg),
         _ptr(loss), _ptr(g), _ptr(stats), _stream(dev)))
+
+
+SPO_TUNE_PAIR_MMA = 0
+SPO_TUNE_GROUP_M = 1
+
+
+def spo_set_tuning(key: int, value: int):
+    """Host-global launch tuning (results do not depend on it)."""
+    _check(lib().spo_set_tuning(int(key), int(value)))

@@ -130,3 +130,18 @@ def test_dw_accumulate_and_skip_outputs():
     torch.testing.assert_close(dW2, base + dW1, rtol=1e-5, atol=1e-6)
     dH, dWn = spo.spo_policy_loss_bwd(H, W, tgt, lse, g, want_dW=False)
     assert dWn is None and dH is not None
+
+
+def test_single_cta_mode_matches_oracle():
+    """The same kernels with one CTA per 128 x 256 tile (no CTA-pair MMA)."""
+    from paper_2607_20908_gb300 import spo
+    spo.spo_set_tuning(spo.SPO_TUNE_PAIR_MMA, 0)
+    spo.spo_set_tuning(spo.SPO_TUNE_GROUP_M, 3)
+    try:
+        _compare(inputs.tiny_case(seed=1071))
+        case = inputs.tiny_case(seed=1072, T_per_seq=125, n_groups=2, rollouts=4, d=320, V=5000)
+        case["mask"] = (torch.rand(case["T"], generator=torch.Generator().manual_seed(9)) > 0.3).to(torch.uint8)
+        _compare(case)
+    finally:
+        spo.spo_set_tuning(spo.SPO_TUNE_PAIR_MMA, 1)
+        spo.spo_set_tuning(spo.SPO_TUNE_GROUP_M, 16)
