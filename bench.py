@@ -57,6 +57,28 @@ KERNEL_NAMES = {0: "logits_lse_fwd", 1: "logits_grad_recompute", 2: "gemm_dH", 3
 SAMPLE_SEQS, SAMPLE_TOKENS = 8, 8   # CPU sample: one group of 8 rollouts, first 8 tokens each
 
 
+# DRAM bytes (read + write) per launch of each tensor-core kernel on this workload, from one
+# `ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum` capture of this command
+# (profiles/launches_full_workload.md), valid only for the kernel sources they were taken on.
+TRAFFIC = {"sources_sha256_16": "91b0e0fcf2f7d7a3",
+           "bytes": {"logits_lse_fwd": 42.808e9, "logits_grad_recompute": 49.241e9,
+                     "gemm_dH": 81.260e9, "gemm_dW": 68.447e9}}
+KERNEL_SOURCES = ["paper_2607_20908_gb300/csrc/gemm.cu", "paper_2607_20908_gb300/csrc/tc.cuh",
+                  "paper_2607_20908_gb300/csrc/internal.h"]
+
+
+def kernel_traffic(name):
+    """ncu DRAM bytes per launch for `name`, or None if the kernel sources changed since."""
+    import hashlib
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, f), "rb") as fh:
+            h.update(fh.read())
+    if h.hexdigest()[:16] != TRAFFIC["sources_sha256_16"]:
+        return None
+    return TRAFFIC["bytes"].get(name)
+
+
 def peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -222,23 +244,71 @@ class Step:
 
 
 class HostIO:
-    """Pinned host copies of every input and output of a step (for e2e)."""
+    """End-to-end step from host buffers: every input copied host -> device and
+    every output copied device -> host, pipelined over two device buffer sets
+    so that the copies of one step overlap the compute of its neighbours
+    (H2D and D2H each on their own stream, compute on the step's stream)."""
 
-    def __init__(self, st: Step):
-        self.st = st
+    def __init__(self, st: "Step"):
+        self.sets = [st, Step(st.case, st.dev)]
+        self.sets[1].old.copy_(st.old)
+        self.sets[1].ref.copy_(st.ref)
         pinned = lambda t: torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
-        self.ins = [(dev_t, pinned(dev_t).copy_(dev_t))
-                    for dev_t in (st.H, st.W, st.tgt, st.mask, st.cu, st.gid, st.rewards, st.old, st.ref)]
-        self.outs = [(dev_t, pinned(dev_t)) for dev_t in (st.loss, st.stats, st.logp, st.ent, st.dH, st.dW)]
-        self.h2d = sum(t.numel() * t.element_size() for t, _ in self.ins)
-        self.d2h = sum(t.numel() * t.element_size() for t, _ in self.outs)
+        ins = lambda x: (x.H, x.W, x.tgt, x.mask, x.cu, x.gid, x.rewards, x.old, x.ref)
+        outs = lambda x: (x.loss, x.stats, x.logp, x.ent, x.dH, x.dW)
+        self.host_in = [pinned(t).copy_(t) for t in ins(st)]
+        self.host_out = [[pinned(t) for t in outs(x)] for x in self.sets]
+        self.dev_in = [ins(x) for x in self.sets]
+        self.dev_out = [outs(x) for x in self.sets]
+        self.h2d = sum(t.numel() * t.element_size() for t in self.host_in)
+        self.d2h = sum(t.numel() * t.element_size() for t in self.host_out[0])
+        self.compute = st.stream
+        self.s_in = torch.cuda.Stream(st.dev)
+        self.s_out = torch.cuda.Stream(st.dev)
+        for x in self.sets:
+            x.stream = self.compute
+        mk = lambda: [torch.cuda.Event() for _ in range(2)]
+        self.in_done, self.comp_done, self.out_done = mk(), mk(), mk()
+        self.i = 0
 
     def step(self):
-        for dev_t, host_t in self.ins:
-            dev_t.copy_(host_t, non_blocking=True)
-        self.st.run()
-        for dev_t, host_t in self.outs:
-            host_t.copy_(dev_t, non_blocking=True)
+        b = self.i & 1
+        x = self.sets[b]
+        if self.i >= 2:
+            self.s_in.wait_event(self.comp_done[b])     # set b's inputs no longer read
+        with torch.cuda.stream(self.s_in):
+            for d, h in zip(self.dev_in[b], self.host_in):
+                d.copy_(h, non_blocking=True)
+            self.in_done[b].record(self.s_in)
+        self.compute.wait_event(self.in_done[b])
+        if self.i >= 2:
+            self.compute.wait_event(self.out_done[b])   # set b's outputs already copied out
+        x.run()
+        self.comp_done[b].record(self.compute)
+        self.s_out.wait_event(self.comp_done[b])
+        with torch.cuda.stream(self.s_out):
+            for d, h in zip(self.dev_out[b], self.host_out[b]):
+                h.copy_(d, non_blocking=True)
+            self.out_done[b].record(self.s_out)
+        self.i += 1
+
+
+def timed_e2e(hio: HostIO, K, dist, dev):
+    """Times K end-to-end steps: from before the first copy in to after the last copy out."""
+    dist.barrier()
+    torch.cuda.synchronize(dev)
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(hio.s_in)
+    hio.compute.wait_event(a)
+    hio.s_out.wait_event(a)
+    for _ in range(K):
+        hio.step()
+    hio.s_in.wait_stream(hio.s_out)
+    hio.s_in.wait_stream(hio.compute)
+    b.record(hio.s_in)
+    torch.cuda.synchronize(dev)
+    dist.barrier()
+    return dist.max(a.elapsed_time(b), dev)
 
 
 def timed(fn, K, dist, dev, stream):
@@ -364,19 +434,29 @@ def ours(args):
                 "peak": pk["bf16_sustained"], "unit": "TFLOP/s", "frac": achieved / pk["bf16_sustained"],
                 "peak_kind": f"bf16 dense sustained, {pk['source']}",
                 "frac_of_burst": achieved / pk["bf16_burst"],
-                "flop_per_launch": flop_gemm, "traffic": None,
-                "traffic_note": "ncu dram bytes: see profiles/ (null here until captured for this build)"}
+                "flop_per_launch": flop_gemm, "traffic": kernel_traffic(dom_name),
+                "traffic_unit": "bytes per launch (ncu dram__bytes_read.sum + dram__bytes_write.sum)",
+                "algorithmic_bytes": None}
+    alg = {"logits_lse_fwd": 2 * T_L * st.d + 2 * st.V * st.d + 16 * T_L * ((st.V + 255) // 256),
+           "logits_grad_recompute": 2 * T_L * st.d + 2 * st.V * st.d + 2 * T_L * st.V,
+           "gemm_dH": 2 * T_L * st.V + 2 * st.V * st.d + 2 * T_L * st.d,
+           "gemm_dW": 2 * T_L * st.V + 2 * T_L * st.d + 4 * st.V * st.d}
+    roofline["algorithmic_bytes"] = alg[dom_name]
+    for name, k in kern.items():
+        k["dram_bytes_ncu"] = kernel_traffic(name)
+        k["algorithmic_bytes"] = alg[name]
 
     # e2e: host buffers, H2D + step + D2H inside the timed region
     hio = HostIO(st)
     for _ in range(2):
         hio.step()
-    ms_e2e, _, _ = timed(hio.step, args.steps, dist, dev, st.stream)
+    ms_e2e = timed_e2e(hio, args.steps, dist, dev)
     e2e = {"value": dist.world * T_L * args.steps / (ms_e2e / 1e3), "unit": UNIT,
            "h2d_bytes_per_step": hio.h2d, "d2h_bytes_per_step": hio.d2h,
            "ms_per_step": ms_e2e / args.steps,
-           "path": "pinned host -> device copies of every input, the C-ABI calls, device -> host copies "
-                   "of loss, stats, logp, entropy, dH, dW"}
+           "path": "pinned host -> device copies of every input (H, W, ids, masks, rewards, old/ref "
+                   "log-probs), the C-ABI calls, device -> host copies of loss, stats, logp, entropy, "
+                   "dH, dW; two buffer sets so copies overlap the neighbouring steps' compute"}
 
     line = {
         "metric": METRIC, "value": tokens_s, "unit": UNIT, "n_gpus": dist.world, "steps": args.steps,
