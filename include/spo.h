@@ -273,10 +273,16 @@ SPO_API spo_status spo_policy_loss_fwd_noalloc(const float* logp, const float* o
 /* Launch tuning, host-global, for every later call on any device:
  *   SPO_TUNE_PAIR_MMA (default 1): 1 = two CTAs of a cluster share one
  *     256 x 256 tile through a cta_group::2 MMA, 0 = one CTA per 128 x 256 tile.
- *   SPO_TUNE_GROUP_M (default 16): output-tile rows walked together by the
+ *   SPO_TUNE_GROUP_M (default 16): output tiles walked together by the
  *     persistent raster (L2 reuse of the streamed operand).
- * Results do not depend on either setting. */
-typedef enum spo_tune_key { SPO_TUNE_PAIR_MMA = 0, SPO_TUNE_GROUP_M = 1 } spo_tune_key;
+ *   SPO_TUNE_RASTER (default 0): 0 = groups of tile rows, 1 = groups of tile
+ *     columns.
+ * Results do not depend on any setting. */
+typedef enum spo_tune_key {
+    SPO_TUNE_PAIR_MMA = 0,
+    SPO_TUNE_GROUP_M = 1,
+    SPO_TUNE_RASTER = 2
+} spo_tune_key;
 SPO_API spo_status spo_set_tuning(int key, int64_t value);
 
 SPO_API spo_status spo_trace_enable(int on);

@@ -174,6 +174,7 @@ BwdWs carve_bwd(void* base, long long T, long long d, long long V) {
 // number of tile rows walked together by the raster.
 int g_tune_pair = 1;
 int g_tune_group_m = 16;
+int g_tune_raster = 0;
 
 // ------------------------------------------------------------ tracing
 // When enabled, a start/stop CUDA event pair is recorded on the launch stream
@@ -225,6 +226,7 @@ spo::GemmArgs base_args(const DevInfo& di) {
   spo::GemmArgs a;
   memset(&a, 0, sizeof(a));
   a.group_m = g_tune_group_m;
+  a.raster = g_tune_raster;
   a.scale = 1.f;
   a.err = di.err;
   return a;
@@ -557,6 +559,10 @@ SPO_API spo_status spo_set_tuning(int key, int64_t value) {
     case SPO_TUNE_GROUP_M:
       if (value < 1 || value > 4096) return fail(SPO_ERR_INVALID_ARG, "group_m must be in [1, 4096]");
       g_tune_group_m = static_cast<int>(value);
+      return ok();
+    case SPO_TUNE_RASTER:
+      if (value != 0 && value != 1) return fail(SPO_ERR_INVALID_ARG, "raster must be 0 or 1");
+      g_tune_raster = static_cast<int>(value);
       return ok();
     default:
       return fail(SPO_ERR_INVALID_ARG, "unknown tuning key %d", key);

@@ -32,16 +32,22 @@ constexpr float kLog2e = 1.4426950408889634f;
 
 __device__ __forceinline__ int clampi(int v, int lo, int hi) { return v < lo ? lo : (v > hi ? hi : v); }
 
-// Grouped raster: `gm` tile rows are walked together across all tile columns,
-// so the A rows of a group stay in L2 while B streams past them.
-__device__ __forceinline__ void tile_coords(int tile, int mt, int nt, int gm, int& mb, int& nb) {
-  const int per_group = gm * nt;
+// Grouped raster.  raster 0: `gm` tile rows are walked together across all
+// tile columns, so the A rows of a group stay in L2 while B streams past them.
+// raster 1: the same with the roles of rows and columns exchanged.
+__device__ __forceinline__ void tile_coords(int tile, int mt, int nt, int gm, int raster, int& mb,
+                                            int& nb) {
+  const int outer = raster ? nt : mt;
+  const int inner = raster ? mt : nt;
+  const int per_group = gm * inner;
   const int group = tile / per_group;
   const int first = group * gm;
-  const int size = min(gm, mt - first);
+  const int size = min(gm, outer - first);
   const int in = tile - group * per_group;
-  mb = first + in % size;
-  nb = in / size;
+  const int o = first + in % size;
+  const int i = in / size;
+  mb = raster ? i : o;
+  nb = raster ? o : i;
 }
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
@@ -291,7 +297,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       bool ok = true;
       for (int tile = unit; tile < num_tiles && ok; tile += n_units) {
         int mb, nb;
-        tile_coords(tile, mt, nt, gm, mb, nb);
+        tile_coords(tile, mt, nt, gm, p.raster, mb, nb);
         const int a_row = mb * G::kTileM + static_cast<int>(rank) * BM;
         const int b_row = nb * BN + static_cast<int>(rank) * G::kBRows;
         for (int kb = 0; kb < num_kb; ++kb) {
@@ -401,7 +407,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const int acc = local & 1;
       const uint32_t acc_phase = (local >> 1) & 1;
       int mb, nb;
-      tile_coords(tile, mt, nt, gm, mb, nb);
+      tile_coords(tile, mt, nt, gm, p.raster, mb, nb);
       const bool ok = mbar_wait(&tfull_bar[acc], acc_phase, abort_flag, p.err, kErrWaitEpilogue);
       if (!__all_sync(0xffffffffu, ok)) break;
       tc_fence_after();

@@ -39,7 +39,8 @@ struct GemmArgs {
   const int* k_count;
   int k_offset;
   int k_cap;
-  int group_m;  // rows of tiles walked together (L2 reuse of the B operand)
+  int group_m;  // tile rows (raster 0) or columns (raster 1) walked together
+  int raster;   // 0: groups of tile rows, 1: groups of tile columns
   float scale;  // inv_temp for EPI_LSE / EPI_GRAD
   // EPI_LSE
   const int* tgt;     // target id of each row
