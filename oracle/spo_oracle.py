@@ -300,6 +300,45 @@ def policy_loss_bwd(H, W, tgt, g, inv_temp: float = 1.0):
 
 
 # --------------------------------------------------------------------------
+# reward composition (§2.2 "Verifiable Reward"; r_i = R_ver(i) + R_str(i), §3)
+# --------------------------------------------------------------------------
+PAPER_REWARD = dict(alpha_comp=3.0, alpha_wrong=2.0, alpha_speed=1.0, alpha_cv=0.5,
+                    s_min=-0.5, s_max=4.0)
+
+
+def reward_compose(compiled, pass_rate, speedup, cv, r_struct=None, params=None):
+    """Composite reward of each candidate program.
+
+    R_comp  = -alpha_comp                         (the program does not compile)
+    R_corr  = -alpha_wrong * (1 - p)              (p = fraction of tests passed)
+    R_speed = alpha_speed * clip(log2 S, s_min, s_max)   (S = speedup)
+    R_cv    = -alpha_cv * cv                       (coefficient of variation)
+    R_ver   = R_comp if not compiled; R_corr if p < 1; R_corr + R_speed + R_cv if p == 1
+    r       = R_ver + R_str
+    A speedup that is not > 0 counts as the lower clip bound.  fp64.
+    """
+    q = dict(PAPER_REWARD if params is None else params)
+    comp = np.asarray(compiled).astype(np.int64)
+    p = np.asarray(pass_rate, dtype=np.float64)
+    S = np.asarray(speedup, dtype=np.float64)
+    c = np.asarray(cv, dtype=np.float64)
+    out = np.zeros(p.size)
+    for i in range(p.size):
+        if comp[i] == 0:
+            r = -q["alpha_comp"]
+        else:
+            r = -q["alpha_wrong"] * (1.0 - p[i])
+            if p[i] >= 1.0:
+                ls = math.log2(S[i]) if S[i] > 0 else -math.inf
+                r += q["alpha_speed"] * min(max(ls, q["s_min"]), q["s_max"])
+                r += -q["alpha_cv"] * c[i]
+        out[i] = r
+    if r_struct is not None:
+        out = out + np.asarray(r_struct, dtype=np.float64)
+    return out
+
+
+# --------------------------------------------------------------------------
 # the whole step (used for the CPU baseline timing)
 # --------------------------------------------------------------------------
 def grpo_step(H, W, tgt, mask, cu_seqlens, group_id, n_groups, rewards, old_logp, ref_logp,

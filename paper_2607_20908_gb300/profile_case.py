@@ -1,17 +1,22 @@
-"""Runs the whole path a few times on a reduced, profiler-friendly case.
+"""Runs the GEMM part of the path (logits + logsumexp forward, then the
+backward) on a chosen size, as a target for ncu captures and launch-tuning
+sweeps.
 
     python -m paper_2607_20908_gb300.profile_case --T 16384 --d 5120 --V 8192 --iters 3
+    python -m paper_2607_20908_gb300.profile_case --V 151936 --iters 1 \\
+        --configs "1,16,0;1,8,0;0,16,0"
 
-Used as the target of ncu captures: the same kernels as the full workload
-with the same reduction lengths (K = d = 5120 for the logits and their
-recompute, K = T = 16384 tokens for dW), but a vocabulary cut to 8192 so one
-launch takes about a millisecond and the device holds about 1 GB.  The
-streamed operands of dW (G = 268 MB, H = 168 MB) stay larger than the
-129 MB L2.  Prints per-GEMM CUDA-event times of the last iteration.
+--configs is a ';'-separated list of "pair,group,raster" launch tunings
+(spo_set_tuning); each is run for --iters iterations of fwd + bwd.  The
+default reduced size keeps the reduction lengths of the full workload
+(K = d = 5120 for the logits and their recompute, K = T = 16384 tokens for
+dW) with a vocabulary cut to 8192, so one launch takes about a millisecond
+and the device holds about 1 GB; the streamed operands of dW (G = 268 MB,
+H = 168 MB) stay larger than the 129 MB L2.  Prints per-GEMM CUDA-event
+times of the last iteration of each configuration.
 """
 
 import argparse
-import ctypes
 import os
 import sys
 
@@ -28,6 +33,7 @@ def main():
     ap.add_argument("--d", type=int, default=5120)
     ap.add_argument("--V", type=int, default=8192)
     ap.add_argument("--iters", type=int, default=3)
+    ap.add_argument("--configs", type=str, default="", help='e.g. "1,16,0;0,16,0"')
     a = ap.parse_args()
     from paper_2607_20908_gb300 import spo
     dev = torch.device("cuda")
@@ -36,13 +42,28 @@ def main():
     W = (torch.randn(a.V, a.d, device=dev, generator=g) * 0.02).to(torch.bfloat16)
     tgt = torch.randint(0, a.V, (a.T,), device=dev, generator=g, dtype=torch.int32)
     gl = torch.randn(a.T, device=dev, generator=g) * 1e-4
-    for i in range(a.iters):
-        spo.spo_trace_enable(i == a.iters - 1)
-        _, _, lse = spo.spo_logprobs_fwd(H, W, tgt)
-        spo.spo_policy_loss_bwd(H, W, tgt, lse, gl)
-    torch.cuda.synchronize()
-    for kind, ms in spo.spo_trace_read():
-        print(f"{spo.TRACE_KINDS[kind]:24s} {ms:8.3f} ms  {2.0 * a.T * a.d * a.V / ms / 1e9:8.1f} TFLOP/s")
+    ws_f = torch.empty(spo.logprobs_workspace_size(a.T, a.d, a.V), dtype=torch.uint8, device=dev)
+    ws_b = torch.empty(spo.policy_loss_bwd_workspace_size(a.T, a.d, a.V), dtype=torch.uint8,
+                       device=dev)
+    dH = torch.empty(a.T, a.d, dtype=torch.bfloat16, device=dev)
+    dW = torch.empty(a.V, a.d, dtype=torch.float32, device=dev)
+    configs = [tuple(int(x) for x in c.split(",")) for c in a.configs.split(";") if c] or [None]
+    for cfg in configs:
+        if cfg is not None:
+            pair, group, raster = cfg
+            spo.spo_set_tuning(spo.SPO_TUNE_PAIR_MMA, pair)
+            spo.spo_set_tuning(spo.SPO_TUNE_GROUP_M, group)
+            spo.spo_set_tuning(spo.SPO_TUNE_RASTER, raster)
+        for i in range(a.iters):
+            spo.spo_trace_enable(i == a.iters - 1)
+            _, _, lse = spo.spo_logprobs_fwd(H, W, tgt, ws=ws_f)
+            spo.spo_policy_loss_bwd(H, W, tgt, lse, gl, dH=dH, dW=dW, ws=ws_b)
+        torch.cuda.synchronize()
+        label = "default" if cfg is None else f"pair={cfg[0]} group={cfg[1]} raster={cfg[2]}"
+        print(f"--- {label}")
+        for kind, ms in spo.spo_trace_read():
+            tflops = 2.0 * a.T * a.d * a.V / ms / 1e9
+            print(f"{spo.TRACE_KINDS[kind]:24s} {ms:8.3f} ms  {tflops:8.1f} TFLOP/s")
     assert spo.spo_device_error() == 0
 
 

@@ -368,3 +368,32 @@ def test_grpo_step_runs_on_tiny_workload():
                       old, ref, case["clip_eps"], case["kl_beta"])
     assert np.isfinite(out["loss"]) and out["stats"]["n_loss_tokens"] == case["T"]
     assert np.all(out["logp"] <= 0)
+
+
+# ---------------------------------------------------------------- reward composition
+def test_verifiable_reward_hand_cases(golden_dir):
+    gold = _golden(golden_dir, "verifiable_reward_hand_cases.json")
+    cs = gold["cases"]
+    r = O.reward_compose([c["compiled"] for c in cs], [c["pass_rate"] for c in cs],
+                         [c["speedup"] for c in cs], [c["cv"] for c in cs],
+                         [c["r_struct"] for c in cs])
+    np.testing.assert_allclose(r, [c["reward"] for c in cs], atol=1e-12)
+
+
+def test_verifiable_reward_properties():
+    rng = np.random.default_rng(20)
+    n = 200
+    S = np.exp2(rng.uniform(-3, 7, n))
+    cv = rng.uniform(0, 1, n)
+    full = O.reward_compose(np.ones(n), np.ones(n), S, cv)
+    # bounded by the clip: alpha_speed*[s_min, s_max] minus the stability term
+    assert np.all(full <= 4.0 + 1e-12) and np.all(full >= -0.5 - 0.5 * 1.0 - 1e-12)
+    # monotone in speedup for fixed cv
+    order = np.argsort(S)
+    fixed = O.reward_compose(np.ones(n), np.ones(n), S[order], np.full(n, 0.2))
+    assert np.all(np.diff(fixed) >= -1e-12)
+    # partial pass rates ignore speed and cv; a non-positive speedup is the lower bound
+    part = O.reward_compose(np.ones(3), [0.5, 0.5, 0.999], [1e6, 1e-6, 5.0], [0.0, 9.0, 0.0])
+    np.testing.assert_allclose(part, [-1.0, -1.0, -0.002], atol=1e-12)
+    z = O.reward_compose([1, 1], [1.0, 1.0], [0.0, -3.0], [0.0, 0.0])
+    np.testing.assert_allclose(z, [-0.5, -0.5], atol=1e-12)
