@@ -339,6 +339,88 @@ def reward_compose(compiled, pass_rate, speedup, cv, r_struct=None, params=None)
 
 
 # --------------------------------------------------------------------------
+# offline structural ranker (§2.1 "Structural Reward", appendix "MLP Ranker
+# Architecture"): s_psi(phi_hat) with an 11 -> 64 -> 32 -> 1 ReLU MLP and the
+# pairwise logistic ranking loss E[softplus(-(s(y+) - s(y-)))]
+# --------------------------------------------------------------------------
+RANKER_SHAPES = (("W1", (64, 11)), ("b1", (64,)), ("W2", (32, 64)), ("b2", (32,)),
+                 ("w3", (32,)), ("b3", (1,)))
+RANKER_NPARAMS = sum(int(np.prod(sh)) for _, sh in RANKER_SHAPES)   # 2881
+
+
+def ranker_unpack(flat):
+    """Packed parameter vector -> dict of arrays (row-major, in RANKER_SHAPES order)."""
+    flat = np.asarray(flat, dtype=np.float64)
+    out, off = {}, 0
+    for name, sh in RANKER_SHAPES:
+        n = int(np.prod(sh))
+        out[name] = flat[off:off + n].reshape(sh)
+        off += n
+    return out
+
+
+def ranker_scores(phi, mu, sigma, flat, keep1=None, keep2=None, drop_p=0.0):
+    """s_psi(phi_hat) for each row of phi [n, 11]; phi_hat = (phi - mu) / sigma.
+
+    keep1 [n, 64] / keep2 [n, 32]: optional dropout keep flags (0/1) of the two
+    hidden layers; kept units are scaled by 1 / (1 - drop_p).
+    Returns (scores [n], cache for the backward).
+    """
+    P = ranker_unpack(flat)
+    x = (np.asarray(phi, dtype=np.float64) - np.asarray(mu, dtype=np.float64)) / np.asarray(
+        sigma, dtype=np.float64)
+    a1 = x @ P["W1"].T + P["b1"]
+    h1 = np.maximum(a1, 0.0)
+    if keep1 is not None:
+        h1 = h1 * np.asarray(keep1, dtype=np.float64) / (1.0 - drop_p)
+    a2 = h1 @ P["W2"].T + P["b2"]
+    h2 = np.maximum(a2, 0.0)
+    if keep2 is not None:
+        h2 = h2 * np.asarray(keep2, dtype=np.float64) / (1.0 - drop_p)
+    s = h2 @ P["w3"] + P["b3"][0]
+    return s, dict(x=x, a1=a1, h1=h1, a2=a2, h2=h2, P=P, keep1=keep1, keep2=keep2, p=drop_p)
+
+
+def _ranker_backward(c, ds):
+    """Gradient of sum_i ds_i * s_i w.r.t. the packed parameters."""
+    P = c["P"]
+    g = {"w3": c["h2"].T @ ds, "b3": np.array([ds.sum()])}
+    dh2 = np.outer(ds, P["w3"])
+    if c["keep2"] is not None:
+        dh2 = dh2 * np.asarray(c["keep2"], dtype=np.float64) / (1.0 - c["p"])
+    da2 = dh2 * (c["a2"] > 0)
+    g["W2"] = da2.T @ c["h1"]
+    g["b2"] = da2.sum(axis=0)
+    dh1 = da2 @ P["W2"]
+    if c["keep1"] is not None:
+        dh1 = dh1 * np.asarray(c["keep1"], dtype=np.float64) / (1.0 - c["p"])
+    da1 = dh1 * (c["a1"] > 0)
+    g["W1"] = da1.T @ c["x"]
+    g["b1"] = da1.sum(axis=0)
+    return np.concatenate([g[name].reshape(-1) for name, _ in RANKER_SHAPES])
+
+
+def ranker_pair_loss(phi, mu, sigma, flat, pos, neg, keep1=None, keep2=None, drop_p=0.0):
+    """L = mean_k softplus(-(s(phi[pos_k]) - s(phi[neg_k]))) and dL/dparams.
+
+    keep1 / keep2 (optional): dropout keep flags per pair member, shaped
+    [P, 2, 64] / [P, 2, 32] (index 0 = the y+ member, 1 = the y- member).
+    """
+    pos = np.asarray(pos).astype(np.int64)
+    neg = np.asarray(neg).astype(np.int64)
+    Pn = pos.size
+    rows = np.concatenate([pos, neg])
+    k1 = None if keep1 is None else np.concatenate([np.asarray(keep1)[:, 0], np.asarray(keep1)[:, 1]])
+    k2 = None if keep2 is None else np.concatenate([np.asarray(keep2)[:, 0], np.asarray(keep2)[:, 1]])
+    s, c = ranker_scores(np.asarray(phi)[rows], mu, sigma, flat, k1, k2, drop_p)
+    delta = s[:Pn] - s[Pn:]
+    loss = float(np.mean(np.logaddexp(0.0, -delta)))        # softplus(-delta)
+    dd = -1.0 / (1.0 + np.exp(delta)) / Pn                   # dL/d delta
+    grad = _ranker_backward(c, np.concatenate([dd, -dd]))
+    return loss, grad
+
+
+# --------------------------------------------------------------------------
 # the whole step (used for the CPU baseline timing)
 # --------------------------------------------------------------------------
 def grpo_step(H, W, tgt, mask, cu_seqlens, group_id, n_groups, rewards, old_logp, ref_logp,

@@ -397,3 +397,67 @@ def test_verifiable_reward_properties():
     np.testing.assert_allclose(part, [-1.0, -1.0, -0.002], atol=1e-12)
     z = O.reward_compose([1, 1], [1.0, 1.0], [0.0, -3.0], [0.0, 0.0])
     np.testing.assert_allclose(z, [-0.5, -0.5], atol=1e-12)
+
+
+# ---------------------------------------------------------------- offline ranker
+def _ranker_case(seed, n=40, P=25):
+    rng = np.random.default_rng(seed)
+    phi = rng.standard_normal((n, 11)) * 3 + 1
+    mu, sigma = phi.mean(axis=0), phi.std(axis=0) + 0.1
+    flat = rng.standard_normal(O.RANKER_NPARAMS) * 0.3
+    pos, neg = rng.integers(0, n, P), rng.integers(0, n, P)
+    return phi, mu, sigma, flat, pos, neg
+
+
+def test_ranker_shapes_and_equal_scores():
+    assert O.RANKER_NPARAMS == 64 * 11 + 64 + 32 * 64 + 32 + 32 + 1
+    phi, mu, sigma, flat, _, _ = _ranker_case(30)
+    # identical members of a pair: loss = softplus(0) = ln 2 and the gradient vanishes
+    loss, grad = O.ranker_pair_loss(phi, mu, sigma, flat, [3, 7], [3, 7])
+    assert abs(loss - math.log(2.0)) < 1e-15 and np.abs(grad).max() < 1e-15
+    # swapping every pair turns softplus(-d) into softplus(d): the sum is mean(|d|) + 2 mean(softplus(-|d|))
+    _, _, _, _, pos, neg = _ranker_case(31)
+    l1, _ = O.ranker_pair_loss(phi, mu, sigma, flat, pos, neg)
+    l2, _ = O.ranker_pair_loss(phi, mu, sigma, flat, neg, pos)
+    s, _ = O.ranker_scores(phi, mu, sigma, flat)
+    d = s[pos] - s[neg]
+    assert abs(l1 + l2 - (np.abs(d).mean() + 2 * np.logaddexp(0, -np.abs(d)).mean())) < 1e-12
+
+
+def test_ranker_vs_torch_autograd():
+    phi, mu, sigma, flat, pos, neg = _ranker_case(32)
+    rng = np.random.default_rng(33)
+    keep1 = (rng.random((pos.size, 2, 64)) > 0.1).astype(np.uint8)
+    keep2 = (rng.random((pos.size, 2, 32)) > 0.1).astype(np.uint8)
+    loss, grad = O.ranker_pair_loss(phi, mu, sigma, flat, pos, neg, keep1, keep2, 0.1)
+    t = torch.tensor(flat, requires_grad=True)
+    off, Pt = 0, {}
+    for name, sh in O.RANKER_SHAPES:
+        n = int(np.prod(sh))
+        Pt[name] = t[off:off + n].reshape(sh)
+        off += n
+    x = (torch.tensor(phi) - torch.tensor(mu)) / torch.tensor(sigma)
+
+    def score(rows, k1, k2):
+        h1 = torch.relu(x[rows] @ Pt["W1"].T + Pt["b1"]) * torch.tensor(k1, dtype=torch.float64) / 0.9
+        h2 = torch.relu(h1 @ Pt["W2"].T + Pt["b2"]) * torch.tensor(k2, dtype=torch.float64) / 0.9
+        return h2 @ Pt["w3"] + Pt["b3"][0]
+
+    d = score(torch.tensor(pos), keep1[:, 0], keep2[:, 0]) - score(torch.tensor(neg), keep1[:, 1], keep2[:, 1])
+    lt = torch.nn.functional.softplus(-d).mean()
+    lt.backward()
+    assert abs(lt.item() - loss) < 1e-12
+    np.testing.assert_allclose(grad, t.grad.numpy(), atol=1e-12)
+
+
+def test_ranker_finite_difference():
+    phi, mu, sigma, flat, pos, neg = _ranker_case(34, n=12, P=9)
+    _, grad = O.ranker_pair_loss(phi, mu, sigma, flat, pos, neg)
+    h = 1e-6
+    for j in np.random.default_rng(35).choice(O.RANKER_NPARAMS, 40, replace=False):
+        fp, fm = flat.copy(), flat.copy()
+        fp[j] += h
+        fm[j] -= h
+        fd = (O.ranker_pair_loss(phi, mu, sigma, fp, pos, neg)[0] -
+              O.ranker_pair_loss(phi, mu, sigma, fm, pos, neg)[0]) / (2 * h)
+        assert abs(fd - grad[j]) < 1e-7, (j, fd, grad[j])
