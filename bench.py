@@ -53,16 +53,20 @@ UNIT = "tokens/s"
 WORKLOAD = ("full loss fwd+bwd: T=16384 tokens (16 groups x 8 rollouts x 128 tokens), d=5120, "
             "V=151936, bf16 H/W, fp32 accumulate, rewards correctness+log-speedup+structural, "
             "clip eps=0.2, KL beta=0.04, window 1024, SEQ_GROUP aggregation")
-KERNEL_NAMES = {0: "logits_lse_fwd", 1: "logits_grad_recompute", 2: "gemm_dH", 3: "gemm_dW"}
+KERNEL_NAMES = {0: "logits_lse_fwd", 1: "logits_grad_recompute", 2: "gemm_dH", 3: "gemm_dW",
+                4: "lse_combine", 5: "select_gather_fwd", 6: "select_gather_bwd",
+                7: "policy_loss_fwd", 8: "group_advantages", 9: "token_select",
+                10: "reward_compose"}
+GEMM_KINDS = ("logits_lse_fwd", "logits_grad_recompute", "gemm_dH", "gemm_dW")
 SAMPLE_SEQS, SAMPLE_TOKENS = 8, 8   # CPU sample: one group of 8 rollouts, first 8 tokens each
 
 
 # DRAM bytes (read + write) per launch of each tensor-core kernel on this workload, from one
 # `ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum` capture of this command
-# (profiles/launches_full_workload.md), valid only for the kernel sources they were taken on.
-TRAFFIC = {"sources_sha256_16": "91b0e0fcf2f7d7a3",
-           "bytes": {"logits_lse_fwd": 42.808e9, "logits_grad_recompute": 49.241e9,
-                     "gemm_dH": 81.260e9, "gemm_dW": 68.447e9}}
+# (profiles/raster_dram_sweep_full_workload.md, first row), valid only for the kernel sources they were taken on.
+TRAFFIC = {"sources_sha256_16": "359a09cc1e70d703",
+           "bytes": {"logits_lse_fwd": 41.135e9, "logits_grad_recompute": 49.551e9,
+                     "gemm_dH": 83.180e9, "gemm_dW": 69.987e9}}
 KERNEL_SOURCES = ["paper_2607_20908_gb300/csrc/gemm.cu", "paper_2607_20908_gb300/csrc/tc.cuh",
                   "paper_2607_20908_gb300/csrc/internal.h"]
 
@@ -372,6 +376,37 @@ def run_cpu_baseline(st: Step, budget_s: float = 12.0):
             "kind": "oracle", "sample": sample_description(s["n"]) + f"; {reps} reps in {el:.1f} s"}
 
 
+def aux_measurements(dev, pk):
+    """Steps outside the timed loop, each timed with CUDA events on its own:
+    the reward composition (section 2.2) at an enlarged synthetic size
+    (2^24 candidates; 21 algorithmic bytes each), HBM-bound."""
+    from paper_2607_20908_gb300 import spo
+    n = 1 << 24
+    gen = torch.Generator(device=dev).manual_seed(5)
+    compiled = (torch.rand(n, device=dev, generator=gen) < 0.8).to(torch.uint8)
+    p = torch.where(torch.rand(n, device=dev, generator=gen) < 0.5, 1.0,
+                    torch.rand(n, device=dev, generator=gen))
+    S = torch.exp2(torch.rand(n, device=dev, generator=gen) * 11 - 3)
+    cv = torch.rand(n, device=dev, generator=gen)
+    rs = torch.randn(n, device=dev, generator=gen)
+    out = torch.empty(n, device=dev)
+    for _ in range(3):
+        spo.spo_reward_compose(compiled, p, S, cv, rs, out=out)
+    torch.cuda.synchronize(dev)
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    reps = 20
+    a.record()
+    for _ in range(reps):
+        spo.spo_reward_compose(compiled, p, S, cv, rs, out=out)
+    b.record()
+    torch.cuda.synchronize(dev)
+    t = a.elapsed_time(b) / reps / 1e3
+    gbs = 21 * n / t / 1e9
+    return {"reward_compose": {"candidates": n, "ms": t * 1e3, "gbs": gbs,
+                               "frac_of_hbm": gbs / pk["hbm"], "bound": "hbm",
+                               "note": "enlarged synthetic size; the workload itself has 128 rollouts"}}
+
+
 # ----------------------------------------------------------------- arms
 def config_block(case, T_L, world):
     return {"workload": WORKLOAD, "T": case["T"], "loss_tokens": T_L, "d": case["d"], "V": case["V"],
@@ -424,11 +459,26 @@ def ours(args):
         k = kern.setdefault(KERNEL_NAMES.get(kind, str(kind)), {"launches": 0, "total_ms": 0.0})
         k["launches"] += 1
         k["total_ms"] += t
-    for k in kern.values():
+    nsplit = (st.V + 255) // 256
+    hbm_bytes = {   # algorithmic bytes per call of the HBM-bound steps
+        "lse_combine": 16 * nsplit * T_L + 8 * T_L + 12 * st.T,
+        "select_gather_fwd": 4 * T_L * st.d + 5 * st.T + 8 * T_L,
+        "select_gather_bwd": 4 * T_L * st.d + 12 * st.T + 16 * T_L,
+    }
+    for name, k in kern.items():
         k["avg_ms"] = k["total_ms"] / k["launches"]
         k["share_of_step"] = k["total_ms"] / ms
-        k["tflops"] = flop_gemm / (k["avg_ms"] / 1e3) / 1e12
-    dom_name, dom = max(kern.items(), key=lambda kv: kv[1]["total_ms"])
+        if name in GEMM_KINDS:
+            k["tflops"] = flop_gemm / (k["avg_ms"] / 1e3) / 1e12
+        elif name in hbm_bytes:
+            k["gbs"] = hbm_bytes[name] / (k["avg_ms"] / 1e3) / 1e9
+            k["frac_of_hbm"] = k["gbs"] / pk["hbm"]
+            k["algorithmic_bytes"] = hbm_bytes[name]
+        else:
+            k["bound"] = "latency"
+            k["avg_us"] = k["avg_ms"] * 1e3
+    dom_name, dom = max(((n, k) for n, k in kern.items() if n in GEMM_KINDS),
+                        key=lambda kv: kv[1]["total_ms"])
     achieved = dom["tflops"]
     roofline = {"bound": "tensor", "kernel": dom_name, "achieved": achieved,
                 "peak": pk["bf16_sustained"], "unit": "TFLOP/s", "frac": achieved / pk["bf16_sustained"],
@@ -443,8 +493,9 @@ def ours(args):
            "gemm_dW": 2 * T_L * st.V + 2 * T_L * st.d + 4 * st.V * st.d}
     roofline["algorithmic_bytes"] = alg[dom_name]
     for name, k in kern.items():
-        k["dram_bytes_ncu"] = kernel_traffic(name)
-        k["algorithmic_bytes"] = alg[name]
+        if name in alg:
+            k["dram_bytes_ncu"] = kernel_traffic(name)
+            k["algorithmic_bytes"] = alg[name]
 
     # e2e: host buffers, H2D + step + D2H inside the timed region
     hio = HostIO(st)
@@ -478,6 +529,7 @@ def ours(args):
         "launches_per_step": n_launch / args.steps,
         "clocks": clocks.summary(t0, t1),
     }
+    line["aux"] = aux_measurements(dev, pk)
     if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = run_cpu_baseline(st)
     if dist.rank == 0:

@@ -151,6 +151,68 @@ SPO_API spo_status spo_logprobs_fwd(const void* H, const void* W, const int32_t*
                                     void* ws, size_t ws_bytes, void* stream);
 
 /* ---------------------------------------------------------------------------
+ * Composite reward (section 2.2, "Verifiable Reward"; r_i = R_ver(i) + R_str(i),
+ * section 3), the input of spo_group_advantages.  Per candidate i:
+ *   R_comp  = -alpha_comp                        if the program does not compile
+ *   R_corr  = -alpha_wrong * (1 - p)             p = fraction of tests passed
+ *   R_speed = alpha_speed * clip(log2 S, s_min, s_max)
+ *   R_cv    = -alpha_cv * cv
+ *   R_ver   = R_comp (not compiled) | R_corr (p < 1) | R_corr + R_speed + R_cv (p = 1)
+ *   r       = R_ver + r_struct
+ *
+ *   compiled  uint8[n]   0 = compilation failed
+ *   pass_rate fp32[n]    in [0, 1]
+ *   speedup   fp32[n]    sequential / CUDA runtime; a value that is not > 0
+ *                        counts as the lower clip bound
+ *   cv        fp32[n]    coefficient of variation of the CUDA runtime
+ *   r_struct  fp32[n]    structural score R_str, or NULL for 0
+ *   params    HOST pointer, or NULL for the paper's values (3.0, 2.0, 1.0,
+ *             0.5, -0.5, 4.0); must be finite with s_min <= s_max
+ *   rewards   fp32[n] out.  fp32 arithmetic (log2f); within 1e-6 of fp64.
+ * ------------------------------------------------------------------------- */
+typedef struct spo_reward_params {
+    float alpha_comp, alpha_wrong, alpha_speed, alpha_cv, s_min, s_max;
+} spo_reward_params;
+SPO_API spo_status spo_reward_compose(const uint8_t* compiled, const float* pass_rate,
+                                      const float* speedup, const float* cv,
+                                      const float* r_struct, int32_t n,
+                                      const spo_reward_params* params, float* rewards,
+                                      void* stream);
+
+/* ---------------------------------------------------------------------------
+ * Offline structural ranker (section 2.1, "Structural Reward"; architecture in
+ * the appendix "MLP Ranker Architecture").  Features phi (11 per program:
+ * coalescing, arithmetic intensity, occupancy, divergence, transfer,
+ * atomics, syncthreads, kernels, threads per block, global accesses, ops)
+ * are z-scored with the training split's mean and std, phi_hat = (phi - mu) /
+ * sigma, and scored by s_psi: 11 -> 64 -> 32 -> 1 with ReLU.  The score is
+ * the structural reward R_str.  Training minimises the pairwise logistic
+ * ranking loss L = mean_k softplus(-(s(y+_k) - s(y-_k))).
+ *
+ * params: fp32[2881] packed row-major: W1[64][11], b1[64], W2[32][64], b2[32],
+ *         w3[32], b3.  phi fp32[n][11]; mu, sigma fp32[11].
+ * spo_ranker_scores: scores fp32[n] = s_psi(phi_hat) (inference, no dropout).
+ * spo_ranker_pair_loss: pos / neg int32[n_pairs] row indices into phi (the
+ *   y+ and y- of each pair; valid rows of phi, not range-checked); keep1
+ *   uint8[n_pairs][2][64] / keep2 uint8[n_pairs][2][32] are optional dropout
+ *   keep flags of the two hidden layers ([k][0] = y+, [k][1] = y-), kept
+ *   units scaled by 1 / (1 - drop_p) (NULL = no dropout); loss fp32[1]; grad
+ *   fp32[2881] = dL/dparams (may be NULL).  One warp per pair; gradients are
+ *   summed in a fixed order (run-to-run deterministic).  fp32 arithmetic.
+ *   ws >= spo_ranker_workspace_size(n_pairs) bytes, 256-byte aligned.
+ * ------------------------------------------------------------------------- */
+#define SPO_RANKER_FEATURES 11
+#define SPO_RANKER_PARAMS 2881
+SPO_API spo_status spo_ranker_scores(const float* phi, const float* mu, const float* sigma,
+                                     int32_t n, const float* params, float* scores, void* stream);
+SPO_API spo_status spo_ranker_workspace_size(int32_t n_pairs, size_t* bytes);
+SPO_API spo_status spo_ranker_pair_loss(const float* phi, const float* mu, const float* sigma,
+                                        const int32_t* pos, const int32_t* neg, int32_t n_pairs,
+                                        const float* params, const uint8_t* keep1,
+                                        const uint8_t* keep2, float drop_p, float* loss,
+                                        float* grad, void* ws, size_t ws_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------
  * a4. Group-normalised advantage (definition under Eq. 3):
  *   A_hat_i = (r_i - mean(r_g)) / (std(r_g) + eps), g = group_id[i].
  * Members of a group are taken in ascending i; the arithmetic is IEEE fp32
@@ -259,14 +321,18 @@ SPO_API spo_status spo_policy_loss_fwd_noalloc(const float* logp, const float* o
  * Measurement hooks (no counterpart in the paper; used to report per-kernel
  * device time against the tensor-core roofline).
  *
- * spo_trace_enable(1): from now on every tensor-core GEMM launch of this
- *   library is bracketed by a start/stop CUDA event pair recorded on the
- *   launch stream.  Host-global; costs two event records per GEMM.
+ * spo_trace_enable(1): from now on every launch sequence of this library
+ *   (each GEMM, and each small-kernel step) is bracketed by a start/stop CUDA
+ *   event pair recorded on the launch stream.  Host-global; two event records
+ *   per traced sequence.
  * spo_trace_read: waits for every recorded pair, writes up to max_records
  *   (kind, milliseconds) in launch order, returns the number recorded in
  *   *n_records (may exceed max_records) and clears the record list.  kind:
  *   0 = logits + online logsumexp (a2), 1 = logits recompute -> G (a6),
- *   2 = dH = G W (a7), 3 = dW = G^T H (a8).
+ *   2 = dH = G W (a7), 3 = dW = G^T H (a8), 4 = split-vocab combine (a3),
+ *   5 = forward row selection + gather, 6 = backward row selection + gather,
+ *   7 = policy-loss forward (a5), 8 = group advantages (a4),
+ *   9 = token selection (a1), 10 = reward composition.
  * spo_launch_count: kernels launched by this library since it was loaded
  *   (host-side counter; every kernel launch adds one).
  * ------------------------------------------------------------------------- */

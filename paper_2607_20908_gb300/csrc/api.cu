@@ -189,21 +189,27 @@ bool g_trace_on = false;
 std::vector<TraceRec> g_trace;
 std::vector<TraceRec> g_trace_pool;  // event pairs ready for reuse
 
-spo_status traced_gemm(int kind, bool a_mn, bool b_mn, const CUtensorMap& ta, const CUtensorMap& tb,
-                       const spo::GemmArgs& args, int grid, cudaStream_t s, const DevInfo& di) {
-  TraceRec rec{kind, di.dev, nullptr, nullptr};
+// Runs `launch` (which enqueues one or more kernels on s and returns the
+// launch status), bracketed by a recorded event pair when tracing is on.
+template <class F>
+spo_status traced(int kind, cudaStream_t s, const char* what, F&& launch) {
+  int dev = 0;
+  TraceRec rec{kind, 0, nullptr, nullptr};
   bool tracing;
   {
     std::lock_guard<std::mutex> lk(g_trace_mu);
     tracing = g_trace_on;
-    if (tracing) {
-      for (size_t i = 0; i < g_trace_pool.size(); ++i) {
-        if (g_trace_pool[i].dev == di.dev) {
-          rec.start = g_trace_pool[i].start;
-          rec.stop = g_trace_pool[i].stop;
-          g_trace_pool.erase(g_trace_pool.begin() + i);
-          break;
-        }
+  }
+  if (tracing) {
+    SPO_CUDA(cudaGetDevice(&dev), "cudaGetDevice");
+    rec.dev = dev;
+    std::lock_guard<std::mutex> lk(g_trace_mu);
+    for (size_t i = 0; i < g_trace_pool.size(); ++i) {
+      if (g_trace_pool[i].dev == dev) {
+        rec.start = g_trace_pool[i].start;
+        rec.stop = g_trace_pool[i].stop;
+        g_trace_pool.erase(g_trace_pool.begin() + i);
+        break;
       }
     }
   }
@@ -212,14 +218,32 @@ spo_status traced_gemm(int kind, bool a_mn, bool b_mn, const CUtensorMap& ta, co
     SPO_CUDA(cudaEventCreate(&rec.stop), "cudaEventCreate");
   }
   if (tracing) SPO_CUDA(cudaEventRecord(rec.start, s), "cudaEventRecord");
-  SPO_CUDA(spo::launch_gemm(kind, a_mn, b_mn, g_tune_pair != 0, ta, tb, args, grid, s),
-           "gemm launch");
+  SPO_CUDA(launch(), what);
   if (tracing) {
     SPO_CUDA(cudaEventRecord(rec.stop, s), "cudaEventRecord");
     std::lock_guard<std::mutex> lk(g_trace_mu);
     g_trace.push_back(rec);
   }
   return SPO_OK;
+}
+
+// Trace kinds (spo_trace_read): the four tensor-core GEMMs keep their EPI ids.
+enum TraceKind : int {
+  kTraceLseCombine = 4,
+  kTraceSelectGatherFwd = 5,
+  kTraceSelectGatherBwd = 6,
+  kTracePolicyLoss = 7,
+  kTraceAdvantages = 8,
+  kTraceTokenSelect = 9,
+  kTraceReward = 10,
+  kTraceRanker = 11,
+};
+
+spo_status traced_gemm(int kind, bool a_mn, bool b_mn, const CUtensorMap& ta, const CUtensorMap& tb,
+                       const spo::GemmArgs& args, int grid, cudaStream_t s) {
+  return traced(kind, s, "gemm launch", [&] {
+    return spo::launch_gemm(kind, a_mn, b_mn, g_tune_pair != 0, ta, tb, args, grid, s);
+  });
 }
 
 spo::GemmArgs base_args(const DevInfo& di) {
@@ -296,9 +320,10 @@ SPO_API spo_status spo_token_select(const int32_t* cu_seqlens, const uint8_t* ma
   if (n_seq < 1 || n_seq > (1 << 24)) return fail(SPO_ERR_SHAPE, "n_seq = %d outside [1, 2^24]", n_seq);
   if (T < 1 || T > (1ll << 31) - 1) return fail(SPO_ERR_SHAPE, "T = %lld out of range", (long long)T);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  SPO_CUDA(spo::launch_token_select(cu_seqlens, mask, tgt, n_seq, window, loss_mask, n_tok, s),
-           "token_select launch");
-  return ok();
+  spo_status st = traced(kTraceTokenSelect, s, "token_select launch", [&] {
+    return spo::launch_token_select(cu_seqlens, mask, tgt, n_seq, window, loss_mask, n_tok, s);
+  });
+  return st == SPO_OK ? ok() : st;
 }
 
 SPO_API spo_status spo_logprobs_workspace_size(int64_t T, int64_t d, int64_t V, size_t* bytes) {
@@ -326,11 +351,14 @@ SPO_API spo_status spo_logprobs_fwd(const void* H, const void* W, const int32_t*
   const FwdWs w = carve_fwd(ws, T, d, V);
 
   // a1 (row selection) + gather of the kept rows into a dense bf16 block
-  SPO_CUDA(spo::launch_compact(0, mask, tgt, nullptr, T, w.scratch, w.idx, w.count, s), "compact");
-  SPO_CUDA(spo::launch_gather(static_cast<const __nv_bfloat16*>(H), static_cast<int>(d), w.idx,
+  st = traced(kTraceSelectGatherFwd, s, "compact/gather", [&] {
+    cudaError_t e = spo::launch_compact(0, mask, tgt, nullptr, T, w.scratch, w.idx, w.count, s);
+    if (e != cudaSuccess) return e;
+    return spo::launch_gather(static_cast<const __nv_bfloat16*>(H), static_cast<int>(d), w.idx,
                               w.count, static_cast<int>(w.T_pad), w.Hc, tgt, w.tgt_c, nullptr,
-                              nullptr, nullptr, nullptr, s),
-           "gather");
+                              nullptr, nullptr, nullptr, s);
+  });
+  if (st != SPO_OK) return st;
   // a2: logits tile by tile + online logsumexp partials
   CUtensorMap ta, tb;
   SPO_CUDA(spo::make_tmap_bf16(&ta, w.Hc, d, w.T_pad, d * 2, spo::BK, spo::BM), "tensor map H");
@@ -344,19 +372,84 @@ SPO_API spo_status spo_logprobs_fwd(const void* H, const void* W, const int32_t*
   a.scale = inv_temp;
   a.tgt = w.tgt_c;
   a.partials = w.partials;
-  a.ld_part = static_cast<int>(w.T_pad);
+  a.nsplit = w.nsplit;
   a.ztgt = w.ztgt;
-  if ((st = traced_gemm(spo::EPI_LSE, false, false, ta, tb, a, grid_for(di, w.T_pad, V), s, di)) !=
+  if ((st = traced_gemm(spo::EPI_LSE, false, false, ta, tb, a, grid_for(di, w.T_pad, V), s)) !=
       SPO_OK)
     return st;
   // a3: split-vocab combine, scattered back to token positions (skipped tokens read 0)
   SPO_CUDA(cudaMemsetAsync(logp, 0, sizeof(float) * T, s), "memset logp");
   if (entropy) SPO_CUDA(cudaMemsetAsync(entropy, 0, sizeof(float) * T, s), "memset entropy");
   if (lse) SPO_CUDA(cudaMemsetAsync(lse, 0, sizeof(float) * T, s), "memset lse");
-  SPO_CUDA(spo::launch_lse_combine(w.partials, static_cast<int>(w.T_pad), w.nsplit, w.ztgt, w.idx,
-                                   w.count, static_cast<int>(w.T_pad), logp, entropy, lse, s),
-           "combine launch");
+  st = traced(kTraceLseCombine, s, "combine launch", [&] {
+    return spo::launch_lse_combine(w.partials, w.nsplit, w.ztgt, w.idx, w.count,
+                                   static_cast<int>(w.T_pad), logp, entropy, lse, s);
+  });
+  return st == SPO_OK ? ok() : st;
+}
+
+SPO_API spo_status spo_reward_compose(const uint8_t* compiled, const float* pass_rate,
+                                      const float* speedup, const float* cv, const float* r_struct,
+                                      int32_t n, const spo_reward_params* params, float* rewards,
+                                      void* stream) {
+  if (!compiled || !pass_rate || !speedup || !cv || !rewards)
+    return fail(SPO_ERR_INVALID_ARG, "compiled, pass_rate, speedup, cv and rewards must be non-NULL");
+  if (n < 1 || n > (1 << 30)) return fail(SPO_ERR_SHAPE, "n = %d out of range", n);
+  spo::RewardParams q{3.0f, 2.0f, 1.0f, 0.5f, -0.5f, 4.0f};  // the paper's constants
+  if (params) {
+    q = spo::RewardParams{params->alpha_comp, params->alpha_wrong, params->alpha_speed,
+                          params->alpha_cv, params->s_min, params->s_max};
+    const float v[6] = {q.alpha_comp, q.alpha_wrong, q.alpha_speed, q.alpha_cv, q.s_min, q.s_max};
+    for (float x : v)
+      if (!isfinite(x)) return fail(SPO_ERR_INVALID_ARG, "reward parameters must be finite");
+    if (q.s_min > q.s_max) return fail(SPO_ERR_INVALID_ARG, "s_min must not exceed s_max");
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  spo_status st = traced(kTraceReward, s, "reward launch", [&] {
+    return spo::launch_reward_compose(compiled, pass_rate, speedup, cv, r_struct, n, q, rewards, s);
+  });
+  return st == SPO_OK ? ok() : st;
+}
+
+SPO_API spo_status spo_ranker_scores(const float* phi, const float* mu, const float* sigma,
+                                     int32_t n, const float* params, float* scores, void* stream) {
+  if (!phi || !mu || !sigma || !params || !scores)
+    return fail(SPO_ERR_INVALID_ARG, "phi, mu, sigma, params and scores must be non-NULL");
+  if (n < 1 || n > (1 << 30)) return fail(SPO_ERR_SHAPE, "n = %d out of range", n);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  spo_status st = traced(kTraceRanker, s, "ranker launch", [&] {
+    return spo::launch_ranker_scores(phi, mu, sigma, n, params, scores, s);
+  });
+  return st == SPO_OK ? ok() : st;
+}
+
+SPO_API spo_status spo_ranker_workspace_size(int32_t n_pairs, size_t* bytes) {
+  if (!bytes) return fail(SPO_ERR_INVALID_ARG, "bytes must be non-NULL");
+  if (n_pairs < 1) return fail(SPO_ERR_SHAPE, "n_pairs must be >= 1");
+  *bytes = spo::ranker_ws_bytes(n_pairs);
   return ok();
+}
+
+SPO_API spo_status spo_ranker_pair_loss(const float* phi, const float* mu, const float* sigma,
+                                        const int32_t* pos, const int32_t* neg, int32_t n_pairs,
+                                        const float* params, const uint8_t* keep1,
+                                        const uint8_t* keep2, float drop_p, float* loss,
+                                        float* grad, void* ws, size_t ws_bytes, void* stream) {
+  if (!phi || !mu || !sigma || !pos || !neg || !params || !loss)
+    return fail(SPO_ERR_INVALID_ARG, "a required pointer is NULL");
+  if (n_pairs < 1 || n_pairs > (1 << 28)) return fail(SPO_ERR_SHAPE, "n_pairs = %d out of range", n_pairs);
+  if (!(drop_p >= 0.f && drop_p < 1.f)) return fail(SPO_ERR_INVALID_ARG, "drop_p must be in [0, 1)");
+  const size_t need = spo::ranker_ws_bytes(n_pairs);
+  if (!ws || ws_bytes < need)
+    return fail(SPO_ERR_WORKSPACE, "workspace needs %zu bytes, got %zu", need, ws_bytes);
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
+    return fail(SPO_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  spo_status st = traced(kTraceRanker, s, "ranker launch", [&] {
+    return spo::launch_ranker_pair_loss(phi, mu, sigma, pos, neg, n_pairs, params, keep1, keep2,
+                                        drop_p, loss, grad, static_cast<float*>(ws), s);
+  });
+  return st == SPO_OK ? ok() : st;
 }
 
 SPO_API spo_status spo_group_advantages(const float* rewards, const int32_t* group_id,
@@ -370,9 +463,10 @@ SPO_API spo_status spo_group_advantages(const float* rewards, const int32_t* gro
     return fail(SPO_ERR_INVALID_ARG, "std_mode %d unknown", std_mode);
   if (!(eps >= 0.f) || !isfinite(eps)) return fail(SPO_ERR_INVALID_ARG, "eps must be finite and >= 0");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  SPO_CUDA(spo::launch_group_advantages(rewards, group_id, n_seq, n_groups, std_mode, eps, adv, s),
-           "advantage launch");
-  return ok();
+  spo_status st = traced(kTraceAdvantages, s, "advantage launch", [&] {
+    return spo::launch_group_advantages(rewards, group_id, n_seq, n_groups, std_mode, eps, adv, s);
+  });
+  return st == SPO_OK ? ok() : st;
 }
 
 SPO_API spo_status spo_policy_loss_workspace_size(int32_t n_seq, int32_t n_groups, size_t* bytes) {
@@ -405,11 +499,12 @@ SPO_API spo_status spo_policy_loss_fwd(const float* logp, const float* old_logp,
     return fail(SPO_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const spo::LossWs w = spo::carve_loss_ws(ws, n_seq, n_groups);
-  SPO_CUDA(spo::launch_policy_loss(logp, old_logp, ref_logp, adv, cu_seqlens, group_id, n_seq,
+  spo_status st = traced(kTracePolicyLoss, s, "policy loss launch", [&] {
+    return spo::launch_policy_loss(logp, old_logp, ref_logp, adv, cu_seqlens, group_id, n_seq,
                                    n_groups, loss_mask, T, clip_eps, kl_beta, agg, loss, g, stats,
-                                   w, s),
-           "policy loss launch");
-  return ok();
+                                   w, s);
+  });
+  return st == SPO_OK ? ok() : st;
 }
 
 SPO_API spo_status spo_policy_loss_bwd_workspace_size(int64_t T, int64_t d, int64_t V,
@@ -441,11 +536,14 @@ SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32
   if (!dH && !dW) return ok();
 
   // rows with g != 0 are the only ones with a non-zero gradient row
-  SPO_CUDA(spo::launch_compact(1, nullptr, nullptr, g, T, w.scratch, w.idx, w.count, s), "compact");
-  SPO_CUDA(spo::launch_gather(static_cast<const __nv_bfloat16*>(H), static_cast<int>(d), w.idx,
+  st = traced(kTraceSelectGatherBwd, s, "compact/gather", [&] {
+    cudaError_t e = spo::launch_compact(1, nullptr, nullptr, g, T, w.scratch, w.idx, w.count, s);
+    if (e != cudaSuccess) return e;
+    return spo::launch_gather(static_cast<const __nv_bfloat16*>(H), static_cast<int>(d), w.idx,
                               w.count, static_cast<int>(w.T_pad), w.Hc, tgt, w.tgt_c, lse, w.lse_c,
-                              g, w.g_c, s),
-           "gather");
+                              g, w.g_c, s);
+  });
+  if (st != SPO_OK) return st;
   if (dH) SPO_CUDA(cudaMemsetAsync(dH, 0, sizeof(uint16_t) * T * d, s), "memset dH");
 
   CUtensorMap tW_k, tW_mn, tG_k, tG_mn;
@@ -476,8 +574,7 @@ SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32
     a.gvec = w.g_c + r0;
     a.G = w.G;
     a.ldG = V;
-    if ((st = traced_gemm(spo::EPI_GRAD, false, false, tH_k, tW_k, a, grid_for(di, rows, V), s,
-                          di)) != SPO_OK)
+    if ((st = traced_gemm(spo::EPI_GRAD, false, false, tH_k, tW_k, a, grid_for(di, rows, V), s)) != SPO_OK)
       return st;
     // a7: dH rows = G W, scattered to token rows
     if (dH) {
@@ -490,8 +587,7 @@ SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32
       b.row_idx = w.idx + r0;
       b.out_bf16 = static_cast<__nv_bfloat16*>(dH);
       b.ld_out = d;
-      if ((st = traced_gemm(spo::EPI_DH, false, true, tG_k, tW_mn, b, grid_for(di, rows, d), s,
-                            di)) != SPO_OK)
+      if ((st = traced_gemm(spo::EPI_DH, false, true, tG_k, tW_mn, b, grid_for(di, rows, d), s)) != SPO_OK)
         return st;
     }
     // a8: dW (+)= G^T Hc over this chunk's rows
@@ -505,7 +601,7 @@ SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32
       b.out_f32 = dW;
       b.ld_out = d;
       b.accumulate = (c == 0) ? (accumulate_dW ? 1 : 0) : 1;
-      if ((st = traced_gemm(spo::EPI_DW, true, true, tG_mn, tH_mn, b, grid_for(di, V, d), s, di)) !=
+      if ((st = traced_gemm(spo::EPI_DW, true, true, tG_mn, tH_mn, b, grid_for(di, V, d), s)) !=
           SPO_OK)
         return st;
     }

@@ -114,7 +114,8 @@ __device__ __forceinline__ void epi_lse(const GemmArgs& p, uint32_t taddr, int r
     run_m = nm;
   }
   if (row_ok) {
-    p.partials[static_cast<size_t>(nb) * p.ld_part + row] = make_float4(run_m, run_s, run_e, 0.f);
+    p.partials[(static_cast<size_t>(row >> 5) * p.nsplit + nb) * 32 + (row & 31)] =
+        make_float4(run_m, run_s, run_e, 0.f);
     if (hit) p.ztgt[row] = zt;
   }
 }

@@ -44,8 +44,10 @@ struct GemmArgs {
   float scale;  // inv_temp for EPI_LSE / EPI_GRAD
   // EPI_LSE
   const int* tgt;     // target id of each row
-  float4* partials;   // [ceil(n / BN)][ld_part]: (max*log2e, sum 2^(t-max), sum 2^(t-max) t, 0)
-  int ld_part;
+  // Per (row, vocab tile) partials (max*log2e, sum 2^(t-max), sum 2^(t-max) t, 0), laid out
+  // [row / 32][vocab tile][row % 32]: a warp's 32 rows of one tile are 512 contiguous bytes.
+  float4* partials;
+  int nsplit;  // number of vocab tiles, ceil(n / BN)
   float* ztgt;        // target logit (natural units) of each row
   // EPI_GRAD
   const float* lse;   // natural-log lse of each row
@@ -96,7 +98,7 @@ cudaError_t launch_gather(const __nv_bfloat16* H, int d, const int* idx, const i
                           const float* a, float* a_c, const float* b, float* b_c,
                           cudaStream_t s);
 
-cudaError_t launch_lse_combine(const float4* partials, int ld_part, int nsplit,
+cudaError_t launch_lse_combine(const float4* partials, int nsplit,
                                const float* ztgt, const int* idx, const int* count,
                                int rows_cap, float* logp, float* entropy, float* lse,
                                cudaStream_t s);
@@ -108,6 +110,28 @@ cudaError_t launch_token_select(const int* cu_seqlens, const uint8_t* mask, cons
 cudaError_t launch_group_advantages(const float* rewards, const int* group_id, int n_seq,
                                     int n_groups, int std_mode, float eps, float* adv,
                                     cudaStream_t s);
+
+// Composite reward (section 2.2 verifiable reward + structural score).
+struct RewardParams {
+  float alpha_comp, alpha_wrong, alpha_speed, alpha_cv, s_min, s_max;
+};
+cudaError_t launch_reward_compose(const uint8_t* compiled, const float* pass_rate,
+                                  const float* speedup, const float* cv, const float* r_struct,
+                                  int n, const RewardParams& q, float* out, cudaStream_t s);
+
+// Offline structural ranker: 11 -> 64 -> 32 -> 1 ReLU MLP, packed parameters
+// W1[64][11], b1[64], W2[32][64], b2[32], w3[32], b3.
+constexpr int kRankerFeatures = 11;
+constexpr int kRankerParams = 64 * 11 + 64 + 32 * 64 + 32 + 32 + 1;  // 2881
+int ranker_blocks(int n_pairs);
+size_t ranker_ws_bytes(int n_pairs);
+cudaError_t launch_ranker_scores(const float* phi, const float* mu, const float* sigma, int n,
+                                 const float* params, float* scores, cudaStream_t s);
+cudaError_t launch_ranker_pair_loss(const float* phi, const float* mu, const float* sigma,
+                                    const int* pos, const int* neg, int n_pairs,
+                                    const float* params, const uint8_t* keep1,
+                                    const uint8_t* keep2, float drop_p, float* loss, float* grad,
+                                    float* ws, cudaStream_t s);
 
 struct LossWs {
   int* gsize;        // [n_groups]

@@ -133,27 +133,30 @@ __global__ void gather_kernel(const uint4* H, int row_vecs, const int* idx, cons
 }
 
 // Merge (m2, s2, e2) into (m, s, e); m in log2 units, s = sum 2^(t-m), e = sum 2^(t-m) t.
+// One exponential: the side with the smaller max is rescaled onto the larger.
 __device__ __forceinline__ void lse_merge(float& m, float& s, float& e, float m2, float s2, float e2) {
   if (m2 == -INFINITY) return;
-  if (m == -INFINITY) {
-    m = m2; s = s2; e = e2;
-    return;
+  if (m2 <= m) {
+    const float r = exp2f(m2 - m);
+    s = fmaf(s2, r, s);
+    e = fmaf(e2, r, e);
+  } else {
+    const float r = exp2f(m - m2);  // m = -inf gives r = 0
+    s = fmaf(s, r, s2);
+    e = fmaf(e, r, e2);
+    m = m2;
   }
-  const float nm = fmaxf(m, m2);
-  const float r1 = exp2f(m - nm), r2 = exp2f(m2 - nm);
-  s = s * r1 + s2 * r2;
-  e = e * r1 + e2 * r2;
-  m = nm;
 }
 
-// Split-vocabulary combine: 32 rows per block, warp w merges vocab tiles
-// w, w+8, ...; the 8 per-warp results are merged through shared memory.
-__global__ void __launch_bounds__(256) lse_combine_kernel(const float4* partials, int ld_part,
-                                                          int nsplit, const float* ztgt,
-                                                          const int* idx, const int* count,
-                                                          float* logp, float* entropy,
-                                                          float* lse_out) {
-  __shared__ float sm[8][32][3];
+constexpr int kCombineWarps = 16;
+
+// Split-vocabulary combine: 32 rows per block (one contiguous [nsplit][32]
+// slab of partials), warp w merges vocab tiles w, w + 16, ...; the per-warp
+// results are merged through shared memory.
+__global__ void __launch_bounds__(kCombineWarps * 32) lse_combine_kernel(
+    const float4* partials, int nsplit, const float* ztgt, const int* idx, const int* count,
+    float* logp, float* entropy, float* lse_out) {
+  __shared__ float sm[kCombineWarps][32][3];
   const int n = *count;
   const int row0 = blockIdx.x * 32;
   if (row0 >= n) return;
@@ -161,9 +164,10 @@ __global__ void __launch_bounds__(256) lse_combine_kernel(const float4* partials
   const int row = row0 + lane;
   float m = -INFINITY, s = 0.f, e = 0.f;
   if (row < n) {
-#pragma unroll 4
-    for (int j = warp; j < nsplit; j += 8) {
-      const float4 pr = partials[static_cast<size_t>(j) * ld_part + row];
+    const float4* slab = partials + static_cast<size_t>(blockIdx.x) * nsplit * 32 + lane;
+#pragma unroll 8
+    for (int j = warp; j < nsplit; j += kCombineWarps) {
+      const float4 pr = slab[static_cast<size_t>(j) * 32];
       lse_merge(m, s, e, pr.x, pr.y, pr.z);
     }
   }
@@ -172,7 +176,8 @@ __global__ void __launch_bounds__(256) lse_combine_kernel(const float4* partials
   sm[warp][lane][2] = e;
   __syncthreads();
   if (warp == 0 && row < n) {
-    for (int w = 1; w < 8; ++w) lse_merge(m, s, e, sm[w][lane][0], sm[w][lane][1], sm[w][lane][2]);
+    for (int w = 1; w < kCombineWarps; ++w)
+      lse_merge(m, s, e, sm[w][lane][0], sm[w][lane][1], sm[w][lane][2]);
     const float lse2 = m + log2f(s);
     const float lse_nat = lse2 * kLn2;
     const int t = idx[row];
@@ -253,6 +258,48 @@ __global__ void group_adv_kernel(const float* rewards, const int* gid, int n_seq
   for (int base = 0; base < n_seq; base += 32) {
     const int i = base + lane;
     if (i < n_seq && gid[i] == g) adv[i] = zero ? 0.f : __fdiv_rn(__fsub_rn(rewards[i], mu), den);
+  }
+}
+
+// Composite reward of one candidate: the piecewise verifiable reward
+// (compile penalty; correctness penalty; clipped log2 speedup and stability
+// penalty once every test passes) plus the structural score.
+__device__ __forceinline__ float composite_reward(uint8_t compiled, float p, float speedup, float cv,
+                                                  float r_struct, const RewardParams& q) {
+  float r;
+  if (compiled == 0) {
+    r = -q.alpha_comp;
+  } else {
+    r = -q.alpha_wrong * (1.f - p);
+    if (p >= 1.f) {
+      const float ls = speedup > 0.f ? log2f(speedup) : -INFINITY;  // no usable speedup: lower bound
+      r += q.alpha_speed * fminf(fmaxf(ls, q.s_min), q.s_max);
+      r += -q.alpha_cv * cv;
+    }
+  }
+  return r + r_struct;
+}
+
+__global__ void reward_kernel(const uint8_t* compiled, const float* pass_rate, const float* speedup,
+                              const float* cv, const float* r_struct, int n, RewardParams q,
+                              float* out) {
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x)
+    out[i] = composite_reward(compiled[i], pass_rate[i], speedup[i], cv[i],
+                              r_struct ? r_struct[i] : 0.f, q);
+}
+
+// Same, four candidates per thread with 16-byte loads (all operands aligned).
+__global__ void reward_kernel_x4(const uchar4* compiled, const float4* pass_rate,
+                                 const float4* speedup, const float4* cv, const float4* r_struct,
+                                 int n4, RewardParams q, float4* out) {
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += gridDim.x * blockDim.x) {
+    const uchar4 c = compiled[i];
+    const float4 p = pass_rate[i], s = speedup[i], v = cv[i];
+    const float4 r = r_struct ? r_struct[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+    out[i] = make_float4(composite_reward(c.x, p.x, s.x, v.x, r.x, q),
+                         composite_reward(c.y, p.y, s.y, v.y, r.y, q),
+                         composite_reward(c.z, p.z, s.z, v.z, r.z, q),
+                         composite_reward(c.w, p.w, s.w, v.w, r.w, q));
   }
 }
 
@@ -426,12 +473,12 @@ cudaError_t launch_gather(const __nv_bfloat16* H, int d, const int* idx, const i
   return cudaGetLastError();
 }
 
-cudaError_t launch_lse_combine(const float4* partials, int ld_part, int nsplit, const float* ztgt,
+cudaError_t launch_lse_combine(const float4* partials, int nsplit, const float* ztgt,
                                const int* idx, const int* count, int rows_cap, float* logp,
                                float* entropy, float* lse, cudaStream_t s) {
   const int blocks = (rows_cap + 31) / 32;
-  lse_combine_kernel<<<blocks, 256, 0, s>>>(partials, ld_part, nsplit, ztgt, idx, count, logp,
-                                            entropy, lse);
+  lse_combine_kernel<<<blocks, kCombineWarps * 32, 0, s>>>(partials, nsplit, ztgt, idx, count,
+                                                           logp, entropy, lse);
   note_launches(1);
   return cudaGetLastError();
 }
@@ -453,6 +500,36 @@ cudaError_t launch_group_advantages(const float* rewards, const int* group_id, i
   group_adv_kernel<<<(n_groups + warps - 1) / warps, warps * 32, 0, s>>>(
       rewards, group_id, n_seq, n_groups, std_mode, eps, adv);
   note_launches(1);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_reward_compose(const uint8_t* compiled, const float* pass_rate,
+                                  const float* speedup, const float* cv, const float* r_struct,
+                                  int n, const RewardParams& q, float* out, cudaStream_t s) {
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  auto al = [](const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; };
+  const bool vec = al(compiled, 4) && al(pass_rate, 16) && al(speedup, 16) && al(cv, 16) &&
+                   al(out, 16) && (r_struct == nullptr || al(r_struct, 16));
+  const int n4 = vec ? n / 4 : 0;
+  if (n4 > 0) {
+    const int blocks = max(1, min((n4 + 255) / 256, sms * 16));
+    reward_kernel_x4<<<blocks, 256, 0, s>>>(
+        reinterpret_cast<const uchar4*>(compiled), reinterpret_cast<const float4*>(pass_rate),
+        reinterpret_cast<const float4*>(speedup), reinterpret_cast<const float4*>(cv),
+        reinterpret_cast<const float4*>(r_struct), n4, q, reinterpret_cast<float4*>(out));
+    note_launches(1);
+  }
+  const int done = 4 * n4;
+  if (done < n) {
+    const int rest = n - done;
+    const int blocks = max(1, min((rest + 255) / 256, sms * 8));
+    reward_kernel<<<blocks, 256, 0, s>>>(compiled + done, pass_rate + done, speedup + done,
+                                         cv + done, r_struct ? r_struct + done : nullptr, rest, q,
+                                         out + done);
+    note_launches(1);
+  }
   return cudaGetLastError();
 }
 

@@ -248,3 +248,45 @@ def large_case(seed: int = 1005, T_total: int = 131072, d: int = 5120, V: int = 
 def bf16_bits(x: torch.Tensor):
     """uint16 numpy view of a bf16 tensor (the exact bit patterns both sides consume)."""
     return x.contiguous().view(torch.int16).cpu().numpy().view("uint16")
+
+
+def ranker_case(n_programs: int = 4096, n_pairs: int = 1000, seed: int = 1006,
+                init_scale: float = 1.0) -> dict:
+    """Synthetic structural-feature vectors and ranking pairs.
+
+    The 11 features follow the appendix's definitions in range and type:
+    coalescing score (mean over two kernels of {1, 0.4, 0.1, -0.5, 0.2, 0}),
+    arithmetic-intensity proxy in [0, 1), occupancy proxy
+    {1, 0.4, -0.3}, divergence (minus a count), transfer-overhead score,
+    atomics count, syncthreads count, kernel count, threads per block,
+    global-memory access count and operation count.  Pairs (y+, y-) are random
+    row indices.  MLP parameters: uniform(+-1/sqrt(fan_in)) * init_scale,
+    packed W1, b1, W2, b2, w3, b3.
+    """
+    g = _gen(seed)
+    n = n_programs
+
+    def pick(vals, k):
+        v = torch.tensor(vals, dtype=torch.float32)
+        return v[torch.randint(0, len(vals), (k,), generator=g)]
+
+    kernels = torch.randint(1, 6, (n,), generator=g).float()
+    coal = (pick([1.0, 0.4, 0.1, -0.5, 0.2, 0.0], n) + pick([1.0, 0.4, 0.1, -0.5, 0.2, 0.0], n)) / 2
+    ai = torch.rand(n, generator=g) * 0.999             # the proxy's range [0, 1)
+    occ = pick([1.0, 0.4, -0.3], n)
+    div = -torch.randint(0, 8, (n,), generator=g).float() * 0.5
+    xfer = -torch.randint(0, 4, (n,), generator=g).float() + (torch.rand(n, generator=g) < 0.5).float()
+    atomics = torch.randint(0, 10, (n,), generator=g).float()
+    sync = torch.randint(0, 20, (n,), generator=g).float()
+    tpb = pick([32.0, 64.0, 128.0, 256.0, 512.0, 1024.0], n)
+    gmem = torch.randint(0, 200, (n,), generator=g).float()
+    ops = torch.randint(0, 2000, (n,), generator=g).float()
+    phi = torch.stack([coal, ai, occ, div, xfer, atomics, sync, kernels, tpb, gmem, ops], dim=1)
+    pos = torch.randint(0, n, (n_pairs,), generator=g, dtype=torch.int64).to(torch.int32)
+    neg = torch.randint(0, n, (n_pairs,), generator=g, dtype=torch.int64).to(torch.int32)
+    parts = []
+    for fan_in, count in ((11, 64 * 11), (11, 64), (64, 32 * 64), (64, 32), (32, 32), (32, 1)):
+        bound = init_scale / math.sqrt(fan_in)
+        parts.append((torch.rand(count, generator=g) * 2 - 1) * bound)
+    params = torch.cat(parts).float()
+    return dict(phi=phi.contiguous(), pos=pos, neg=neg, params=params, n=n, n_pairs=n_pairs)

@@ -53,11 +53,19 @@ _SIGS = {
                         ctypes.POINTER(ctypes.c_int)], ctypes.c_int),
     "spo_launch_count": ([], ctypes.c_longlong),
     "spo_set_tuning": ([ctypes.c_int, ctypes.c_int64], ctypes.c_int),
+    "spo_reward_compose": ([_vp, _vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp], ctypes.c_int),
+    "spo_ranker_scores": ([_vp, _vp, _vp, _i32, _vp, _vp, _vp], ctypes.c_int),
+    "spo_ranker_workspace_size": ([_i32, ctypes.POINTER(_c_size)], ctypes.c_int),
+    "spo_ranker_pair_loss": ([_vp, _vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp, _f32, _vp, _vp, _vp,
+                              _c_size, _vp], ctypes.c_int),
     "spo_policy_loss_fwd_noalloc": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, _i32, _vp, _i64, _f32,
                                      _f32, ctypes.c_int, _vp, _vp, _vp, _vp], ctypes.c_int),
 }
 
-TRACE_KINDS = {0: "logits_lse_fwd", 1: "logits_grad_recompute", 2: "gemm_dH", 3: "gemm_dW"}
+TRACE_KINDS = {0: "logits_lse_fwd", 1: "logits_grad_recompute", 2: "gemm_dH", 3: "gemm_dW",
+               4: "lse_combine", 5: "select_gather_fwd", 6: "select_gather_bwd",
+               7: "policy_loss_fwd", 8: "group_advantages", 9: "token_select",
+               10: "reward_compose", 11: "ranker"}
 
 
 class SpoError(RuntimeError):
@@ -316,3 +324,75 @@ SPO_TUNE_RASTER = 2
 def spo_set_tuning(key: int, value: int):
     """Host-global launch tuning (results do not depend on it)."""
     _check(lib().spo_set_tuning(int(key), int(value)))
+
+
+class RewardParams(ctypes.Structure):
+    """spo_reward_params (section 2.2 constants; the defaults are the paper's)."""
+    _fields_ = [("alpha_comp", ctypes.c_float), ("alpha_wrong", ctypes.c_float),
+                ("alpha_speed", ctypes.c_float), ("alpha_cv", ctypes.c_float),
+                ("s_min", ctypes.c_float), ("s_max", ctypes.c_float)]
+
+
+def spo_reward_compose(compiled, pass_rate, speedup, cv, r_struct=None, params=None, out=None):
+    """Composite reward r = R_ver + R_str per candidate, fp32[n]."""
+    dev = pass_rate.device
+    n = pass_rate.numel()
+    _need(compiled, "compiled", torch.uint8, n, dev)
+    _need(pass_rate, "pass_rate", torch.float32, n, dev)
+    _need(speedup, "speedup", torch.float32, n, dev)
+    _need(cv, "cv", torch.float32, n, dev)
+    if r_struct is not None:
+        _need(r_struct, "r_struct", torch.float32, n, dev)
+    out = torch.empty(n, dtype=torch.float32, device=dev) if out is None else out
+    _need(out, "rewards", torch.float32, n, dev)
+    prm = None
+    if params is not None:
+        prm = ctypes.byref(RewardParams(**params) if isinstance(params, dict) else params)
+    _check(lib().spo_reward_compose(_ptr(compiled), _ptr(pass_rate), _ptr(speedup), _ptr(cv),
+                                    _ptr(r_struct), n, prm, _ptr(out), _stream(dev)))
+    return out
+
+
+RANKER_FEATURES = 11
+RANKER_PARAMS = 2881
+
+
+def spo_ranker_scores(phi, mu, sigma, params):
+    """Structural score s_psi(phi_hat) per program, fp32[n]."""
+    dev = phi.device
+    n = phi.shape[0]
+    _need(phi, "phi", torch.float32, n * RANKER_FEATURES, dev)
+    _need(mu, "mu", torch.float32, RANKER_FEATURES, dev)
+    _need(sigma, "sigma", torch.float32, RANKER_FEATURES, dev)
+    _need(params, "params", torch.float32, RANKER_PARAMS, dev)
+    out = torch.empty(n, dtype=torch.float32, device=dev)
+    _check(lib().spo_ranker_scores(_ptr(phi), _ptr(mu), _ptr(sigma), n, _ptr(params), _ptr(out),
+                                   _stream(dev)))
+    return out
+
+
+def spo_ranker_pair_loss(phi, mu, sigma, params, pos, neg, keep1=None, keep2=None,
+                         drop_p: float = 0.0, want_grad=True, ws=None):
+    """Pairwise logistic ranking loss and its gradient: (loss fp32[1], grad fp32[2881])."""
+    dev = phi.device
+    n_pairs = pos.numel()
+    _need(phi, "phi", torch.float32, phi.shape[0] * RANKER_FEATURES, dev)
+    _need(mu, "mu", torch.float32, RANKER_FEATURES, dev)
+    _need(sigma, "sigma", torch.float32, RANKER_FEATURES, dev)
+    _need(params, "params", torch.float32, RANKER_PARAMS, dev)
+    _need(pos, "pos", torch.int32, n_pairs, dev)
+    _need(neg, "neg", torch.int32, n_pairs, dev)
+    if keep1 is not None:
+        _need(keep1, "keep1", torch.uint8, n_pairs * 2 * 64, dev)
+    if keep2 is not None:
+        _need(keep2, "keep2", torch.uint8, n_pairs * 2 * 32, dev)
+    loss = torch.empty(1, dtype=torch.float32, device=dev)
+    grad = torch.empty(RANKER_PARAMS, dtype=torch.float32, device=dev) if want_grad else None
+    n = ctypes.c_size_t(0)
+    _check(lib().spo_ranker_workspace_size(n_pairs, ctypes.byref(n)))
+    w = _workspace(n.value, dev, ws)
+    _check(lib().spo_ranker_pair_loss(_ptr(phi), _ptr(mu), _ptr(sigma), _ptr(pos), _ptr(neg),
+                                      n_pairs, _ptr(params), _ptr(keep1), _ptr(keep2),
+                                      float(drop_p), _ptr(loss), _ptr(grad), _ptr(w), w.numel(),
+                                      _stream(dev)))
+    return loss, grad
