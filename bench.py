@@ -18,8 +18,10 @@ a bounded sample of the same workload on this machine's host cores.
 
 --impl reference times the fp64 oracle itself (host cores) on bounded
 samples of the same workload and prints the same line with impl=reference.
-Under torchrun each rank runs its own batch (weak scaling, no collective on
-the data path); only the timing uses a barrier and a max over ranks.
+Under torchrun every rank owns 16 whole groups of a data-parallel batch (weak
+scaling): its loss and dL/dlogp carry weight 1/N and dW is summed across
+ranks with one NCCL all-reduce per step; the timing adds a barrier and a max
+over ranks.
 """
 
 from __future__ import annotations
@@ -186,9 +188,13 @@ class ClockSampler:
 class Step:
     """Device buffers + workspaces for one batch, driven through the C ABI."""
 
-    def __init__(self, case, dev):
+    def __init__(self, case, dev, dist=None):
         from paper_2607_20908_gb300 import spo
         self.spo = spo
+        # data parallel over whole groups: every rank owns the same number of groups, so each
+        # rank's share of Eq. 3's group average is exactly 1 / world
+        self.dist = dist if dist is not None and dist.world > 1 else None
+        self.dp_weight = 1.0 / dist.world if self.dist else 1.0
         self.L = spo.lib()
         self.dev = dev
         self.case = case
@@ -242,9 +248,15 @@ class Step:
                                   p(self.gid), self.n_seq, self.n_groups, p(self.loss_mask), self.T,
                                   c["clip_eps"], c["kl_beta"], 0, p(self.loss), p(self.g),
                                   p(self.stats), p(self.ws_l), self.ws_l.numel(), s))
+        if self.dist:
+            chk(L.spo_scale_f32(p(self.g), self.T, self.dp_weight, None, s))
+            chk(L.spo_scale_f32(p(self.loss), 1, self.dp_weight, None, s))
         chk(L.spo_policy_loss_bwd(p(self.H), p(self.W), p(self.tgt), p(self.lse), p(self.g), self.T,
                                   self.d, self.V, c["inv_temp"], p(self.dH), p(self.dW), 0,
                                   p(self.ws_b), self.ws_b.numel(), s))
+        if self.dist:   # the one real exchange of data-parallel training: sum of dW (and the loss)
+            self.dist.pg.all_reduce(self.dW)
+            self.dist.pg.all_reduce(self.loss)
 
 
 class HostIO:
@@ -254,7 +266,7 @@ class HostIO:
     (H2D and D2H each on their own stream, compute on the step's stream)."""
 
     def __init__(self, st: "Step"):
-        self.sets = [st, Step(st.case, st.dev)]
+        self.sets = [st, Step(st.case, st.dev, st.dist)]
         self.sets[1].old.copy_(st.old)
         self.sets[1].ref.copy_(st.ref)
         pinned = lambda t: torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
@@ -413,7 +425,8 @@ def config_block(case, T_L, world):
             "groups": case["n_groups"], "rollouts_per_group": 8, "tokens_per_rollout": 128,
             "clip_eps": case["clip_eps"], "kl_beta": case["kl_beta"], "window": case["window"],
             "l2": "inputs larger than L2 (W alone is 1.56 GB; each step also streams a 5 GB bf16 G buffer)",
-            "parallelism": f"{world} replica(s), independent batch per GPU" if world > 1 else "1 GPU"}
+            "parallelism": (f"dp{world}: 16 whole groups per GPU, dW and loss all-reduced (NCCL) "
+                            f"every step" if world > 1 else "1 GPU")}
 
 
 def ours(args):
@@ -426,7 +439,7 @@ def ours(args):
         build.build()
     dist.barrier()
     case = inputs.full_case(seed=1003 + dist.rank, device=str(dev))
-    st = Step(case, dev)
+    st = Step(case, dev, dist)
     st.prepare_old_ref()
     torch.cuda.synchronize(dev)
     T_L = int(st.loss_mask.sum().item())

@@ -213,6 +213,14 @@ SPO_API spo_status spo_ranker_pair_loss(const float* phi, const float* mu, const
                                         float* grad, void* ws, size_t ws_bytes, void* stream);
 
 /* ---------------------------------------------------------------------------
+ * x[i] *= alpha for i < n (alpha_dev: device fp32 scalar used instead of alpha
+ * when non-NULL).  Used by the data-parallel step to weight a rank's loss and
+ * dL/dlogp by its share of the global normaliser of Eq. 3's average.
+ * ------------------------------------------------------------------------- */
+SPO_API spo_status spo_scale_f32(float* x, int64_t n, float alpha, const float* alpha_dev,
+                                 void* stream);
+
+/* ---------------------------------------------------------------------------
  * a4. Group-normalised advantage (definition under Eq. 3):
  *   A_hat_i = (r_i - mean(r_g)) / (std(r_g) + eps), g = group_id[i].
  * Members of a group are taken in ascending i; the arithmetic is IEEE fp32

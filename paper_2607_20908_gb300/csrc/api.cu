@@ -452,6 +452,17 @@ SPO_API spo_status spo_ranker_pair_loss(const float* phi, const float* mu, const
   return st == SPO_OK ? ok() : st;
 }
 
+SPO_API spo_status spo_scale_f32(float* x, int64_t n, float alpha, const float* alpha_dev,
+                                 void* stream) {
+  if (!x) return fail(SPO_ERR_INVALID_ARG, "x must be non-NULL");
+  if (n < 0 || n > (1ll << 40)) return fail(SPO_ERR_SHAPE, "n = %lld out of range", (long long)n);
+  if (!alpha_dev && !isfinite(alpha)) return fail(SPO_ERR_INVALID_ARG, "alpha must be finite");
+  if (n == 0) return ok();
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  SPO_CUDA(spo::launch_scale(x, n, alpha, alpha_dev, s), "scale launch");
+  return ok();
+}
+
 SPO_API spo_status spo_group_advantages(const float* rewards, const int32_t* group_id,
                                         int32_t n_seq, int32_t n_groups, int std_mode, float eps,
                                         float* adv, void* stream) {

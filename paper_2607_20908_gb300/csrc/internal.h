@@ -133,6 +133,9 @@ cudaError_t launch_ranker_pair_loss(const float* phi, const float* mu, const flo
                                     const uint8_t* keep2, float drop_p, float* loss, float* grad,
                                     float* ws, cudaStream_t s);
 
+// x[i] *= alpha (alpha read from device memory when alpha_dev != NULL).
+cudaError_t launch_scale(float* x, long long n, float alpha, const float* alpha_dev, cudaStream_t s);
+
 struct LossWs {
   int* gsize;        // [n_groups]
   int* n_tok;        // [n_seq]

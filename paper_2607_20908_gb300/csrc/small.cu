@@ -303,6 +303,13 @@ __global__ void reward_kernel_x4(const uchar4* compiled, const float4* pass_rate
   }
 }
 
+__global__ void scale_kernel(float* x, long long n, float alpha, const float* alpha_dev) {
+  const float a = alpha_dev ? *alpha_dev : alpha;
+  for (long long i = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; i < n;
+       i += static_cast<long long>(gridDim.x) * blockDim.x)
+    x[i] *= a;
+}
+
 // ---------------------------------------------------------------- policy loss
 constexpr int kLossThreads = 256;
 
@@ -530,6 +537,17 @@ cudaError_t launch_reward_compose(const uint8_t* compiled, const float* pass_rat
                                          out + done);
     note_launches(1);
   }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_scale(float* x, long long n, float alpha, const float* alpha_dev, cudaStream_t s) {
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const long long want = (n + 255) / 256;
+  const int blocks = static_cast<int>(want < sms * 8 ? (want < 1 ? 1 : want) : sms * 8);
+  scale_kernel<<<blocks, 256, 0, s>>>(x, n, alpha, alpha_dev);
+  note_launches(1);
   return cudaGetLastError();
 }
 

@@ -1,0 +1,150 @@
+"""Data-parallel form of the GRPO step: whole groups per rank.
+
+Groups (the g candidates of one task and all their turns, section 3) are
+independent for the advantages and for every per-token term of Eq. 3, so a
+batch shards over ranks by whole groups with no exchange inside the step.
+Two things cross ranks:
+
+  * the normaliser of Eq. 3's average.  With SEQ_GROUP aggregation the loss
+    is a mean over non-empty groups, so rank r's local loss (a mean over its
+    own N_r groups) enters the global loss with weight N_r / N; with TOKEN
+    aggregation the weight is the rank's share of loss tokens.  One
+    all-reduce of two counts per step gives N (and the token total).
+  * dW = sum over ranks of the weighted local dW (an all-reduce of V x d
+    fp32).  dH rows stay on the rank that owns the tokens.
+
+The per-rank compute is an engine object (``SpoEngine`` runs libspo's CUDA
+kernels); the collectives are ``torch.distributed`` on whatever backend the
+process group uses (NCCL between GPUs).
+"""
+
+from __future__ import annotations
+
+from dataclasses import dataclass
+
+import numpy as np
+import torch
+
+AGG_SEQ_GROUP = 0
+AGG_TOKEN = 1
+
+
+def shard_groups(tokens_per_group, world: int):
+    """Assign every group to one rank, balancing loss tokens (greedy, largest
+    first, ties to the lowest rank; deterministic).  Returns sorted group ids
+    per rank."""
+    if world < 1:
+        raise ValueError("world must be >= 1")
+    tokens = [int(t) for t in tokens_per_group]
+    order = sorted(range(len(tokens)), key=lambda g: (-tokens[g], g))
+    loads = [0] * world
+    out = [[] for _ in range(world)]
+    for g in order:
+        r = min(range(world), key=lambda k: (loads[k], k))
+        out[r].append(g)
+        loads[r] += tokens[g]
+    return [sorted(x) for x in out]
+
+
+@dataclass
+class RankBatch:
+    seq_index: np.ndarray     # global sequence ids owned by the rank, ascending
+    token_index: np.ndarray   # global token ids of those sequences, in order
+    cu_seqlens: np.ndarray    # local int32 [n_seq + 1]
+    group_id: np.ndarray      # local int32 [n_seq], remapped to 0..n_groups-1
+    n_groups: int             # groups owned (each has >= 1 sequence)
+
+
+def rank_batch(cu_seqlens, group_id, groups) -> RankBatch:
+    """The sequences and tokens of the given groups, in their global order."""
+    cu = np.asarray(cu_seqlens).astype(np.int64)
+    gid = np.asarray(group_id).astype(np.int64)
+    remap = {int(g): k for k, g in enumerate(sorted(int(x) for x in groups))}
+    seqs = np.array([i for i in range(gid.size) if int(gid[i]) in remap], dtype=np.int64)
+    lens = np.array([cu[i + 1] - cu[i] for i in seqs], dtype=np.int64)
+    tok = (np.concatenate([np.arange(cu[i], cu[i + 1]) for i in seqs]) if seqs.size
+           else np.zeros(0, dtype=np.int64))
+    local_cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    local_gid = np.array([remap[int(gid[i])] for i in seqs], dtype=np.int32)
+    return RankBatch(seqs, tok, local_cu, local_gid, len(remap))
+
+
+def loss_weight(agg: int, local_groups: float, global_groups: float, local_tokens: float,
+                global_tokens: float) -> float:
+    """Weight of a rank's local loss (and dL/dlogp) in the global objective."""
+    if agg == AGG_SEQ_GROUP:
+        return local_groups / global_groups if global_groups > 0 else 0.0
+    return local_tokens / global_tokens if global_tokens > 0 else 0.0
+
+
+class SpoEngine:
+    """libspo (CUDA) as the per-rank compute of a data-parallel step."""
+
+    def __init__(self):
+        from paper_2607_20908_gb300 import spo
+        self.spo = spo
+
+    def step_local(self, b: dict, agg: int):
+        s = self.spo
+        lm, _ = s.spo_token_select(b["cu_seqlens"], b["mask"], b["tgt"], b["window"])
+        logp, _, lse = s.spo_logprobs_fwd(b["H"], b["W"], b["tgt"], lm, b["inv_temp"])
+        adv = s.spo_group_advantages(b["rewards"], b["group_id"], b["n_groups"])
+        loss, g, stats = s.spo_policy_loss_fwd(logp, b["old"], b["ref"], adv, b["cu_seqlens"],
+                                               b["group_id"], b["n_groups"], lm, b["clip_eps"],
+                                               b["kl_beta"], agg)
+        return dict(loss=loss, g=g, lse=lse, n_loss_tokens=stats[3:4].to(torch.float64))
+
+    def scale(self, x, w: float):
+        self.spo.spo_scale_f32(x, alpha=w)
+        return x
+
+    def backward(self, b: dict, lse, g):
+        return self.spo.spo_policy_loss_bwd(b["H"], b["W"], b["tgt"], lse, g, b["inv_temp"])
+
+    def zeros_dW(self, V: int, d: int, like):
+        return torch.zeros((V, d), dtype=torch.float32, device=like.device)
+
+
+class DataParallelStep:
+    """One GRPO step over a process group, whole groups per rank.
+
+    run(b) takes this rank's batch (dict with H, W, tgt, mask, cu_seqlens,
+    group_id, n_groups, rewards, old, ref, window, inv_temp, clip_eps,
+    kl_beta; n_groups may be 0) and returns (global loss, local dH, global dW).
+    Collectives: one all-reduce of [groups, loss tokens], one of the loss,
+    one of dW.
+    """
+
+    def __init__(self, engine, agg: int = AGG_SEQ_GROUP, process_group=None):
+        self.engine = engine
+        self.agg = agg
+        self.pg = process_group
+
+    def run(self, b: dict):
+        import torch.distributed as dist
+        e = self.engine
+        V, d = b["W"].shape
+        if b["n_groups"] > 0:
+            loc = e.step_local(b, self.agg)
+            counts = torch.cat([torch.tensor([float(b["n_groups"])], dtype=torch.float64,
+                                             device=loc["n_loss_tokens"].device),
+                                loc["n_loss_tokens"].reshape(1)])
+        else:
+            loc = None
+            counts = torch.zeros(2, dtype=torch.float64, device=b["W"].device)
+        local = counts.clone()
+        dist.all_reduce(counts, group=self.pg)
+        w = loss_weight(self.agg, float(local[0]), float(counts[0]), float(local[1]),
+                        float(counts[1]))
+        if loc is not None:
+            e.scale(loc["g"], w)
+            e.scale(loc["loss"], w)
+            dH, dW = e.backward(b, loc["lse"], loc["g"])
+            loss = loc["loss"]
+        else:
+            dH = None
+            dW = e.zeros_dW(V, d, b["W"])
+            loss = torch.zeros(1, dtype=dW.dtype, device=dW.device)
+        dist.all_reduce(loss, group=self.pg)
+        dist.all_reduce(dW, group=self.pg)
+        return loss, dH, dW

@@ -55,6 +55,7 @@ _SIGS = {
     "spo_set_tuning": ([ctypes.c_int, ctypes.c_int64], ctypes.c_int),
     "spo_reward_compose": ([_vp, _vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp], ctypes.c_int),
     "spo_ranker_scores": ([_vp, _vp, _vp, _i32, _vp, _vp, _vp], ctypes.c_int),
+    "spo_scale_f32": ([_vp, _i64, _f32, _vp, _vp], ctypes.c_int),
     "spo_ranker_workspace_size": ([_i32, ctypes.POINTER(_c_size)], ctypes.c_int),
     "spo_ranker_pair_loss": ([_vp, _vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp, _f32, _vp, _vp, _vp,
                               _c_size, _vp], ctypes.c_int),
@@ -396,3 +397,13 @@ def spo_ranker_pair_loss(phi, mu, sigma, params, pos, neg, keep1=None, keep2=Non
                                       float(drop_p), _ptr(loss), _ptr(grad), _ptr(w), w.numel(),
                                       _stream(dev)))
     return loss, grad
+
+
+def spo_scale_f32(x, alpha=None, alpha_dev=None):
+    """In place x *= alpha (host float) or x *= alpha_dev[0] (device fp32 scalar)."""
+    _need(x, "x", torch.float32, device=x.device)
+    if alpha_dev is not None:
+        _need(alpha_dev, "alpha_dev", torch.float32, 1, x.device)
+    _check(lib().spo_scale_f32(_ptr(x), x.numel(), float(alpha if alpha is not None else 1.0),
+                               _ptr(alpha_dev), _stream(x.device)))
+    return x
