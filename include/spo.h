@@ -351,11 +351,15 @@ SPO_API spo_status spo_policy_loss_fwd_noalloc(const float* logp, const float* o
  *     persistent raster (L2 reuse of the streamed operand).
  *   SPO_TUNE_RASTER (default 0): 0 = groups of tile rows, 1 = groups of tile
  *     columns.
+ *   SPO_TUNE_DYNAMIC_MASK (default 15): bit k set = GEMM kind k (trace kinds
+ *     0-3) takes its tiles in raster order from an atomic counter instead of
+ *     a static round robin, so in-flight tiles stay a contiguous window.
  * Results do not depend on any setting. */
 typedef enum spo_tune_key {
     SPO_TUNE_PAIR_MMA = 0,
     SPO_TUNE_GROUP_M = 1,
-    SPO_TUNE_RASTER = 2
+    SPO_TUNE_RASTER = 2,
+    SPO_TUNE_DYNAMIC_MASK = 3
 } spo_tune_key;
 SPO_API spo_status spo_set_tuning(int key, int64_t value);
 

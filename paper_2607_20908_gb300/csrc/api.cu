@@ -96,6 +96,7 @@ spo_status check_hwv(const void* H, const void* W, const int32_t* tgt, int64_t T
 struct FwdWs {
   int* idx;
   int* count;
+  int* counters;  // tile counter of the dynamic schedule
   int* scratch;
   int* tgt_c;
   float* ztgt;
@@ -120,6 +121,7 @@ FwdWs carve_fwd(void* base, long long T, long long d, long long V) {
   };
   w.idx = reinterpret_cast<int*>(take(sizeof(int) * w.T_pad));
   w.count = reinterpret_cast<int*>(take(sizeof(int)));
+  w.counters = reinterpret_cast<int*>(take(sizeof(int) * 4));
   w.scratch = reinterpret_cast<int*>(take(sizeof(int) * 2 * nb));
   w.tgt_c = reinterpret_cast<int*>(take(sizeof(int) * w.T_pad));
   w.ztgt = reinterpret_cast<float*>(take(sizeof(float) * w.T_pad));
@@ -134,6 +136,7 @@ constexpr long long kBwdChunkRows = 32768;  // G scratch rows per chunk (multipl
 struct BwdWs {
   int* idx;
   int* count;
+  int* counters;  // tile counters of the dynamic schedule, one per GEMM kind
   int* scratch;
   int* tgt_c;
   float* lse_c;
@@ -159,6 +162,7 @@ BwdWs carve_bwd(void* base, long long T, long long d, long long V) {
   };
   w.idx = reinterpret_cast<int*>(take(sizeof(int) * w.T_pad));
   w.count = reinterpret_cast<int*>(take(sizeof(int)));
+  w.counters = reinterpret_cast<int*>(take(sizeof(int) * 4));
   w.scratch = reinterpret_cast<int*>(take(sizeof(int) * 2 * nb));
   w.tgt_c = reinterpret_cast<int*>(take(sizeof(int) * w.T_pad));
   w.lse_c = reinterpret_cast<float*>(take(sizeof(float) * w.T_pad));
@@ -175,6 +179,10 @@ BwdWs carve_bwd(void* base, long long T, long long d, long long V) {
 int g_tune_pair = 1;
 int g_tune_group_m = 16;
 int g_tune_raster = 0;
+// Bit k set: GEMM kind k takes its tiles from an atomic counter (dynamic
+// schedule) instead of the static round robin, so the tiles in flight stay a
+// contiguous window of the raster however the CTA pairs drift.  Default: all.
+int g_tune_dynamic_mask = 0xF;
 
 // ------------------------------------------------------------ tracing
 // When enabled, a start/stop CUDA event pair is recorded on the launch stream
@@ -239,8 +247,16 @@ enum TraceKind : int {
   kTraceRanker = 11,
 };
 
+// counters: the workspace's four tile counters (the one of this kind is
+// zeroed on the stream and used when the kind's dynamic-schedule bit is set).
 spo_status traced_gemm(int kind, bool a_mn, bool b_mn, const CUtensorMap& ta, const CUtensorMap& tb,
-                       const spo::GemmArgs& args, int grid, cudaStream_t s) {
+                       const spo::GemmArgs& args_in, int grid, cudaStream_t s, int* counters) {
+  spo::GemmArgs args = args_in;
+  args.tile_counter = nullptr;
+  if (counters && ((g_tune_dynamic_mask >> kind) & 1)) {
+    args.tile_counter = counters + kind;
+    SPO_CUDA(cudaMemsetAsync(args.tile_counter, 0, sizeof(int), s), "memset tile counter");
+  }
   return traced(kind, s, "gemm launch", [&] {
     return spo::launch_gemm(kind, a_mn, b_mn, g_tune_pair != 0, ta, tb, args, grid, s);
   });
@@ -374,7 +390,8 @@ SPO_API spo_status spo_logprobs_fwd(const void* H, const void* W, const int32_t*
   a.partials = w.partials;
   a.nsplit = w.nsplit;
   a.ztgt = w.ztgt;
-  if ((st = traced_gemm(spo::EPI_LSE, false, false, ta, tb, a, grid_for(di, w.T_pad, V), s)) !=
+  if ((st = traced_gemm(spo::EPI_LSE, false, false, ta, tb, a, grid_for(di, w.T_pad, V), s,
+                        w.counters)) !=
       SPO_OK)
     return st;
   // a3: split-vocab combine, scattered back to token positions (skipped tokens read 0)
@@ -585,7 +602,8 @@ SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32
     a.gvec = w.g_c + r0;
     a.G = w.G;
     a.ldG = V;
-    if ((st = traced_gemm(spo::EPI_GRAD, false, false, tH_k, tW_k, a, grid_for(di, rows, V), s)) != SPO_OK)
+    if ((st = traced_gemm(spo::EPI_GRAD, false, false, tH_k, tW_k, a, grid_for(di, rows, V), s,
+                          w.counters)) != SPO_OK)
       return st;
     // a7: dH rows = G W, scattered to token rows
     if (dH) {
@@ -598,7 +616,8 @@ SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32
       b.row_idx = w.idx + r0;
       b.out_bf16 = static_cast<__nv_bfloat16*>(dH);
       b.ld_out = d;
-      if ((st = traced_gemm(spo::EPI_DH, false, true, tG_k, tW_mn, b, grid_for(di, rows, d), s)) != SPO_OK)
+      if ((st = traced_gemm(spo::EPI_DH, false, true, tG_k, tW_mn, b, grid_for(di, rows, d), s,
+                            w.counters)) != SPO_OK)
         return st;
     }
     // a8: dW (+)= G^T Hc over this chunk's rows
@@ -612,7 +631,8 @@ SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32
       b.out_f32 = dW;
       b.ld_out = d;
       b.accumulate = (c == 0) ? (accumulate_dW ? 1 : 0) : 1;
-      if ((st = traced_gemm(spo::EPI_DW, true, true, tG_mn, tH_mn, b, grid_for(di, V, d), s)) !=
+      if ((st = traced_gemm(spo::EPI_DW, true, true, tG_mn, tH_mn, b, grid_for(di, V, d), s,
+                            w.counters)) !=
           SPO_OK)
         return st;
     }
@@ -666,6 +686,10 @@ SPO_API spo_status spo_set_tuning(int key, int64_t value) {
     case SPO_TUNE_GROUP_M:
       if (value < 1 || value > 4096) return fail(SPO_ERR_INVALID_ARG, "group_m must be in [1, 4096]");
       g_tune_group_m = static_cast<int>(value);
+      return ok();
+    case SPO_TUNE_DYNAMIC_MASK:
+      if (value < 0 || value > 15) return fail(SPO_ERR_INVALID_ARG, "dynamic mask must be in [0, 15]");
+      g_tune_dynamic_mask = static_cast<int>(value);
       return ok();
     case SPO_TUNE_RASTER:
       if (value != 0 && value != 1) return fail(SPO_ERR_INVALID_ARG, "raster must be 0 or 1");

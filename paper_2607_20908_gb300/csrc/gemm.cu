@@ -222,7 +222,7 @@ struct Geo {
   static constexpr uint32_t kStageBytes = kABytes + kBBytes;
   static constexpr int kTileM = PAIR ? 2 * BM : BM;         // output rows per tile
   static constexpr uint32_t kTxBytes = PAIR ? 2 * kStageBytes : kStageBytes;  // per full barrier
-  static constexpr size_t kSmem = 1024 + kStages * kStageBytes + 256;
+  static constexpr size_t kSmem = 1024 + kStages * kStageBytes + 512;
 };
 
 template <int EPI, bool A_MN, bool B_MN, bool PAIR>
@@ -241,8 +241,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   uint64_t* tfull_bar = empty_bar + S;
   uint64_t* tempty_bar = tfull_bar + 2;
   uint64_t* drain_bar = tempty_bar + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
+  // Dynamic tile schedule: the leader's producer takes tile ids from a global
+  // counter and publishes them through a ring of kRing slots to every other
+  // role (the peer CTA's through its own copy of the ring).
+  constexpr int kRing = 8;
+  uint64_t* ring_full = drain_bar + 1;
+  uint64_t* ring_empty = ring_full + kRing;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(ring_empty + kRing);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  volatile int* ring = reinterpret_cast<volatile int*>(tmem_slot + 2);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -270,6 +277,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       mbar_init(&tempty_bar[a], PAIR ? 8 : 4);  // one arrival per epilogue warp of the pair
     }
     mbar_init(drain_bar, 1);
+    for (int r = 0; r < kRing; ++r) {
+      mbar_init(&ring_full[r], 1);
+      // consumers: MMA + 4 epilogue warps (+ the peer's producer and 4 epilogue warps)
+      mbar_init(&ring_empty[r], PAIR ? 10 : 5);
+    }
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -288,6 +300,42 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  const bool dyn = p.tile_counter != nullptr;
+
+  // i-th tile of this CTA (pair) or -1 when done.  Static: unit + i * n_units.
+  auto static_tile = [&](int i) { const int t = unit + i * n_units; return t < num_tiles ? t : -1; };
+  // Leader producer: take the next tile id and publish it in slot i % kRing.
+  auto publish = [&](int i, bool& ok) -> int {
+    const int slot = i % kRing;
+    if (!mbar_wait(&ring_empty[slot], ((i / kRing) & 1) ^ 1u, abort_flag, p.err, kErrWaitProducer,
+                   PAIR)) {
+      ok = false;
+      return -1;
+    }
+    int t = atomicAdd(p.tile_counter, 1);
+    if (t >= num_tiles) t = -1;
+    ring[slot] = t;
+    if (PAIR) {
+      st_shared_cluster(mapa_shared(smem_u32(const_cast<int*>(&ring[slot])), 1), t);
+      mbar_arrive_cluster(mapa_shared(smem_u32(&ring_full[slot]), 1));  // release: orders the store
+    }
+    mbar_arrive(&ring_full[slot]);
+    return t;
+  };
+  // Any other role (one thread): read slot i % kRing and hand it back.
+  auto take = [&](int i, bool& ok, int code) -> int {
+    const int slot = i % kRing;
+    if (!mbar_wait(&ring_full[slot], (i / kRing) & 1, abort_flag, p.err, code, PAIR)) {
+      ok = false;
+      return -1;
+    }
+    const int t = ring[slot];
+    if (PAIR)
+      mbar_arrive_cluster(mapa_shared(smem_u32(&ring_empty[slot]), 0));  // leader's barrier
+    else
+      mbar_arrive(&ring_empty[slot]);
+    return t;
+  };
 
   if (warp == 0) {
     // ------------------------------------------------ TMA producer (both CTAs)
@@ -296,7 +344,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       uint32_t phase = 0;
       int issued = 0;
       bool ok = true;
-      for (int tile = unit; tile < num_tiles && ok; tile += n_units) {
+      for (int i = 0; ok; ++i) {
+        const int tile = !dyn ? static_tile(i)
+                              : (rank == 0 ? publish(i, ok) : take(i, ok, kErrWaitProducer));
+        if (tile < 0) break;
         int mb, nb;
         tile_coords(tile, mt, nt, gm, p.raster, mb, nb);
         const int a_row = mb * G::kTileM + static_cast<int>(rank) * BM;
@@ -355,9 +406,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       constexpr uint32_t kIdesc = idesc_bf16_f32(G::kTileM, BN, A_MN, B_MN);
       int stage = 0;
       uint32_t phase = 0;
-      int local = 0;
       bool ok = true;
-      for (int tile = unit; tile < num_tiles; tile += n_units, ++local) {
+      for (int local = 0;; ++local) {
+        const int tile = dyn ? take(local, ok, kErrWaitMma) : static_tile(local);
+        if (tile < 0) break;
         const int acc = local & 1;
         const uint32_t acc_phase = (local >> 1) & 1;
         if (!mbar_wait(&tempty_bar[acc], acc_phase ^ 1u, abort_flag, p.err, kErrWaitMma)) {
@@ -403,8 +455,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   } else {
     // ------------------------------------------------ epilogue warps 2..5 (both CTAs)
     const int q = warp & 3;  // TMEM lanes [32q, 32q+32) are reachable from this warp
-    int local = 0;
-    for (int tile = unit; tile < num_tiles; tile += n_units, ++local) {
+    for (int local = 0;; ++local) {
+      int tile;
+      if (dyn) {
+        bool got = true;
+        int t = -1;
+        if (lane == 0) t = take(local, got, kErrWaitEpilogue);
+        tile = __shfl_sync(0xffffffffu, got ? t : -1, 0);
+      } else {
+        tile = static_tile(local);
+      }
+      if (tile < 0) break;
       const int acc = local & 1;
       const uint32_t acc_phase = (local >> 1) & 1;
       int mb, nb;

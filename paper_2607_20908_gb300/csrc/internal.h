@@ -41,6 +41,7 @@ struct GemmArgs {
   int k_cap;
   int group_m;  // tile rows (raster 0) or columns (raster 1) walked together
   int raster;   // 0: groups of tile rows, 1: groups of tile columns
+  int* tile_counter;  // zeroed int: tiles are taken in raster order from it; NULL = static
   float scale;  // inv_temp for EPI_LSE / EPI_GRAD
   // EPI_LSE
   const int* tgt;     // target id of each row

@@ -6,9 +6,9 @@ sweeps.
     python -m paper_2607_20908_gb300.profile_case --V 151936 --iters 1 \\
         --configs "1,16,0;1,8,0;0,16,0"
 
---configs is a ';'-separated list of "pair,group,raster" launch tunings
-(spo_set_tuning); each is run for --iters iterations of fwd + bwd.  The
-default reduced size keeps the reduction lengths of the full workload
+--configs is a ';'-separated list of "pair,group,raster[,dynamic_mask]"
+launch tunings (spo_set_tuning); each is run for --iters iterations of
+fwd + bwd.  The default reduced size keeps the reduction lengths of the full workload
 (K = d = 5120 for the logits and their recompute, K = T = 16384 tokens for
 dW) with a vocabulary cut to 8192, so one launch takes about a millisecond
 and the device holds about 1 GB; the streamed operands of dW (G = 268 MB,
@@ -50,18 +50,22 @@ def main():
     configs = [tuple(int(x) for x in c.split(",")) for c in a.configs.split(";") if c] or [None]
     for cfg in configs:
         if cfg is not None:
-            pair, group, raster = cfg
+            pair, group, raster = cfg[:3]
             spo.spo_set_tuning(spo.SPO_TUNE_PAIR_MMA, pair)
             spo.spo_set_tuning(spo.SPO_TUNE_GROUP_M, group)
             spo.spo_set_tuning(spo.SPO_TUNE_RASTER, raster)
+            if len(cfg) > 3:
+                spo.spo_set_tuning(spo.SPO_TUNE_DYNAMIC_MASK, cfg[3])
         for i in range(a.iters):
             spo.spo_trace_enable(i == a.iters - 1)
             _, _, lse = spo.spo_logprobs_fwd(H, W, tgt, ws=ws_f)
             spo.spo_policy_loss_bwd(H, W, tgt, lse, gl, dH=dH, dW=dW, ws=ws_b)
         torch.cuda.synchronize()
-        label = "default" if cfg is None else f"pair={cfg[0]} group={cfg[1]} raster={cfg[2]}"
+        label = "default" if cfg is None else "pair,group,raster,dynamic=" + ",".join(map(str, cfg))
         print(f"--- {label}")
         for kind, ms in spo.spo_trace_read():
+            if kind > 3:
+                continue
             tflops = 2.0 * a.T * a.d * a.V / ms / 1e9
             print(f"{spo.TRACE_KINDS[kind]:24s} {ms:8.3f} ms  {tflops:8.1f} TFLOP/s")
     assert spo.spo_device_error() == 0

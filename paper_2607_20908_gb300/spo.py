@@ -320,6 +320,7 @@ def spo_policy_loss_fwd_noalloc(logp, old_logp, ref_logp, adv, cu_seqlens, group
 SPO_TUNE_PAIR_MMA = 0
 SPO_TUNE_GROUP_M = 1
 SPO_TUNE_RASTER = 2
+SPO_TUNE_DYNAMIC_MASK = 3
 
 
 def spo_set_tuning(key: int, value: int):

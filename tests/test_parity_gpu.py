@@ -145,3 +145,20 @@ def test_single_cta_mode_matches_oracle():
     finally:
         spo.spo_set_tuning(spo.SPO_TUNE_PAIR_MMA, 1)
         spo.spo_set_tuning(spo.SPO_TUNE_GROUP_M, 16)
+
+
+@pytest.mark.parametrize("mask", [0, 15])
+def test_static_and_dynamic_tile_schedules(mask):
+    """Every GEMM on the static round robin (mask 0) or on the atomic-counter
+    schedule (mask 15), with a small raster group so tiles of several groups
+    are in flight at once."""
+    from paper_2607_20908_gb300 import spo
+    spo.spo_set_tuning(spo.SPO_TUNE_DYNAMIC_MASK, mask)
+    spo.spo_set_tuning(spo.SPO_TUNE_GROUP_M, 2)
+    try:
+        _compare(inputs.tiny_case(seed=1081))
+        case = inputs.tiny_case(seed=1082, T_per_seq=125, n_groups=2, rollouts=4, d=320, V=5000)
+        _compare(case)
+    finally:
+        spo.spo_set_tuning(spo.SPO_TUNE_DYNAMIC_MASK, 15)
+        spo.spo_set_tuning(spo.SPO_TUNE_GROUP_M, 16)
