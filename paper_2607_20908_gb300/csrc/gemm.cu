@@ -212,10 +212,14 @@ __device__ __forceinline__ void epi_dw(const GemmArgs& p, uint32_t taddr, int ro
 // Stage geometry.  Solo: one CTA stages A (128 x 64) and B (256 x 64).  Pair:
 // the two CTAs of a cluster compute one 256 x 256 tile with a shared
 // cta_group::2 MMA; each stages its own 128 rows of A and 128 of the 256 B
-// rows, so a stage is 32 KB and six fit in shared memory.
+// rows, so a stage is 32 KB and seven fit in shared memory (~2 us of MMA
+// work buffered against operand latency).
+#ifndef SPO_PAIR_STAGES
+#define SPO_PAIR_STAGES 7
+#endif
 template <bool PAIR>
 struct Geo {
-  static constexpr int kStages = PAIR ? 6 : 4;
+  static constexpr int kStages = PAIR ? SPO_PAIR_STAGES : 4;
   static constexpr int kBRows = PAIR ? BN / 2 : BN;        // B rows staged per CTA
   static constexpr uint32_t kABytes = BM * BK * 2;         // 16 KB
   static constexpr uint32_t kBBytes = kBRows * BK * 2;     // 16 or 32 KB
