@@ -213,6 +213,25 @@ SPO_API spo_status spo_ranker_pair_loss(const float* phi, const float* mu, const
                                         float* grad, void* ws, size_t ws_bytes, void* stream);
 
 /* ---------------------------------------------------------------------------
+ * Content checks of device inputs that the other calls take on trust (the
+ * host cannot read device data without a synchronisation).  Enqueues one
+ * pass and writes counts (DEVICE int32[6], zeroed first) of:
+ *   [0] tokens with tgt[t] >= V (tgt < 0 is the valid "ignore" marker)
+ *   [1] violations of cu_seqlens: decreasing steps, cu[0] != 0, cu[n_seq] != T
+ *   [2] group ids outside [0, n_groups)
+ *   [3] non-finite rewards
+ *   [4] non-finite old / reference log-probs
+ *   [5] mask bytes other than 0 and 1
+ * Every array pointer may be NULL to skip its checks.  All zero = valid.
+ * ------------------------------------------------------------------------- */
+SPO_API spo_status spo_validate_inputs(const int32_t* tgt, int64_t T, int64_t V,
+                                       const int32_t* cu_seqlens, int32_t n_seq,
+                                       const int32_t* group_id, int32_t n_groups,
+                                       const float* rewards, const float* old_logp,
+                                       const float* ref_logp, const uint8_t* mask,
+                                       int32_t* counts, void* stream);
+
+/* ---------------------------------------------------------------------------
  * x[i] *= alpha for i < n (alpha_dev: device fp32 scalar used instead of alpha
  * when non-NULL).  Used by the data-parallel step to weight a rank's loss and
  * dL/dlogp by its share of the global normaliser of Eq. 3's average.

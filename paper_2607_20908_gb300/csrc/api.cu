@@ -480,6 +480,23 @@ SPO_API spo_status spo_scale_f32(float* x, int64_t n, float alpha, const float* 
   return ok();
 }
 
+SPO_API spo_status spo_validate_inputs(const int32_t* tgt, int64_t T, int64_t V,
+                                       const int32_t* cu_seqlens, int32_t n_seq,
+                                       const int32_t* group_id, int32_t n_groups,
+                                       const float* rewards, const float* old_logp,
+                                       const float* ref_logp, const uint8_t* mask,
+                                       int32_t* counts, void* stream) {
+  if (!counts) return fail(SPO_ERR_INVALID_ARG, "counts must be non-NULL");
+  if (T < 0 || V < 0 || n_seq < 0 || n_groups < 0) return fail(SPO_ERR_SHAPE, "sizes must be >= 0");
+  if ((cu_seqlens || group_id || rewards) && n_seq < 1)
+    return fail(SPO_ERR_SHAPE, "n_seq must be >= 1 when per-sequence arrays are given");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  SPO_CUDA(spo::launch_validate(tgt, T, V, cu_seqlens, n_seq, group_id, n_groups, rewards, old_logp,
+                                ref_logp, mask, counts, s),
+           "validate launch");
+  return ok();
+}
+
 SPO_API spo_status spo_group_advantages(const float* rewards, const int32_t* group_id,
                                         int32_t n_seq, int32_t n_groups, int std_mode, float eps,
                                         float* adv, void* stream) {

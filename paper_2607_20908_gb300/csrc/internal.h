@@ -137,6 +137,11 @@ cudaError_t launch_ranker_pair_loss(const float* phi, const float* mu, const flo
 // x[i] *= alpha (alpha read from device memory when alpha_dev != NULL).
 cudaError_t launch_scale(float* x, long long n, float alpha, const float* alpha_dev, cudaStream_t s);
 
+// Counts of invalid device inputs into counts[6] (zeroed here first); see spo_validate_inputs.
+cudaError_t launch_validate(const int* tgt, long long T, long long V, const int* cu, int n_seq,
+                            const int* gid, int n_groups, const float* rewards, const float* old_logp,
+                            const float* ref_logp, const uint8_t* mask, int* counts, cudaStream_t s);
+
 struct LossWs {
   int* gsize;        // [n_groups]
   int* n_tok;        // [n_seq]

@@ -310,6 +310,31 @@ __global__ void scale_kernel(float* x, long long n, float alpha, const float* al
     x[i] *= a;
 }
 
+// Input validation: one grid-stride pass, integer atomics (counts are exact).
+__global__ void validate_kernel(const int* tgt, long long T, long long V, const int* cu, int n_seq,
+                                const int* gid, int n_groups, const float* rewards,
+                                const float* old_logp, const float* ref_logp, const uint8_t* mask,
+                                int* counts) {
+  int c[6] = {0, 0, 0, 0, 0, 0};
+  const long long stride = static_cast<long long>(gridDim.x) * blockDim.x;
+  const long long i0 = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x;
+  for (long long t = i0; t < T; t += stride) {
+    if (tgt && tgt[t] >= V) ++c[0];
+    if (old_logp && !isfinite(old_logp[t])) ++c[4];
+    if (ref_logp && !isfinite(ref_logp[t])) ++c[4];
+    if (mask && mask[t] > 1) ++c[5];
+  }
+  for (long long i = i0; i < n_seq; i += stride) {
+    if (cu && cu[i + 1] < cu[i]) ++c[1];
+    if (gid && (gid[i] < 0 || gid[i] >= n_groups)) ++c[2];
+    if (rewards && !isfinite(rewards[i])) ++c[3];
+  }
+  if (i0 == 0 && cu) c[1] += (cu[0] != 0) + (cu[n_seq] != T);
+#pragma unroll
+  for (int k = 0; k < 6; ++k)
+    if (c[k]) atomicAdd(&counts[k], c[k]);
+}
+
 // ---------------------------------------------------------------- policy loss
 constexpr int kLossThreads = 256;
 
@@ -547,6 +572,23 @@ cudaError_t launch_scale(float* x, long long n, float alpha, const float* alpha_
   const long long want = (n + 255) / 256;
   const int blocks = static_cast<int>(want < sms * 8 ? (want < 1 ? 1 : want) : sms * 8);
   scale_kernel<<<blocks, 256, 0, s>>>(x, n, alpha, alpha_dev);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_validate(const int* tgt, long long T, long long V, const int* cu, int n_seq,
+                            const int* gid, int n_groups, const float* rewards, const float* old_logp,
+                            const float* ref_logp, const uint8_t* mask, int* counts, cudaStream_t s) {
+  cudaError_t e = cudaMemsetAsync(counts, 0, 6 * sizeof(int), s);
+  if (e != cudaSuccess) return e;
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const long long n = T > n_seq ? T : n_seq;
+  const long long want = (n + 255) / 256;
+  const int blocks = static_cast<int>(want < sms * 4 ? (want < 1 ? 1 : want) : sms * 4);
+  validate_kernel<<<blocks, 256, 0, s>>>(tgt, T, V, cu, n_seq, gid, n_groups, rewards, old_logp,
+                                         ref_logp, mask, counts);
   note_launches(1);
   return cudaGetLastError();
 }

@@ -56,6 +56,8 @@ _SIGS = {
     "spo_reward_compose": ([_vp, _vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp], ctypes.c_int),
     "spo_ranker_scores": ([_vp, _vp, _vp, _i32, _vp, _vp, _vp], ctypes.c_int),
     "spo_scale_f32": ([_vp, _i64, _f32, _vp, _vp], ctypes.c_int),
+    "spo_validate_inputs": ([_vp, _i64, _i64, _vp, _i32, _vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp],
+                            ctypes.c_int),
     "spo_ranker_workspace_size": ([_i32, ctypes.POINTER(_c_size)], ctypes.c_int),
     "spo_ranker_pair_loss": ([_vp, _vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp, _f32, _vp, _vp, _vp,
                               _c_size, _vp], ctypes.c_int),
@@ -408,3 +410,29 @@ def spo_scale_f32(x, alpha=None, alpha_dev=None):
     _check(lib().spo_scale_f32(_ptr(x), x.numel(), float(alpha if alpha is not None else 1.0),
                                _ptr(alpha_dev), _stream(x.device)))
     return x
+
+
+VALIDATION_FIELDS = ("tgt_out_of_range", "bad_cu_seqlens", "bad_group_id", "nonfinite_rewards",
+                     "nonfinite_old_ref_logp", "bad_mask")
+
+
+def spo_validate_inputs(tgt=None, V=0, cu_seqlens=None, group_id=None, n_groups=0, rewards=None,
+                        old_logp=None, ref_logp=None, mask=None, T=None, sync=True):
+    """Counts of invalid device inputs (see include/spo.h); a dict when sync, else the
+    device int32[6] counts tensor."""
+    ref = next(t for t in (tgt, cu_seqlens, group_id, rewards, old_logp, ref_logp, mask)
+               if t is not None)
+    dev = ref.device
+    if T is None:
+        T = (tgt if tgt is not None else old_logp if old_logp is not None else
+             mask if mask is not None else torch.empty(0)).numel()
+    n_seq = (cu_seqlens.numel() - 1 if cu_seqlens is not None else
+             group_id.numel() if group_id is not None else
+             rewards.numel() if rewards is not None else 0)
+    counts = torch.empty(6, dtype=torch.int32, device=dev)
+    _check(lib().spo_validate_inputs(_ptr(tgt), T, V, _ptr(cu_seqlens), n_seq, _ptr(group_id),
+                                     n_groups, _ptr(rewards), _ptr(old_logp), _ptr(ref_logp),
+                                     _ptr(mask), _ptr(counts), _stream(dev)))
+    if not sync:
+        return counts
+    return dict(zip(VALIDATION_FIELDS, counts.cpu().tolist()))

@@ -162,3 +162,37 @@ def test_static_and_dynamic_tile_schedules(mask):
     finally:
         spo.spo_set_tuning(spo.SPO_TUNE_DYNAMIC_MASK, 15)
         spo.spo_set_tuning(spo.SPO_TUNE_GROUP_M, 16)
+
+
+def test_validate_inputs_counts_planted_errors():
+    from paper_2607_20908_gb300 import spo
+    case = inputs.tiny_case(seed=1091)
+    T, V = case["T"], case["V"]
+    c = lambda t: t.cuda()
+    clean = spo.spo_validate_inputs(c(case["tgt"]), V, c(case["cu_seqlens"]), c(case["group_id"]),
+                                    case["n_groups"], c(case["rewards"]), c(case["old_noise"]),
+                                    c(case["ref_noise"]), c(case["mask"]))
+    assert all(v == 0 for v in clean.values()), clean
+    tgt = case["tgt"].clone(); tgt[[3, 77]] = V; tgt[5] = -100          # -100 stays valid
+    cu = case["cu_seqlens"].clone(); cu[4] = cu[3] - 1; cu[-1] = T + 1   # one decrease, wrong end
+    gid = case["group_id"].clone(); gid[0] = case["n_groups"]; gid[1] = -1
+    rw = case["rewards"].clone(); rw[2] = float("nan")
+    old = case["old_noise"].clone(); old[9] = float("inf")
+    mask = case["mask"].clone(); mask[10] = 2
+    bad = spo.spo_validate_inputs(c(tgt), V, c(cu), c(gid), case["n_groups"], c(rw), c(old),
+                                  c(case["ref_noise"]), c(mask))
+    assert bad == dict(tgt_out_of_range=2, bad_cu_seqlens=2, bad_group_id=2, nonfinite_rewards=1,
+                       nonfinite_old_ref_logp=1, bad_mask=1), bad
+
+
+def test_minimum_sizes():
+    """T = 1 token, d = 64, V = 256: one partial tile everywhere."""
+    case = inputs.tiny_case(seed=1101, T_per_seq=1, n_groups=1, rollouts=1, d=64, V=256)
+    _compare(case)
+
+
+def test_two_rollout_group_and_long_window():
+    """Groups of two (the smallest with a non-zero advantage), sequences longer than the window."""
+    case = inputs.tiny_case(seed=1111, T_per_seq=300, n_groups=3, rollouts=2, d=128, V=1024)
+    case["window"] = 256
+    _compare(case)
