@@ -65,10 +65,10 @@ SAMPLE_SEQS, SAMPLE_TOKENS = 8, 8   # CPU sample: one group of 8 rollouts, first
 
 # DRAM bytes (read + write) per launch of each tensor-core kernel on this workload, from one
 # `ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum` capture of this command
-# (profiles/raster_dram_sweep_full_workload.md, row 1,16,0,15), valid only for the kernel sources they were taken on.
-TRAFFIC = {"sources_sha256_16": "c504859b24a49bac",
-           "bytes": {"logits_lse_fwd": 6.961e9, "logits_grad_recompute": 12.824e9,
-                     "gemm_dH": 69.058e9, "gemm_dW": 53.124e9}}
+# (profiles/launches_full_workload.md), valid only for the kernel sources they were taken on.
+TRAFFIC = {"sources_sha256_16": "6bc21f98b1841f5a",
+           "bytes": {"logits_lse_fwd": 6.942e9, "logits_grad_recompute": 12.863e9,
+                     "gemm_dH": 83.132e9, "gemm_dW": 67.302e9}}
 KERNEL_SOURCES = ["paper_2607_20908_gb300/csrc/gemm.cu", "paper_2607_20908_gb300/csrc/tc.cuh",
                   "paper_2607_20908_gb300/csrc/internal.h"]
 
