@@ -51,10 +51,22 @@ if ROOT not in sys.path:
 from paper_2607_20908_gb300 import inputs  # noqa: E402
 
 METRIC = "tokens/s fused logprob+PG loss fwd+bwd (d=5120,V=151936); % BF16 tensor peak"
+METRIC_FWD = "tokens/s forward logprobs + entropy (d=4096,V=151936); % BF16 tensor peak"
 UNIT = "tokens/s"
 WORKLOAD = ("full loss fwd+bwd: T=16384 tokens (16 groups x 8 rollouts x 128 tokens), d=5120, "
             "V=151936, bf16 H/W, fp32 accumulate, rewards correctness+log-speedup+structural, "
             "clip eps=0.2, KL beta=0.04, window 1024, SEQ_GROUP aggregation")
+# Supplementary workloads (--workload); the default is the one the metric is quoted on.
+WORKLOADS = {
+    "full": WORKLOAD,
+    "forward": "forward logprobs only: T=8192 tokens (8 rollouts x 1024), d=4096, V=151936, bf16; "
+               "outputs fp32 per-token logprob and entropy",
+    "ragged": "multi-turn ragged: 32 groups x 8 rollouts x 1-4 turns packed to 65536 tokens, ~40% "
+              "prompt/feedback tokens masked, per-turn rewards, d=5120, V=151936, bf16 fwd+bwd",
+    "large": "large batch: T=131072 packed tokens, groups of 4/8/16, 5% of rollouts in zero-variance "
+             "groups, KL to reference log-probs, d=5120, V=151936, bf16 fwd+bwd (4 backward chunks)",
+}
+
 KERNEL_NAMES = {0: "logits_lse_fwd", 1: "logits_grad_recompute", 2: "gemm_dH", 3: "gemm_dW",
                 4: "lse_combine", 5: "select_gather_fwd", 6: "select_gather_bwd",
                 7: "policy_loss_fwd", 8: "group_advantages", 9: "token_select",
@@ -191,6 +203,7 @@ class Step:
     def __init__(self, case, dev, dist=None):
         from paper_2607_20908_gb300 import spo
         self.spo = spo
+        self.forward_only = case.get("forward_only", "cu_seqlens" not in case)
         # data parallel over whole groups: every rank owns the same number of groups, so each
         # rank's share of Eq. 3's group average is exactly 1 / world
         self.dist = dist if dist is not None and dist.world > 1 else None
@@ -200,15 +213,21 @@ class Step:
         self.case = case
         T, d, V = case["T"], case["d"], case["V"]
         self.T, self.d, self.V = T, d, V
-        self.n_seq = case["cu_seqlens"].numel() - 1
-        self.n_groups = case["n_groups"]
         to = lambda t: t.to(dev).contiguous()
         self.H, self.W = to(case["H"]), to(case["W"])
         self.tgt, self.mask = to(case["tgt"]), to(case["mask"])
+        f32 = dict(dtype=torch.float32, device=dev)
+        if self.forward_only:
+            case = dict(case, cu_seqlens=torch.tensor([0, T], dtype=torch.int32),
+                        group_id=torch.zeros(1, dtype=torch.int32), n_groups=1,
+                        rewards=torch.zeros(1), old_noise=torch.zeros(T), ref_noise=torch.zeros(T),
+                        window=0, clip_eps=0.2, kl_beta=0.0, forward_only=True)
+            self.case = case
+        self.n_seq = case["cu_seqlens"].numel() - 1
+        self.n_groups = case["n_groups"]
         self.cu, self.gid = to(case["cu_seqlens"]), to(case["group_id"])
         self.rewards = to(case["rewards"])
-        f32 = dict(dtype=torch.float32, device=dev)
-        self.loss_mask = torch.empty(T, dtype=torch.uint8, device=dev)
+        self.loss_mask = self.mask if self.forward_only else torch.empty(T, dtype=torch.uint8, device=dev)
         self.n_tok = torch.empty(self.n_seq, dtype=torch.int32, device=dev)
         self.logp, self.ent, self.lse = (torch.empty(T, **f32) for _ in range(3))
         self.adv = torch.empty(self.n_seq, **f32)
@@ -226,6 +245,8 @@ class Step:
 
     def prepare_old_ref(self):
         """Old / reference log-probs = current log-probs + noise (one forward, untimed)."""
+        if self.forward_only:
+            return
         self.run(stop_after_fwd=True)
         torch.cuda.synchronize(self.dev)
         self.old.copy_(self.logp + self.case["old_noise"].to(self.dev))
@@ -235,6 +256,11 @@ class Step:
         L, p, c = self.L, lambda t: ctypes.c_void_p(t.data_ptr()), self.case
         s = ctypes.c_void_p(self.stream.cuda_stream)
         chk = self.spo._check
+        if self.forward_only:   # log-probs and entropy only (old-policy / rescoring pass)
+            chk(L.spo_logprobs_fwd(p(self.H), p(self.W), p(self.tgt), p(self.mask), self.T, self.d,
+                                   self.V, c["inv_temp"], p(self.logp), p(self.ent), p(self.lse),
+                                   p(self.ws_f), self.ws_f.numel(), s))
+            return
         chk(L.spo_token_select(p(self.cu), p(self.mask), p(self.tgt), self.n_seq, self.T, c["window"],
                                p(self.loss_mask), p(self.n_tok), s))
         chk(L.spo_logprobs_fwd(p(self.H), p(self.W), p(self.tgt), p(self.loss_mask), self.T, self.d,
@@ -270,8 +296,12 @@ class HostIO:
         self.sets[1].old.copy_(st.old)
         self.sets[1].ref.copy_(st.ref)
         pinned = lambda t: torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
-        ins = lambda x: (x.H, x.W, x.tgt, x.mask, x.cu, x.gid, x.rewards, x.old, x.ref)
-        outs = lambda x: (x.loss, x.stats, x.logp, x.ent, x.dH, x.dW)
+        if st.forward_only:
+            ins = lambda x: (x.H, x.W, x.tgt, x.mask)
+            outs = lambda x: (x.logp, x.ent, x.lse)
+        else:
+            ins = lambda x: (x.H, x.W, x.tgt, x.mask, x.cu, x.gid, x.rewards, x.old, x.ref)
+            outs = lambda x: (x.loss, x.stats, x.logp, x.ent, x.dH, x.dW)
         self.host_in = [pinned(t).copy_(t) for t in ins(st)]
         self.host_out = [[pinned(t) for t in outs(x)] for x in self.sets]
         self.dev_in = [ins(x) for x in self.sets]
@@ -420,13 +450,19 @@ def aux_measurements(dev, pk):
 
 
 # ----------------------------------------------------------------- arms
-def config_block(case, T_L, world):
-    return {"workload": WORKLOAD, "T": case["T"], "loss_tokens": T_L, "d": case["d"], "V": case["V"],
-            "groups": case["n_groups"], "rollouts_per_group": 8, "tokens_per_rollout": 128,
-            "clip_eps": case["clip_eps"], "kl_beta": case["kl_beta"], "window": case["window"],
-            "l2": "inputs larger than L2 (W alone is 1.56 GB; each step also streams a 5 GB bf16 G buffer)",
-            "parallelism": (f"dp{world}: 16 whole groups per GPU, dW and loss all-reduced (NCCL) "
-                            f"every step" if world > 1 else "1 GPU")}
+def config_block(case, T_L, world, workload="full"):
+    cfg = {"workload": WORKLOADS[workload], "T": case["T"], "loss_tokens": T_L, "d": case["d"],
+           "V": case["V"]}
+    if workload == "full":
+        cfg.update(groups=case["n_groups"], rollouts_per_group=8, tokens_per_rollout=128)
+    elif workload != "forward":
+        cfg.update(groups=case["n_groups"], sequences=int(case["cu_seqlens"].numel() - 1))
+    if workload != "forward":
+        cfg.update(clip_eps=case["clip_eps"], kl_beta=case["kl_beta"], window=case["window"])
+    cfg["l2"] = "inputs larger than L2 (W alone is 1.2-1.56 GB and is streamed every step)"
+    cfg["parallelism"] = (f"dp{world}: whole groups per GPU, dW and loss all-reduced (NCCL) every step"
+                          if world > 1 else "1 GPU")
+    return cfg
 
 
 def ours(args):
@@ -438,13 +474,19 @@ def ours(args):
     if dist.rank == 0 and not os.path.exists(spo.LIB_PATH):
         build.build()
     dist.barrier()
-    case = inputs.full_case(seed=1003 + dist.rank, device=str(dev))
+    maker = {"full": inputs.full_case, "forward": inputs.forward_case, "ragged": inputs.ragged_case,
+             "large": inputs.large_case}[args.workload]
+    seed0 = {"full": 1003, "forward": 1002, "ragged": 1004, "large": 1005}[args.workload]
+    case = maker(seed=seed0 + dist.rank, device=str(dev))
+    if args.workload == "forward" and dist.world > 1:
+        raise SystemExit("--workload forward runs on one GPU")
     st = Step(case, dev, dist)
     st.prepare_old_ref()
     torch.cuda.synchronize(dev)
     T_L = int(st.loss_mask.sum().item())
     flop_gemm = 2.0 * T_L * st.d * st.V          # one GEMM-equivalent (algorithmic)
-    flop_metric = 3.0 * flop_gemm                 # fwd + dH + dW (the recompute is not counted)
+    # fwd + dH + dW (the backward's recompute is not counted); the forward-only workload: fwd
+    flop_metric = (1.0 if st.forward_only else 3.0) * flop_gemm
     pk = peaks()
 
     for _ in range(args.warmup):
@@ -523,18 +565,20 @@ def ours(args):
                    "dH, dW; two buffer sets so copies overlap the neighbouring steps' compute"}
 
     line = {
-        "metric": METRIC, "value": tokens_s, "unit": UNIT, "n_gpus": dist.world, "steps": args.steps,
+        "metric": METRIC_FWD if st.forward_only else METRIC, "value": tokens_s, "unit": UNIT,
+        "n_gpus": dist.world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded; H~N(0,1), W~N(0,0.02^2) rounded to bf16: random-init stand-in for "
                 "the policy's final hidden states and LM head)",
-        "config": config_block(case, T_L, dist.world),
+        "config": config_block(case, T_L, dist.world, args.workload),
         "tensor_peak_frac": {"metric_tflops": flop_metric * args.steps / (ms / 1e3) / 1e12,
                              "of_burst": flop_metric * args.steps / (ms / 1e3) / 1e12 / pk["bf16_burst"],
                              "of_sustained": flop_metric * args.steps / (ms / 1e3) / 1e12 / pk["bf16_sustained"],
                              "flop_per_step": flop_metric,
-                             "note": "algorithmic 3 x 2*T*d*V per step; the backward's logit recompute "
-                                     "is done but not counted"},
+                             "note": ("algorithmic 2*T*d*V per step (forward only)" if st.forward_only else
+                                      "algorithmic 3 x 2*T*d*V per step; the backward's logit "
+                                      "recompute is done but not counted")},
         "roofline": roofline,
         "kernels": kern,
         "e2e": e2e,
@@ -542,8 +586,9 @@ def ours(args):
         "launches_per_step": n_launch / args.steps,
         "clocks": clocks.summary(t0, t1),
     }
-    line["aux"] = aux_measurements(dev, pk)
-    if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:
+    if args.workload == "full":
+        line["aux"] = aux_measurements(dev, pk)
+    if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline and args.workload == "full":
         line["cpu_baseline"] = run_cpu_baseline(st)
     if dist.rank == 0:
         print(json.dumps(line), flush=True)
@@ -596,6 +641,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle timing")
+    ap.add_argument("--workload", choices=sorted(WORKLOADS), default="full",
+                    help="supplementary workloads; the default is the one the metric is quoted on")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
