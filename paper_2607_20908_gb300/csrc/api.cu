@@ -250,7 +250,8 @@ enum TraceKind : int {
 // counters: the workspace's four tile counters (the one of this kind is
 // zeroed on the stream and used when the kind's dynamic-schedule bit is set).
 spo_status traced_gemm(int kind, bool a_mn, bool b_mn, const CUtensorMap& ta, const CUtensorMap& tb,
-                       const spo::GemmArgs& args_in, int grid, cudaStream_t s, int* counters) {
+                       const CUtensorMap& tc, const spo::GemmArgs& args_in, int grid, cudaStream_t s,
+                       int* counters) {
   spo::GemmArgs args = args_in;
   args.tile_counter = nullptr;
   if (counters && ((g_tune_dynamic_mask >> kind) & 1)) {
@@ -258,7 +259,7 @@ spo_status traced_gemm(int kind, bool a_mn, bool b_mn, const CUtensorMap& ta, co
     SPO_CUDA(cudaMemsetAsync(args.tile_counter, 0, sizeof(int), s), "memset tile counter");
   }
   return traced(kind, s, "gemm launch", [&] {
-    return spo::launch_gemm(kind, a_mn, b_mn, g_tune_pair != 0, ta, tb, args, grid, s);
+    return spo::launch_gemm(kind, a_mn, b_mn, g_tune_pair != 0, ta, tb, tc, args, grid, s);
   });
 }
 
@@ -390,7 +391,7 @@ SPO_API spo_status spo_logprobs_fwd(const void* H, const void* W, const int32_t*
   a.partials = w.partials;
   a.nsplit = w.nsplit;
   a.ztgt = w.ztgt;
-  if ((st = traced_gemm(spo::EPI_LSE, false, false, ta, tb, a, grid_for(di, w.T_pad, V), s,
+  if ((st = traced_gemm(spo::EPI_LSE, false, false, ta, tb, ta, a, grid_for(di, w.T_pad, V), s,
                         w.counters)) !=
       SPO_OK)
     return st;
@@ -591,11 +592,18 @@ SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32
   if (st != SPO_OK) return st;
   if (dH) SPO_CUDA(cudaMemsetAsync(dH, 0, sizeof(uint16_t) * T * d, s), "memset dH");
 
-  CUtensorMap tW_k, tW_mn, tG_k, tG_mn;
+  CUtensorMap tW_k, tW_mn, tG_k, tG_mn;  // operand maps
   SPO_CUDA(spo::make_tmap_bf16(&tW_k, W, d, V, d * 2, spo::BK, b_box_rows()), "tensor map W");
   SPO_CUDA(spo::make_tmap_bf16(&tW_mn, W, d, V, d * 2, 64, spo::BK), "tensor map W (MN)");
   SPO_CUDA(spo::make_tmap_bf16(&tG_k, w.G, V, w.chunk, V * 2, spo::BK, spo::BM), "tensor map G");
   SPO_CUDA(spo::make_tmap_bf16(&tG_mn, w.G, V, w.chunk, V * 2, 64, spo::BK), "tensor map G (MN)");
+  CUtensorMap tG_store, tdW;
+  SPO_CUDA(spo::make_tmap_bf16(&tG_store, w.G, V, w.chunk, V * 2, 64, spo::kStoreBoxRows),
+           "tensor map G (store)");
+  if (dW)
+    SPO_CUDA(spo::make_tmap_f32(&tdW, dW, d, V, d * 4, 32, spo::kStoreBoxRows), "tensor map dW");
+  else
+    tdW = tG_store;
 
   const long long n_chunks = (w.T_pad + w.chunk - 1) / w.chunk;
   for (long long c = 0; c < n_chunks; ++c) {
@@ -619,7 +627,7 @@ SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32
     a.gvec = w.g_c + r0;
     a.G = w.G;
     a.ldG = V;
-    if ((st = traced_gemm(spo::EPI_GRAD, false, false, tH_k, tW_k, a, grid_for(di, rows, V), s,
+    if ((st = traced_gemm(spo::EPI_GRAD, false, false, tH_k, tW_k, tG_store, a, grid_for(di, rows, V), s,
                           w.counters)) != SPO_OK)
       return st;
     // a7: dH rows = G W, scattered to token rows
@@ -633,7 +641,7 @@ SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32
       b.row_idx = w.idx + r0;
       b.out_bf16 = static_cast<__nv_bfloat16*>(dH);
       b.ld_out = d;
-      if ((st = traced_gemm(spo::EPI_DH, false, true, tG_k, tW_mn, b, grid_for(di, rows, d), s,
+      if ((st = traced_gemm(spo::EPI_DH, false, true, tG_k, tW_mn, tG_k, b, grid_for(di, rows, d), s,
                             w.counters)) != SPO_OK)
         return st;
     }
@@ -648,7 +656,7 @@ SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32
       b.out_f32 = dW;
       b.ld_out = d;
       b.accumulate = (c == 0) ? (accumulate_dW ? 1 : 0) : 1;
-      if ((st = traced_gemm(spo::EPI_DW, true, true, tG_mn, tH_mn, b, grid_for(di, V, d), s,
+      if ((st = traced_gemm(spo::EPI_DW, true, true, tG_mn, tH_mn, tdW, b, grid_for(di, V, d), s,
                             w.counters)) !=
           SPO_OK)
         return st;

@@ -120,39 +120,6 @@ __device__ __forceinline__ void epi_lse(const GemmArgs& p, uint32_t taddr, int r
   }
 }
 
-__device__ __forceinline__ void epi_grad(const GemmArgs& p, uint32_t taddr, int row, int M, int nb) {
-  const bool row_ok = row < M;
-  const float gl = row_ok ? p.gvec[row] : 0.f;
-  const float l2 = row_ok ? p.lse[row] * kLog2e : 0.f;
-  const int y = row_ok ? p.tgt[row] : -1;
-  const float coef = p.scale * gl;
-  const float sc2 = p.scale * kLog2e;
-  const int col_base = nb * BN;
-  __nv_bfloat16* grow = p.G + static_cast<size_t>(row) * p.ldG;
-#pragma unroll 1
-  for (int c = 0; c < BN / 32; ++c) {
-    const int c0 = col_base + c * 32;
-    if (c0 >= p.n) break;  // warp-uniform
-    float v[32];
-    tmem_ld32(taddr + c * 32, v);
-    uint32_t pk[16];
-#pragma unroll
-    for (int j = 0; j < 16; ++j) {
-      const int ca = c0 + 2 * j;
-      const float pa = exp2f(fmaf(v[2 * j], sc2, -l2));
-      const float pb = exp2f(fmaf(v[2 * j + 1], sc2, -l2));
-      const float ga = coef * ((ca == y ? 1.f : 0.f) - pa);
-      const float gb = coef * ((ca + 1 == y ? 1.f : 0.f) - pb);
-      pk[j] = pack_bf16x2(ga, gb);
-    }
-#pragma unroll
-    for (int q = 0; q < 4; ++q)
-      if (c0 + 8 * q < p.n)
-        *reinterpret_cast<uint4*>(grow + c0 + 8 * q) =
-            make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
-  }
-}
-
 __device__ __forceinline__ void epi_dh(const GemmArgs& p, uint32_t taddr, int row, int M, int nb) {
   const bool row_ok = row < M;
   const int out_row = row_ok ? (p.row_idx ? p.row_idx[row] : row) : 0;
@@ -176,10 +143,81 @@ __device__ __forceinline__ void epi_dh(const GemmArgs& p, uint32_t taddr, int ro
   }
 }
 
-__device__ __forceinline__ void epi_dw(const GemmArgs& p, uint32_t taddr, int row, int M, int nb,
-                                       bool kzero) {
+// TMA-store epilogues: each epilogue warp stages its 32 rows x 128 bytes in a
+// [32][128 B] shared slot with the 128-byte swizzle (chunk j of row r at
+// position j ^ (r % 8): conflict-free writes, and the layout a swizzled
+// tensor map expects), then one lane issues a bulk tensor store (or
+// reduce-add) of the 32 x 128 B box.  Two slots per warp alternate.
+constexpr uint32_t kEpiSlotBytes = 32 * 128;
+
+__device__ __forceinline__ void stage_row128(uint8_t* slot, int lane, const uint32_t (&w)[32]) {
+  uint4* row = reinterpret_cast<uint4*>(slot + lane * 128);
+#pragma unroll
+  for (int j = 0; j < 8; ++j)
+    row[j ^ (lane & 7)] = make_uint4(w[4 * j], w[4 * j + 1], w[4 * j + 2], w[4 * j + 3]);
+}
+
+// Hands slot (slab & 1) back after staging: fence the generic writes for the
+// async proxy, then one lane issues the store.  `reduce` selects add.
+__device__ __forceinline__ void flush_slot(const CUtensorMap* tm, uint8_t* slot, int x, int y,
+                                           bool reduce, int lane) {
+  fence_proxy_async_smem();
+  __syncwarp();
+  if (lane == 0) {
+    if (reduce)
+      tma_reduce_add_2d(tm, slot, x, y);
+    else
+      tma_store_2d(tm, slot, x, y);
+    bulk_commit();
+  }
+}
+
+__device__ __forceinline__ uint8_t* acquire_slot(uint8_t* slots, int slab, int lane) {
+  if (lane == 0) bulk_wait_read<1>();  // the store issued from this slot two slabs ago has read it
+  __syncwarp();
+  return slots + (slab & 1) * kEpiSlotBytes;
+}
+
+// G rows as bf16 through 64-column (128-byte) slabs.
+__device__ __forceinline__ void epi_grad_tma(const GemmArgs& p, const CUtensorMap* tmC, uint32_t taddr,
+                                             int row, int row0, int M, int nb, uint8_t* slots,
+                                             int& slab, int lane) {
   const bool row_ok = row < M;
-  float* dst = p.out_f32 + static_cast<size_t>(row_ok ? row : 0) * p.ld_out;
+  const float gl = row_ok ? p.gvec[row] : 0.f;
+  const float l2 = row_ok ? p.lse[row] * kLog2e : 0.f;
+  const int y = row_ok ? p.tgt[row] : -1;
+  const float coef = p.scale * gl;
+  const float sc2 = p.scale * kLog2e;
+  const int col_base = nb * BN;
+#pragma unroll 1
+  for (int c2 = 0; c2 < BN / 64; ++c2) {
+    const int c0 = col_base + c2 * 64;
+    if (c0 >= p.n) break;  // warp-uniform; columns past n inside a slab are clipped by the store
+    uint32_t w[32];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      float v[32];
+      tmem_ld32(taddr + c2 * 64 + h * 32, v);
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const int ca = c0 + h * 32 + 2 * j;
+        const float pa = exp2f(fmaf(v[2 * j], sc2, -l2));
+        const float pb = exp2f(fmaf(v[2 * j + 1], sc2, -l2));
+        w[h * 16 + j] = pack_bf16x2(coef * ((ca == y ? 1.f : 0.f) - pa),
+                                    coef * ((ca + 1 == y ? 1.f : 0.f) - pb));
+      }
+    }
+    uint8_t* slot = acquire_slot(slots, slab, lane);
+    stage_row128(slot, lane, w);
+    flush_slot(tmC, slot, c0, row0, false, lane);
+    ++slab;
+  }
+}
+
+// dW rows as fp32 through 32-column (128-byte) slabs; accumulate = reduce-add.
+__device__ __forceinline__ void epi_dw_tma(const GemmArgs& p, const CUtensorMap* tmC, uint32_t taddr,
+                                           int row0, int nb, bool kzero, uint8_t* slots, int& slab,
+                                           int lane) {
   const int col_base = nb * BN;
 #pragma unroll 1
   for (int c = 0; c < BN / 32; ++c) {
@@ -192,19 +230,13 @@ __device__ __forceinline__ void epi_dw(const GemmArgs& p, uint32_t taddr, int ro
     } else {
       tmem_ld32(taddr + c * 32, v);
     }
-    if (!row_ok) continue;
+    uint32_t w[32];
 #pragma unroll
-    for (int q = 0; q < 8; ++q) {
-      if (c0 + 4 * q < p.n) {
-        float4* d4 = reinterpret_cast<float4*>(dst + c0 + 4 * q);
-        float4 o = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-        if (p.accumulate) {
-          const float4 a = *d4;
-          o.x += a.x; o.y += a.y; o.z += a.z; o.w += a.w;
-        }
-        *d4 = o;
-      }
-    }
+    for (int j = 0; j < 32; ++j) w[j] = __float_as_uint(v[j]);
+    uint8_t* slot = acquire_slot(slots, slab, lane);
+    stage_row128(slot, lane, w);
+    flush_slot(tmC, slot, c0, row0, p.accumulate != 0, lane);
+    ++slab;
   }
 }
 
@@ -214,33 +246,35 @@ __device__ __forceinline__ void epi_dw(const GemmArgs& p, uint32_t taddr, int ro
 // cta_group::2 MMA; each stages its own 128 rows of A and 128 of the 256 B
 // rows, so a stage is 32 KB and seven fit in shared memory (~2 us of MMA
 // work buffered against operand latency).
-#ifndef SPO_PAIR_STAGES
-#define SPO_PAIR_STAGES 7
-#endif
-template <bool PAIR>
+// The G and dW epilogues store through TMA and need 32 KB of staging, so
+// their pair-mode ring has six stages.
+template <bool PAIR, int EPI = EPI_LSE>
 struct Geo {
-  static constexpr int kStages = PAIR ? SPO_PAIR_STAGES : 4;
+  static constexpr bool kTmaStore = EPI == EPI_GRAD || EPI == EPI_DW;
+  static constexpr int kStages = PAIR ? (kTmaStore ? 6 : 7) : 4;
+  static constexpr uint32_t kEpiBytes = kTmaStore ? 4 * 2 * kEpiSlotBytes : 0;  // 4 warps x 2 slots
   static constexpr int kBRows = PAIR ? BN / 2 : BN;        // B rows staged per CTA
   static constexpr uint32_t kABytes = BM * BK * 2;         // 16 KB
   static constexpr uint32_t kBBytes = kBRows * BK * 2;     // 16 or 32 KB
   static constexpr uint32_t kStageBytes = kABytes + kBBytes;
   static constexpr int kTileM = PAIR ? 2 * BM : BM;         // output rows per tile
   static constexpr uint32_t kTxBytes = PAIR ? 2 * kStageBytes : kStageBytes;  // per full barrier
-  static constexpr size_t kSmem = 1024 + kStages * kStageBytes + 512;
+  static constexpr size_t kSmem = 1024 + kStages * kStageBytes + kEpiBytes + 512;
 };
 
 template <int EPI, bool A_MN, bool B_MN, bool PAIR>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                const GemmArgs p) {
-  using G = Geo<PAIR>;
+                const __grid_constant__ CUtensorMap tmC, const GemmArgs p) {
+  using G = Geo<PAIR, EPI>;
   constexpr int S = G::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + S * G::kABytes;
-  uint64_t* full_bar = reinterpret_cast<uint64_t*>(sB + S * G::kBBytes);
+  uint8_t* sEpi = sB + S * G::kBBytes;  // TMA-store staging (1024-byte aligned)
+  uint64_t* full_bar = reinterpret_cast<uint64_t*>(sEpi + G::kEpiBytes);
   uint64_t* empty_bar = full_bar + S;
   uint64_t* tfull_bar = empty_bar + S;
   uint64_t* tempty_bar = tfull_bar + 2;
@@ -459,6 +493,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   } else {
     // ------------------------------------------------ epilogue warps 2..5 (both CTAs)
     const int q = warp & 3;  // TMEM lanes [32q, 32q+32) are reachable from this warp
+    uint8_t* slots = sEpi + (warp - 2) * 2 * kEpiSlotBytes;  // unused unless G::kTmaStore
+    int slab = 0;
     for (int local = 0;; ++local) {
       int tile;
       if (dyn) {
@@ -480,10 +516,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const int row = mb * G::kTileM + static_cast<int>(rank) * BM + q * 32 + lane;
       const uint32_t taddr =
           tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN);
+      const int row0 = row - lane;  // first row of this warp
       if (EPI == EPI_LSE) epi_lse(p, taddr, row, M, nb);
-      if (EPI == EPI_GRAD) epi_grad(p, taddr, row, M, nb);
+      if (EPI == EPI_GRAD) epi_grad_tma(p, &tmC, taddr, row, row0, M, nb, slots, slab, lane);
       if (EPI == EPI_DH) epi_dh(p, taddr, row, M, nb);
-      if (EPI == EPI_DW) epi_dw(p, taddr, row, M, nb, num_kb == 0);
+      if (EPI == EPI_DW) epi_dw_tma(p, &tmC, taddr, row0, nb, num_kb == 0, slots, slab, lane);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) {
@@ -492,6 +529,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         else
           mbar_arrive(&tempty_bar[acc]);
       }
+    }
+    if (G::kTmaStore) {
+      if (lane == 0) bulk_wait_all();  // stores complete before the CTA exits
+      __syncwarp();
     }
   }
 
@@ -527,10 +568,10 @@ EncodeTiledFn encode_fn() {
 }
 
 template <int EPI, bool A_MN, bool B_MN, bool PAIR>
-cudaError_t launch_one(const CUtensorMap& ta, const CUtensorMap& tb, const GemmArgs& args, int grid,
-                       cudaStream_t s) {
+cudaError_t launch_one(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc,
+                       const GemmArgs& args, int grid, cudaStream_t s) {
   auto k = gemm_kernel<EPI, A_MN, B_MN, PAIR>;
-  const size_t smem = Geo<PAIR>::kSmem;
+  const size_t smem = Geo<PAIR, EPI>::kSmem;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
@@ -546,7 +587,7 @@ cudaError_t launch_one(const CUtensorMap& ta, const CUtensorMap& tb, const GemmA
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  e = cudaLaunchKernelEx(&cfg, k, ta, tb, args);
+  e = cudaLaunchKernelEx(&cfg, k, ta, tb, tc, args);
   note_launches(1);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
@@ -554,32 +595,47 @@ cudaError_t launch_one(const CUtensorMap& ta, const CUtensorMap& tb, const GemmA
 
 }  // namespace
 
-size_t gemm_smem_bytes(bool pair) { return pair ? Geo<true>::kSmem : Geo<false>::kSmem; }
+size_t gemm_smem_bytes(bool pair) { return pair ? Geo<true, EPI_GRAD>::kSmem : Geo<false, EPI_GRAD>::kSmem; }
 
 int gemm_tile_m(bool pair) { return pair ? Geo<true>::kTileM : Geo<false>::kTileM; }
 
 int gemm_b_box_rows(bool pair) { return pair ? Geo<true>::kBRows : Geo<false>::kBRows; }
 
-cudaError_t make_tmap_bf16(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer,
-                           uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer) {
+namespace {
+cudaError_t make_tmap_2d(CUtensorMap* tm, CUtensorMapDataType type, const void* base, uint64_t inner,
+                         uint64_t outer, uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return cudaErrorNotSupported;
   cuuint64_t dims[2] = {inner, outer};
   cuuint64_t strides[1] = {row_bytes};
   cuuint32_t box[2] = {box_inner, box_outer};
   cuuint32_t estr[2] = {1, 1};
-  CUresult r = fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
-                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+  CUresult r = fn(tm, type, 2, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
+}  // namespace
+
+cudaError_t make_tmap_bf16(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer,
+                           uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer) {
+  return make_tmap_2d(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, base, inner, outer, row_bytes, box_inner,
+                      box_outer);
+}
+
+cudaError_t make_tmap_f32(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer,
+                          uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer) {
+  return make_tmap_2d(tm, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, base, inner, outer, row_bytes, box_inner,
+                      box_outer);
+}
 
 cudaError_t launch_gemm(int epi, bool a_mn, bool b_mn, bool pair, const CUtensorMap& ta,
-                        const CUtensorMap& tb, const GemmArgs& args, int grid, cudaStream_t s) {
+                        const CUtensorMap& tb, const CUtensorMap& tc, const GemmArgs& args, int grid,
+                        cudaStream_t s) {
 #define SPO_GEMM_CASE(E, AM, BMN)                                                        \
   if (epi == E && a_mn == AM && b_mn == BMN)                                             \
-    return pair ? launch_one<E, AM, BMN, true>(ta, tb, args, grid, s)                    \
-                : launch_one<E, AM, BMN, false>(ta, tb, args, grid, s);
+    return pair ? launch_one<E, AM, BMN, true>(ta, tb, tc, args, grid, s)                \
+                : launch_one<E, AM, BMN, false>(ta, tb, tc, args, grid, s);
   SPO_GEMM_CASE(EPI_LSE, false, false)
   SPO_GEMM_CASE(EPI_GRAD, false, false)
   SPO_GEMM_CASE(EPI_DH, false, true)

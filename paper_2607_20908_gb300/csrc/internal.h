@@ -59,9 +59,9 @@ struct GemmArgs {
   const int* row_idx;         // output row of each row (NULL: identity)
   __nv_bfloat16* out_bf16;
   long long ld_out;
-  // EPI_DW
+  // EPI_DW (the output itself goes through the tc tensor map)
   float* out_f32;
-  int accumulate;
+  int accumulate;  // 1: reduce-add into the output, 0: overwrite
   int* err;  // device error word
 };
 
@@ -77,11 +77,16 @@ long long launches();
 // extents in elements / rows, row_bytes the pitch, box the staged tile.
 cudaError_t make_tmap_bf16(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer,
                            uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer);
+cudaError_t make_tmap_f32(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer,
+                          uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer);
 
 // Supported (epi, a_mn, b_mn): (LSE,0,0) (GRAD,0,0) (DH,0,1) (DW,1,1).  With
-// `pair` the grid must be even (clusters of two CTAs).
+// `pair` the grid must be even (clusters of two CTAs).  tc is the output's
+// tensor map for the TMA-store epilogues (GRAD: G as bf16, box 64 x 32; DW:
+// dW as fp32, box 32 x 32; both 128-byte swizzled); ignored by LSE and DH.
+constexpr uint32_t kStoreBoxRows = 32;
 cudaError_t launch_gemm(int epi, bool a_mn, bool b_mn, bool pair, const CUtensorMap& ta,
-                        const CUtensorMap& tb, const GemmArgs& args, int grid,
+                        const CUtensorMap& tb, const CUtensorMap& tc, const GemmArgs& args, int grid,
                         cudaStream_t s);
 
 // ---------------------------------------------------------------- small kernels
