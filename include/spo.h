@@ -373,12 +373,16 @@ SPO_API spo_status spo_policy_loss_fwd_noalloc(const float* logp, const float* o
  *   SPO_TUNE_DYNAMIC_MASK (default 15): bit k set = GEMM kind k (trace kinds
  *     0-3) takes its tiles in raster order from an atomic counter instead of
  *     a static round robin, so in-flight tiles stay a contiguous window.
- * Results do not depend on any setting. */
+ *   SPO_TUNE_DW_SPLIT_ROWS (default 8192; multiple of 256, 0 = off): dW =
+ *     G^T H is reduced over at most this many token rows per pass, later
+ *     passes adding into dW (smaller operand slabs stay in L2).
+ * Results do not depend on any setting beyond fp32 summation order. */
 typedef enum spo_tune_key {
     SPO_TUNE_PAIR_MMA = 0,
     SPO_TUNE_GROUP_M = 1,
     SPO_TUNE_RASTER = 2,
-    SPO_TUNE_DYNAMIC_MASK = 3
+    SPO_TUNE_DYNAMIC_MASK = 3,
+    SPO_TUNE_DW_SPLIT_ROWS = 4
 } spo_tune_key;
 SPO_API spo_status spo_set_tuning(int key, int64_t value);
 

@@ -183,6 +183,9 @@ int g_tune_raster = 0;
 // schedule) instead of the static round robin, so the tiles in flight stay a
 // contiguous window of the raster however the CTA pairs drift.  Default: all.
 int g_tune_dynamic_mask = 0xF;
+// dW = G^T H runs as passes over at most this many token rows (0: one pass
+// per chunk): smaller operand slabs keep a wave's working set inside L2.
+int g_tune_dw_split = 8192;
 
 // ------------------------------------------------------------ tracing
 // When enabled, a start/stop CUDA event pair is recorded on the launch stream
@@ -645,21 +648,32 @@ SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32
                             w.counters)) != SPO_OK)
         return st;
     }
-    // a8: dW (+)= G^T Hc over this chunk's rows
+    // a8: dW (+)= G^T Hc over this chunk's rows, in passes of at most
+    // g_tune_dw_split rows (later passes reduce-add into dW)
     if (dW) {
-      spo::GemmArgs b = base_args(di);
-      b.m_static = static_cast<int>(V);
-      b.n = static_cast<int>(d);
-      b.k_count = w.count;
-      b.k_offset = static_cast<int>(r0);
-      b.k_cap = static_cast<int>(w.chunk);
-      b.out_f32 = dW;
-      b.ld_out = d;
-      b.accumulate = (c == 0) ? (accumulate_dW ? 1 : 0) : 1;
-      if ((st = traced_gemm(spo::EPI_DW, true, true, tG_mn, tH_mn, tdW, b, grid_for(di, V, d), s,
-                            w.counters)) !=
-          SPO_OK)
-        return st;
+      const long long split = g_tune_dw_split > 0 ? g_tune_dw_split : rows;
+      for (long long q0 = 0; q0 < rows; q0 += split) {
+        const long long qrows = (rows - q0) < split ? (rows - q0) : split;
+        CUtensorMap tGq = tG_mn, tHq = tH_mn;
+        if (q0 > 0 || qrows < rows) {
+          SPO_CUDA(spo::make_tmap_bf16(&tGq, w.G + q0 * V, V, qrows, V * 2, 64, spo::BK),
+                   "tensor map G (MN, pass)");
+          SPO_CUDA(spo::make_tmap_bf16(&tHq, Hc0 + q0 * d, d, qrows, d * 2, 64, spo::BK),
+                   "tensor map Hc (MN, pass)");
+        }
+        spo::GemmArgs b = base_args(di);
+        b.m_static = static_cast<int>(V);
+        b.n = static_cast<int>(d);
+        b.k_count = w.count;
+        b.k_offset = static_cast<int>(r0 + q0);
+        b.k_cap = static_cast<int>(qrows);
+        b.out_f32 = dW;
+        b.ld_out = d;
+        b.accumulate = (c == 0 && q0 == 0) ? (accumulate_dW ? 1 : 0) : 1;
+        if ((st = traced_gemm(spo::EPI_DW, true, true, tGq, tHq, tdW, b, grid_for(di, V, d), s,
+                              w.counters)) != SPO_OK)
+          return st;
+      }
     }
   }
   return ok();
@@ -715,6 +729,11 @@ SPO_API spo_status spo_set_tuning(int key, int64_t value) {
     case SPO_TUNE_DYNAMIC_MASK:
       if (value < 0 || value > 15) return fail(SPO_ERR_INVALID_ARG, "dynamic mask must be in [0, 15]");
       g_tune_dynamic_mask = static_cast<int>(value);
+      return ok();
+    case SPO_TUNE_DW_SPLIT_ROWS:
+      if (value < 0 || value > (1 << 24) || value % 256 != 0)
+        return fail(SPO_ERR_INVALID_ARG, "dW split rows must be a multiple of 256 in [0, 2^24]");
+      g_tune_dw_split = static_cast<int>(value);
       return ok();
     case SPO_TUNE_RASTER:
       if (value != 0 && value != 1) return fail(SPO_ERR_INVALID_ARG, "raster must be 0 or 1");

@@ -6,7 +6,7 @@ sweeps.
     python -m paper_2607_20908_gb300.profile_case --V 151936 --iters 1 \\
         --configs "1,16,0;1,8,0;0,16,0"
 
---configs is a ';'-separated list of "pair,group,raster[,dynamic_mask]"
+--configs is a ';'-separated list of "pair,group,raster[,dynamic_mask[,dw_split_rows]]"
 launch tunings (spo_set_tuning); each is run for --iters iterations of
 fwd + bwd.  The default reduced size keeps the reduction lengths of the full workload
 (K = d = 5120 for the logits and their recompute, K = T = 16384 tokens for
@@ -56,6 +56,8 @@ def main():
             spo.spo_set_tuning(spo.SPO_TUNE_RASTER, raster)
             if len(cfg) > 3:
                 spo.spo_set_tuning(spo.SPO_TUNE_DYNAMIC_MASK, cfg[3])
+            if len(cfg) > 4:
+                spo.spo_set_tuning(spo.SPO_TUNE_DW_SPLIT_ROWS, cfg[4])
         for i in range(a.iters):
             spo.spo_trace_enable(i == a.iters - 1)
             _, _, lse = spo.spo_logprobs_fwd(H, W, tgt, ws=ws_f)

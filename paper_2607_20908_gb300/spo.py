@@ -323,6 +323,7 @@ SPO_TUNE_PAIR_MMA = 0
 SPO_TUNE_GROUP_M = 1
 SPO_TUNE_RASTER = 2
 SPO_TUNE_DYNAMIC_MASK = 3
+SPO_TUNE_DW_SPLIT_ROWS = 4
 
 
 def spo_set_tuning(key: int, value: int):

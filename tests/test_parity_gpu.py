@@ -196,3 +196,14 @@ def test_two_rollout_group_and_long_window():
     case = inputs.tiny_case(seed=1111, T_per_seq=300, n_groups=3, rollouts=2, d=128, V=1024)
     case["window"] = 256
     _compare(case)
+
+
+def test_dw_split_passes():
+    """dW reduced over token passes of 256 rows (several reduce-add passes per chunk)."""
+    from paper_2607_20908_gb300 import spo
+    spo.spo_set_tuning(spo.SPO_TUNE_DW_SPLIT_ROWS, 256)
+    try:
+        case = inputs.tiny_case(seed=1121, T_per_seq=125, n_groups=2, rollouts=4, d=320, V=5000)
+        _compare(case)
+    finally:
+        spo.spo_set_tuning(spo.SPO_TUNE_DW_SPLIT_ROWS, 8192)
