@@ -78,9 +78,9 @@ SAMPLE_SEQS, SAMPLE_TOKENS = 8, 8   # CPU sample: one group of 8 rollouts, first
 # DRAM bytes (read + write) per launch of each tensor-core kernel on this workload, from one
 # `ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum` capture of this command
 # (profiles/launches_full_workload.md), valid only for the kernel sources they were taken on.
-TRAFFIC = {"sources_sha256_16": "6bc21f98b1841f5a",
-           "bytes": {"logits_lse_fwd": 6.942e9, "logits_grad_recompute": 12.863e9,
-                     "gemm_dH": 83.132e9, "gemm_dW": 67.302e9}}
+TRAFFIC = {"sources_sha256_16": "1a250a0dc6cf6892",
+           "bytes": {"logits_lse_fwd": 6.964e9, "logits_grad_recompute": 13.367e9,
+                     "gemm_dH": 90.246e9, "gemm_dW": 20.725e9}}
 KERNEL_SOURCES = ["paper_2607_20908_gb300/csrc/gemm.cu", "paper_2607_20908_gb300/csrc/tc.cuh",
                   "paper_2607_20908_gb300/csrc/internal.h"]
 
@@ -524,7 +524,10 @@ def ours(args):
         k["avg_ms"] = k["total_ms"] / k["launches"]
         k["share_of_step"] = k["total_ms"] / ms
         if name in GEMM_KINDS:
-            k["tflops"] = flop_gemm / (k["avg_ms"] / 1e3) / 1e12
+            # a GEMM may run as several launches per step (token chunks, dW passes)
+            k["launches_per_step"] = k["launches"] / args.steps
+            k["flop_per_launch"] = flop_gemm / k["launches_per_step"]
+            k["tflops"] = k["flop_per_launch"] / (k["avg_ms"] / 1e3) / 1e12
         elif name in hbm_bytes:
             k["gbs"] = hbm_bytes[name] / (k["avg_ms"] / 1e3) / 1e9
             k["frac_of_hbm"] = k["gbs"] / pk["hbm"]
@@ -539,18 +542,19 @@ def ours(args):
                 "peak": pk["bf16_sustained"], "unit": "TFLOP/s", "frac": achieved / pk["bf16_sustained"],
                 "peak_kind": f"bf16 dense sustained, {pk['source']}",
                 "frac_of_burst": achieved / pk["bf16_burst"],
-                "flop_per_launch": flop_gemm, "traffic": kernel_traffic(dom_name),
+                "flop_per_launch": dom["flop_per_launch"], "traffic": kernel_traffic(dom_name),
                 "traffic_unit": "bytes per launch (ncu dram__bytes_read.sum + dram__bytes_write.sum)",
                 "algorithmic_bytes": None}
     alg = {"logits_lse_fwd": 2 * T_L * st.d + 2 * st.V * st.d + 16 * T_L * ((st.V + 255) // 256),
            "logits_grad_recompute": 2 * T_L * st.d + 2 * st.V * st.d + 2 * T_L * st.V,
            "gemm_dH": 2 * T_L * st.V + 2 * st.V * st.d + 2 * T_L * st.d,
            "gemm_dW": 2 * T_L * st.V + 2 * T_L * st.d + 4 * st.V * st.d}
-    roofline["algorithmic_bytes"] = alg[dom_name]
+    # per launch: a step's operand and output bytes spread over its launches of that GEMM
+    roofline["algorithmic_bytes"] = alg[dom_name] / dom["launches_per_step"]
     for name, k in kern.items():
         if name in alg:
             k["dram_bytes_ncu"] = kernel_traffic(name)
-            k["algorithmic_bytes"] = alg[name]
+            k["algorithmic_bytes"] = alg[name] / k["launches_per_step"]
 
     # e2e: host buffers, H2D + step + D2H inside the timed region
     hio = HostIO(st)

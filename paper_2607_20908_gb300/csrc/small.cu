@@ -148,41 +148,47 @@ __device__ __forceinline__ void lse_merge(float& m, float& s, float& e, float m2
   }
 }
 
-constexpr int kCombineWarps = 16;
+constexpr int kCombineRows = 16;   // rows per block: 1024 blocks at T = 16384 balance 152 SMs
+constexpr int kCombineGroups = 16; // split groups per row (8 warps x 2 half-warps)
 
-// Split-vocabulary combine: 32 rows per block (one contiguous [nsplit][32]
-// slab of partials), warp w merges vocab tiles w, w + 16, ...; the per-warp
-// results are merged through shared memory.
-__global__ void __launch_bounds__(kCombineWarps * 32) lse_combine_kernel(
-    const float4* partials, int nsplit, const float* ztgt, const int* idx, const int* count,
-    float* logp, float* entropy, float* lse_out) {
-  __shared__ float sm[kCombineWarps][32][3];
+// Split-vocabulary combine.  A block owns 16 rows; half-warp h of warp w
+// merges vocab tiles 2w + h, 2w + h + 16, ... of those rows (each load is a
+// contiguous 256-byte run of the row-block-major partials), and the 16
+// per-group results are merged through shared memory.
+__global__ void __launch_bounds__(256) lse_combine_kernel(const float4* partials, int nsplit,
+                                                          const float* ztgt, const int* idx,
+                                                          const int* count, float* logp,
+                                                          float* entropy, float* lse_out) {
+  __shared__ float sm[kCombineGroups][kCombineRows][3];
   const int n = *count;
-  const int row0 = blockIdx.x * 32;
+  const int row0 = blockIdx.x * kCombineRows;
   if (row0 >= n) return;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int row = row0 + lane;
+  const int r = lane & 15, grp = warp * 2 + (lane >> 4);
+  const int row = row0 + r;
   float m = -INFINITY, s = 0.f, e = 0.f;
   if (row < n) {
-    const float4* slab = partials + static_cast<size_t>(blockIdx.x) * nsplit * 32 + lane;
+    const float4* slab = partials + static_cast<size_t>(row >> 5) * nsplit * 32 + (row & 31);
 #pragma unroll 8
-    for (int j = warp; j < nsplit; j += kCombineWarps) {
+    for (int j = grp; j < nsplit; j += kCombineGroups) {
       const float4 pr = slab[static_cast<size_t>(j) * 32];
       lse_merge(m, s, e, pr.x, pr.y, pr.z);
     }
   }
-  sm[warp][lane][0] = m;
-  sm[warp][lane][1] = s;
-  sm[warp][lane][2] = e;
+  sm[grp][r][0] = m;
+  sm[grp][r][1] = s;
+  sm[grp][r][2] = e;
   __syncthreads();
-  if (warp == 0 && row < n) {
-    for (int w = 1; w < kCombineWarps; ++w)
-      lse_merge(m, s, e, sm[w][lane][0], sm[w][lane][1], sm[w][lane][2]);
-    const float lse2 = m + log2f(s);
+  if (threadIdx.x < kCombineRows && row0 + static_cast<int>(threadIdx.x) < n) {
+    const int rr = threadIdx.x;
+    float M = sm[0][rr][0], S = sm[0][rr][1], E = sm[0][rr][2];
+    for (int g = 1; g < kCombineGroups; ++g) lse_merge(M, S, E, sm[g][rr][0], sm[g][rr][1], sm[g][rr][2]);
+    const float lse2 = M + log2f(S);
     const float lse_nat = lse2 * kLn2;
-    const int t = idx[row];
-    logp[t] = ztgt[row] - lse_nat;
-    if (entropy) entropy[t] = (lse2 - e / s) * kLn2;
+    const int crow = row0 + rr;
+    const int t = idx[crow];
+    logp[t] = ztgt[crow] - lse_nat;
+    if (entropy) entropy[t] = (lse2 - E / S) * kLn2;
     if (lse_out) lse_out[t] = lse_nat;
   }
 }
@@ -508,9 +514,8 @@ cudaError_t launch_gather(const __nv_bfloat16* H, int d, const int* idx, const i
 cudaError_t launch_lse_combine(const float4* partials, int nsplit, const float* ztgt,
                                const int* idx, const int* count, int rows_cap, float* logp,
                                float* entropy, float* lse, cudaStream_t s) {
-  const int blocks = (rows_cap + 31) / 32;
-  lse_combine_kernel<<<blocks, kCombineWarps * 32, 0, s>>>(partials, nsplit, ztgt, idx, count,
-                                                           logp, entropy, lse);
+  const int blocks = (rows_cap + kCombineRows - 1) / kCombineRows;
+  lse_combine_kernel<<<blocks, 256, 0, s>>>(partials, nsplit, ztgt, idx, count, logp, entropy, lse);
   note_launches(1);
   return cudaGetLastError();
 }
