@@ -101,7 +101,7 @@ struct FwdWs {
   int* tgt_c;
   float* ztgt;
   __nv_bfloat16* Hc;
-  float4* partials;
+  float* partials;
   long long T_pad;
   int nsplit;
   size_t bytes;
@@ -126,7 +126,8 @@ FwdWs carve_fwd(void* base, long long T, long long d, long long V) {
   w.tgt_c = reinterpret_cast<int*>(take(sizeof(int) * w.T_pad));
   w.ztgt = reinterpret_cast<float*>(take(sizeof(float) * w.T_pad));
   w.Hc = reinterpret_cast<__nv_bfloat16*>(take(sizeof(__nv_bfloat16) * w.T_pad * d));
-  w.partials = reinterpret_cast<float4*>(take(sizeof(float4) * w.nsplit * w.T_pad));
+  w.partials = reinterpret_cast<float*>(
+      take(sizeof(float) * spo::kPartialBlock / 32 * w.nsplit * w.T_pad));
   w.bytes = off;
   return w;
 }

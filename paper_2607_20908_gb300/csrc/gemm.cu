@@ -114,8 +114,11 @@ __device__ __forceinline__ void epi_lse(const GemmArgs& p, uint32_t taddr, int r
     run_m = nm;
   }
   if (row_ok) {
-    p.partials[(static_cast<size_t>(row >> 5) * p.nsplit + nb) * 32 + (row & 31)] =
-        make_float4(run_m, run_s, run_e, 0.f);
+    float* q = p.partials + (static_cast<size_t>(row >> 5) * p.nsplit + nb) * kPartialBlock +
+               (row & 31);
+    q[0] = run_m;    // each of the three stores is one 128-byte line per warp
+    q[32] = run_s;
+    q[64] = run_e;
     if (hit) p.ztgt[row] = zt;
   }
 }

@@ -18,6 +18,8 @@ constexpr int BK = 64;
 // Compacted row buffers are padded (and zero-filled) to this many rows so a
 // pair tile never reads rows past the buffer.
 constexpr int kRowPad = 256;
+// Floats of logsumexp partials per 32 rows and vocab tile: three planes of 32.
+constexpr int kPartialBlock = 96;
 
 // What the epilogue does with a finished 128 x 256 fp32 accumulator tile.
 enum EpiKind : int {
@@ -45,9 +47,9 @@ struct GemmArgs {
   float scale;  // inv_temp for EPI_LSE / EPI_GRAD
   // EPI_LSE
   const int* tgt;     // target id of each row
-  // Per (row, vocab tile) partials (max*log2e, sum 2^(t-max), sum 2^(t-max) t, 0), laid out
-  // [row / 32][vocab tile][row % 32]: a warp's 32 rows of one tile are 512 contiguous bytes.
-  float4* partials;
+  // Per (row, vocab tile) partials m = max*log2e, s = sum 2^(t-m), e = sum 2^(t-m) t, laid out
+  // [row / 32][vocab tile][m, s, e][row % 32] (kPartialBlock floats per 32 rows and tile).
+  float* partials;
   int nsplit;  // number of vocab tiles, ceil(n / BN)
   float* ztgt;        // target logit (natural units) of each row
   // EPI_GRAD
@@ -104,7 +106,7 @@ cudaError_t launch_gather(const __nv_bfloat16* H, int d, const int* idx, const i
                           const float* a, float* a_c, const float* b, float* b_c,
                           cudaStream_t s);
 
-cudaError_t launch_lse_combine(const float4* partials, int nsplit,
+cudaError_t launch_lse_combine(const float* partials, int nsplit,
                                const float* ztgt, const int* idx, const int* count,
                                int rows_cap, float* logp, float* entropy, float* lse,
                                cudaStream_t s);

@@ -150,12 +150,14 @@ __device__ __forceinline__ void lse_merge(float& m, float& s, float& e, float m2
 
 constexpr int kCombineRows = 16;   // rows per block: 1024 blocks at T = 16384 balance 152 SMs
 constexpr int kCombineGroups = 16; // split groups per row (8 warps x 2 half-warps)
+constexpr int kCombineUnroll = 4;  // vocab tiles whose loads a thread has in flight at once
 
 // Split-vocabulary combine.  A block owns 16 rows; half-warp h of warp w
-// merges vocab tiles 2w + h, 2w + h + 16, ... of those rows (each load is a
-// contiguous 256-byte run of the row-block-major partials), and the 16
-// per-group results are merged through shared memory.
-__global__ void __launch_bounds__(256) lse_combine_kernel(const float4* partials, int nsplit,
+// merges vocab tiles 2w + h, 2w + h + 16, ... of those rows in ascending
+// order (each load is a contiguous 64-byte run of one plane of the
+// row-block-major partials), and the 16 per-group results are merged through
+// shared memory.  The partials are read once, so the loads stream past L1/L2.
+__global__ void __launch_bounds__(256) lse_combine_kernel(const float* partials, int nsplit,
                                                           const float* ztgt, const int* idx,
                                                           const int* count, float* logp,
                                                           float* entropy, float* lse_out) {
@@ -168,11 +170,23 @@ __global__ void __launch_bounds__(256) lse_combine_kernel(const float4* partials
   const int row = row0 + r;
   float m = -INFINITY, s = 0.f, e = 0.f;
   if (row < n) {
-    const float4* slab = partials + static_cast<size_t>(row >> 5) * nsplit * 32 + (row & 31);
-#pragma unroll 8
-    for (int j = grp; j < nsplit; j += kCombineGroups) {
-      const float4 pr = slab[static_cast<size_t>(j) * 32];
-      lse_merge(m, s, e, pr.x, pr.y, pr.z);
+    const float* slab = partials + static_cast<size_t>(row >> 5) * nsplit * kPartialBlock + (row & 31);
+    int j = grp;
+    for (; j + (kCombineUnroll - 1) * kCombineGroups < nsplit; j += kCombineUnroll * kCombineGroups) {
+      float pm[kCombineUnroll], ps[kCombineUnroll], pe[kCombineUnroll];
+#pragma unroll
+      for (int u = 0; u < kCombineUnroll; ++u) {
+        const float* q = slab + static_cast<size_t>(j + u * kCombineGroups) * kPartialBlock;
+        pm[u] = __ldcs(q);
+        ps[u] = __ldcs(q + 32);
+        pe[u] = __ldcs(q + 64);
+      }
+#pragma unroll
+      for (int u = 0; u < kCombineUnroll; ++u) lse_merge(m, s, e, pm[u], ps[u], pe[u]);
+    }
+    for (; j < nsplit; j += kCombineGroups) {
+      const float* q = slab + static_cast<size_t>(j) * kPartialBlock;
+      lse_merge(m, s, e, __ldcs(q), __ldcs(q + 32), __ldcs(q + 64));
     }
   }
   sm[grp][r][0] = m;
@@ -511,7 +525,7 @@ cudaError_t launch_gather(const __nv_bfloat16* H, int d, const int* idx, const i
   return cudaGetLastError();
 }
 
-cudaError_t launch_lse_combine(const float4* partials, int nsplit, const float* ztgt,
+cudaError_t launch_lse_combine(const float* partials, int nsplit, const float* ztgt,
                                const int* idx, const int* count, int rows_cap, float* logp,
                                float* entropy, float* lse, cudaStream_t s) {
   const int blocks = (rows_cap + kCombineRows - 1) / kCombineRows;
