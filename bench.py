@@ -419,23 +419,26 @@ def run_cpu_baseline(st: Step, budget_s: float = 12.0):
 
 
 def read_ceiling_gbs(dev, nbytes, reps=15):
-    """Achievable DRAM read rate for one transfer of nbytes: a library reduction
-    (torch.sum) over that many fp32 bytes, each rep after a 256 MB write that
-    evicts L2, timed with CUDA events like the library's own launches.  The
-    measured copy peak is reached only by multi-GB transfers; this is the
-    denominator's value at the size a small HBM-bound step actually moves."""
-    x = torch.rand(max(1, nbytes // 4), device=dev)
+    """Achievable DRAM rate for one transfer of nbytes: a library copy
+    (torch's vectorised copy kernel) that reads nbytes / 2 and writes
+    nbytes / 2 -- the same kind of transfer as the measured copy peak, at the
+    size a small HBM-bound step actually moves.  Each rep follows a 256 MB
+    write that evicts L2; CUDA events as for the library's own launches.
+    The copy peak itself is reached only by multi-GB transfers."""
+    n = max(1, nbytes // 8)
+    x = torch.rand(n, device=dev)
+    y = torch.empty_like(x)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
           for _ in range(reps)]
     for i, (a, b) in enumerate(ev):
         flush.fill_(i & 0xFF)
         a.record()
-        torch.sum(x)
+        y.copy_(x)
         b.record()
     torch.cuda.synchronize(dev)
     ms = sorted(a.elapsed_time(b) for a, b in ev[3:])[(reps - 3) // 2]
-    return x.numel() * 4 / (ms / 1e3) / 1e9
+    return 2 * n * 4 / (ms / 1e3) / 1e9
 
 
 def aux_measurements(dev, pk):

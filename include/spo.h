@@ -316,6 +316,64 @@ SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32
                                        int accumulate_dW, void* ws, size_t ws_bytes, void* stream);
 
 /* ---------------------------------------------------------------------------
+ * Vocabulary-split form of a2/a3 and a6-a8: the LM head's V rows split into
+ * contiguous slices, one per GPU (tensor-parallel LM head).  The paper trains
+ * on two GPUs (section 3, "Base Models") without describing this split; it is
+ * the form of the path that shards W instead of the batch.  Because the
+ * softmax normaliser couples all V logits of a token, the slices exchange one
+ * 16-byte record per token in the forward and sum their dH in the backward:
+ *
+ *   rank k:  rec_k = spo_logprobs_fwd_slice(H, W[v0_k : v0_k + V_k], ...)
+ *   all:     all-gather rec_0 .. rec_{R-1} (T x 16 bytes each)
+ *            spo_logprobs_merge_slices -> logp, entropy, lse (identical on every rank)
+ *            spo_policy_loss_fwd as in the unsplit path
+ *   rank k:  spo_policy_loss_bwd_slice -> dH_k (fp32), dW[v0_k : v0_k + V_k]
+ *   all:     all-reduce (sum) of dH_k -> dH; dW stays sharded with W
+ *
+ * The three calls run on any device; nothing here communicates.
+ *
+ * spo_logprobs_fwd_slice: the forward over vocabulary rows [v_offset,
+ * v_offset + V_slice) of the full head, W_slice pointing at row v_offset.
+ * Sizes, alignment, mask and workspace (spo_logprobs_workspace_size(T, d,
+ * V_slice)) as in spo_logprobs_fwd with V = V_slice; 0 <= v_offset.  tgt holds
+ * ids of the full vocabulary.  Writes rec float32[T][4], 16-byte aligned: for a
+ * kept token, with u = z log2(e) over the slice's logits,
+ *   rec[t] = { max u,  sum 2^(u - max u),  sum 2^(u - max u) u,
+ *              z[tgt[t]] if tgt[t] is in the slice, else -inf }
+ * and {0, 0, 0, 0} for a skipped token (mask 0 or tgt < 0).
+ * ------------------------------------------------------------------------- */
+SPO_API spo_status spo_logprobs_fwd_slice(const void* H, const void* W_slice, const int32_t* tgt,
+                                          const uint8_t* mask, int64_t T, int64_t d,
+                                          int64_t V_slice, int64_t v_offset, float inv_temp,
+                                          float* rec, void* ws, size_t ws_bytes, void* stream);
+
+/* spo_logprobs_merge_slices: rec float32[n_slices][T][4] (the slices' records
+ * back to back, in any slice order) -> logp, entropy, lse exactly as
+ * spo_logprobs_fwd defines them over the union of the slices.  A token whose
+ * records all have a zero second entry (skipped) gets 0.  The slices must
+ * together cover the vocabulary once and contain every kept token's target
+ * (otherwise that token's logp is -inf).  entropy and lse may be NULL;
+ * 1 <= n_slices <= 1024, 1 <= T <= 2^24. */
+SPO_API spo_status spo_logprobs_merge_slices(const float* rec, int32_t n_slices, int64_t T,
+                                             float* logp, float* entropy, float* lse,
+                                             void* stream);
+
+/* spo_policy_loss_bwd_slice: the backward restricted to the slice's columns of
+ * G, with lse the full-vocabulary lse from spo_logprobs_merge_slices:
+ *   G_k     = inv_temp * g[t] * (1[v0 + j == tgt[t]] - exp(z_t[v0 + j] - lse[t])), j < V_slice
+ *   dH_part = G_k W_slice   fp32[T, d] out (the slices' parts sum to dH; NULL to skip)
+ *   dW_slice = G_k^T H      fp32[V_slice, d] out (+= if accumulate_dW; NULL to skip)
+ * Arguments otherwise as in spo_policy_loss_bwd with V = V_slice; workspace
+ * spo_policy_loss_bwd_workspace_size(T, d, V_slice).  Rows with g[t] == 0 get
+ * dH_part = 0. */
+SPO_API spo_status spo_policy_loss_bwd_slice(const void* H, const void* W_slice,
+                                             const int32_t* tgt, const float* lse, const float* g,
+                                             int64_t T, int64_t d, int64_t V_slice,
+                                             int64_t v_offset, float inv_temp, float* dH_part,
+                                             float* dW_slice, int accumulate_dW, void* ws,
+                                             size_t ws_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------
  * spo_policy_loss_fwd without a caller workspace.  The paper has no
  * counterpart: this is a convenience for callers that cannot hand out device
  * scratch memory -- for example code running under a framework whose memory
@@ -359,7 +417,8 @@ SPO_API spo_status spo_policy_loss_fwd_noalloc(const float* logp, const float* o
  *   2 = dH = G W (a7), 3 = dW = G^T H (a8), 4 = split-vocab combine (a3),
  *   5 = forward row selection + gather, 6 = backward row selection + gather,
  *   7 = policy-loss forward (a5), 8 = group advantages (a4),
- *   9 = token selection (a1), 10 = reward composition.
+ *   9 = token selection (a1), 10 = reward composition, 11 = ranker,
+ *   12 = merge of vocabulary-slice records.
  * spo_launch_count: kernels launched by this library since it was loaded
  *   (host-side counter; every kernel launch adds one).
  * ------------------------------------------------------------------------- */

@@ -123,6 +123,60 @@ def logprobs(H, W, tgt, inv_temp: float = 1.0, mask=None):
 
 
 # --------------------------------------------------------------------------
+# a2/a3 with the vocabulary split into slices (LM-head rows per device)
+# --------------------------------------------------------------------------
+def logprobs_slice_record(H, W_slice, v_offset: int, tgt, inv_temp: float = 1.0, mask=None):
+    """What one vocabulary slice [v_offset, v_offset + V_slice) knows of each token:
+    (max_v z, sum_v exp(z - max), sum_v exp(z - max) z, z[y] if y is in the slice
+    else -inf), z over the slice's logits only.  Skipped tokens: (0, 0, 0, 0).
+    Returns fp64 [T, 4]."""
+    T = H.shape[0]
+    tgt = np.asarray(tgt).astype(np.int64)
+    keep = tgt >= 0
+    if mask is not None:
+        keep &= np.asarray(mask).astype(np.int64) == 1
+    rows = np.nonzero(keep)[0]
+    rec = np.zeros((T, 4))
+    if rows.size == 0:
+        return rec
+    z = logits(H[rows], W_slice, inv_temp)                 # [n, V_slice]
+    m = z.max(axis=1)
+    w = np.exp(z - m[:, None])
+    rec[rows, 0] = m
+    rec[rows, 1] = w.sum(axis=1)
+    rec[rows, 2] = (w * z).sum(axis=1)
+    local = tgt[rows] - v_offset
+    hit = (local >= 0) & (local < W_slice.shape[0])
+    zt = np.full(rows.size, -np.inf)
+    zt[hit] = z[np.nonzero(hit)[0], local[hit]]
+    rec[rows, 3] = zt
+    return rec
+
+
+def merge_slice_records(recs):
+    """(logp, entropy, lse) from the records of slices that together cover the
+    vocabulary once: with M = max_k m_k and S = sum_k s_k exp(m_k - M),
+    lse = M + log S; sum_v p_v z_v = (sum_k e_k exp(m_k - M)) / S; the target
+    logit is the one finite z[y].  Tokens whose records are all empty get 0."""
+    recs = np.asarray(recs, dtype=np.float64)              # [R, T, 4]
+    T = recs.shape[1]
+    logp, ent, lse = np.zeros(T), np.zeros(T), np.zeros(T)
+    live = recs[:, :, 1] > 0
+    for t in range(T):
+        k = np.nonzero(live[:, t])[0]
+        if k.size == 0:
+            continue
+        m, s, e, zt = recs[k, t, 0], recs[k, t, 1], recs[k, t, 2], recs[k, t, 3]
+        M = m.max()
+        S = (s * np.exp(m - M)).sum()
+        E = (e * np.exp(m - M)).sum()
+        lse[t] = M + math.log(S)
+        logp[t] = zt.max() - lse[t]
+        ent[t] = lse[t] - E / S
+    return logp, ent, lse
+
+
+# --------------------------------------------------------------------------
 # a4: group-normalised advantage (the definition of A_hat under Eq. 3)
 # --------------------------------------------------------------------------
 def group_advantages(rewards, group_id, n_groups: int, std_mode: int = STD_UNBIASED,
@@ -295,6 +349,34 @@ def policy_loss_bwd(H, W, tgt, g, inv_temp: float = 1.0):
     onehot[np.arange(rows.size), tgt[rows]] = 1.0
     G = inv_temp * g[rows][:, None] * (onehot - p)
     dH[rows] = G @ W
+    dW = G.T @ H[rows]
+    return dH, dW
+
+
+def policy_loss_bwd_slice(H, W_slice, v_offset: int, tgt, lse, g, inv_temp: float = 1.0):
+    """One vocabulary slice's share of the backward: G restricted to columns
+    [v_offset, v_offset + V_slice), G[t, j] = tau^-1 g_t (1[v_offset + j == y_t]
+    - exp(z_t[v_offset + j] - lse_t)) with the full-vocabulary lse.  Returns
+    (dH part = G W_slice [T, d], dW rows of the slice = G^T H [V_slice, d]);
+    the parts of all slices sum to policy_loss_bwd's dH."""
+    T, d = H.shape
+    Vs = W_slice.shape[0]
+    tgt = np.asarray(tgt).astype(np.int64)
+    g = np.asarray(g, dtype=np.float64)
+    lse = np.asarray(lse, dtype=np.float64)
+    rows = np.nonzero(g != 0.0)[0]
+    dH = np.zeros((T, d))
+    dW = np.zeros((Vs, d))
+    if rows.size == 0:
+        return dH, dW
+    z = logits(H[rows], W_slice, inv_temp)
+    p = np.exp(z - lse[rows][:, None])
+    onehot = np.zeros_like(p)
+    local = tgt[rows] - v_offset
+    hit = np.nonzero((local >= 0) & (local < Vs))[0]
+    onehot[hit, local[hit]] = 1.0
+    G = inv_temp * g[rows][:, None] * (onehot - p)
+    dH[rows] = G @ W_slice
     dW = G.T @ H[rows]
     return dH, dW
 

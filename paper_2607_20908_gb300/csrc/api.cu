@@ -249,6 +249,7 @@ enum TraceKind : int {
   kTraceTokenSelect = 9,
   kTraceReward = 10,
   kTraceRanker = 11,
+  kTraceMergeSlices = 12,
 };
 
 // counters: the workspace's four tile counters (the one of this kind is
@@ -289,6 +290,200 @@ int grid_for(const DevInfo& di, long long max_m, long long n) {
 }
 
 uint32_t b_box_rows() { return static_cast<uint32_t>(spo::gemm_b_box_rows(g_tune_pair != 0)); }
+
+// a1 selection + gather, a2 and a3 over vocabulary rows [v_offset, v_offset + V)
+// (W points at row v_offset).  rec == NULL: logp / entropy / lse; otherwise the
+// slice records.  Arguments are validated by the caller.
+spo_status logprobs_impl(const void* H, const void* W, const int32_t* tgt, const uint8_t* mask,
+                         int64_t T, int64_t d, int64_t V, int64_t v_offset, float inv_temp,
+                         float* logp, float* entropy, float* lse, float* rec, void* ws,
+                         cudaStream_t s) {
+  spo_status st;
+  DevInfo di;
+  if ((st = device_info(&di)) != SPO_OK) return st;
+  const FwdWs w = carve_fwd(ws, T, d, V);
+
+  // a1 (row selection) + gather of the kept rows into a dense bf16 block
+  st = traced(kTraceSelectGatherFwd, s, "compact/gather", [&] {
+    cudaError_t e = spo::launch_compact(0, mask, tgt, nullptr, T, w.scratch, w.idx, w.count, s);
+    if (e != cudaSuccess) return e;
+    return spo::launch_gather(static_cast<const __nv_bfloat16*>(H), static_cast<int>(d), w.idx,
+                              w.count, static_cast<int>(w.T_pad), w.Hc, tgt, w.tgt_c, v_offset, V,
+                              nullptr, nullptr, nullptr, nullptr, s);
+  });
+  if (st != SPO_OK) return st;
+  // a2: logits tile by tile + online logsumexp partials
+  CUtensorMap ta, tb;
+  SPO_CUDA(spo::make_tmap_bf16(&ta, w.Hc, d, w.T_pad, d * 2, spo::BK, spo::BM), "tensor map H");
+  SPO_CUDA(spo::make_tmap_bf16(&tb, W, d, V, d * 2, spo::BK, b_box_rows()), "tensor map W");
+  spo::GemmArgs a = base_args(di);
+  a.m_count = w.count;
+  a.m_offset = 0;
+  a.m_cap = static_cast<int>(w.T_pad);
+  a.n = static_cast<int>(V);
+  a.k_static = static_cast<int>(d);
+  a.scale = inv_temp;
+  a.tgt = w.tgt_c;
+  a.partials = w.partials;
+  a.nsplit = w.nsplit;
+  a.ztgt = w.ztgt;
+  if ((st = traced_gemm(spo::EPI_LSE, false, false, ta, tb, ta, a, grid_for(di, w.T_pad, V), s,
+                        w.counters)) !=
+      SPO_OK)
+    return st;
+  // a3: split-vocab combine, scattered back to token positions (skipped tokens read 0)
+  if (rec) {
+    SPO_CUDA(cudaMemsetAsync(rec, 0, sizeof(float) * 4 * T, s), "memset rec");
+  } else {
+    SPO_CUDA(cudaMemsetAsync(logp, 0, sizeof(float) * T, s), "memset logp");
+    if (entropy) SPO_CUDA(cudaMemsetAsync(entropy, 0, sizeof(float) * T, s), "memset entropy");
+    if (lse) SPO_CUDA(cudaMemsetAsync(lse, 0, sizeof(float) * T, s), "memset lse");
+  }
+  st = traced(kTraceLseCombine, s, "combine launch", [&] {
+    return spo::launch_lse_combine(w.partials, w.nsplit, w.ztgt, w.idx, w.count,
+                                   static_cast<int>(w.T_pad), logp, entropy, lse, w.tgt_c,
+                                   reinterpret_cast<float4*>(rec), s);
+  });
+  return st == SPO_OK ? ok() : st;
+}
+
+spo_status check_fwd_ws(int64_t T, int64_t d, int64_t V, const void* ws, size_t ws_bytes) {
+  const FwdWs need = carve_fwd(nullptr, T, d, V);
+  if (!ws || ws_bytes < need.bytes)
+    return fail(SPO_ERR_WORKSPACE, "workspace needs %zu bytes, got %zu", need.bytes, ws_bytes);
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
+    return fail(SPO_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
+  return SPO_OK;
+}
+
+// a6-a8 over vocabulary rows [v_offset, v_offset + V) (W points at row
+// v_offset); dH is bf16, or fp32 with dH_f32.  Arguments are validated by the caller.
+spo_status bwd_impl(const void* H, const void* W, const int32_t* tgt, const float* lse,
+                    const float* g, int64_t T, int64_t d, int64_t V, int64_t v_offset,
+                    float inv_temp, void* dH, bool dH_f32, float* dW, int accumulate_dW, void* ws,
+                    cudaStream_t s) {
+  spo_status st;
+  DevInfo di;
+  if ((st = device_info(&di)) != SPO_OK) return st;
+  const BwdWs w = carve_bwd(ws, T, d, V);
+  if (!dH && !dW) return ok();
+
+  // rows with g != 0 are the only ones with a non-zero gradient row
+  st = traced(kTraceSelectGatherBwd, s, "compact/gather", [&] {
+    cudaError_t e = spo::launch_compact(1, nullptr, nullptr, g, T, w.scratch, w.idx, w.count, s);
+    if (e != cudaSuccess) return e;
+    return spo::launch_gather(static_cast<const __nv_bfloat16*>(H), static_cast<int>(d), w.idx,
+                              w.count, static_cast<int>(w.T_pad), w.Hc, tgt, w.tgt_c, v_offset, V,
+                              lse, w.lse_c, g, w.g_c, s);
+  });
+  if (st != SPO_OK) return st;
+  if (dH)
+    SPO_CUDA(cudaMemsetAsync(dH, 0, (dH_f32 ? sizeof(float) : sizeof(uint16_t)) * T * d, s),
+             "memset dH");
+
+  CUtensorMap tW_k, tW_mn, tG_k, tG_mn;  // operand maps
+  SPO_CUDA(spo::make_tmap_bf16(&tW_k, W, d, V, d * 2, spo::BK, b_box_rows()), "tensor map W");
+  SPO_CUDA(spo::make_tmap_bf16(&tW_mn, W, d, V, d * 2, 64, spo::BK), "tensor map W (MN)");
+  SPO_CUDA(spo::make_tmap_bf16(&tG_k, w.G, V, w.chunk, V * 2, spo::BK, spo::BM), "tensor map G");
+  SPO_CUDA(spo::make_tmap_bf16(&tG_mn, w.G, V, w.chunk, V * 2, 64, spo::BK), "tensor map G (MN)");
+  CUtensorMap tG_store, tdW;
+  SPO_CUDA(spo::make_tmap_bf16(&tG_store, w.G, V, w.chunk, V * 2, 64, spo::kStoreBoxRows),
+           "tensor map G (store)");
+  if (dW)
+    SPO_CUDA(spo::make_tmap_f32(&tdW, dW, d, V, d * 4, 32, spo::kStoreBoxRows), "tensor map dW");
+  else
+    tdW = tG_store;
+
+  const long long n_chunks = (w.T_pad + w.chunk - 1) / w.chunk;
+  for (long long c = 0; c < n_chunks; ++c) {
+    const long long r0 = c * w.chunk;
+    const long long rows = (w.T_pad - r0) < w.chunk ? (w.T_pad - r0) : w.chunk;
+    const __nv_bfloat16* Hc0 = w.Hc + r0 * d;
+    CUtensorMap tH_k, tH_mn;
+    SPO_CUDA(spo::make_tmap_bf16(&tH_k, Hc0, d, rows, d * 2, spo::BK, spo::BM), "tensor map Hc");
+    SPO_CUDA(spo::make_tmap_bf16(&tH_mn, Hc0, d, rows, d * 2, 64, spo::BK), "tensor map Hc (MN)");
+
+    // a6: G = inv_temp * g * (onehot - softmax), logits recomputed
+    spo::GemmArgs a = base_args(di);
+    a.m_count = w.count;
+    a.m_offset = static_cast<int>(r0);
+    a.m_cap = static_cast<int>(w.chunk);
+    a.n = static_cast<int>(V);
+    a.k_static = static_cast<int>(d);
+    a.scale = inv_temp;
+    a.tgt = w.tgt_c + r0;
+    a.lse = w.lse_c + r0;
+    a.gvec = w.g_c + r0;
+    a.G = w.G;
+    a.ldG = V;
+    if ((st = traced_gemm(spo::EPI_GRAD, false, false, tH_k, tW_k, tG_store, a, grid_for(di, rows, V), s,
+                          w.counters)) != SPO_OK)
+      return st;
+    // a7: dH rows = G W, scattered to token rows
+    if (dH) {
+      spo::GemmArgs b = base_args(di);
+      b.m_count = w.count;
+      b.m_offset = static_cast<int>(r0);
+      b.m_cap = static_cast<int>(w.chunk);
+      b.n = static_cast<int>(d);
+      b.k_static = static_cast<int>(V);
+      b.row_idx = w.idx + r0;
+      if (dH_f32)
+        b.out_f32 = static_cast<float*>(dH);
+      else
+        b.out_bf16 = static_cast<__nv_bfloat16*>(dH);
+      b.ld_out = d;
+      if ((st = traced_gemm(spo::EPI_DH, false, true, tG_k, tW_mn, tG_k, b, grid_for(di, rows, d), s,
+                            w.counters)) != SPO_OK)
+        return st;
+    }
+    // a8: dW (+)= G^T Hc over this chunk's rows, in passes of at most
+    // g_tune_dw_split rows (later passes reduce-add into dW)
+    if (dW) {
+      const long long split = g_tune_dw_split > 0 ? g_tune_dw_split : rows;
+      for (long long q0 = 0; q0 < rows; q0 += split) {
+        const long long qrows = (rows - q0) < split ? (rows - q0) : split;
+        CUtensorMap tGq = tG_mn, tHq = tH_mn;
+        if (q0 > 0 || qrows < rows) {
+          SPO_CUDA(spo::make_tmap_bf16(&tGq, w.G + q0 * V, V, qrows, V * 2, 64, spo::BK),
+                   "tensor map G (MN, pass)");
+          SPO_CUDA(spo::make_tmap_bf16(&tHq, Hc0 + q0 * d, d, qrows, d * 2, 64, spo::BK),
+                   "tensor map Hc (MN, pass)");
+        }
+        spo::GemmArgs b = base_args(di);
+        b.m_static = static_cast<int>(V);
+        b.n = static_cast<int>(d);
+        b.k_count = w.count;
+        b.k_offset = static_cast<int>(r0 + q0);
+        b.k_cap = static_cast<int>(qrows);
+        b.out_f32 = dW;
+        b.ld_out = d;
+        b.accumulate = (c == 0 && q0 == 0) ? (accumulate_dW ? 1 : 0) : 1;
+        if ((st = traced_gemm(spo::EPI_DW, true, true, tGq, tHq, tdW, b, grid_for(di, V, d), s,
+                              w.counters)) != SPO_OK)
+          return st;
+      }
+    }
+  }
+  return ok();
+}
+
+
+spo_status check_bwd_args(const void* H, const void* W, const int32_t* tgt, const float* lse,
+                          const float* g, int64_t T, int64_t d, int64_t V, float inv_temp,
+                          const void* dH, const float* dW, const void* ws, size_t ws_bytes) {
+  spo_status st = check_hwv(H, W, tgt, T, d, V, inv_temp);
+  if (st != SPO_OK) return st;
+  if (!lse || !g) return fail(SPO_ERR_INVALID_ARG, "lse and g must be non-NULL");
+  if (dH && !aligned16(dH)) return fail(SPO_ERR_ALIGNMENT, "dH must be 16-byte aligned");
+  if (dW && !aligned16(dW)) return fail(SPO_ERR_ALIGNMENT, "dW must be 16-byte aligned");
+  const BwdWs need = carve_bwd(nullptr, T, d, V);
+  if (!ws || ws_bytes < need.bytes)
+    return fail(SPO_ERR_WORKSPACE, "workspace needs %zu bytes, got %zu", need.bytes, ws_bytes);
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
+    return fail(SPO_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
+  return SPO_OK;
+}
 
 }  // namespace
 
@@ -361,51 +556,38 @@ SPO_API spo_status spo_logprobs_fwd(const void* H, const void* W, const int32_t*
   spo_status st = check_hwv(H, W, tgt, T, d, V, inv_temp);
   if (st != SPO_OK) return st;
   if (!logp) return fail(SPO_ERR_INVALID_ARG, "logp must be non-NULL");
-  const FwdWs need = carve_fwd(nullptr, T, d, V);
-  if (!ws || ws_bytes < need.bytes)
-    return fail(SPO_ERR_WORKSPACE, "workspace needs %zu bytes, got %zu", need.bytes, ws_bytes);
-  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
-    return fail(SPO_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
-  DevInfo di;
-  if ((st = device_info(&di)) != SPO_OK) return st;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const FwdWs w = carve_fwd(ws, T, d, V);
+  if ((st = check_fwd_ws(T, d, V, ws, ws_bytes)) != SPO_OK) return st;
+  return logprobs_impl(H, W, tgt, mask, T, d, V, 0, inv_temp, logp, entropy, lse, nullptr, ws,
+                       static_cast<cudaStream_t>(stream));
+}
 
-  // a1 (row selection) + gather of the kept rows into a dense bf16 block
-  st = traced(kTraceSelectGatherFwd, s, "compact/gather", [&] {
-    cudaError_t e = spo::launch_compact(0, mask, tgt, nullptr, T, w.scratch, w.idx, w.count, s);
-    if (e != cudaSuccess) return e;
-    return spo::launch_gather(static_cast<const __nv_bfloat16*>(H), static_cast<int>(d), w.idx,
-                              w.count, static_cast<int>(w.T_pad), w.Hc, tgt, w.tgt_c, nullptr,
-                              nullptr, nullptr, nullptr, s);
-  });
+SPO_API spo_status spo_logprobs_fwd_slice(const void* H, const void* W_slice, const int32_t* tgt,
+                                          const uint8_t* mask, int64_t T, int64_t d,
+                                          int64_t V_slice, int64_t v_offset, float inv_temp,
+                                          float* rec, void* ws, size_t ws_bytes, void* stream) {
+  spo_status st = check_hwv(H, W_slice, tgt, T, d, V_slice, inv_temp);
   if (st != SPO_OK) return st;
-  // a2: logits tile by tile + online logsumexp partials
-  CUtensorMap ta, tb;
-  SPO_CUDA(spo::make_tmap_bf16(&ta, w.Hc, d, w.T_pad, d * 2, spo::BK, spo::BM), "tensor map H");
-  SPO_CUDA(spo::make_tmap_bf16(&tb, W, d, V, d * 2, spo::BK, b_box_rows()), "tensor map W");
-  spo::GemmArgs a = base_args(di);
-  a.m_count = w.count;
-  a.m_offset = 0;
-  a.m_cap = static_cast<int>(w.T_pad);
-  a.n = static_cast<int>(V);
-  a.k_static = static_cast<int>(d);
-  a.scale = inv_temp;
-  a.tgt = w.tgt_c;
-  a.partials = w.partials;
-  a.nsplit = w.nsplit;
-  a.ztgt = w.ztgt;
-  if ((st = traced_gemm(spo::EPI_LSE, false, false, ta, tb, ta, a, grid_for(di, w.T_pad, V), s,
-                        w.counters)) !=
-      SPO_OK)
-    return st;
-  // a3: split-vocab combine, scattered back to token positions (skipped tokens read 0)
-  SPO_CUDA(cudaMemsetAsync(logp, 0, sizeof(float) * T, s), "memset logp");
-  if (entropy) SPO_CUDA(cudaMemsetAsync(entropy, 0, sizeof(float) * T, s), "memset entropy");
-  if (lse) SPO_CUDA(cudaMemsetAsync(lse, 0, sizeof(float) * T, s), "memset lse");
-  st = traced(kTraceLseCombine, s, "combine launch", [&] {
-    return spo::launch_lse_combine(w.partials, w.nsplit, w.ztgt, w.idx, w.count,
-                                   static_cast<int>(w.T_pad), logp, entropy, lse, s);
+  if (v_offset < 0 || v_offset > (1ll << 31) - 1)
+    return fail(SPO_ERR_SHAPE, "v_offset = %lld outside [0, 2^31)", (long long)v_offset);
+  if (!rec) return fail(SPO_ERR_INVALID_ARG, "rec must be non-NULL");
+  if (!aligned16(rec)) return fail(SPO_ERR_ALIGNMENT, "rec must be 16-byte aligned");
+  if ((st = check_fwd_ws(T, d, V_slice, ws, ws_bytes)) != SPO_OK) return st;
+  return logprobs_impl(H, W_slice, tgt, mask, T, d, V_slice, v_offset, inv_temp, nullptr, nullptr,
+                       nullptr, rec, ws, static_cast<cudaStream_t>(stream));
+}
+
+SPO_API spo_status spo_logprobs_merge_slices(const float* rec, int32_t n_slices, int64_t T,
+                                             float* logp, float* entropy, float* lse,
+                                             void* stream) {
+  if (!rec || !logp) return fail(SPO_ERR_INVALID_ARG, "rec and logp must be non-NULL");
+  if (!aligned16(rec)) return fail(SPO_ERR_ALIGNMENT, "rec must be 16-byte aligned");
+  if (n_slices < 1 || n_slices > 1024)
+    return fail(SPO_ERR_SHAPE, "n_slices = %d outside [1, 1024]", n_slices);
+  if (T < 1 || T > (1ll << 24)) return fail(SPO_ERR_SHAPE, "T = %lld outside [1, 2^24]", (long long)T);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  spo_status st = traced(kTraceMergeSlices, s, "merge launch", [&] {
+    return spo::launch_merge_slices(reinterpret_cast<const float4*>(rec), n_slices, T, logp,
+                                    entropy, lse, s);
   });
   return st == SPO_OK ? ok() : st;
 }
@@ -569,115 +751,25 @@ SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32
                                        const float* lse, const float* g, int64_t T, int64_t d,
                                        int64_t V, float inv_temp, void* dH, float* dW,
                                        int accumulate_dW, void* ws, size_t ws_bytes, void* stream) {
-  spo_status st = check_hwv(H, W, tgt, T, d, V, inv_temp);
+  spo_status st = check_bwd_args(H, W, tgt, lse, g, T, d, V, inv_temp, dH, dW, ws, ws_bytes);
   if (st != SPO_OK) return st;
-  if (!lse || !g) return fail(SPO_ERR_INVALID_ARG, "lse and g must be non-NULL");
-  if (dH && !aligned16(dH)) return fail(SPO_ERR_ALIGNMENT, "dH must be 16-byte aligned");
-  if (dW && !aligned16(dW)) return fail(SPO_ERR_ALIGNMENT, "dW must be 16-byte aligned");
-  const BwdWs need = carve_bwd(nullptr, T, d, V);
-  if (!ws || ws_bytes < need.bytes)
-    return fail(SPO_ERR_WORKSPACE, "workspace needs %zu bytes, got %zu", need.bytes, ws_bytes);
-  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
-    return fail(SPO_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
-  DevInfo di;
-  if ((st = device_info(&di)) != SPO_OK) return st;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const BwdWs w = carve_bwd(ws, T, d, V);
-  if (!dH && !dW) return ok();
+  return bwd_impl(H, W, tgt, lse, g, T, d, V, 0, inv_temp, dH, false, dW, accumulate_dW, ws,
+                  static_cast<cudaStream_t>(stream));
+}
 
-  // rows with g != 0 are the only ones with a non-zero gradient row
-  st = traced(kTraceSelectGatherBwd, s, "compact/gather", [&] {
-    cudaError_t e = spo::launch_compact(1, nullptr, nullptr, g, T, w.scratch, w.idx, w.count, s);
-    if (e != cudaSuccess) return e;
-    return spo::launch_gather(static_cast<const __nv_bfloat16*>(H), static_cast<int>(d), w.idx,
-                              w.count, static_cast<int>(w.T_pad), w.Hc, tgt, w.tgt_c, lse, w.lse_c,
-                              g, w.g_c, s);
-  });
+SPO_API spo_status spo_policy_loss_bwd_slice(const void* H, const void* W_slice,
+                                             const int32_t* tgt, const float* lse, const float* g,
+                                             int64_t T, int64_t d, int64_t V_slice,
+                                             int64_t v_offset, float inv_temp, float* dH_part,
+                                             float* dW_slice, int accumulate_dW, void* ws,
+                                             size_t ws_bytes, void* stream) {
+  spo_status st = check_bwd_args(H, W_slice, tgt, lse, g, T, d, V_slice, inv_temp, dH_part,
+                                 dW_slice, ws, ws_bytes);
   if (st != SPO_OK) return st;
-  if (dH) SPO_CUDA(cudaMemsetAsync(dH, 0, sizeof(uint16_t) * T * d, s), "memset dH");
-
-  CUtensorMap tW_k, tW_mn, tG_k, tG_mn;  // operand maps
-  SPO_CUDA(spo::make_tmap_bf16(&tW_k, W, d, V, d * 2, spo::BK, b_box_rows()), "tensor map W");
-  SPO_CUDA(spo::make_tmap_bf16(&tW_mn, W, d, V, d * 2, 64, spo::BK), "tensor map W (MN)");
-  SPO_CUDA(spo::make_tmap_bf16(&tG_k, w.G, V, w.chunk, V * 2, spo::BK, spo::BM), "tensor map G");
-  SPO_CUDA(spo::make_tmap_bf16(&tG_mn, w.G, V, w.chunk, V * 2, 64, spo::BK), "tensor map G (MN)");
-  CUtensorMap tG_store, tdW;
-  SPO_CUDA(spo::make_tmap_bf16(&tG_store, w.G, V, w.chunk, V * 2, 64, spo::kStoreBoxRows),
-           "tensor map G (store)");
-  if (dW)
-    SPO_CUDA(spo::make_tmap_f32(&tdW, dW, d, V, d * 4, 32, spo::kStoreBoxRows), "tensor map dW");
-  else
-    tdW = tG_store;
-
-  const long long n_chunks = (w.T_pad + w.chunk - 1) / w.chunk;
-  for (long long c = 0; c < n_chunks; ++c) {
-    const long long r0 = c * w.chunk;
-    const long long rows = (w.T_pad - r0) < w.chunk ? (w.T_pad - r0) : w.chunk;
-    const __nv_bfloat16* Hc0 = w.Hc + r0 * d;
-    CUtensorMap tH_k, tH_mn;
-    SPO_CUDA(spo::make_tmap_bf16(&tH_k, Hc0, d, rows, d * 2, spo::BK, spo::BM), "tensor map Hc");
-    SPO_CUDA(spo::make_tmap_bf16(&tH_mn, Hc0, d, rows, d * 2, 64, spo::BK), "tensor map Hc (MN)");
-
-    // a6: G = inv_temp * g * (onehot - softmax), logits recomputed
-    spo::GemmArgs a = base_args(di);
-    a.m_count = w.count;
-    a.m_offset = static_cast<int>(r0);
-    a.m_cap = static_cast<int>(w.chunk);
-    a.n = static_cast<int>(V);
-    a.k_static = static_cast<int>(d);
-    a.scale = inv_temp;
-    a.tgt = w.tgt_c + r0;
-    a.lse = w.lse_c + r0;
-    a.gvec = w.g_c + r0;
-    a.G = w.G;
-    a.ldG = V;
-    if ((st = traced_gemm(spo::EPI_GRAD, false, false, tH_k, tW_k, tG_store, a, grid_for(di, rows, V), s,
-                          w.counters)) != SPO_OK)
-      return st;
-    // a7: dH rows = G W, scattered to token rows
-    if (dH) {
-      spo::GemmArgs b = base_args(di);
-      b.m_count = w.count;
-      b.m_offset = static_cast<int>(r0);
-      b.m_cap = static_cast<int>(w.chunk);
-      b.n = static_cast<int>(d);
-      b.k_static = static_cast<int>(V);
-      b.row_idx = w.idx + r0;
-      b.out_bf16 = static_cast<__nv_bfloat16*>(dH);
-      b.ld_out = d;
-      if ((st = traced_gemm(spo::EPI_DH, false, true, tG_k, tW_mn, tG_k, b, grid_for(di, rows, d), s,
-                            w.counters)) != SPO_OK)
-        return st;
-    }
-    // a8: dW (+)= G^T Hc over this chunk's rows, in passes of at most
-    // g_tune_dw_split rows (later passes reduce-add into dW)
-    if (dW) {
-      const long long split = g_tune_dw_split > 0 ? g_tune_dw_split : rows;
-      for (long long q0 = 0; q0 < rows; q0 += split) {
-        const long long qrows = (rows - q0) < split ? (rows - q0) : split;
-        CUtensorMap tGq = tG_mn, tHq = tH_mn;
-        if (q0 > 0 || qrows < rows) {
-          SPO_CUDA(spo::make_tmap_bf16(&tGq, w.G + q0 * V, V, qrows, V * 2, 64, spo::BK),
-                   "tensor map G (MN, pass)");
-          SPO_CUDA(spo::make_tmap_bf16(&tHq, Hc0 + q0 * d, d, qrows, d * 2, 64, spo::BK),
-                   "tensor map Hc (MN, pass)");
-        }
-        spo::GemmArgs b = base_args(di);
-        b.m_static = static_cast<int>(V);
-        b.n = static_cast<int>(d);
-        b.k_count = w.count;
-        b.k_offset = static_cast<int>(r0 + q0);
-        b.k_cap = static_cast<int>(qrows);
-        b.out_f32 = dW;
-        b.ld_out = d;
-        b.accumulate = (c == 0 && q0 == 0) ? (accumulate_dW ? 1 : 0) : 1;
-        if ((st = traced_gemm(spo::EPI_DW, true, true, tGq, tHq, tdW, b, grid_for(di, V, d), s,
-                              w.counters)) != SPO_OK)
-          return st;
-      }
-    }
-  }
-  return ok();
+  if (v_offset < 0 || v_offset > (1ll << 31) - 1)
+    return fail(SPO_ERR_SHAPE, "v_offset = %lld outside [0, 2^31)", (long long)v_offset);
+  return bwd_impl(H, W_slice, tgt, lse, g, T, d, V_slice, v_offset, inv_temp, dH_part, true,
+                  dW_slice, accumulate_dW, ws, static_cast<cudaStream_t>(stream));
 }
 
 SPO_API spo_status spo_trace_enable(int on) {

@@ -126,7 +126,9 @@ __device__ __forceinline__ void epi_lse(const GemmArgs& p, uint32_t taddr, int r
 __device__ __forceinline__ void epi_dh(const GemmArgs& p, uint32_t taddr, int row, int M, int nb) {
   const bool row_ok = row < M;
   const int out_row = row_ok ? (p.row_idx ? p.row_idx[row] : row) : 0;
-  __nv_bfloat16* dst = p.out_bf16 + static_cast<size_t>(out_row) * p.ld_out;
+  const size_t off = static_cast<size_t>(out_row) * p.ld_out;
+  __nv_bfloat16* dst = p.out_f32 ? nullptr : p.out_bf16 + off;
+  float* dst32 = p.out_f32 ? p.out_f32 + off : nullptr;
   const int col_base = nb * BN;
 #pragma unroll 1
   for (int c = 0; c < BN / 32; ++c) {
@@ -135,6 +137,14 @@ __device__ __forceinline__ void epi_dh(const GemmArgs& p, uint32_t taddr, int ro
     float v[32];
     tmem_ld32(taddr + c * 32, v);
     if (!row_ok) continue;
+    if (p.out_f32) {
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        if (c0 + 4 * q < p.n)
+          *reinterpret_cast<float4*>(dst32 + c0 + 4 * q) =
+              make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+      continue;
+    }
     uint32_t pk[16];
 #pragma unroll
     for (int j = 0; j < 16; ++j) pk[j] = pack_bf16x2(v[2 * j], v[2 * j + 1]);

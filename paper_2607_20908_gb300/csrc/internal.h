@@ -57,7 +57,8 @@ struct GemmArgs {
   const float* gvec;  // dL/dlogp of each row
   __nv_bfloat16* G;   // [rows][ldG]
   long long ldG;
-  // EPI_DH
+  // EPI_DH: rows scattered to row_idx[row], bf16 to out_bf16 or, when out_f32
+  // is set, fp32 to out_f32 (the per-slice partial of the vocabulary split)
   const int* row_idx;         // output row of each row (NULL: identity)
   __nv_bfloat16* out_bf16;
   long long ld_out;
@@ -101,15 +102,26 @@ cudaError_t launch_compact(int kind, const uint8_t* mask, const int* tgt, const 
 
 // Hc[r] = H[idx[r]] for r < count and 0 for count <= r < round_up(count, kRowPad)
 // (r < rows_cap); also gathers up to three per-row vectors (NULL to skip).
+// tgt_c[r] = tgt[idx[r]] - tgt_off when that lies in [0, tgt_lim), else -1 (the
+// target is outside this vocabulary slice: no logit of the slice is the target).
 cudaError_t launch_gather(const __nv_bfloat16* H, int d, const int* idx, const int* count,
                           int rows_cap, __nv_bfloat16* Hc, const int* tgt, int* tgt_c,
-                          const float* a, float* a_c, const float* b, float* b_c,
-                          cudaStream_t s);
+                          long long tgt_off, long long tgt_lim, const float* a, float* a_c,
+                          const float* b, float* b_c, cudaStream_t s);
 
+// Merges each kept row's vocab-tile partials.  With rec == NULL writes logp,
+// entropy, lse at the row's token position; otherwise writes the slice record
+// rec[t] = (m, s, e, z_tgt) (log2 units for m and e; z_tgt natural, -inf when
+// tgt_c < 0) and leaves the three outputs untouched.
 cudaError_t launch_lse_combine(const float* partials, int nsplit,
                                const float* ztgt, const int* idx, const int* count,
                                int rows_cap, float* logp, float* entropy, float* lse,
-                               cudaStream_t s);
+                               const int* tgt_c, float4* rec, cudaStream_t s);
+
+// Merges n_slices slice records per token, rec[k * T + t], into logp, entropy
+// and lse; a token whose records all have s == 0 (skipped) gets 0.
+cudaError_t launch_merge_slices(const float4* rec, int n_slices, long long T, float* logp,
+                                float* entropy, float* lse, cudaStream_t s);
 
 cudaError_t launch_token_select(const int* cu_seqlens, const uint8_t* mask, const int* tgt,
                                 int n_seq, int window, uint8_t* loss_mask, int* n_tok,

@@ -103,8 +103,9 @@ __global__ void compact_write_kernel(int kind, const uint8_t* mask, const int* t
 
 // One warp per compacted row: copy the bf16 row in 16-byte pieces.
 __global__ void gather_kernel(const uint4* H, int row_vecs, const int* idx, const int* count,
-                              int rows_cap, uint4* Hc, const int* tgt, int* tgt_c, const float* a,
-                              float* a_c, const float* b, float* b_c) {
+                              int rows_cap, uint4* Hc, const int* tgt, int* tgt_c,
+                              long long tgt_off, long long tgt_lim, const float* a, float* a_c,
+                              const float* b, float* b_c) {
   const int n = *count;
   const int zero_end = min(rows_cap, (n + kRowPad - 1) / kRowPad * kRowPad);
   const int warps_per_block = blockDim.x >> 5;
@@ -117,7 +118,10 @@ __global__ void gather_kernel(const uint4* H, int row_vecs, const int* idx, cons
       const uint4* src = H + static_cast<size_t>(src_row) * row_vecs;
       for (int i = lane; i < row_vecs; i += 32) dst[i] = src[i];
       if (lane == 0) {
-        if (tgt_c) tgt_c[r] = tgt[src_row];
+        if (tgt_c) {
+          const long long y = static_cast<long long>(tgt[src_row]) - tgt_off;
+          tgt_c[r] = (y >= 0 && y < tgt_lim) ? static_cast<int>(y) : -1;
+        }
         if (a_c) a_c[r] = a[src_row];
         if (b_c) b_c[r] = b[src_row];
       }
@@ -160,7 +164,8 @@ constexpr int kCombineUnroll = 4;  // vocab tiles whose loads a thread has in fl
 __global__ void __launch_bounds__(256) lse_combine_kernel(const float* partials, int nsplit,
                                                           const float* ztgt, const int* idx,
                                                           const int* count, float* logp,
-                                                          float* entropy, float* lse_out) {
+                                                          float* entropy, float* lse_out,
+                                                          const int* tgt_c, float4* rec) {
   __shared__ float sm[kCombineGroups][kCombineRows][3];
   const int n = *count;
   const int row0 = blockIdx.x * kCombineRows;
@@ -197,13 +202,44 @@ __global__ void __launch_bounds__(256) lse_combine_kernel(const float* partials,
     const int rr = threadIdx.x;
     float M = sm[0][rr][0], S = sm[0][rr][1], E = sm[0][rr][2];
     for (int g = 1; g < kCombineGroups; ++g) lse_merge(M, S, E, sm[g][rr][0], sm[g][rr][1], sm[g][rr][2]);
-    const float lse2 = M + log2f(S);
-    const float lse_nat = lse2 * kLn2;
     const int crow = row0 + rr;
     const int t = idx[crow];
+    if (rec) {  // one vocabulary slice: hand the merged partial on
+      rec[t] = make_float4(M, S, E, tgt_c[crow] >= 0 ? ztgt[crow] : -INFINITY);
+      return;
+    }
+    const float lse2 = M + log2f(S);
+    const float lse_nat = lse2 * kLn2;
     logp[t] = ztgt[crow] - lse_nat;
     if (entropy) entropy[t] = (lse2 - E / S) * kLn2;
     if (lse_out) lse_out[t] = lse_nat;
+  }
+}
+
+// Merge of the vocabulary slices' records: one thread per token, slices in
+// ascending order.  The target logit is the one finite z_tgt among them.
+__global__ void merge_slices_kernel(const float4* rec, int n_slices, long long T, float* logp,
+                                    float* entropy, float* lse_out) {
+  const long long t = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (t >= T) return;
+  float m = -INFINITY, s = 0.f, e = 0.f, zt = -INFINITY;
+  for (int k = 0; k < n_slices; ++k) {
+    const float4 q = rec[static_cast<long long>(k) * T + t];
+    if (q.y > 0.f) {
+      lse_merge(m, s, e, q.x, q.y, q.z);
+      zt = fmaxf(zt, q.w);
+    }
+  }
+  if (s > 0.f) {
+    const float lse2 = m + log2f(s);
+    const float lse_nat = lse2 * kLn2;
+    logp[t] = zt - lse_nat;
+    if (entropy) entropy[t] = (lse2 - e / s) * kLn2;
+    if (lse_out) lse_out[t] = lse_nat;
+  } else {
+    logp[t] = 0.f;
+    if (entropy) entropy[t] = 0.f;
+    if (lse_out) lse_out[t] = 0.f;
   }
 }
 
@@ -512,24 +548,36 @@ cudaError_t launch_compact(int kind, const uint8_t* mask, const int* tgt, const 
 
 cudaError_t launch_gather(const __nv_bfloat16* H, int d, const int* idx, const int* count,
                           int rows_cap, __nv_bfloat16* Hc, const int* tgt, int* tgt_c,
-                          const float* a, float* a_c, const float* b, float* b_c, cudaStream_t s) {
+                          long long tgt_off, long long tgt_lim, const float* a, float* a_c,
+                          const float* b, float* b_c, cudaStream_t s) {
   const int row_vecs = d / 8;  // 16-byte pieces per row
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const int blocks = max(1, min((rows_cap + 7) / 8, sms * 8));
   gather_kernel<<<blocks, 256, 0, s>>>(reinterpret_cast<const uint4*>(H), row_vecs, idx, count,
-                                       rows_cap, reinterpret_cast<uint4*>(Hc), tgt, tgt_c, a, a_c,
-                                       b, b_c);
+                                       rows_cap, reinterpret_cast<uint4*>(Hc), tgt, tgt_c,
+                                       tgt_off, tgt_lim, a, a_c, b, b_c);
   note_launches(1);
   return cudaGetLastError();
 }
 
 cudaError_t launch_lse_combine(const float* partials, int nsplit, const float* ztgt,
                                const int* idx, const int* count, int rows_cap, float* logp,
-                               float* entropy, float* lse, cudaStream_t s) {
+                               float* entropy, float* lse, const int* tgt_c, float4* rec,
+                               cudaStream_t s) {
   const int blocks = (rows_cap + kCombineRows - 1) / kCombineRows;
-  lse_combine_kernel<<<blocks, 256, 0, s>>>(partials, nsplit, ztgt, idx, count, logp, entropy, lse);
+  lse_combine_kernel<<<blocks, 256, 0, s>>>(partials, nsplit, ztgt, idx, count, logp, entropy, lse,
+                                            tgt_c, rec);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_merge_slices(const float4* rec, int n_slices, long long T, float* logp,
+                                float* entropy, float* lse, cudaStream_t s) {
+  const long long blocks = (T + 255) / 256;
+  merge_slices_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(rec, n_slices, T, logp,
+                                                                    entropy, lse);
   note_launches(1);
   return cudaGetLastError();
 }

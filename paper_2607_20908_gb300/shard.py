@@ -1,4 +1,6 @@
-"""Data-parallel form of the GRPO step: whole groups per rank.
+"""Multi-GPU forms of the GRPO step.
+
+Data-parallel (``DataParallelStep``): whole groups per rank.
 
 Groups (the g candidates of one task and all their turns, section 3) are
 independent for the advantages and for every per-token term of Eq. 3, so a
@@ -13,9 +15,20 @@ Two things cross ranks:
   * dW = sum over ranks of the weighted local dW (an all-reduce of V x d
     fp32).  dH rows stay on the rank that owns the tokens.
 
-The per-rank compute is an engine object (``SpoEngine`` runs libspo's CUDA
-kernels); the collectives are ``torch.distributed`` on whatever backend the
-process group uses (NCCL between GPUs).
+Vocabulary-parallel (``VocabParallelStep``): the LM head's V rows split into
+contiguous slices, one per rank, the batch replicated.  The softmax
+normaliser couples all V logits of a token, so each rank's forward ends in a
+16-byte record per token (max, sum-exp, sum-exp*z, target logit of its slice);
+one all-gather of T x 16 bytes lets every rank merge the records into the
+full-vocabulary logp / entropy / lse, and the loss is then computed
+redundantly on every rank.  In the backward each rank forms G for its own
+columns: dW stays sharded with W, and dH = sum over ranks of G_k W_k (one
+all-reduce of T x d fp32).
+
+The per-rank compute is an engine object (``SpoEngine`` and
+``SpoVocabEngine`` run libspo's CUDA kernels); the collectives are
+``torch.distributed`` on whatever backend the process group uses (NCCL
+between GPUs).
 """
 
 from __future__ import annotations
@@ -148,3 +161,84 @@ class DataParallelStep:
         dist.all_reduce(loss, group=self.pg)
         dist.all_reduce(dW, group=self.pg)
         return loss, dH, dW
+
+
+def vocab_slices(V: int, world: int, align: int = 8):
+    """Contiguous [offset, offset + size) slices of V rows, one per rank, sizes
+    multiples of `align` (the tensor-map rule for W's rows) and as even as
+    that allows; the first slices take the remainder."""
+    if world < 1:
+        raise ValueError("world must be >= 1")
+    if V % align != 0:
+        raise ValueError(f"V = {V} is not a multiple of {align}")
+    units = V // align
+    if units < world:
+        raise ValueError(f"V = {V} has fewer than {world} blocks of {align} rows")
+    base, extra = divmod(units, world)
+    out, off = [], 0
+    for r in range(world):
+        n = (base + (1 if r < extra else 0)) * align
+        out.append((off, n))
+        off += n
+    return out
+
+
+class SpoVocabEngine:
+    """libspo (CUDA) as the per-rank compute of a vocabulary-parallel step."""
+
+    def __init__(self):
+        from paper_2607_20908_gb300 import spo
+        self.spo = spo
+
+    def forward_slice(self, b: dict):
+        s = self.spo
+        lm, _ = s.spo_token_select(b["cu_seqlens"], b["mask"], b["tgt"], b["window"])
+        rec = s.spo_logprobs_fwd_slice(b["H"], b["W_slice"], b["v_offset"], b["tgt"], lm,
+                                       b["inv_temp"])
+        return lm, rec
+
+    def merge(self, recs):
+        return self.spo.spo_logprobs_merge_slices(recs)
+
+    def loss(self, b: dict, lm, logp, agg: int):
+        s = self.spo
+        adv = s.spo_group_advantages(b["rewards"], b["group_id"], b["n_groups"])
+        loss, g, _ = s.spo_policy_loss_fwd(logp, b["old"], b["ref"], adv, b["cu_seqlens"],
+                                           b["group_id"], b["n_groups"], lm, b["clip_eps"],
+                                           b["kl_beta"], agg)
+        return loss, g
+
+    def backward_slice(self, b: dict, lse, g):
+        return self.spo.spo_policy_loss_bwd_slice(b["H"], b["W_slice"], b["v_offset"], b["tgt"],
+                                                  lse, g, b["inv_temp"])
+
+
+class VocabParallelStep:
+    """One GRPO step with W's rows split over the ranks of a process group.
+
+    run(b) takes this rank's inputs (dict with the whole batch -- H, tgt,
+    mask, cu_seqlens, group_id, n_groups, rewards, old, ref, window,
+    inv_temp, clip_eps, kl_beta -- plus W_slice and v_offset of this rank's
+    rows) and returns (loss, logp, dH, dW_slice): loss, logp and dH are the
+    same on every rank, dW_slice holds the gradient of this rank's rows.
+    Collectives: one all-gather of the per-token records, one all-reduce of
+    dH.
+    """
+
+    def __init__(self, engine, agg: int = AGG_SEQ_GROUP, process_group=None):
+        self.engine = engine
+        self.agg = agg
+        self.pg = process_group
+
+    def run(self, b: dict):
+        import torch.distributed as dist
+        e = self.engine
+        lm, rec = e.forward_slice(b)
+        world = dist.get_world_size(self.pg)
+        parts = [torch.empty_like(rec) for _ in range(world)]
+        dist.all_gather(parts, rec.contiguous(), group=self.pg)
+        logp, _, lse = e.merge(torch.stack(parts))
+        loss, g = e.loss(b, lm, logp, self.agg)
+        dH, dW = e.backward_slice(b, lse, g)
+        dist.all_reduce(dH, group=self.pg)
+        return loss, logp, dH, dW

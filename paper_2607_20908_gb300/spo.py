@@ -63,12 +63,17 @@ _SIGS = {
                               _c_size, _vp], ctypes.c_int),
     "spo_policy_loss_fwd_noalloc": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, _i32, _vp, _i64, _f32,
                                      _f32, ctypes.c_int, _vp, _vp, _vp, _vp], ctypes.c_int),
+    "spo_logprobs_fwd_slice": ([_vp, _vp, _vp, _vp, _i64, _i64, _i64, _i64, _f32, _vp, _vp,
+                                _c_size, _vp], ctypes.c_int),
+    "spo_logprobs_merge_slices": ([_vp, _i32, _i64, _vp, _vp, _vp, _vp], ctypes.c_int),
+    "spo_policy_loss_bwd_slice": ([_vp, _vp, _vp, _vp, _vp, _i64, _i64, _i64, _i64, _f32, _vp,
+                                   _vp, ctypes.c_int, _vp, _c_size, _vp], ctypes.c_int),
 }
 
 TRACE_KINDS = {0: "logits_lse_fwd", 1: "logits_grad_recompute", 2: "gemm_dH", 3: "gemm_dW",
                4: "lse_combine", 5: "select_gather_fwd", 6: "select_gather_bwd",
                7: "policy_loss_fwd", 8: "group_advantages", 9: "token_select",
-               10: "reward_compose", 11: "ranker"}
+               10: "reward_compose", 11: "ranker", 12: "merge_slices"}
 
 
 class SpoError(RuntimeError):
@@ -273,6 +278,75 @@ def spo_policy_loss_bwd(H, W, tgt, lse, g, inv_temp: float = 1.0, dH=None, dW=No
                                      float(inv_temp), _ptr(dH), _ptr(dW), int(bool(accumulate_dW)),
                                      _ptr(w), w.numel(), _stream(dev)))
     return dH, dW
+
+
+def spo_logprobs_fwd_slice(H, W_slice, v_offset: int, tgt, mask=None, inv_temp: float = 1.0,
+                           rec=None, ws=None):
+    """Vocabulary-split a2+a3 over rows [v_offset, v_offset + V_slice) of the
+    head: returns this slice's per-token records, fp32[T, 4]."""
+    dev = H.device
+    T, d = H.shape
+    V = W_slice.shape[0]
+    _need(H, "H", torch.bfloat16, device=dev)
+    _need(W_slice, "W_slice", torch.bfloat16, device=dev)
+    if W_slice.shape[1] != d:
+        raise ValueError(f"W_slice has {W_slice.shape[1]} columns, H has {d}")
+    _need(tgt, "tgt", torch.int32, T, dev)
+    if mask is not None:
+        _need(mask, "mask", torch.uint8, T, dev)
+    if rec is None:
+        rec = torch.empty((T, 4), dtype=torch.float32, device=dev)
+    _need(rec, "rec", torch.float32, T * 4, dev)
+    w = _workspace(logprobs_workspace_size(T, d, V), dev, ws)
+    _check(lib().spo_logprobs_fwd_slice(_ptr(H), _ptr(W_slice), _ptr(tgt), _ptr(mask), T, d, V,
+                                        int(v_offset), float(inv_temp), _ptr(rec), _ptr(w),
+                                        w.numel(), _stream(dev)))
+    return rec
+
+
+def spo_logprobs_merge_slices(rec, want_entropy=True):
+    """rec fp32[n_slices, T, 4] (the slices' records stacked) -> (logp, entropy or None, lse)."""
+    dev = rec.device
+    if rec.dim() != 3 or rec.shape[2] != 4:
+        raise ValueError("rec must have shape [n_slices, T, 4]")
+    n, T = rec.shape[0], rec.shape[1]
+    _need(rec, "rec", torch.float32, n * T * 4, dev)
+    logp = torch.empty(T, dtype=torch.float32, device=dev)
+    ent = torch.empty(T, dtype=torch.float32, device=dev) if want_entropy else None
+    lse = torch.empty(T, dtype=torch.float32, device=dev)
+    _check(lib().spo_logprobs_merge_slices(_ptr(rec), n, T, _ptr(logp), _ptr(ent), _ptr(lse),
+                                           _stream(dev)))
+    return logp, ent, lse
+
+
+def spo_policy_loss_bwd_slice(H, W_slice, v_offset: int, tgt, lse, g, inv_temp: float = 1.0,
+                              dH_part=None, dW_slice=None, accumulate_dW: bool = False,
+                              want_dH=True, want_dW=True, ws=None):
+    """Vocabulary-split a6-a8: returns (this slice's fp32 part of dH [T, d] or
+    None, dW rows of the slice fp32[V_slice, d] or None)."""
+    dev = H.device
+    T, d = H.shape
+    V = W_slice.shape[0]
+    _need(H, "H", torch.bfloat16, device=dev)
+    _need(W_slice, "W_slice", torch.bfloat16, device=dev)
+    _need(tgt, "tgt", torch.int32, T, dev)
+    _need(lse, "lse", torch.float32, T, dev)
+    _need(g, "g", torch.float32, T, dev)
+    if want_dH and dH_part is None:
+        dH_part = torch.empty((T, d), dtype=torch.float32, device=dev)
+    if want_dW and dW_slice is None:
+        dW_slice = (torch.zeros if accumulate_dW else torch.empty)((V, d), dtype=torch.float32,
+                                                                   device=dev)
+    if dH_part is not None:
+        _need(dH_part, "dH_part", torch.float32, T * d, dev)
+    if dW_slice is not None:
+        _need(dW_slice, "dW_slice", torch.float32, V * d, dev)
+    w = _workspace(policy_loss_bwd_workspace_size(T, d, V), dev, ws)
+    _check(lib().spo_policy_loss_bwd_slice(_ptr(H), _ptr(W_slice), _ptr(tgt), _ptr(lse), _ptr(g),
+                                           T, d, V, int(v_offset), float(inv_temp), _ptr(dH_part),
+                                           _ptr(dW_slice), int(bool(accumulate_dW)), _ptr(w),
+                                           w.numel(), _stream(dev)))
+    return dH_part, dW_slice
 
 
 def spo_trace_enable(on: bool = True):

@@ -87,3 +87,25 @@ def test_host_validation_without_gpu(lib):
     bw = lib.spo_policy_loss_bwd
     assert bw(p, p, p, nul, p, 256, 256, 4096, 1.0, p, p, 0, p, 1 << 40, nul) == 1
     assert bw(p, p, p, p, p, 256, 256, 4096, 1.0, ctypes.c_void_p(4098), p, 0, p, 1 << 40, nul) == 3
+
+
+def test_vocab_split_host_validation_without_gpu(lib):
+    p = ctypes.c_void_p(4096)  # never dereferenced: validation fails first
+    nul = ctypes.c_void_p(0)
+    fs = lib.spo_logprobs_fwd_slice
+    assert fs(p, p, p, nul, 256, 256, 2048, 1024, 1.0, nul, p, 1 << 30, nul) == 1
+    assert fs(p, p, p, nul, 256, 256, 2048, 1024, 1.0, ctypes.c_void_p(4100), p, 1 << 30, nul) == 3
+    assert fs(p, p, p, nul, 256, 256, 2048, -8, 1.0, p, p, 1 << 30, nul) == 2
+    assert "v_offset" in _err(lib)[1]
+    assert fs(p, p, p, nul, 256, 256, 128, 0, 1.0, p, p, 1 << 30, nul) == 2
+    assert fs(p, p, p, nul, 256, 256, 2048, 0, 1.0, p, p, 64, nul) == 4
+    mg = lib.spo_logprobs_merge_slices
+    assert mg(p, 0, 256, p, nul, nul, nul) == 2
+    assert mg(p, 2, 0, p, nul, nul, nul) == 2
+    assert mg(ctypes.c_void_p(4104), 2, 256, p, nul, nul, nul) == 3
+    assert mg(p, 2, 256, nul, nul, nul, nul) == 1
+    bs = lib.spo_policy_loss_bwd_slice
+    assert bs(p, p, p, p, p, 256, 256, 2048, -1, 1.0, p, p, 0, p, 1 << 40, nul) == 2
+    assert bs(p, p, p, nul, p, 256, 256, 2048, 0, 1.0, p, p, 0, p, 1 << 40, nul) == 1
+    assert bs(p, p, p, p, p, 256, 256, 2048, 0, 1.0, ctypes.c_void_p(4100), p, 0, p, 1 << 40,
+              nul) == 3

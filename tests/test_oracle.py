@@ -370,6 +370,78 @@ def test_grpo_step_runs_on_tiny_workload():
     assert np.all(out["logp"] <= 0)
 
 
+# ---------------------------------------------------------------- vocabulary split
+def _slices(V, cuts):
+    edges = [0] + list(cuts) + [V]
+    return list(zip(edges[:-1], edges[1:]))
+
+
+@pytest.mark.parametrize("cuts", [[], [40], [8, 56], [32, 64, 88]])
+def test_slice_records_merge_to_the_full_softmax(cuts):
+    """The logsumexp of a union of slices, assembled from per-slice (max, sumexp,
+    sumexp*z, target) records, against the full-vocabulary definition and
+    torch.log_softmax; uneven slices, a skipped token, an ignored target."""
+    T, d, V = 24, 12, 96
+    H, W = _rand_hw(T, d, V, seed=11, scale_w=1.5)
+    rng = np.random.default_rng(12)
+    tgt = rng.integers(0, V, T)
+    tgt[5] = -1
+    mask = (rng.random(T) > 0.2).astype(np.uint8)
+    recs = [O.logprobs_slice_record(H, W[a:b], a, tgt, 0.8, mask) for a, b in _slices(V, cuts)]
+    lp, ent, lse = O.merge_slice_records(recs)
+    keep = (tgt >= 0) & (mask == 1)
+    z = torch.from_numpy(0.8 * H @ W.T)
+    ls = torch.log_softmax(z, dim=1).numpy()
+    ref_lp = np.where(keep, ls[np.arange(T), np.where(keep, tgt, 0)], 0.0)
+    ref_ent = np.where(keep, -(np.exp(ls) * ls).sum(axis=1), 0.0)
+    ref_lse = np.where(keep, torch.logsumexp(z, dim=1).numpy(), 0.0)
+    np.testing.assert_allclose(lp, ref_lp, atol=1e-12)
+    np.testing.assert_allclose(ent, ref_ent, atol=1e-12)
+    np.testing.assert_allclose(lse, ref_lse, atol=1e-12)
+    # the merge does not depend on the order of the slices
+    lp2, ent2, lse2 = O.merge_slice_records(recs[::-1])
+    np.testing.assert_allclose(lp2, lp, atol=1e-13)
+    np.testing.assert_allclose(ent2, ent, atol=1e-13)
+
+
+def test_slice_record_fields_brute_force():
+    """One token, one slice, written out element by element."""
+    H = np.array([[0.5, -1.0, 2.0]])
+    W = np.array([[1.0, 0.0, 0.0], [0.0, 1.0, 0.0], [0.0, 0.0, 1.0], [1.0, 1.0, 1.0]])
+    rec = O.logprobs_slice_record(H, W[1:3], 1, np.array([2]))[0]
+    z = [-1.0, 2.0]                         # logits of vocabulary ids 1 and 2
+    assert rec[0] == 2.0
+    assert math.isclose(rec[1], math.exp(-3.0) + 1.0, rel_tol=1e-15)
+    assert math.isclose(rec[2], math.exp(-3.0) * z[0] + z[1], rel_tol=1e-15)
+    assert rec[3] == 2.0
+    other = O.logprobs_slice_record(H, W[3:4], 3, np.array([2]))[0]
+    assert other[3] == -np.inf and other[1] == 1.0
+
+
+@pytest.mark.parametrize("cuts", [[48], [16, 24, 72]])
+def test_backward_slices_sum_to_the_full_backward(cuts):
+    """Sum over slices of the dH parts is dH; the slices' dW rows stacked are dW
+    (both against autograd of the fp64 log_softmax, not the oracle)."""
+    T, d, V = 16, 10, 96
+    H, W = _rand_hw(T, d, V, seed=21, scale_w=1.0)
+    rng = np.random.default_rng(22)
+    tgt = rng.integers(0, V, T)
+    g = rng.standard_normal(T)
+    g[[2, 9]] = 0.0
+    tau = 0.7
+    Ht = torch.from_numpy(H).requires_grad_(True)
+    Wt = torch.from_numpy(W).requires_grad_(True)
+    ls = torch.log_softmax(tau * Ht @ Wt.T, dim=1)
+    (ls[torch.arange(T), torch.from_numpy(tgt)] * torch.from_numpy(g)).sum().backward()
+    lse = torch.logsumexp(torch.from_numpy(tau * H @ W.T), dim=1).numpy()
+    parts = [O.policy_loss_bwd_slice(H, W[a:b], a, tgt, lse, g, tau) for a, b in _slices(V, cuts)]
+    dH = sum(p[0] for p in parts)
+    dW = np.concatenate([p[1] for p in parts])
+    np.testing.assert_allclose(dH, Ht.grad.numpy(), atol=1e-12)
+    np.testing.assert_allclose(dW, Wt.grad.numpy(), atol=1e-12)
+    assert not dH[[2, 9]].any()
+
+
 # ---------------------------------------------------------------- reward composition
 def test_verifiable_reward_hand_cases(golden_dir):
     gold = _golden(golden_dir, "verifiable_reward_hand_cases.json")

@@ -171,3 +171,88 @@ def test_lost_rank_ends_the_next_collective_with_an_error():
             p.join(60)
         status = open(os.path.join(d, "rank0.txt")).read()
         assert status.startswith("error"), status
+
+
+# ---------------------------------------------------------------- vocabulary-parallel form
+class OracleVocabEngine:
+    """The fp64 oracle as a rank's compute for the vocabulary split."""
+
+    def forward_slice(self, b):
+        lm, _ = O.token_select(b["cu_seqlens"], b["mask"], b["tgt"], b["window"])
+        rec = O.logprobs_slice_record(b["H"], b["W_slice"], b["v_offset"], b["tgt"], b["inv_temp"],
+                                      lm)
+        return lm, torch.from_numpy(rec)
+
+    def merge(self, recs):
+        return tuple(torch.from_numpy(x) for x in O.merge_slice_records(recs.numpy()))
+
+    def loss(self, b, lm, logp, agg):
+        adv = O.group_advantages(b["rewards"], b["group_id"], b["n_groups"])
+        loss, g, _ = O.policy_loss(logp.numpy(), b["old"], b["ref"], adv, b["cu_seqlens"],
+                                   b["group_id"], b["n_groups"], lm, b["clip_eps"], b["kl_beta"], agg)
+        return torch.tensor([loss], dtype=torch.float64), torch.from_numpy(g)
+
+    def backward_slice(self, b, lse, g):
+        dH, dW = O.policy_loss_bwd_slice(b["H"], b["W_slice"], b["v_offset"], b["tgt"],
+                                         lse.numpy(), g.numpy(), b["inv_temp"])
+        return torch.from_numpy(dH), torch.from_numpy(dW)
+
+
+def _vocab_batch():
+    b = _batch(seed=3)
+    rng = np.random.default_rng(4)
+    V = 72
+    b["W"] = 0.3 * rng.standard_normal((V, b["H"].shape[1]))
+    b["tgt"] = rng.integers(0, V, b["H"].shape[0])
+    b["tgt"][[4, 17]] = -1
+    return b
+
+
+def _vocab_worker(rank, world, port, outdir, agg):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world, timeout=timedelta(seconds=60))
+    b = _vocab_batch()
+    _, _, _, old, ref = _reference(b, agg)
+    off, n = shard.vocab_slices(b["W"].shape[0], world)[rank]
+    inp = dict(H=b["H"], W_slice=b["W"][off:off + n], v_offset=off, tgt=b["tgt"], mask=b["mask"],
+               cu_seqlens=b["cu"], group_id=b["gid"], n_groups=b["n_groups"],
+               rewards=b["rewards"], old=old, ref=ref, window=b["window"], inv_temp=1.0,
+               clip_eps=b["eps"], kl_beta=b["beta"])
+    loss, logp, dH, dW = shard.VocabParallelStep(OracleVocabEngine(), agg).run(inp)
+    np.save(os.path.join(outdir, f"loss{rank}.npy"), loss.numpy())
+    np.save(os.path.join(outdir, f"logp{rank}.npy"), logp.numpy())
+    np.save(os.path.join(outdir, f"dH{rank}.npy"), dH.numpy())
+    np.save(os.path.join(outdir, f"dW{rank}.npy"), dW.numpy())
+    dist.destroy_process_group()
+
+
+@pytest.mark.parametrize("world,agg", [(2, O.AGG_SEQ_GROUP), (3, O.AGG_TOKEN)])
+def test_vocab_parallel_step_matches_unsplit(world, agg):
+    with tempfile.TemporaryDirectory() as d:
+        mp.start_processes(_vocab_worker, args=(world, _free_port(), d, agg), nprocs=world,
+                           join=True, start_method="spawn")
+        b = _vocab_batch()
+        loss, dH, dW, _, _ = _reference(b, agg)
+        lm, _ = O.token_select(b["cu"], b["mask"], b["tgt"], b["window"])
+        lp, _, _ = O.logprobs(b["H"], b["W"], b["tgt"], 1.0, lm)
+        rows = []
+        for r in range(world):
+            assert abs(float(np.load(os.path.join(d, f"loss{r}.npy"))[0]) - loss) < 1e-12
+            np.testing.assert_allclose(np.load(os.path.join(d, f"logp{r}.npy")), lp, atol=1e-12)
+            np.testing.assert_allclose(np.load(os.path.join(d, f"dH{r}.npy")), dH, atol=1e-13)
+            rows.append(np.load(os.path.join(d, f"dW{r}.npy")))
+        np.testing.assert_allclose(np.concatenate(rows), dW, atol=1e-13)
+
+
+def test_vocab_slices_cover_the_vocabulary():
+    for V, world in ((151936, 2), (151936, 3), (151936, 7), (4096, 8), (72, 9)):
+        sl = shard.vocab_slices(V, world)
+        assert len(sl) == world and sl[0][0] == 0
+        assert all(o1 + n1 == o2 for (o1, n1), (o2, _) in zip(sl[:-1], sl[1:]))
+        assert sl[-1][0] + sl[-1][1] == V
+        assert all(n % 8 == 0 and n > 0 for _, n in sl)
+        assert max(n for _, n in sl) - min(n for _, n in sl) <= 8
+    with pytest.raises(ValueError):
+        shard.vocab_slices(4100, 2)
+    with pytest.raises(ValueError):
+        shard.vocab_slices(16, 3)
