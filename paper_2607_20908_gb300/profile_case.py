@@ -65,10 +65,11 @@ def main():
         torch.cuda.synchronize()
         label = "default" if cfg is None else "pair,group,raster,dynamic=" + ",".join(map(str, cfg))
         print(f"--- {label}")
-        for kind, ms in spo.spo_trace_read():
-            if kind > 3:
-                continue
-            tflops = 2.0 * a.T * a.d * a.V / ms / 1e9
+        recs = [(k, ms) for k, ms in spo.spo_trace_read() if k <= 3]
+        per_kind = {k: sum(1 for kk, _ in recs if kk == k) for k, _ in recs}
+        for kind, ms in recs:
+            # a GEMM run as several launches (dW passes) splits its FLOPs evenly
+            tflops = 2.0 * a.T * a.d * a.V / per_kind[kind] / ms / 1e9
             print(f"{spo.TRACE_KINDS[kind]:24s} {ms:8.3f} ms  {tflops:8.1f} TFLOP/s")
     assert spo.spo_device_error() == 0
 
