@@ -442,12 +442,31 @@ def read_ceiling_gbs(dev, nbytes, reps=15):
 
 
 def aux_measurements(dev, pk):
-    """Steps outside the timed loop, each timed with CUDA events on its own:
-    the reward composition (section 2.2) at an enlarged synthetic size
-    (2^24 candidates; 21 algorithmic bytes each), HBM-bound."""
+    """HBM-bound steps at enlarged synthetic sizes, outside the timed loop:
+    the reward composition (section 2.2; 2^24 candidates, 21 algorithmic bytes
+    each), the group advantages (2^24 rollouts in contiguous groups of 16,
+    12 algorithmic bytes each: group id, reward, advantage) and the loss
+    forward (2^24 tokens, 17 bytes each).  Each rep runs
+    after a 256 MB write that evicts L2 and is timed on its own with CUDA
+    events; the median is reported."""
     from paper_2607_20908_gb300 import spo
     n = 1 << 24
     gen = torch.Generator(device=dev).manual_seed(5)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+
+    def median_ms(fn, reps=12):
+        for _ in range(3):
+            fn()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(reps)]
+        for i, (a, b) in enumerate(ev):
+            flush.fill_(i & 0xFF)
+            a.record()
+            fn()
+            b.record()
+        torch.cuda.synchronize(dev)
+        return sorted(a.elapsed_time(b) for a, b in ev)[reps // 2]
+
     compiled = (torch.rand(n, device=dev, generator=gen) < 0.8).to(torch.uint8)
     p = torch.where(torch.rand(n, device=dev, generator=gen) < 0.5, 1.0,
                     torch.rand(n, device=dev, generator=gen))
@@ -455,21 +474,47 @@ def aux_measurements(dev, pk):
     cv = torch.rand(n, device=dev, generator=gen)
     rs = torch.randn(n, device=dev, generator=gen)
     out = torch.empty(n, device=dev)
-    for _ in range(3):
-        spo.spo_reward_compose(compiled, p, S, cv, rs, out=out)
-    torch.cuda.synchronize(dev)
-    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    reps = 20
-    a.record()
-    for _ in range(reps):
-        spo.spo_reward_compose(compiled, p, S, cv, rs, out=out)
-    b.record()
-    torch.cuda.synchronize(dev)
-    t = a.elapsed_time(b) / reps / 1e3
-    gbs = 21 * n / t / 1e9
-    return {"reward_compose": {"candidates": n, "ms": t * 1e3, "gbs": gbs,
+    ms = median_ms(lambda: spo.spo_reward_compose(compiled, p, S, cv, rs, out=out))
+    gbs = 21 * n / (ms / 1e3) / 1e9
+    res = {"reward_compose": {"candidates": n, "ms": ms, "gbs": gbs, "frac_of_hbm": gbs / pk["hbm"],
+                              "bound": "hbm",
+                              "note": "enlarged synthetic size; the workload itself has 128 rollouts"}}
+    del compiled, p, S, cv, rs, out
+
+    groups = n // 16
+    gid = torch.arange(n, device=dev, dtype=torch.int32) // 16
+    r = torch.randn(n, device=dev, generator=gen)
+    adv = torch.empty(n, device=dev)
+    ws = torch.empty(spo.group_advantages_workspace_size(n, groups), dtype=torch.uint8, device=dev)
+    ms = median_ms(lambda: spo.spo_group_advantages_ws(r, gid, groups, adv=adv, ws=ws))
+    gbs = 12 * n / (ms / 1e3) / 1e9
+    res["group_advantages"] = {"rollouts": n, "groups": groups, "ms": ms, "gbs": gbs,
                                "frac_of_hbm": gbs / pk["hbm"], "bound": "hbm",
-                               "note": "enlarged synthetic size; the workload itself has 128 rollouts"}}
+                               "note": "enlarged synthetic size, contiguous groups of 16 "
+                                       "(spo_group_advantages_ws); a step has 128-640 sequences"}
+    del gid, r, adv, ws
+
+    # a5 at 2^24 loss tokens (131072 sequences of 128, groups of 8): per token
+    # logp, old, ref (fp32), the loss mask (u8) in and g (fp32) out = 17 bytes
+    L = 128
+    ns = n // L
+    ng = ns // 8
+    cu = torch.arange(0, n + 1, L, device=dev, dtype=torch.int32)
+    gid = torch.arange(ns, device=dev, dtype=torch.int32) // 8
+    lp = -8.0 * torch.rand(n, device=dev, generator=gen)
+    old = lp + 0.05 * torch.randn(n, device=dev, generator=gen)
+    ref = lp + 0.05 * torch.randn(n, device=dev, generator=gen)
+    a_seq = torch.randn(ns, device=dev, generator=gen)
+    lm = torch.ones(n, dtype=torch.uint8, device=dev)
+    ws = torch.empty(spo.policy_loss_workspace_size(ns, ng), dtype=torch.uint8, device=dev)
+    ms = median_ms(lambda: spo.spo_policy_loss_fwd(lp, old, ref, a_seq, cu, gid, ng, lm, 0.2, 0.04,
+                                                   ws=ws))
+    alg = 17 * n + 12 * ns
+    gbs = alg / (ms / 1e3) / 1e9
+    res["policy_loss_fwd"] = {"tokens": n, "sequences": ns, "groups": ng, "ms": ms, "gbs": gbs,
+                              "frac_of_hbm": gbs / pk["hbm"], "bound": "hbm",
+                              "note": "enlarged synthetic size; a step has 16384-131072 tokens"}
+    return res
 
 
 # ----------------------------------------------------------------- arms

@@ -485,6 +485,18 @@ spo_status check_bwd_args(const void* H, const void* W, const int32_t* tgt, cons
   return SPO_OK;
 }
 
+spo_status check_adv_args(const float* rewards, const int32_t* group_id, int32_t n_seq,
+                          int32_t n_groups, int std_mode, float eps, const float* adv) {
+  if (!rewards || !group_id || !adv)
+    return fail(SPO_ERR_INVALID_ARG, "rewards, group_id and adv must be non-NULL");
+  if (n_seq < 1 || n_groups < 1 || n_seq > (1 << 26) || n_groups > (1 << 26))
+    return fail(SPO_ERR_SHAPE, "n_seq = %d, n_groups = %d out of range", n_seq, n_groups);
+  if (std_mode != SPO_STD_UNBIASED && std_mode != SPO_STD_POPULATION)
+    return fail(SPO_ERR_INVALID_ARG, "std_mode %d unknown", std_mode);
+  if (!(eps >= 0.f) || !isfinite(eps)) return fail(SPO_ERR_INVALID_ARG, "eps must be finite and >= 0");
+  return SPO_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -687,16 +699,39 @@ SPO_API spo_status spo_validate_inputs(const int32_t* tgt, int64_t T, int64_t V,
 SPO_API spo_status spo_group_advantages(const float* rewards, const int32_t* group_id,
                                         int32_t n_seq, int32_t n_groups, int std_mode, float eps,
                                         float* adv, void* stream) {
-  if (!rewards || !group_id || !adv)
-    return fail(SPO_ERR_INVALID_ARG, "rewards, group_id and adv must be non-NULL");
+  spo_status st = check_adv_args(rewards, group_id, n_seq, n_groups, std_mode, eps, adv);
+  if (st != SPO_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  st = traced(kTraceAdvantages, s, "advantage launch", [&] {
+    return spo::launch_group_advantages(rewards, group_id, n_seq, n_groups, std_mode, eps, adv, s);
+  });
+  return st == SPO_OK ? ok() : st;
+}
+
+SPO_API spo_status spo_group_advantages_workspace_size(int32_t n_seq, int32_t n_groups,
+                                                       size_t* bytes) {
+  if (!bytes) return fail(SPO_ERR_INVALID_ARG, "bytes must be non-NULL");
   if (n_seq < 1 || n_groups < 1 || n_seq > (1 << 26) || n_groups > (1 << 26))
     return fail(SPO_ERR_SHAPE, "n_seq = %d, n_groups = %d out of range", n_seq, n_groups);
-  if (std_mode != SPO_STD_UNBIASED && std_mode != SPO_STD_POPULATION)
-    return fail(SPO_ERR_INVALID_ARG, "std_mode %d unknown", std_mode);
-  if (!(eps >= 0.f) || !isfinite(eps)) return fail(SPO_ERR_INVALID_ARG, "eps must be finite and >= 0");
+  *bytes = spo::adv_ws_bytes(n_groups);
+  return ok();
+}
+
+SPO_API spo_status spo_group_advantages_ws(const float* rewards, const int32_t* group_id,
+                                           int32_t n_seq, int32_t n_groups, int std_mode,
+                                           float eps, float* adv, void* ws, size_t ws_bytes,
+                                           void* stream) {
+  spo_status st = check_adv_args(rewards, group_id, n_seq, n_groups, std_mode, eps, adv);
+  if (st != SPO_OK) return st;
+  const size_t need = spo::adv_ws_bytes(n_groups);
+  if (!ws || ws_bytes < need)
+    return fail(SPO_ERR_WORKSPACE, "workspace needs %zu bytes, got %zu", need, ws_bytes);
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
+    return fail(SPO_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  spo_status st = traced(kTraceAdvantages, s, "advantage launch", [&] {
-    return spo::launch_group_advantages(rewards, group_id, n_seq, n_groups, std_mode, eps, adv, s);
+  st = traced(kTraceAdvantages, s, "advantage launch", [&] {
+    return spo::launch_group_advantages_runs(rewards, group_id, n_seq, n_groups, std_mode, eps,
+                                             adv, ws, s);
   });
   return st == SPO_OK ? ok() : st;
 }

@@ -130,6 +130,13 @@ cudaError_t launch_token_select(const int* cu_seqlens, const uint8_t* mask, cons
 cudaError_t launch_group_advantages(const float* rewards, const int* group_id, int n_seq,
                                     int n_groups, int std_mode, float eps, float* adv,
                                     cudaStream_t s);
+// The same advantages in O(n_seq + n_groups) when every group's members are
+// contiguous (one run of equal ids), falling back to the per-group scan
+// otherwise; ws holds adv_ws_bytes(n_groups) bytes.
+size_t adv_ws_bytes(int n_groups);
+cudaError_t launch_group_advantages_runs(const float* rewards, const int* group_id, int n_seq,
+                                         int n_groups, int std_mode, float eps, float* adv,
+                                         void* ws, cudaStream_t s);
 
 // Composite reward (section 2.2 verifiable reward + structural score).
 struct RewardParams {
@@ -162,11 +169,12 @@ cudaError_t launch_validate(const int* tgt, long long T, long long V, const int*
                             const float* ref_logp, const uint8_t* mask, int* counts, cudaStream_t s);
 
 struct LossWs {
-  int* gsize;        // [n_groups]
-  int* n_tok;        // [n_seq]
-  long long* scal;   // [2]: non-empty groups, total loss tokens
-  double* part;      // [n_seq][3]: sum c*l, sum rho, sum kl
-  int* part_clip;    // [n_seq]
+  int* gsize;                // [n_groups]
+  int* n_tok;                // [n_seq]
+  unsigned long long* scal;  // [2]: non-empty groups, total loss tokens
+  double* part;              // [n_seq][3]: sum c*l, sum rho, sum kl
+  int* part_clip;            // [n_seq]
+  double* bpart;             // [64][4]: first-stage sums of the final reduction
 };
 size_t loss_ws_bytes(int n_seq, int n_groups);
 LossWs carve_loss_ws(void* ws, int n_seq, int n_groups);

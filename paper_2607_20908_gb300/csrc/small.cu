@@ -264,21 +264,20 @@ __global__ void token_select_kernel(const int* cu, const uint8_t* mask, const in
   if (lane == 0) n_tok[seq] = (window > 0 && kept > window) ? window : kept;
 }
 
-// One warp per group.  Members are visited in ascending sequence index and
-// every operation is a single IEEE fp32 operation in a fixed order, so the
-// result is reproducible bit for bit (the _rn intrinsics also keep the
-// compiler from contracting into fused multiply-adds).
-__global__ void group_adv_kernel(const float* rewards, const int* gid, int n_seq, int n_groups,
-                                 int std_mode, float eps, float* adv) {
-  const int warps = blockDim.x >> 5;
-  const int g = blockIdx.x * warps + (threadIdx.x >> 5);
-  const int lane = threadIdx.x & 31;
-  if (g >= n_groups) return;
+// Group-normalised advantages of one group g, computed by one warp.  The
+// members are the indices i in [b, e) (with gid[i] == g when check_gid) and
+// are visited in ascending index; every operation is a single IEEE fp32
+// operation in a fixed order, so the result is reproducible bit for bit (the
+// _rn intrinsics also keep the compiler from contracting into fused
+// multiply-adds).
+__device__ __forceinline__ void group_adv_warp(const float* rewards, const int* gid, int g, int b,
+                                               int e, bool check_gid, int std_mode, float eps,
+                                               float* adv, int lane) {
   float acc = 0.f, lo = INFINITY, hi = -INFINITY;
   int n = 0;
-  for (int base = 0; base < n_seq; base += 32) {
+  for (int base = b; base < e; base += 32) {
     const int i = base + lane;
-    const bool mem = i < n_seq && gid[i] == g;
+    const bool mem = i < e && (!check_gid || gid[i] == g);
     const float r = mem ? rewards[i] : 0.f;
     unsigned bal = __ballot_sync(0xffffffffu, mem);
     while (bal) {
@@ -296,9 +295,9 @@ __global__ void group_adv_kernel(const float* rewards, const int* gid, int n_seq
   if (!zero) {
     mu = __fdiv_rn(acc, static_cast<float>(n));
     float ss = 0.f;
-    for (int base = 0; base < n_seq; base += 32) {
+    for (int base = b; base < e; base += 32) {
       const int i = base + lane;
-      const bool mem = i < n_seq && gid[i] == g;
+      const bool mem = i < e && (!check_gid || gid[i] == g);
       const float dv = mem ? __fsub_rn(rewards[i], mu) : 0.f;
       unsigned bal = __ballot_sync(0xffffffffu, mem);
       while (bal) {
@@ -311,9 +310,161 @@ __global__ void group_adv_kernel(const float* rewards, const int* gid, int n_seq
     const float var = __fdiv_rn(ss, static_cast<float>(std_mode == 0 ? n - 1 : n));
     den = __fadd_rn(__fsqrt_rn(var), eps);
   }
-  for (int base = 0; base < n_seq; base += 32) {
+  for (int base = b; base < e; base += 32) {
     const int i = base + lane;
-    if (i < n_seq && gid[i] == g) adv[i] = zero ? 0.f : __fdiv_rn(__fsub_rn(rewards[i], mu), den);
+    if (i < e && (!check_gid || gid[i] == g))
+      adv[i] = zero ? 0.f : __fdiv_rn(__fsub_rn(rewards[i], mu), den);
+  }
+}
+
+// One warp per group, scanning every sequence: O(n_groups * n_seq) reads, no
+// scratch memory; the right shape for the few hundred sequences of a step.
+__global__ void group_adv_kernel(const float* rewards, const int* gid, int n_seq, int n_groups,
+                                 int std_mode, float eps, float* adv) {
+  const int warps = blockDim.x >> 5;
+  const int g = blockIdx.x * warps + (threadIdx.x >> 5);
+  if (g >= n_groups) return;
+  group_adv_warp(rewards, gid, g, 0, n_seq, true, std_mode, eps, adv, threadIdx.x & 31);
+}
+
+// Runs of equal group ids: the number of runs of each group and the start /
+// end of its run (meaningful when it has one).  The atomics' results are not
+// waited for.
+__global__ void adv_runs_kernel(const int* gid, int n_seq, int n_groups, int* runs, int* start,
+                                int* end) {
+  const int stride = gridDim.x * blockDim.x;
+  for (int i0 = blockIdx.x * blockDim.x + threadIdx.x; i0 < n_seq; i0 += 4 * stride) {
+    int gv[4], gp[4], gn[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {  // the loads of four elements in flight together
+      const int i = i0 + u * stride;
+      gv[u] = i < n_seq ? gid[i] : -1;
+      gp[u] = i < n_seq && i > 0 ? gid[i - 1] : -1;
+      gn[u] = i + 1 < n_seq ? gid[i + 1] : -1;
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int i = i0 + u * stride;
+      const int g = gv[u];
+      if (i >= n_seq || g < 0 || g >= n_groups) continue;  // no group: no advantage
+      if (i == 0 || gp[u] != g) {
+        atomicAdd(&runs[g], 1);
+        start[g] = i;
+      }
+      if (i == n_seq - 1 || gn[u] != g) end[g] = i + 1;
+    }
+  }
+}
+
+// Raises *split when some group has more than one run (its members are not
+// contiguous).
+__global__ void adv_split_kernel(const int* runs, int n_groups, int* split) {
+  bool multi = false;
+  for (int g = blockIdx.x * blockDim.x + threadIdx.x; g < n_groups; g += gridDim.x * blockDim.x)
+    multi |= runs[g] > 1;
+  if (__any_sync(0xffffffffu, multi) && (threadIdx.x & 31) == 0) atomicOr(split, 1);
+}
+
+// The same fold by one thread over a contiguous run [b, e): the identical
+// sequence of fp32 operations, without the warp's shuffles, so a warp
+// handles 32 groups at once.  Element i lives at src[at(i)] and its advantage
+// goes to dst[at(i)].
+template <class At>
+__device__ __forceinline__ void group_adv_thread(const float* src, int b, int e, int std_mode,
+                                                 float eps, float* dst, At at) {
+  constexpr int kB = 8;  // loads issued before the fold consumes them
+  float acc = 0.f, lo = INFINITY, hi = -INFINITY;
+  for (int i0 = b; i0 < e; i0 += kB) {
+    float r[kB];
+#pragma unroll
+    for (int u = 0; u < kB; ++u) r[u] = i0 + u < e ? src[at(i0 + u)] : 0.f;
+#pragma unroll
+    for (int u = 0; u < kB; ++u) {
+      if (i0 + u < e) {
+        acc = __fadd_rn(acc, r[u]);
+        lo = fminf(lo, r[u]);
+        hi = fmaxf(hi, r[u]);
+      }
+    }
+  }
+  const int n = e - b;
+  const bool zero = n <= 1 || lo == hi;
+  float mu = 0.f, den = 1.f;
+  if (!zero) {
+    mu = __fdiv_rn(acc, static_cast<float>(n));
+    float ss = 0.f;
+    for (int i0 = b; i0 < e; i0 += kB) {
+      float r[kB];
+#pragma unroll
+      for (int u = 0; u < kB; ++u) r[u] = i0 + u < e ? src[at(i0 + u)] : 0.f;
+#pragma unroll
+      for (int u = 0; u < kB; ++u) {
+        if (i0 + u < e) {
+          const float dv = __fsub_rn(r[u], mu);
+          ss = __fadd_rn(ss, __fmul_rn(dv, dv));
+        }
+      }
+    }
+    const float var = __fdiv_rn(ss, static_cast<float>(std_mode == 0 ? n - 1 : n));
+    den = __fadd_rn(__fsqrt_rn(var), eps);
+  }
+  for (int i = b; i < e; ++i)
+    dst[at(i)] = zero ? 0.f : __fdiv_rn(__fsub_rn(src[at(i)], mu), den);
+}
+
+struct AtIdentity {
+  __device__ int operator()(int i) const { return i; }
+};
+// one pad word per 32: consecutive threads' runs fall in different banks
+struct AtPadded {
+  __device__ int operator()(int i) const { return i + (i >> 5); }
+};
+
+// Second pass of the run path.  When every group is one run, a block takes 256
+// consecutive group ids; if their runs lie back to back in memory (the usual
+// packing) and span at most kAdvStage rewards, the block stages that span in
+// shared memory with coalesced loads, each thread folds its own group there,
+// and the advantages go back with coalesced stores.  Other blocks fold each
+// group straight from memory, one thread per group.  When some group has
+// several runs, one warp per group scans every sequence.  In every case the
+// members are folded in ascending index: the same bits.
+constexpr int kAdvStage = 8192;
+
+__global__ void __launch_bounds__(256) group_adv_runs_kernel(
+    const float* rewards, const int* gid, int n_seq, int n_groups, int std_mode, float eps,
+    const int* runs, const int* start, const int* end, const int* split, float* adv) {
+  __shared__ float st[kAdvStage + kAdvStage / 32];
+  if (*split) {
+    const int lane = threadIdx.x & 31;
+    const int warps = (gridDim.x * blockDim.x) >> 5;
+    for (int g = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; g < n_groups; g += warps)
+      group_adv_warp(rewards, gid, g, 0, n_seq, true, std_mode, eps, adv, lane);
+    return;
+  }
+  for (int g0 = blockIdx.x * blockDim.x; g0 < n_groups; g0 += gridDim.x * blockDim.x) {
+    const int g = g0 + threadIdx.x;
+    const bool live = g < n_groups;
+    const int b = live && runs[g] > 0 ? start[g] : 0;
+    const int e = live && runs[g] > 0 ? end[g] : 0;
+    // back to back: every group of the block non-empty, each run starting where
+    // the previous group's ends
+    const int g_last = min(n_groups, g0 + static_cast<int>(blockDim.x)) - 1;
+    const int lo = runs[g0] > 0 ? start[g0] : 0;
+    const int hi = runs[g_last] > 0 ? end[g_last] : 0;
+    const bool chained =
+        !live || (runs[g] > 0 && (g == g0 || (runs[g - 1] > 0 && end[g - 1] == b)));
+    const bool staged = __syncthreads_and(chained) && hi - lo > 0 && hi - lo <= kAdvStage;
+    if (!staged) {
+      if (live && e > b) group_adv_thread(rewards, b, e, std_mode, eps, adv, AtIdentity());
+      continue;
+    }
+    const AtPadded at;
+    for (int k = threadIdx.x; k < hi - lo; k += blockDim.x) st[at(k)] = rewards[lo + k];
+    __syncthreads();
+    if (live) group_adv_thread(st, b - lo, e - lo, std_mode, eps, st, at);
+    __syncthreads();
+    for (int k = threadIdx.x; k < hi - lo; k += blockDim.x) adv[lo + k] = st[at(k)];
+    __syncthreads();
   }
 }
 
@@ -407,105 +558,185 @@ __device__ __forceinline__ double block_sum_d(double v, double* sh) {
   return r;
 }
 
-// (a) loss tokens per sequence and sequences per group.
-__global__ void loss_count_kernel(const int* cu, const int* gid, const uint8_t* lm, int* n_tok,
-                                  int* gsize) {
-  __shared__ double sh[kLossThreads];
-  const int i = blockIdx.x;
-  const int b = cu[i], e = cu[i + 1];
-  double c = 0;
-  for (int t = b + threadIdx.x; t < e; t += kLossThreads) c += lm[t] ? 1.0 : 0.0;
-  const double tot = block_sum_d(c, sh);
-  if (threadIdx.x == 0) {
-    n_tok[i] = static_cast<int>(tot);
-    atomicAdd(&gsize[gid[i]], 1);
+// One warp per sequence; the grid strides over sequences.
+__device__ __forceinline__ int warp_seq0() { return (blockIdx.x * blockDim.x + threadIdx.x) >> 5; }
+__device__ __forceinline__ int warp_seq_stride() { return (gridDim.x * blockDim.x) >> 5; }
+
+// Sum over a warp by a fixed xor butterfly: every lane ends with the same bits.
+__device__ __forceinline__ float warp_sum_f(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = __fadd_rn(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+__device__ __forceinline__ long long warp_sum_ll(long long v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// (a) loss tokens per sequence and sequences per group (integers).
+__global__ void loss_count_kernel(const int* cu, const int* gid, const uint8_t* lm, int n_seq,
+                                  int n_groups, int* n_tok, int* gsize) {
+  const int lane = threadIdx.x & 31;
+  for (int i = warp_seq0(); i < n_seq; i += warp_seq_stride()) {
+    const int b = cu[i], e = cu[i + 1];
+    int c = 0;
+    for (int t0 = b + lane; t0 < e; t0 += 128) {
+      uint8_t m[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) m[u] = t0 + 32 * u < e ? lm[t0 + 32 * u] : 0;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) c += m[u] ? 1 : 0;
+    }
+    c = __reduce_add_sync(0xffffffffu, c);
+    if (lane == 0) {
+      n_tok[i] = c;
+      const int g = gid[i];
+      if (g >= 0 && g < n_groups) atomicAdd(&gsize[g], 1);
+    }
   }
 }
 
-// (b) number of non-empty groups and of loss tokens.
+// (b) number of non-empty groups and of loss tokens (integer sums; scal zeroed).
 __global__ void loss_scalars_kernel(const int* gsize, int n_groups, const int* n_tok, int n_seq,
-                                    long long* scal) {
-  __shared__ double sh[kLossThreads];
-  double ng = 0, nt = 0;
-  for (int g = threadIdx.x; g < n_groups; g += kLossThreads) ng += gsize[g] > 0 ? 1.0 : 0.0;
-  for (int i = threadIdx.x; i < n_seq; i += kLossThreads) nt += n_tok[i];
-  ng = block_sum_d(ng, sh);
-  nt = block_sum_d(nt, sh);
-  if (threadIdx.x == 0) {
-    scal[0] = static_cast<long long>(ng);
-    scal[1] = static_cast<long long>(nt);
+                                    unsigned long long* scal) {
+  long long ng = 0, nt = 0;
+  for (int k = blockIdx.x * blockDim.x + threadIdx.x; k < max(n_groups, n_seq);
+       k += gridDim.x * blockDim.x) {
+    if (k < n_groups) ng += gsize[k] > 0 ? 1 : 0;
+    if (k < n_seq) nt += n_tok[k];
+  }
+  ng = warp_sum_ll(ng);
+  nt = warp_sum_ll(nt);
+  if ((threadIdx.x & 31) == 0) {
+    if (ng) atomicAdd(&scal[0], static_cast<unsigned long long>(ng));
+    if (nt) atomicAdd(&scal[1], static_cast<unsigned long long>(nt));
   }
 }
 
-// (c) per-token surrogate, KL, dL/dlogp; per-sequence fp64 partial sums.
+// (c) per-token surrogate, KL, dL/dlogp; per-sequence fp64 partial sums (each
+// lane over tokens b + lane, b + lane + 32, ..., then the fixed butterfly).
 __global__ void loss_token_kernel(const float* logp, const float* old_logp, const float* ref_logp,
-                                  const float* adv, const int* cu, const int* gid,
-                                  const uint8_t* lm, float clip_eps, float kl_beta, int agg,
-                                  const int* n_tok, const int* gsize, const long long* scal,
-                                  float* g, double* part, int* part_clip) {
-  __shared__ double sh[kLossThreads];
-  const int i = blockIdx.x;
-  const int b = cu[i], e = cu[i + 1];
-  const int ni = n_tok[i];
-  float c = 0.f;
-  if (agg == 0) {
-    const long long ng = scal[0];
-    if (ni > 0 && ng > 0)
-      c = static_cast<float>(1.0 / (static_cast<double>(ng) * gsize[gid[i]] * ni));
-  } else {
-    const long long nt = scal[1];
-    if (nt > 0) c = static_cast<float>(1.0 / static_cast<double>(nt));
-  }
-  const float A = adv[i];
+                                  const float* adv, const int* cu, const int* gid, int n_seq,
+                                  int n_groups, const uint8_t* lm, float clip_eps, float kl_beta,
+                                  int agg, const int* n_tok, const int* gsize,
+                                  const unsigned long long* scal, float* g, double* part,
+                                  int* part_clip) {
+  const int lane = threadIdx.x & 31;
   const bool use_kl = ref_logp != nullptr && kl_beta != 0.f;
   const float lo = 1.f - clip_eps, hi = 1.f + clip_eps;
-  double s_l = 0, s_rho = 0, s_kl = 0, s_clip = 0;
-  for (int t = b + threadIdx.x; t < e; t += kLossThreads) {
-    if (!lm[t]) {
-      g[t] = 0.f;
-      continue;
+  for (int i = warp_seq0(); i < n_seq; i += warp_seq_stride()) {
+    const int b = cu[i], e = cu[i + 1];
+    const int ni = n_tok[i];
+    // c_t of Eq. 3's average; fp32 (GB300's fp64 unit is narrow, and every
+    // lane of the warp computes it)
+    float c = 0.f;
+    if (agg == 0) {
+      const unsigned long long ng = scal[0];
+      const int gi = gid[i];
+      if (ni > 0 && ng > 0 && gi >= 0 && gi < n_groups)
+        c = __frcp_rn(static_cast<float>(ng) * static_cast<float>(gsize[gi]) *
+                      static_cast<float>(ni));
+    } else {
+      const unsigned long long nt = scal[1];
+      if (nt > 0) c = __frcp_rn(static_cast<float>(nt));
     }
-    const float lp = logp[t];
-    const float rho = expf(lp - old_logp[t]);
-    const float clipped = fminf(fmaxf(rho, lo), hi);
-    const float surr = fminf(rho * A, clipped * A);
-    const bool binds = (A > 0.f && rho > hi) || (A < 0.f && rho < lo);
-    float kl = 0.f, dkl = 0.f;
-    if (use_kl) {
-      const float delta = ref_logp[t] - lp;
-      const float em1 = expm1f(delta);
-      kl = em1 - delta;  // exp(delta) - delta - 1
-      dkl = -em1;        // 1 - exp(delta)
+    const float A = adv[i];
+    // a lane sums its own tokens and the warp its lanes in fp32 (fixed
+    // butterfly); the sums over sequences are fp64
+    float s_l = 0.f, s_rho = 0.f, s_kl = 0.f;
+    int n_clip = 0;
+    // a lane's tokens b + lane, b + lane + 32, ... in order, four loads in flight
+    for (int t0 = b + lane; t0 < e; t0 += 128) {
+      uint8_t mk[4];
+      float lpv[4], olv[4], rfv[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int t = t0 + 32 * u;
+        mk[u] = t < e ? lm[t] : 0;
+        lpv[u] = mk[u] ? logp[t] : 0.f;
+        olv[u] = mk[u] ? old_logp[t] : 0.f;
+        rfv[u] = mk[u] && use_kl ? ref_logp[t] : 0.f;
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int t = t0 + 32 * u;
+        if (t >= e) break;
+        if (!mk[u]) {
+          g[t] = 0.f;
+          continue;
+        }
+        const float lp = lpv[u];
+        const float rho = expf(lp - olv[u]);
+        const float clipped = fminf(fmaxf(rho, lo), hi);
+        const float surr = fminf(rho * A, clipped * A);
+        const bool binds = (A > 0.f && rho > hi) || (A < 0.f && rho < lo);
+        float kl = 0.f, dkl = 0.f;
+        if (use_kl) {
+          const float delta = rfv[u] - lp;
+          const float em1 = expm1f(delta);
+          kl = em1 - delta;  // exp(delta) - delta - 1
+          dkl = -em1;        // 1 - exp(delta)
+        }
+        const float ell = -(surr - kl_beta * kl);
+        g[t] = c * ((binds ? 0.f : -A * rho) + (use_kl ? kl_beta * dkl : 0.f));
+        s_l += ell;
+        s_rho += rho;
+        s_kl += kl;
+        n_clip += binds ? 1 : 0;
+      }
     }
-    const float ell = -(surr - kl_beta * kl);
-    g[t] = c * ((binds ? 0.f : -A * rho) + (use_kl ? kl_beta * dkl : 0.f));
-    s_l += static_cast<double>(c) * ell;
-    s_rho += rho;
-    s_kl += kl;
-    s_clip += binds ? 1.0 : 0.0;
-  }
-  s_l = block_sum_d(s_l, sh);
-  s_rho = block_sum_d(s_rho, sh);
-  s_kl = block_sum_d(s_kl, sh);
-  s_clip = block_sum_d(s_clip, sh);
-  if (threadIdx.x == 0) {
-    part[3 * i + 0] = s_l;
-    part[3 * i + 1] = s_rho;
-    part[3 * i + 2] = s_kl;
-    part_clip[i] = static_cast<int>(s_clip);
+    s_l = warp_sum_f(s_l);
+    s_rho = warp_sum_f(s_rho);
+    s_kl = warp_sum_f(s_kl);
+    n_clip = __reduce_add_sync(0xffffffffu, n_clip);
+    if (lane == 0) {
+      part[3 * i + 0] = static_cast<double>(s_l) * static_cast<double>(c);
+      part[3 * i + 1] = s_rho;
+      part[3 * i + 2] = s_kl;
+      part_clip[i] = n_clip;
+    }
   }
 }
 
-// (d) fixed-order sum over sequences -> loss and stats.
-__global__ void loss_final_kernel(const double* part, const int* part_clip, int n_seq,
-                                  const long long* scal, float* loss, float* stats) {
+// (d) fixed-order sum over sequences in two stages: block k sums the
+// sequences of its contiguous chunk (thread-strided, then a fixed tree), and
+// one block sums the kLossFinalBlocks block results.  The split depends only
+// on n_seq, so the loss is the same bits on any device.
+constexpr int kLossFinalBlocks = 64;
+
+__global__ void loss_final_partial_kernel(const double* part, const int* part_clip, int n_seq,
+                                          int chunk, double* bpart) {
   __shared__ double sh[kLossThreads];
+  const int i0 = blockIdx.x * chunk, i1 = min(n_seq, i0 + chunk);
   double l = 0, r = 0, k = 0, c = 0;
-  for (int i = threadIdx.x; i < n_seq; i += kLossThreads) {
+  for (int i = i0 + threadIdx.x; i < i1; i += kLossThreads) {
     l += part[3 * i];
     r += part[3 * i + 1];
     k += part[3 * i + 2];
     c += part_clip[i];
+  }
+  l = block_sum_d(l, sh);
+  r = block_sum_d(r, sh);
+  k = block_sum_d(k, sh);
+  c = block_sum_d(c, sh);
+  if (threadIdx.x == 0) {
+    bpart[4 * blockIdx.x + 0] = l;
+    bpart[4 * blockIdx.x + 1] = r;
+    bpart[4 * blockIdx.x + 2] = k;
+    bpart[4 * blockIdx.x + 3] = c;
+  }
+}
+
+__global__ void loss_final_kernel(const double* bpart, int nb, const unsigned long long* scal,
+                                  float* loss, float* stats) {
+  __shared__ double sh[kLossThreads];
+  double l = 0, r = 0, k = 0, c = 0;
+  for (int j = threadIdx.x; j < nb; j += kLossThreads) {
+    l += bpart[4 * j];
+    r += bpart[4 * j + 1];
+    k += bpart[4 * j + 2];
+    c += bpart[4 * j + 3];
   }
   l = block_sum_d(l, sh);
   r = block_sum_d(r, sh);
@@ -602,6 +833,33 @@ cudaError_t launch_group_advantages(const float* rewards, const int* group_id, i
   return cudaGetLastError();
 }
 
+size_t adv_ws_bytes(int n_groups) { return align256(sizeof(int) * (3 * static_cast<size_t>(n_groups) + 1)); }
+
+cudaError_t launch_group_advantages_runs(const float* rewards, const int* group_id, int n_seq,
+                                         int n_groups, int std_mode, float eps, float* adv,
+                                         void* ws, cudaStream_t s) {
+  int* runs = static_cast<int*>(ws);
+  int* start = runs + n_groups;
+  int* end = start + n_groups;
+  int* split = end + n_groups;
+  cudaError_t e = cudaMemsetAsync(runs, 0, sizeof(int) * n_groups, s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(split, 0, sizeof(int), s);
+  if (e != cudaSuccess) return e;
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  adv_runs_kernel<<<max(1, min((n_seq + 1023) / 1024, sms * 8)), 256, 0, s>>>(
+      group_id, n_seq, n_groups, runs, start, end);
+  adv_split_kernel<<<max(1, min((n_groups + 255) / 256, sms * 4)), 256, 0, s>>>(runs, n_groups,
+                                                                               split);
+  // enough warps for the per-group scan of the fallback, one thread per group otherwise
+  const int blocks2 = max(1, min((n_groups + 7) / 8, sms * 16));
+  group_adv_runs_kernel<<<blocks2, 256, 0, s>>>(rewards, group_id, n_seq, n_groups, std_mode, eps,
+                                                runs, start, end, split, adv);
+  note_launches(3);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_reward_compose(const uint8_t* compiled, const float* pass_rate,
                                   const float* speedup, const float* cv, const float* r_struct,
                                   int n, const RewardParams& q, float* out, cudaStream_t s) {
@@ -663,7 +921,7 @@ cudaError_t launch_validate(const int* tgt, long long T, long long V, const int*
 size_t loss_ws_bytes(int n_seq, int n_groups) {
   return align256(sizeof(int) * n_groups) + align256(sizeof(int) * n_seq) +
          align256(2 * sizeof(long long)) + align256(3 * sizeof(double) * n_seq) +
-         align256(sizeof(int) * n_seq);
+         align256(sizeof(int) * n_seq) + align256(4 * sizeof(double) * kLossFinalBlocks);
 }
 
 LossWs carve_loss_ws(void* ws, int n_seq, int n_groups) {
@@ -673,11 +931,13 @@ LossWs carve_loss_ws(void* ws, int n_seq, int n_groups) {
   p += align256(sizeof(int) * n_groups);
   w.n_tok = reinterpret_cast<int*>(p);
   p += align256(sizeof(int) * n_seq);
-  w.scal = reinterpret_cast<long long*>(p);
+  w.scal = reinterpret_cast<unsigned long long*>(p);
   p += align256(2 * sizeof(long long));
   w.part = reinterpret_cast<double*>(p);
   p += align256(3 * sizeof(double) * n_seq);
   w.part_clip = reinterpret_cast<int*>(p);
+  p += align256(sizeof(int) * n_seq);
+  w.bpart = reinterpret_cast<double*>(p);
   return w;
 }
 
@@ -688,16 +948,28 @@ cudaError_t launch_policy_loss(const float* logp, const float* old_logp, const f
                                float* stats, const LossWs& w, cudaStream_t s) {
   (void)T;
   cudaError_t e = cudaMemsetAsync(w.gsize, 0, sizeof(int) * n_groups, s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(w.scal, 0, 2 * sizeof(unsigned long long), s);
   if (e != cudaSuccess) return e;
-  loss_count_kernel<<<n_seq, kLossThreads, 0, s>>>(cu_seqlens, group_id, loss_mask, w.n_tok,
-                                                   w.gsize);
-  loss_scalars_kernel<<<1, kLossThreads, 0, s>>>(w.gsize, n_groups, w.n_tok, n_seq, w.scal);
-  loss_token_kernel<<<n_seq, kLossThreads, 0, s>>>(logp, old_logp, ref_logp, adv, cu_seqlens,
-                                                   group_id, loss_mask, clip_eps, kl_beta, agg,
-                                                   w.n_tok, w.gsize, w.scal, g, w.part,
-                                                   w.part_clip);
-  loss_final_kernel<<<1, kLossThreads, 0, s>>>(w.part, w.part_clip, n_seq, w.scal, loss, stats);
-  note_launches(4);
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int per_block = kLossThreads / 32;  // sequences in flight per block
+  const int seq_blocks = max(1, min((n_seq + per_block - 1) / per_block, sms * 8));
+  loss_count_kernel<<<seq_blocks, kLossThreads, 0, s>>>(cu_seqlens, group_id, loss_mask, n_seq,
+                                                        n_groups, w.n_tok, w.gsize);
+  const int nmax = n_seq > n_groups ? n_seq : n_groups;
+  loss_scalars_kernel<<<max(1, min((nmax + kLossThreads - 1) / kLossThreads, sms * 4)), kLossThreads,
+                        0, s>>>(w.gsize, n_groups, w.n_tok, n_seq, w.scal);
+  loss_token_kernel<<<seq_blocks, kLossThreads, 0, s>>>(logp, old_logp, ref_logp, adv, cu_seqlens,
+                                                        group_id, n_seq, n_groups, loss_mask,
+                                                        clip_eps, kl_beta, agg, w.n_tok, w.gsize,
+                                                        w.scal, g, w.part, w.part_clip);
+  const int chunk = (n_seq + kLossFinalBlocks - 1) / kLossFinalBlocks;
+  const int nb = (n_seq + chunk - 1) / chunk;
+  loss_final_partial_kernel<<<nb, kLossThreads, 0, s>>>(w.part, w.part_clip, n_seq, chunk,
+                                                        w.bpart);
+  loss_final_kernel<<<1, kLossThreads, 0, s>>>(w.bpart, nb, w.scal, loss, stats);
+  note_launches(5);
   return cudaGetLastError();
 }
 

@@ -63,6 +63,9 @@ _SIGS = {
                               _c_size, _vp], ctypes.c_int),
     "spo_policy_loss_fwd_noalloc": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, _i32, _vp, _i64, _f32,
                                      _f32, ctypes.c_int, _vp, _vp, _vp, _vp], ctypes.c_int),
+    "spo_group_advantages_workspace_size": ([_i32, _i32, ctypes.POINTER(_c_size)], ctypes.c_int),
+    "spo_group_advantages_ws": ([_vp, _vp, _i32, _i32, ctypes.c_int, _f32, _vp, _vp, _c_size, _vp],
+                                ctypes.c_int),
     "spo_logprobs_fwd_slice": ([_vp, _vp, _vp, _vp, _i64, _i64, _i64, _i64, _f32, _vp, _vp,
                                 _c_size, _vp], ctypes.c_int),
     "spo_logprobs_merge_slices": ([_vp, _i32, _i64, _vp, _vp, _vp, _vp], ctypes.c_int),
@@ -211,6 +214,30 @@ def spo_group_advantages(rewards, group_id, n_groups: int, std_mode: int = SPO_S
     adv = torch.empty(n, dtype=torch.float32, device=dev)
     _check(lib().spo_group_advantages(_ptr(rewards), _ptr(group_id), n, int(n_groups),
                                       int(std_mode), float(eps), _ptr(adv), _stream(dev)))
+    return adv
+
+
+def group_advantages_workspace_size(n_seq: int, n_groups: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().spo_group_advantages_workspace_size(n_seq, n_groups, ctypes.byref(n)))
+    return n.value
+
+
+def spo_group_advantages_ws(rewards, group_id, n_groups: int, std_mode: int = SPO_STD_UNBIASED,
+                            eps: float = 1e-6, adv=None, ws=None):
+    """a4 in O(n_seq + n_groups) for contiguous groups (same bits as
+    spo_group_advantages); fp32[n_seq]."""
+    dev = rewards.device
+    n = rewards.numel()
+    _need(rewards, "rewards", torch.float32, device=dev)
+    _need(group_id, "group_id", torch.int32, n, dev)
+    if adv is None:
+        adv = torch.empty(n, dtype=torch.float32, device=dev)
+    _need(adv, "adv", torch.float32, n, dev)
+    w = _workspace(group_advantages_workspace_size(n, int(n_groups)), dev, ws)
+    _check(lib().spo_group_advantages_ws(_ptr(rewards), _ptr(group_id), n, int(n_groups),
+                                         int(std_mode), float(eps), _ptr(adv), _ptr(w), w.numel(),
+                                         _stream(dev)))
     return adv
 
 

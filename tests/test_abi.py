@@ -109,3 +109,16 @@ def test_vocab_split_host_validation_without_gpu(lib):
     assert bs(p, p, p, nul, p, 256, 256, 2048, 0, 1.0, p, p, 0, p, 1 << 40, nul) == 1
     assert bs(p, p, p, p, p, 256, 256, 2048, 0, 1.0, ctypes.c_void_p(4100), p, 0, p, 1 << 40,
               nul) == 3
+
+
+def test_group_advantages_ws_host_validation(lib):
+    from paper_2607_20908_gb300 import spo
+    p = ctypes.c_void_p(4096)
+    nul = ctypes.c_void_p(0)
+    assert spo.group_advantages_workspace_size(1 << 24, 1 << 20) >= 4 * 3 * (1 << 20)
+    f = lib.spo_group_advantages_ws
+    assert f(p, p, 16, 4, 0, 1e-6, p, p, 16, nul) == 4
+    assert f(p, p, 16, 4, 0, 1e-6, p, ctypes.c_void_p(4100), 1 << 20, nul) == 3
+    assert f(p, p, 16, 4, 5, 1e-6, p, p, 1 << 20, nul) == 1
+    assert f(p, nul, 16, 4, 0, 1e-6, p, p, 1 << 20, nul) == 1
+    assert f(p, p, 0, 4, 0, 1e-6, p, p, 1 << 20, nul) == 2

@@ -98,6 +98,38 @@ def test_advantages_bit_exact_fp32_order():
     assert np.all(got[gid == 11] == 0)
 
 
+@pytest.mark.parametrize("layout", ["contiguous", "scattered", "empty_and_invalid"])
+def test_advantages_run_path_bit_exact(layout):
+    """The workspace variant: one pass over the runs of equal group ids, then
+    each group folded over its own run (contiguous layout) or the per-group
+    scan (scattered ids); the same bits as the fp32-order oracle either way."""
+    from paper_2607_20908_gb300 import spo
+    rng = np.random.default_rng(4)
+    sizes = rng.integers(1, 40, 300)                  # groups of 1..39 sequences
+    sizes[[5, 6]] = [1, 64]
+    ng = sizes.size
+    gid = np.repeat(np.arange(ng), sizes).astype(np.int32)
+    n = gid.size
+    r = rng.normal(0.3, 1.0, n).astype(np.float32)
+    r[gid == 9] = -0.5                                 # zero-variance group
+    if layout == "scattered":
+        gid = gid[rng.permutation(n)]
+    if layout == "empty_and_invalid":
+        gid = np.where(gid >= 100, gid + 2, gid).astype(np.int32)   # groups 100, 101 empty
+        ng += 2
+        gid[[0, n - 1]] = [ng, -1]                      # no group: adv left untouched; every
+                                                        # group still one run (the run path)
+    want = O.group_advantages_f32(r, np.where((gid >= 0) & (gid < ng), gid, ng), ng + 1)
+    adv = torch.full((n,), 7.0, device="cuda")
+    got = spo.spo_group_advantages_ws(torch.from_numpy(r).cuda(), torch.from_numpy(gid).cuda(), ng,
+                                      adv=adv).cpu().numpy()
+    ok = (gid >= 0) & (gid < ng)
+    np.testing.assert_array_equal(got[ok].view(np.uint32), want[ok].view(np.uint32))
+    assert np.all(got[~ok] == 7.0)
+    base = spo.spo_group_advantages(torch.from_numpy(r).cuda(), torch.from_numpy(gid).cuda(), ng)
+    np.testing.assert_array_equal(got[ok].view(np.uint32), base.cpu().numpy()[ok].view(np.uint32))
+
+
 def test_no_loss_tokens():
     """Every token masked: log-probs, loss, g, dH and dW are exactly zero."""
     case = inputs.tiny_case(seed=1041)
