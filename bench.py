@@ -82,7 +82,7 @@ TRAFFIC = {"sources_sha256_16": "2ade601110b09cba",
            "bytes": {"logits_lse_fwd": 6.859e9, "logits_grad_recompute": 13.740e9,
                      "gemm_dH": 79.425e9, "gemm_dW": 20.412e9}}
 KERNEL_SOURCES = ["paper_2607_20908_gb300/csrc/gemm.cu", "paper_2607_20908_gb300/csrc/tc.cuh",
-                  "paper_2607_20908_gb300/csrc/internal.h"]
+                  "paper_2607_20908_gb300/csrc/gemm.h"]
 
 
 def kernel_traffic(name):

@@ -19,7 +19,7 @@
 //   EPI_DW   : dW = G^T H rows, fp32, overwrite or accumulate.
 #include <math.h>
 
-#include "internal.h"
+#include "gemm.h"
 #include "tc.cuh"
 
 namespace spo {
