@@ -97,6 +97,14 @@ SPO_API int spo_last_error(char* buf, size_t n);
  * Returns SPO_ERR_TIMEOUT if a wait expired, else SPO_OK / SPO_ERR_CUDA. */
 SPO_API spo_status spo_device_error(int* code, void* stream);
 
+/* Failure-detection self-test: enqueues one thread that waits, through the
+ * tensor-core kernels' own bounded wait, on a shared-memory barrier nothing
+ * ever arrives on.  The wait gives up after its limit (1 s), records code
+ * 0x1ff in the error word and the kernel returns, so the context stays
+ * usable; the next spo_device_error reports SPO_ERR_TIMEOUT with that code.
+ * Faults, traps and hangs nothing. */
+SPO_API spo_status spo_selftest_bounded_wait(void* stream);
+
 /* ---------------------------------------------------------------------------
  * a1. Loss-token selection (section 3, "Multi-turn RL Training": the loss uses
  * only unmasked tokens within a 1024-token window of each generation).

@@ -540,6 +540,15 @@ SPO_API spo_status spo_device_error(int* code, void* stream) {
   return ok();
 }
 
+SPO_API spo_status spo_selftest_bounded_wait(void* stream) {
+  DevInfo di;
+  spo_status st = device_info(&di);
+  if (st != SPO_OK) return st;
+  SPO_CUDA(spo::launch_bounded_wait_selftest(di.err, static_cast<cudaStream_t>(stream)),
+           "self-test launch");
+  return ok();
+}
+
 SPO_API spo_status spo_token_select(const int32_t* cu_seqlens, const uint8_t* mask,
                                     const int32_t* tgt, int32_t n_seq, int64_t T, int32_t window,
                                     uint8_t* loss_mask, int32_t* n_tok, void* stream) {

@@ -642,6 +642,25 @@ cudaError_t make_tmap_f32(CUtensorMap* tm, const void* base, uint64_t inner, uin
                       box_outer);
 }
 
+namespace {
+// One thread waits, through the kernels' own bounded wait, on an mbarrier that
+// nothing arrives on: the wait gives up after kWaitTimeoutNs and records
+// kErrWaitSelftest in the error word, and the kernel returns.
+__global__ void bounded_wait_selftest_kernel(int* err) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  abort_flag = 0;
+  mbar_init(&bar, 1);
+  mbar_wait(&bar, 0, &abort_flag, err, kErrWaitSelftest);
+}
+}  // namespace
+
+cudaError_t launch_bounded_wait_selftest(int* err, cudaStream_t s) {
+  bounded_wait_selftest_kernel<<<1, 1, 0, s>>>(err);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_gemm(int epi, bool a_mn, bool b_mn, bool pair, const CUtensorMap& ta,
                         const CUtensorMap& tb, const CUtensorMap& tc, const GemmArgs& args, int grid,
                         cudaStream_t s) {

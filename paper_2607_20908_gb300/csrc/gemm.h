@@ -89,6 +89,9 @@ cudaError_t make_tmap_f32(CUtensorMap* tm, const void* base, uint64_t inner, uin
 // tensor map for the TMA-store epilogues (GRAD: G as bf16, box 64 x 32; DW:
 // dW as fp32, box 32 x 32; both 128-byte swizzled); ignored by LSE and DH.
 constexpr uint32_t kStoreBoxRows = 32;
+// One thread waits on a barrier nothing arrives on (bounded-wait self-test).
+cudaError_t launch_bounded_wait_selftest(int* err, cudaStream_t s);
+
 cudaError_t launch_gemm(int epi, bool a_mn, bool b_mn, bool pair, const CUtensorMap& ta,
                         const CUtensorMap& tb, const CUtensorMap& tc, const GemmArgs& args, int grid,
                         cudaStream_t s);

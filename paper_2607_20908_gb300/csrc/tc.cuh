@@ -20,6 +20,7 @@ enum DevErr : int {
   kErrWaitMma = 0x102,
   kErrWaitEpilogue = 0x103,
   kErrWaitDrain = 0x104,
+  kErrWaitSelftest = 0x1ff,  // the self-test's wait on a barrier nothing arrives on
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {

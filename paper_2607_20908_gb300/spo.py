@@ -63,6 +63,7 @@ _SIGS = {
                               _c_size, _vp], ctypes.c_int),
     "spo_policy_loss_fwd_noalloc": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, _i32, _vp, _i64, _f32,
                                      _f32, ctypes.c_int, _vp, _vp, _vp, _vp], ctypes.c_int),
+    "spo_selftest_bounded_wait": ([_vp], ctypes.c_int),
     "spo_group_advantages_workspace_size": ([_i32, _i32, ctypes.POINTER(_c_size)], ctypes.c_int),
     "spo_group_advantages_ws": ([_vp, _vp, _i32, _i32, ctypes.c_int, _f32, _vp, _vp, _c_size, _vp],
                                 ctypes.c_int),
@@ -374,6 +375,13 @@ def spo_policy_loss_bwd_slice(H, W_slice, v_offset: int, tgt, lse, g, inv_temp: 
                                            _ptr(dW_slice), int(bool(accumulate_dW)), _ptr(w),
                                            w.numel(), _stream(dev)))
     return dH_part, dW_slice
+
+
+def spo_selftest_bounded_wait(device=None):
+    """Enqueue the bounded-wait self-test on the current stream (returns at once;
+    the kernel gives up after about a second and records code 0x1ff)."""
+    dev = torch.device("cuda", torch.cuda.current_device()) if device is None else device
+    _check(lib().spo_selftest_bounded_wait(_stream(dev)))
 
 
 def spo_trace_enable(on: bool = True):
