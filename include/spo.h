@@ -452,23 +452,36 @@ SPO_API spo_status spo_policy_loss_fwd_noalloc(const float* logp, const float* o
 /* Launch tuning, host-global, for every later call on any device:
  *   SPO_TUNE_PAIR_MMA (default 1): 1 = two CTAs of a cluster share one
  *     256 x 256 tile through a cta_group::2 MMA, 0 = one CTA per 128 x 256 tile.
- *   SPO_TUNE_GROUP_M (default 16): output tiles walked together by the
- *     persistent raster (L2 reuse of the streamed operand).
- *   SPO_TUNE_RASTER (default 0): 0 = groups of tile rows, 1 = groups of tile
- *     columns.
+ *   SPO_TUNE_GROUP_M: tile rows (or columns) walked together by the
+ *     persistent raster (L2 reuse of the streamed operand), for every GEMM;
+ *     SPO_TUNE_GROUP_M_FWD / _GRAD / _DH / _DW set one GEMM (trace kinds 0-3;
+ *     defaults 16, 16, 4, 8).
+ *   SPO_TUNE_RASTER: 0 = groups of tile rows, 1 = groups of tile columns, for
+ *     every GEMM; SPO_TUNE_RASTER_FWD / _GRAD / _DH / _DW one GEMM (defaults
+ *     0, 0, 0, 1).
  *   SPO_TUNE_DYNAMIC_MASK (default 15): bit k set = GEMM kind k (trace kinds
  *     0-3) takes its tiles in raster order from an atomic counter instead of
  *     a static round robin, so in-flight tiles stay a contiguous window.
  *   SPO_TUNE_DW_SPLIT_ROWS (default 8192; multiple of 256, 0 = off): dW =
  *     G^T H is reduced over at most this many token rows per pass, later
  *     passes adding into dW (smaller operand slabs stay in L2).
+ *   SPO_TUNE_DEFAULTS (value ignored): every setting back to its default.
  * Results do not depend on any setting beyond fp32 summation order. */
 typedef enum spo_tune_key {
     SPO_TUNE_PAIR_MMA = 0,
     SPO_TUNE_GROUP_M = 1,
     SPO_TUNE_RASTER = 2,
     SPO_TUNE_DYNAMIC_MASK = 3,
-    SPO_TUNE_DW_SPLIT_ROWS = 4
+    SPO_TUNE_DW_SPLIT_ROWS = 4,
+    SPO_TUNE_GROUP_M_FWD = 5,
+    SPO_TUNE_GROUP_M_GRAD = 6,
+    SPO_TUNE_GROUP_M_DH = 7,
+    SPO_TUNE_GROUP_M_DW = 8,
+    SPO_TUNE_RASTER_FWD = 9,
+    SPO_TUNE_RASTER_GRAD = 10,
+    SPO_TUNE_RASTER_DH = 11,
+    SPO_TUNE_RASTER_DW = 12,
+    SPO_TUNE_DEFAULTS = 13
 } spo_tune_key;
 SPO_API spo_status spo_set_tuning(int key, int64_t value);
 

@@ -178,8 +178,14 @@ BwdWs carve_bwd(void* base, long long T, long long d, long long V) {
 // Host-global launch choices (spo_set_tuning): CTA-pair MMA on/off and the
 // number of tile rows walked together by the raster.
 int g_tune_pair = 1;
-int g_tune_group_m = 16;
-int g_tune_raster = 0;
+// Per GEMM kind (0 logits + logsumexp, 1 recompute -> G, 2 dH, 3 dW), from
+// DRAM-traffic sweeps at the full workload: the logits GEMMs walk 16 tile rows
+// together; dH, whose tiles reduce over the whole vocabulary, re-reads least
+// with 4; dW with groups of 8 tile columns.
+constexpr int kDefaultGroupM[4] = {16, 16, 4, 8};
+constexpr int kDefaultRaster[4] = {0, 0, 0, 1};
+int g_tune_group_m[4] = {kDefaultGroupM[0], kDefaultGroupM[1], kDefaultGroupM[2], kDefaultGroupM[3]};
+int g_tune_raster[4] = {kDefaultRaster[0], kDefaultRaster[1], kDefaultRaster[2], kDefaultRaster[3]};
 // Bit k set: GEMM kind k takes its tiles from an atomic counter (dynamic
 // schedule) instead of the static round robin, so the tiles in flight stay a
 // contiguous window of the raster however the CTA pairs drift.  Default: all.
@@ -258,6 +264,8 @@ spo_status traced_gemm(int kind, bool a_mn, bool b_mn, const CUtensorMap& ta, co
                        const CUtensorMap& tc, const spo::GemmArgs& args_in, int grid, cudaStream_t s,
                        int* counters) {
   spo::GemmArgs args = args_in;
+  args.group_m = g_tune_group_m[kind];
+  args.raster = g_tune_raster[kind];
   args.tile_counter = nullptr;
   if (counters && ((g_tune_dynamic_mask >> kind) & 1)) {
     args.tile_counter = counters + kind;
@@ -271,8 +279,7 @@ spo_status traced_gemm(int kind, bool a_mn, bool b_mn, const CUtensorMap& ta, co
 spo::GemmArgs base_args(const DevInfo& di) {
   spo::GemmArgs a;
   memset(&a, 0, sizeof(a));
-  a.group_m = g_tune_group_m;
-  a.raster = g_tune_raster;
+  a.group_m = 1;  // set per kind at launch
   a.scale = 1.f;
   a.err = di.err;
   return a;
@@ -861,7 +868,7 @@ SPO_API spo_status spo_set_tuning(int key, int64_t value) {
       return ok();
     case SPO_TUNE_GROUP_M:
       if (value < 1 || value > 4096) return fail(SPO_ERR_INVALID_ARG, "group_m must be in [1, 4096]");
-      g_tune_group_m = static_cast<int>(value);
+      for (int k = 0; k < 4; ++k) g_tune_group_m[k] = static_cast<int>(value);
       return ok();
     case SPO_TUNE_DYNAMIC_MASK:
       if (value < 0 || value > 15) return fail(SPO_ERR_INVALID_ARG, "dynamic mask must be in [0, 15]");
@@ -872,9 +879,32 @@ SPO_API spo_status spo_set_tuning(int key, int64_t value) {
         return fail(SPO_ERR_INVALID_ARG, "dW split rows must be a multiple of 256 in [0, 2^24]");
       g_tune_dw_split = static_cast<int>(value);
       return ok();
+    case SPO_TUNE_GROUP_M_FWD:
+    case SPO_TUNE_GROUP_M_GRAD:
+    case SPO_TUNE_GROUP_M_DH:
+    case SPO_TUNE_GROUP_M_DW:
+      if (value < 1 || value > 4096) return fail(SPO_ERR_INVALID_ARG, "group_m must be in [1, 4096]");
+      g_tune_group_m[key - SPO_TUNE_GROUP_M_FWD] = static_cast<int>(value);
+      return ok();
+    case SPO_TUNE_RASTER_FWD:
+    case SPO_TUNE_RASTER_GRAD:
+    case SPO_TUNE_RASTER_DH:
+    case SPO_TUNE_RASTER_DW:
+      if (value != 0 && value != 1) return fail(SPO_ERR_INVALID_ARG, "raster must be 0 or 1");
+      g_tune_raster[key - SPO_TUNE_RASTER_FWD] = static_cast<int>(value);
+      return ok();
+    case SPO_TUNE_DEFAULTS:
+      g_tune_pair = 1;
+      for (int k = 0; k < 4; ++k) {
+        g_tune_group_m[k] = kDefaultGroupM[k];
+        g_tune_raster[k] = kDefaultRaster[k];
+      }
+      g_tune_dynamic_mask = 0xF;
+      g_tune_dw_split = 8192;
+      return ok();
     case SPO_TUNE_RASTER:
       if (value != 0 && value != 1) return fail(SPO_ERR_INVALID_ARG, "raster must be 0 or 1");
-      g_tune_raster = static_cast<int>(value);
+      for (int k = 0; k < 4; ++k) g_tune_raster[k] = static_cast<int>(value);
       return ok();
     default:
       return fail(SPO_ERR_INVALID_ARG, "unknown tuning key %d", key);

@@ -175,8 +175,7 @@ def test_single_cta_mode_matches_oracle():
         case["mask"] = (torch.rand(case["T"], generator=torch.Generator().manual_seed(9)) > 0.3).to(torch.uint8)
         _compare(case)
     finally:
-        spo.spo_set_tuning(spo.SPO_TUNE_PAIR_MMA, 1)
-        spo.spo_set_tuning(spo.SPO_TUNE_GROUP_M, 16)
+        spo.spo_set_tuning(spo.SPO_TUNE_DEFAULTS, 0)
 
 
 @pytest.mark.parametrize("mask", [0, 15])
@@ -192,8 +191,7 @@ def test_static_and_dynamic_tile_schedules(mask):
         case = inputs.tiny_case(seed=1082, T_per_seq=125, n_groups=2, rollouts=4, d=320, V=5000)
         _compare(case)
     finally:
-        spo.spo_set_tuning(spo.SPO_TUNE_DYNAMIC_MASK, 15)
-        spo.spo_set_tuning(spo.SPO_TUNE_GROUP_M, 16)
+        spo.spo_set_tuning(spo.SPO_TUNE_DEFAULTS, 0)
 
 
 def test_validate_inputs_counts_planted_errors():
@@ -238,4 +236,4 @@ def test_dw_split_passes():
         case = inputs.tiny_case(seed=1121, T_per_seq=125, n_groups=2, rollouts=4, d=320, V=5000)
         _compare(case)
     finally:
-        spo.spo_set_tuning(spo.SPO_TUNE_DW_SPLIT_ROWS, 8192)
+        spo.spo_set_tuning(spo.SPO_TUNE_DEFAULTS, 0)
