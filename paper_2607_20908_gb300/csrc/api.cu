@@ -178,21 +178,17 @@ BwdWs carve_bwd(void* base, long long T, long long d, long long V) {
 // Host-global launch choices (spo_set_tuning): CTA-pair MMA on/off and the
 // number of tile rows walked together by the raster.
 int g_tune_pair = 1;
-// Per GEMM kind (0 logits + logsumexp, 1 recompute -> G, 2 dH, 3 dW), from
-// DRAM-traffic sweeps at the full workload: the logits GEMMs walk 16 tile rows
-// together; dH, whose tiles reduce over the whole vocabulary, re-reads least
-// with 4; dW with groups of 8 tile columns.
-constexpr int kDefaultGroupM[4] = {16, 16, 4, 8};
-constexpr int kDefaultRaster[4] = {0, 0, 0, 1};
+using spo::kDefaultGroupM;
+using spo::kDefaultRaster;
 int g_tune_group_m[4] = {kDefaultGroupM[0], kDefaultGroupM[1], kDefaultGroupM[2], kDefaultGroupM[3]};
 int g_tune_raster[4] = {kDefaultRaster[0], kDefaultRaster[1], kDefaultRaster[2], kDefaultRaster[3]};
 // Bit k set: GEMM kind k takes its tiles from an atomic counter (dynamic
 // schedule) instead of the static round robin, so the tiles in flight stay a
 // contiguous window of the raster however the CTA pairs drift.  Default: all.
-int g_tune_dynamic_mask = 0xF;
+int g_tune_dynamic_mask = spo::kDefaultDynamicMask;
 // dW = G^T H runs as passes over at most this many token rows (0: one pass
 // per chunk): smaller operand slabs keep a wave's working set inside L2.
-int g_tune_dw_split = 8192;
+int g_tune_dw_split = spo::kDefaultDwSplitRows;
 
 // ------------------------------------------------------------ tracing
 // When enabled, a start/stop CUDA event pair is recorded on the launch stream
@@ -899,8 +895,8 @@ SPO_API spo_status spo_set_tuning(int key, int64_t value) {
         g_tune_group_m[k] = kDefaultGroupM[k];
         g_tune_raster[k] = kDefaultRaster[k];
       }
-      g_tune_dynamic_mask = 0xF;
-      g_tune_dw_split = 8192;
+      g_tune_dynamic_mask = spo::kDefaultDynamicMask;
+      g_tune_dw_split = spo::kDefaultDwSplitRows;
       return ok();
     case SPO_TUNE_RASTER:
       if (value != 0 && value != 1) return fail(SPO_ERR_INVALID_ARG, "raster must be 0 or 1");

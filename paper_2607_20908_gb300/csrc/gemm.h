@@ -22,6 +22,17 @@ constexpr int kRowPad = 256;
 // Floats of logsumexp partials per 32 rows and vocab tile: three planes of 32.
 constexpr int kPartialBlock = 96;
 
+// Default launch schedule per GEMM kind (0 logits + logsumexp, 1 recompute
+// -> G, 2 dH, 3 dW), from DRAM-traffic sweeps at the full workload: the
+// logits GEMMs walk 16 tile rows together, dH (whose tiles reduce over the
+// whole vocabulary) re-reads least with 4, dW with groups of 8 tile columns;
+// every GEMM takes its tiles from an atomic counter; dW reduces over passes
+// of at most 8192 token rows.
+constexpr int kDefaultGroupM[4] = {16, 16, 4, 8};
+constexpr int kDefaultRaster[4] = {0, 0, 0, 1};
+constexpr int kDefaultDynamicMask = 0xF;
+constexpr int kDefaultDwSplitRows = 8192;
+
 // What the epilogue does with a finished 128 x 256 fp32 accumulator tile.
 enum EpiKind : int {
   EPI_LSE = 0,   // online max / sum-exp / sum-exp*z per row + target logit -> partials
