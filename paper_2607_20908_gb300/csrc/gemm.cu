@@ -3,10 +3,16 @@
 //
 //   C[M, N] = A[M, K] * B[N, K]^T    (bf16 in, fp32 accumulate in TMEM)
 //
-// One CTA per SM walks output tiles of 128 x 256.  Warp 0 issues TMA loads
-// into a 4-stage shared-memory ring, warp 1 issues tcgen05.mma (one thread)
-// into one of two TMEM accumulators (2 x 256 columns), warps 2-5 drain the
-// other accumulator through the epilogue, so MMA and epilogue overlap.
+// One CTA per SM.  By default two CTAs of a cluster share each 256 x 256
+// output tile through a cta_group::2 MMA (each stages 128 rows of A and half
+// of the tile's B rows); with SPO_TUNE_PAIR_MMA = 0 a CTA owns a 128 x 256
+// tile alone.  Warp 0 issues TMA loads into a shared-memory ring (7 stages of
+// 32 KB per CTA in pair mode, 6 when the epilogue stages its TMA stores, 4 of
+// 48 KB alone), warp 1 issues tcgen05.mma from one thread into one of two TMEM
+// accumulators (2 x 256 columns), and warps 2-5 drain the other accumulator
+// through the epilogue, so MMA and epilogue overlap.  Tiles are taken in a
+// grouped raster order, statically or from an atomic counter whose values the
+// leader's producer publishes to both CTAs through a shared-memory ring.
 // Operands may be K-major (rows of K contiguous) or MN-major (rows of M or N
 // contiguous); both are staged with the 128-byte swizzle.
 //
@@ -14,9 +20,11 @@
 //   EPI_LSE  : forward. Online max / sum-exp / sum-exp*z of each row over the
 //              tile plus the target logit; writes one partial per
 //              (vocab tile, row).  The logits themselves never leave TMEM.
-//   EPI_GRAD : backward. G = inv_temp * g_t * (onehot - exp(z - lse_t)) in bf16.
-//   EPI_DH   : dH = G W rows, bf16, scattered back to token rows.
-//   EPI_DW   : dW = G^T H rows, fp32, overwrite or accumulate.
+//   EPI_GRAD : backward. G = inv_temp * g_t * (onehot - exp(z - lse_t)) in
+//              bf16, through TMA bulk stores.
+//   EPI_DH   : dH = G W rows scattered back to token rows, bf16 (or fp32 for
+//              one vocabulary slice's part).
+//   EPI_DW   : dW = G^T H, fp32 through TMA bulk stores or reduce-adds.
 #include <math.h>
 
 #include "gemm.h"

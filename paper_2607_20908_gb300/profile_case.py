@@ -6,9 +6,11 @@ sweeps.
     python -m paper_2607_20908_gb300.profile_case --V 151936 --iters 1 \\
         --configs "1,16,0;1,8,0;0,16,0"
 
---configs is a ';'-separated list of "pair,group,raster[,dynamic_mask[,dw_split_rows]]"
-launch tunings (spo_set_tuning); each is run for --iters iterations of
-fwd + bwd.  The default reduced size keeps the reduction lengths of the full workload
+--configs is a ';'-separated list of launch tunings (spo_set_tuning), each
+either "pair,group,raster[,dynamic_mask[,dw_split_rows]]" applied to every
+GEMM, or '|'-separated "key=value" settings (spo_tune_key numbers, e.g.
+"7=4|11=0" for dH's raster group and direction) applied after the defaults;
+each is run for --iters iterations of fwd + bwd.  The default reduced size keeps the reduction lengths of the full workload
 (K = d = 5120 for the logits and their recompute, K = T = 16384 tokens for
 dW) with a vocabulary cut to 8192, so one launch takes about a millisecond
 and the device holds about 1 GB; the streamed operands of dW (G = 268 MB,
@@ -47,9 +49,15 @@ def main():
                        device=dev)
     dH = torch.empty(a.T, a.d, dtype=torch.bfloat16, device=dev)
     dW = torch.empty(a.V, a.d, dtype=torch.float32, device=dev)
-    configs = [tuple(int(x) for x in c.split(",")) for c in a.configs.split(";") if c] or [None]
+    configs = [c if "=" in c else tuple(int(x) for x in c.split(","))
+               for c in a.configs.split(";") if c] or [None]
     for cfg in configs:
-        if cfg is not None:
+        if isinstance(cfg, str):
+            spo.spo_set_tuning(spo.SPO_TUNE_DEFAULTS, 0)
+            for kv in cfg.split("|"):
+                key, value = kv.split("=")
+                spo.spo_set_tuning(int(key), int(value))
+        elif cfg is not None:
             pair, group, raster = cfg[:3]
             spo.spo_set_tuning(spo.SPO_TUNE_PAIR_MMA, pair)
             spo.spo_set_tuning(spo.SPO_TUNE_GROUP_M, group)
@@ -63,7 +71,8 @@ def main():
             _, _, lse = spo.spo_logprobs_fwd(H, W, tgt, ws=ws_f)
             spo.spo_policy_loss_bwd(H, W, tgt, lse, gl, dH=dH, dW=dW, ws=ws_b)
         torch.cuda.synchronize()
-        label = "default" if cfg is None else "pair,group,raster,dynamic=" + ",".join(map(str, cfg))
+        label = ("default" if cfg is None else cfg if isinstance(cfg, str)
+                 else "pair,group,raster,dynamic=" + ",".join(map(str, cfg)))
         print(f"--- {label}")
         recs = [(k, ms) for k, ms in spo.spo_trace_read() if k <= 3]
         per_kind = {k: sum(1 for kk, _ in recs if kk == k) for k, _ in recs}
