@@ -65,12 +65,15 @@ WORKLOADS = {
               "prompt/feedback tokens masked, per-turn rewards, d=5120, V=151936, bf16 fwd+bwd",
     "large": "large batch: T=131072 packed tokens, groups of 4/8/16, 5% of rollouts in zero-variance "
              "groups, KL to reference log-probs, d=5120, V=151936, bf16 fwd+bwd (4 backward chunks)",
+    "vocab-split": WORKLOAD + "; vocabulary-split form: the head's rows as 2 slices of 75968, run "
+                   "in turn on one GPU (per-slice log-prob records merged, fp32 dH parts summed on "
+                   "the device where ranks would all-gather / all-reduce, dW written per slice)",
 }
 
 KERNEL_NAMES = {0: "logits_lse_fwd", 1: "logits_grad_recompute", 2: "gemm_dH", 3: "gemm_dW",
                 4: "lse_combine", 5: "select_gather_fwd", 6: "select_gather_bwd",
                 7: "policy_loss_fwd", 8: "group_advantages", 9: "token_select",
-                10: "reward_compose"}
+                10: "reward_compose", 12: "merge_slices"}
 GEMM_KINDS = ("logits_lse_fwd", "logits_grad_recompute", "gemm_dH", "gemm_dW")
 SAMPLE_SEQS, SAMPLE_TOKENS = 8, 8   # CPU sample: one group of 8 rollouts, first 8 tokens each
 
@@ -235,6 +238,14 @@ class Step:
         self.g = torch.empty(T, **f32)
         self.dH = torch.empty((T, d), dtype=torch.bfloat16, device=dev)
         self.dW = torch.empty((V, d), **f32)
+        # vocabulary-split form: slices of W's rows run in turn, records merged
+        self.slices = []
+        if case.get("vocab_slices"):
+            from paper_2607_20908_gb300 import shard
+            self.slices = shard.vocab_slices(V, case["vocab_slices"])
+            self.rec = torch.empty((len(self.slices), T, 4), **f32)
+            self.dH_parts = [torch.empty((T, d), **f32) for _ in self.slices]
+            self.dH = torch.empty((T, d), **f32)   # the sum of the parts (fp32)
         self.ws_f = torch.empty(spo.logprobs_workspace_size(T, d, V), dtype=torch.uint8, device=dev)
         self.ws_l = torch.empty(max(256, spo.policy_loss_workspace_size(self.n_seq, self.n_groups)),
                                 dtype=torch.uint8, device=dev)
@@ -263,9 +274,17 @@ class Step:
             return
         chk(L.spo_token_select(p(self.cu), p(self.mask), p(self.tgt), self.n_seq, self.T, c["window"],
                                p(self.loss_mask), p(self.n_tok), s))
-        chk(L.spo_logprobs_fwd(p(self.H), p(self.W), p(self.tgt), p(self.loss_mask), self.T, self.d,
-                               self.V, c["inv_temp"], p(self.logp), p(self.ent), p(self.lse),
-                               p(self.ws_f), self.ws_f.numel(), s))
+        if self.slices:
+            for k, (off, n) in enumerate(self.slices):
+                chk(L.spo_logprobs_fwd_slice(p(self.H), p(self.W[off:off + n]), p(self.tgt),
+                                             p(self.loss_mask), self.T, self.d, n, off, c["inv_temp"],
+                                             p(self.rec[k]), p(self.ws_f), self.ws_f.numel(), s))
+            chk(L.spo_logprobs_merge_slices(p(self.rec), len(self.slices), self.T, p(self.logp),
+                                            p(self.ent), p(self.lse), s))
+        else:
+            chk(L.spo_logprobs_fwd(p(self.H), p(self.W), p(self.tgt), p(self.loss_mask), self.T,
+                                   self.d, self.V, c["inv_temp"], p(self.logp), p(self.ent),
+                                   p(self.lse), p(self.ws_f), self.ws_f.numel(), s))
         if stop_after_fwd:
             return
         chk(L.spo_group_advantages(p(self.rewards), p(self.gid), self.n_seq, self.n_groups, 0, 1e-6,
@@ -277,9 +296,22 @@ class Step:
         if self.dist:
             chk(L.spo_scale_f32(p(self.g), self.T, self.dp_weight, None, s))
             chk(L.spo_scale_f32(p(self.loss), 1, self.dp_weight, None, s))
-        chk(L.spo_policy_loss_bwd(p(self.H), p(self.W), p(self.tgt), p(self.lse), p(self.g), self.T,
-                                  self.d, self.V, c["inv_temp"], p(self.dH), p(self.dW), 0,
-                                  p(self.ws_b), self.ws_b.numel(), s))
+        if self.slices:
+            for k, (off, n) in enumerate(self.slices):
+                chk(L.spo_policy_loss_bwd_slice(p(self.H), p(self.W[off:off + n]), p(self.tgt),
+                                                p(self.lse), p(self.g), self.T, self.d, n, off,
+                                                c["inv_temp"], p(self.dH_parts[k]),
+                                                p(self.dW[off:off + n]), 0, p(self.ws_b),
+                                                self.ws_b.numel(), s))
+            # stands in for the ranks' all-reduce of their dH parts
+            with torch.cuda.stream(self.stream):
+                torch.add(self.dH_parts[0], self.dH_parts[1], out=self.dH)
+                for part in self.dH_parts[2:]:
+                    self.dH.add_(part)
+        else:
+            chk(L.spo_policy_loss_bwd(p(self.H), p(self.W), p(self.tgt), p(self.lse), p(self.g),
+                                      self.T, self.d, self.V, c["inv_temp"], p(self.dH),
+                                      p(self.dW), 0, p(self.ws_b), self.ws_b.numel(), s))
         if self.dist:   # the one real exchange of data-parallel training: sum of dW (and the loss)
             self.dist.pg.all_reduce(self.dW)
             self.dist.pg.all_reduce(self.loss)
@@ -527,6 +559,8 @@ def config_block(case, T_L, world, workload="full"):
         cfg.update(groups=case["n_groups"], sequences=int(case["cu_seqlens"].numel() - 1))
     if workload != "forward":
         cfg.update(clip_eps=case["clip_eps"], kl_beta=case["kl_beta"], window=case["window"])
+    if case.get("vocab_slices"):
+        cfg["vocab_slices"] = case["vocab_slices"]
     cfg["l2"] = "inputs larger than L2 (W alone is 1.2-1.56 GB and is streamed every step)"
     cfg["parallelism"] = (f"dp{world}: whole groups per GPU, dW and loss all-reduced (NCCL) every step"
                           if world > 1 else "1 GPU")
@@ -543,11 +577,14 @@ def ours(args):
         build.build()
     dist.barrier()
     maker = {"full": inputs.full_case, "forward": inputs.forward_case, "ragged": inputs.ragged_case,
-             "large": inputs.large_case}[args.workload]
-    seed0 = {"full": 1003, "forward": 1002, "ragged": 1004, "large": 1005}[args.workload]
+             "large": inputs.large_case, "vocab-split": inputs.full_case}[args.workload]
+    seed0 = {"full": 1003, "forward": 1002, "ragged": 1004, "large": 1005,
+             "vocab-split": 1003}[args.workload]
     case = maker(seed=seed0 + dist.rank, device=str(dev))
-    if args.workload == "forward" and dist.world > 1:
-        raise SystemExit("--workload forward runs on one GPU")
+    if args.workload in ("forward", "vocab-split") and dist.world > 1:
+        raise SystemExit(f"--workload {args.workload} runs on one GPU")
+    if args.workload == "vocab-split":
+        case["vocab_slices"] = 2
     st = Step(case, dev, dist)
     st.prepare_old_ref()
     torch.cuda.synchronize(dev)
