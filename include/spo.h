@@ -35,6 +35,11 @@
  *   - A launch failure returns SPO_ERR_CUDA.  Every device-side wait in the
  *     tensor-core kernels is bounded; a wait that expires records a code that
  *     spo_device_error() returns (SPO_ERR_TIMEOUT) instead of hanging.
+ *   - Results are bit-reproducible run to run: every output element is
+ *     reduced in one fixed order whatever the order in which tiles are
+ *     scheduled.  The compute calls make no host synchronisation and no
+ *     allocation, so a sequence of them can be captured into a CUDA graph
+ *     (workspaces and buffers fixed) and replayed.
  *   - The sign convention is that of an optimiser: `loss` = -J_GRPO, to be
  *     minimised.
  *

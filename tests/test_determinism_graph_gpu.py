@@ -1,0 +1,122 @@
+"""Run-to-run determinism and CUDA-graph capture of the whole step.
+
+The tile schedule hands tiles to whichever CTA pair asks first, but every
+output element is still reduced in one fixed order (one CTA per output tile,
+fixed K order; the combine, advantages and loss in fixed orders; dW passes in
+stream order), so two runs give the same bits.  The step makes no host
+synchronisation and no allocation of its own, so it captures into a CUDA
+graph whose replays give the same bits as eager calls and re-read inputs
+updated in place."""
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2607_20908_gb300 import inputs
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def spo():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    from paper_2607_20908_gb300 import build
+    build.build()
+    from paper_2607_20908_gb300 import spo as mod
+    return mod
+
+
+def _tensors(spo, case):
+    dev = torch.device("cuda")
+    t = {k: case[k].to(dev) for k in ("H", "W", "tgt", "mask", "rewards")}
+    t["cu"], t["gid"] = case["cu_seqlens"].to(dev), case["group_id"].to(dev)
+    for k in ("n_groups", "window", "inv_temp", "clip_eps", "kl_beta"):
+        t[k] = case[k]
+    T, d, V = case["T"], case["d"], case["V"]
+    n_seq = t["cu"].numel() - 1
+    u8 = dict(dtype=torch.uint8, device=dev)
+    t["ws_f"] = torch.empty(spo.logprobs_workspace_size(T, d, V), **u8)
+    t["ws_l"] = torch.empty(max(256, spo.policy_loss_workspace_size(n_seq, case["n_groups"])), **u8)
+    t["ws_b"] = torch.empty(spo.policy_loss_bwd_workspace_size(T, d, V), **u8)
+    lm, _ = spo.spo_token_select(t["cu"], t["mask"], t["tgt"], t["window"])
+    logp, _, _ = spo.spo_logprobs_fwd(t["H"], t["W"], t["tgt"], lm, t["inv_temp"], ws=t["ws_f"])
+    t["old"] = (logp + case["old_noise"].to(dev)).contiguous()
+    t["ref"] = (logp + case["ref_noise"].to(dev)).contiguous()
+    return t
+
+
+def _step(spo, t):
+    lm, _ = spo.spo_token_select(t["cu"], t["mask"], t["tgt"], t["window"])
+    logp, ent, lse = spo.spo_logprobs_fwd(t["H"], t["W"], t["tgt"], lm, t["inv_temp"], ws=t["ws_f"])
+    adv = spo.spo_group_advantages(t["rewards"], t["gid"], t["n_groups"])
+    loss, g, stats = spo.spo_policy_loss_fwd(logp, t["old"], t["ref"], adv, t["cu"], t["gid"],
+                                             t["n_groups"], lm, t["clip_eps"], t["kl_beta"], 0,
+                                             ws=t["ws_l"])
+    dH, dW = spo.spo_policy_loss_bwd(t["H"], t["W"], t["tgt"], lse, g, t["inv_temp"], ws=t["ws_b"])
+    return dict(logp=logp, ent=ent, lse=lse, adv=adv, loss=loss, g=g, stats=stats, dH=dH, dW=dW)
+
+
+def _same_bits(a, b):
+    for k in a:
+        assert torch.equal(a[k].view(torch.uint8) if a[k].dtype == torch.bfloat16 else a[k],
+                           b[k].view(torch.uint8) if b[k].dtype == torch.bfloat16 else b[k]), k
+
+
+def _medium_case():
+    """1600 tokens (7 tile rows, ragged), d = 256, V = 5000 (20 vocab tiles, ragged)."""
+    case = inputs.tiny_case(seed=1301, T_per_seq=100, n_groups=4, rollouts=4, V=5000)
+    case["mask"] = (torch.rand(case["T"], generator=torch.Generator().manual_seed(3)) > 0.25).to(
+        torch.uint8)
+    return case
+
+
+def test_two_runs_give_the_same_bits(spo):
+    t = _tensors(spo, _medium_case())
+    a = {k: v.clone() for k, v in _step(spo, t).items()}
+    b = _step(spo, t)
+    torch.cuda.synchronize()
+    _same_bits(a, b)
+    assert spo.spo_device_error() == 0
+
+
+def test_full_workload_backward_is_deterministic(spo):
+    """The benchmark's launch shape: dW (3.1 GB) and dH bit-identical across runs."""
+    case = inputs.full_case(device="cuda")
+    H, W, tgt = case["H"], case["W"], case["tgt"].cuda()
+    _, _, lse = spo.spo_logprobs_fwd(H, W, tgt)
+    gen = torch.Generator().manual_seed(11)
+    g = (torch.randn(case["T"], generator=gen) * 1e-4).float().cuda()
+    dH1, dW1 = spo.spo_policy_loss_bwd(H, W, tgt, lse, g)
+    dH1, dW1 = dH1.clone(), dW1.clone()
+    dH2, dW2 = spo.spo_policy_loss_bwd(H, W, tgt, lse, g)
+    torch.cuda.synchronize()
+    assert torch.equal(dW1, dW2)
+    assert torch.equal(dH1.view(torch.int16), dH2.view(torch.int16))
+    del H, W, dW1, dW2
+    torch.cuda.empty_cache()
+
+
+def test_step_captures_into_a_cuda_graph(spo):
+    t = _tensors(spo, _medium_case())
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):          # warm-up off the capture stream
+        _step(spo, t)
+    torch.cuda.current_stream().wait_stream(side)
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        out = _step(spo, t)
+    graph.replay()
+    torch.cuda.synchronize()
+    _same_bits({k: v.clone() for k, v in _step(spo, t).items()}, out)
+    # new rewards written in place: the replay reads them
+    gen = torch.Generator().manual_seed(5)
+    t["rewards"].copy_(torch.rand(t["rewards"].numel(), generator=gen) * 3.0)
+    graph.replay()
+    torch.cuda.synchronize()
+    eager = _step(spo, t)
+    torch.cuda.synchronize()
+    _same_bits(eager, out)
+    assert not np.allclose(eager["adv"].cpu().numpy(), 0)
+    assert spo.spo_device_error() == 0
