@@ -105,8 +105,9 @@ def _loss_check(spo, case, loss_mask_gpu, loss_mask_np, seed, agg=0):
     loss, g, stats = spo.spo_policy_loss_fwd(
         logp.cuda(), old.cuda(), ref.cuda(), adv, case["cu_seqlens"].cuda(), case["group_id"].cuda(),
         case["n_groups"], loss_mask_gpu, case["clip_eps"], case["kl_beta"], agg)
+    # the oracle's own fp32-order advantages (the same bits as the kernel's, checked above)
     loss_o, g_o, st_o = O.policy_loss(logp.double().numpy(), old.double().numpy(),
-                                      ref.double().numpy(), adv.cpu().double().numpy(),
+                                      ref.double().numpy(), adv32.astype(np.float64),
                                       case["cu_seqlens"].numpy(), case["group_id"].numpy(),
                                       case["n_groups"], loss_mask_np, case["clip_eps"],
                                       case["kl_beta"], agg)
