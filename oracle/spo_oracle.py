@@ -70,17 +70,16 @@ def token_select(cu_seqlens, mask, tgt, window: int):
 
     Returns (loss_mask uint8[T], n_tok int64[n_seq]).
     """
-    cu = [int(v) for v in cu_seqlens]
-    T = cu[-1]
-    loss_mask = np.zeros(T, dtype=np.uint8)
-    n_tok = np.zeros(len(cu) - 1, dtype=np.int64)
-    for i in range(len(cu) - 1):
-        kept = 0
-        for t in range(cu[i], cu[i + 1]):
-            if int(mask[t]) == 1 and int(tgt[t]) >= 0 and (window <= 0 or kept < window):
-                loss_mask[t] = 1
-                kept += 1
-        n_tok[i] = kept
+    cu = np.asarray(cu_seqlens).astype(np.int64)
+    n_seq = cu.size - 1
+    eligible = (np.asarray(mask).astype(np.int64) == 1) & (np.asarray(tgt).astype(np.int64) >= 0)
+    seq = np.repeat(np.arange(n_seq), np.diff(cu))             # the sequence of every token
+    upto = np.cumsum(eligible)                                  # eligible tokens in [0, t]
+    at_start = np.concatenate([[0], upto])[cu[:-1]]             # eligible tokens before each sequence
+    earlier = upto - eligible - at_start[seq]                   # earlier eligible tokens of t's sequence
+    keep = eligible & ((window <= 0) | (earlier < window))
+    loss_mask = keep.astype(np.uint8)
+    n_tok = np.bincount(seq, weights=keep, minlength=n_seq).astype(np.int64)
     return loss_mask, n_tok
 
 
