@@ -167,6 +167,12 @@ def test_advantage_degenerate_groups():
         assert a[0] == 0 and a[1] == 0 and a[2] == 0      # zero variance
         assert a[3] == 0                                   # singleton group
         assert a[4] > 0 > a[5]
+    # identical rewards whose mean is not exact in binary (3 x 0.1 sums to 0.30000000000000004):
+    # the zero-variance rule, not the arithmetic, gives exactly 0, even with eps = 0
+    r = np.array([0.1, 0.1, 0.1, 0.7, 0.7, 0.7])
+    gid = np.array([0, 0, 0, 1, 1, 1])
+    for fn in (O.group_advantages, O.group_advantages_f32):
+        assert not fn(r, gid, 2, O.STD_UNBIASED, 0.0).any()
 
 
 def test_advantage_f32_matches_f64():
@@ -215,6 +221,15 @@ def test_ratio_one_no_kl_is_minus_mean_advantage():
     want_t = -(np.repeat(adv, lens)).mean()
     assert abs(loss_t - want_t) < 1e-12
     assert st["clip_frac"] == 0 and abs(st["mean_ratio"] - 1) < 1e-15
+    # with masked tokens the means run over loss tokens only
+    lm = (rng.random(T) > 0.4).astype(np.uint8)
+    lm[cu[:-1]] = 1                               # every output keeps at least one token
+    per_tok = np.repeat(adv, lens)
+    loss_t, _, st = O.policy_loss(lp, lp, None, adv, cu, gid, 3, lm, 0.2, 0.0, O.AGG_TOKEN)
+    assert abs(loss_t + per_tok[lm == 1].mean()) < 1e-12
+    loss_s, _, _ = O.policy_loss(lp, lp, None, adv, cu, gid, 3, lm, 0.2, 0.0, O.AGG_SEQ_GROUP)
+    assert abs(loss_s - want) < 1e-12              # per-output token means: masks cancel
+    assert st["n_loss_tokens"] == int(lm.sum())
 
 
 def test_kl_properties():
