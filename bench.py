@@ -118,16 +118,27 @@ class Dist:
         self.rank = int(os.environ.get("RANK", "0"))
         self.local = int(os.environ.get("LOCAL_RANK", "0"))
         self.pg = None
+        self.device = None
 
-    def init(self, backend):
+    def init(self, backend, device=None):
+        """Joins the process group; with NCCL the group is bound to this rank's
+        GPU (set as the current device first) so no collective guesses GPU 0."""
+        self.device = device
         if self.world > 1:
             import torch.distributed as dist
-            dist.init_process_group(backend)
+            if device is not None and device.type == "cuda":
+                torch.cuda.set_device(device)
+                dist.init_process_group(backend, device_id=device)
+            else:
+                dist.init_process_group(backend)
             self.pg = dist
 
     def barrier(self):
         if self.pg:
-            self.pg.barrier()
+            if self.device is not None and self.device.type == "cuda":
+                self.pg.barrier(device_ids=[self.device.index])
+            else:
+                self.pg.barrier()
 
     def max(self, x: float, device) -> float:
         if not self.pg:
@@ -569,9 +580,9 @@ def config_block(case, T_L, world, workload="full"):
 
 def ours(args):
     dist = Dist()
-    dist.init("nccl")
     dev = torch.device("cuda", dist.local)
     torch.cuda.set_device(dev)
+    dist.init("nccl", dev)
     from paper_2607_20908_gb300 import build, spo
     if dist.rank == 0 and not os.path.exists(spo.LIB_PATH):
         build.build()
