@@ -6,6 +6,9 @@
 
 namespace spo {
 
+// SM count of the current device, cached per ordinal (1 if the query fails).
+int sm_count();
+
 // ---------------------------------------------------------------- small kernels
 // Compaction of selected rows: kind 0 selects (mask == NULL || mask[t]) &&
 // tgt[t] >= 0, kind 1 selects g[t] != 0.  Writes idx[0..count) ascending and

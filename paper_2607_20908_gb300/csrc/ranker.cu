@@ -223,18 +223,13 @@ __global__ void ranker_reduce_kernel(const float* block_part, int n_blocks, int 
   }
 }
 
-int sms_of_current_device() {
-  int dev = 0, sms = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  return sms > 0 ? sms : 1;
-}
+
 
 }  // namespace
 
 int ranker_blocks(int n_pairs) {
   const int want = (n_pairs + kWarps - 1) / kWarps;
-  const int cap = 2 * sms_of_current_device();
+  const int cap = 2 * sm_count();
   return want < 1 ? 1 : (want < cap ? want : cap);
 }
 
@@ -245,7 +240,7 @@ size_t ranker_ws_bytes(int n_pairs) {
 cudaError_t launch_ranker_scores(const float* phi, const float* mu, const float* sigma, int n,
                                  const float* params, float* scores, cudaStream_t s) {
   const int want = (n + kWarps - 1) / kWarps;
-  const int cap = 8 * sms_of_current_device();
+  const int cap = 8 * sm_count();
   ranker_scores_kernel<<<want < cap ? want : cap, kWarps * 32, 0, s>>>(phi, mu, sigma, n, params,
                                                                        scores);
   note_launches(1);

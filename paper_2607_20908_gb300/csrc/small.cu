@@ -756,9 +756,26 @@ __global__ void loss_final_kernel(const double* bpart, int nb, const unsigned lo
 
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
+
+
 std::atomic<long long> g_launches{0};
 
 }  // namespace
+
+// SM count of the current device, cached per ordinal (1 if the query fails:
+// grids stay valid, only smaller).
+int sm_count() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
+  static int cache[64] = {0};
+  if (cache[dev] == 0) {
+    int n = 0;
+    cache[dev] = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && n > 0
+                     ? n
+                     : 1;
+  }
+  return cache[dev];
+}
 
 void note_launches(int n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
 long long launches() { return g_launches.load(std::memory_order_relaxed); }
@@ -782,9 +799,7 @@ cudaError_t launch_gather(const __nv_bfloat16* H, int d, const int* idx, const i
                           long long tgt_off, long long tgt_lim, const float* a, float* a_c,
                           const float* b, float* b_c, cudaStream_t s) {
   const int row_vecs = d / 8;  // 16-byte pieces per row
-  int dev = 0, sms = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int sms = sm_count();
   const int blocks = max(1, min((rows_cap + 7) / 8, sms * 8));
   gather_kernel<<<blocks, 256, 0, s>>>(reinterpret_cast<const uint4*>(H), row_vecs, idx, count,
                                        rows_cap, reinterpret_cast<uint4*>(Hc), tgt, tgt_c,
@@ -845,9 +860,7 @@ cudaError_t launch_group_advantages_runs(const float* rewards, const int* group_
   cudaError_t e = cudaMemsetAsync(runs, 0, sizeof(int) * n_groups, s);
   if (e == cudaSuccess) e = cudaMemsetAsync(split, 0, sizeof(int), s);
   if (e != cudaSuccess) return e;
-  int dev = 0, sms = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int sms = sm_count();
   adv_runs_kernel<<<max(1, min((n_seq + 1023) / 1024, sms * 8)), 256, 0, s>>>(
       group_id, n_seq, n_groups, runs, start, end);
   adv_split_kernel<<<max(1, min((n_groups + 255) / 256, sms * 4)), 256, 0, s>>>(runs, n_groups,
@@ -863,9 +876,7 @@ cudaError_t launch_group_advantages_runs(const float* rewards, const int* group_
 cudaError_t launch_reward_compose(const uint8_t* compiled, const float* pass_rate,
                                   const float* speedup, const float* cv, const float* r_struct,
                                   int n, const RewardParams& q, float* out, cudaStream_t s) {
-  int dev = 0, sms = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int sms = sm_count();
   auto al = [](const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; };
   const bool vec = al(compiled, 4) && al(pass_rate, 16) && al(speedup, 16) && al(cv, 16) &&
                    al(out, 16) && (r_struct == nullptr || al(r_struct, 16));
@@ -891,9 +902,7 @@ cudaError_t launch_reward_compose(const uint8_t* compiled, const float* pass_rat
 }
 
 cudaError_t launch_scale(float* x, long long n, float alpha, const float* alpha_dev, cudaStream_t s) {
-  int dev = 0, sms = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int sms = sm_count();
   const long long want = (n + 255) / 256;
   const int blocks = static_cast<int>(want < sms * 8 ? (want < 1 ? 1 : want) : sms * 8);
   scale_kernel<<<blocks, 256, 0, s>>>(x, n, alpha, alpha_dev);
@@ -906,9 +915,7 @@ cudaError_t launch_validate(const int* tgt, long long T, long long V, const int*
                             const float* ref_logp, const uint8_t* mask, int* counts, cudaStream_t s) {
   cudaError_t e = cudaMemsetAsync(counts, 0, 6 * sizeof(int), s);
   if (e != cudaSuccess) return e;
-  int dev = 0, sms = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int sms = sm_count();
   const long long n = T > n_seq ? T : n_seq;
   const long long want = (n + 255) / 256;
   const int blocks = static_cast<int>(want < sms * 4 ? (want < 1 ? 1 : want) : sms * 4);
@@ -950,9 +957,7 @@ cudaError_t launch_policy_loss(const float* logp, const float* old_logp, const f
   cudaError_t e = cudaMemsetAsync(w.gsize, 0, sizeof(int) * n_groups, s);
   if (e == cudaSuccess) e = cudaMemsetAsync(w.scal, 0, 2 * sizeof(unsigned long long), s);
   if (e != cudaSuccess) return e;
-  int dev = 0, sms = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int sms = sm_count();
   const int per_block = kLossThreads / 32;  // sequences in flight per block
   const int seq_blocks = max(1, min((n_seq + per_block - 1) / per_block, sms * 8));
   loss_count_kernel<<<seq_blocks, kLossThreads, 0, s>>>(cu_seqlens, group_id, loss_mask, n_seq,
