@@ -1,4 +1,5 @@
-"""Run-to-run determinism and CUDA-graph capture of the whole step.
+"""Run-to-run determinism, CUDA-graph capture of the whole step, and calls on
+two streams at once.
 
 The tile schedule hands tiles to whichever CTA pair asks first, but every
 output element is still reduced in one fixed order (one CTA per output tile,
@@ -119,4 +120,30 @@ def test_step_captures_into_a_cuda_graph(spo):
     torch.cuda.synchronize()
     _same_bits(eager, out)
     assert not np.allclose(eager["adv"].cpu().numpy(), 0)
+    assert spo.spo_device_error() == 0
+
+
+def test_two_streams_at_once_match_serial_runs(spo):
+    """Two different batches, each with its own workspaces, on two streams at
+    the same time: the library's persistent grids interleave on the SMs and
+    each result is the same bits as a run alone."""
+    ta = _tensors(spo, _medium_case())
+    tb = _tensors(spo, inputs.tiny_case(seed=1302, T_per_seq=75, n_groups=3, rollouts=4, d=320,
+                                        V=4104))
+    torch.cuda.synchronize()
+    alone_a = {k: v.clone() for k, v in _step(spo, ta).items()}
+    alone_b = {k: v.clone() for k, v in _step(spo, tb).items()}
+    torch.cuda.synchronize()
+    sa, sb = torch.cuda.Stream(), torch.cuda.Stream()
+    outs = []
+    for _ in range(3):
+        with torch.cuda.stream(sa):
+            oa = _step(spo, ta)
+        with torch.cuda.stream(sb):
+            ob = _step(spo, tb)
+        outs.append((oa, ob))
+    torch.cuda.synchronize()
+    for oa, ob in outs:
+        _same_bits(alone_a, oa)
+        _same_bits(alone_b, ob)
     assert spo.spo_device_error() == 0
