@@ -65,6 +65,8 @@ WORKLOADS = {
               "prompt/feedback tokens masked, per-turn rewards, d=5120, V=151936, bf16 fwd+bwd",
     "large": "large batch: T=131072 packed tokens, groups of 4/8/16, 5% of rollouts in zero-variance "
              "groups, KL to reference log-probs, d=5120, V=151936, bf16 fwd+bwd (4 backward chunks)",
+    "kept": WORKLOAD + "; kept-exponential form: the forward also keeps exp(z - tile max) in bf16 "
+            "(5 GB) and the backward forms G from it instead of recomputing the logits",
     "vocab-split": WORKLOAD + "; vocabulary-split form: the head's rows as 2 slices of 75968, run "
                    "in turn on one GPU (per-slice log-prob records merged, fp32 dH parts summed on "
                    "the device where ranks would all-gather / all-reduce, dW written per slice)",
@@ -73,7 +75,7 @@ WORKLOADS = {
 KERNEL_NAMES = {0: "logits_lse_fwd", 1: "logits_grad_recompute", 2: "gemm_dH", 3: "gemm_dW",
                 4: "lse_combine", 5: "select_gather_fwd", 6: "select_gather_bwd",
                 7: "policy_loss_fwd", 8: "group_advantages", 9: "token_select",
-                10: "reward_compose", 12: "merge_slices"}
+                10: "reward_compose", 12: "merge_slices", 13: "form_g"}
 GEMM_KINDS = ("logits_lse_fwd", "logits_grad_recompute", "gemm_dH", "gemm_dW")
 SAMPLE_SEQS, SAMPLE_TOKENS = 8, 8   # CPU sample: one group of 8 rollouts, first 8 tokens each
 
@@ -249,6 +251,10 @@ class Step:
         self.g = torch.empty(T, **f32)
         self.dH = torch.empty((T, d), dtype=torch.bfloat16, device=dev)
         self.dW = torch.empty((V, d), **f32)
+        # kept-exponential form: the forward keeps exp(z - tile max) for the backward
+        self.keep = None
+        if case.get("keep"):
+            self.keep = torch.empty(spo.logprobs_keep_size(T, V), dtype=torch.uint8, device=dev)
         # vocabulary-split form: slices of W's rows run in turn, records merged
         self.slices = []
         if case.get("vocab_slices"):
@@ -292,6 +298,11 @@ class Step:
                                              p(self.rec[k]), p(self.ws_f), self.ws_f.numel(), s))
             chk(L.spo_logprobs_merge_slices(p(self.rec), len(self.slices), self.T, p(self.logp),
                                             p(self.ent), p(self.lse), s))
+        elif self.keep is not None:
+            chk(L.spo_logprobs_fwd_keep(p(self.H), p(self.W), p(self.tgt), p(self.loss_mask),
+                                        self.T, self.d, self.V, c["inv_temp"], p(self.logp),
+                                        p(self.ent), p(self.lse), p(self.keep), self.keep.numel(),
+                                        p(self.ws_f), self.ws_f.numel(), s))
         else:
             chk(L.spo_logprobs_fwd(p(self.H), p(self.W), p(self.tgt), p(self.loss_mask), self.T,
                                    self.d, self.V, c["inv_temp"], p(self.logp), p(self.ent),
@@ -319,6 +330,11 @@ class Step:
                 torch.add(self.dH_parts[0], self.dH_parts[1], out=self.dH)
                 for part in self.dH_parts[2:]:
                     self.dH.add_(part)
+        elif self.keep is not None:
+            chk(L.spo_policy_loss_bwd_kept(p(self.W), p(self.lse), p(self.g), self.T, self.d,
+                                           self.V, c["inv_temp"], p(self.keep), self.keep.numel(),
+                                           p(self.ws_f), self.ws_f.numel(), p(self.dH), p(self.dW),
+                                           0, s))
         else:
             chk(L.spo_policy_loss_bwd(p(self.H), p(self.W), p(self.tgt), p(self.lse), p(self.g),
                                       self.T, self.d, self.V, c["inv_temp"], p(self.dH),
@@ -588,14 +604,17 @@ def ours(args):
         build.build()
     dist.barrier()
     maker = {"full": inputs.full_case, "forward": inputs.forward_case, "ragged": inputs.ragged_case,
-             "large": inputs.large_case, "vocab-split": inputs.full_case}[args.workload]
+             "large": inputs.large_case, "vocab-split": inputs.full_case,
+             "kept": inputs.full_case}[args.workload]
     seed0 = {"full": 1003, "forward": 1002, "ragged": 1004, "large": 1005,
-             "vocab-split": 1003}[args.workload]
+             "vocab-split": 1003, "kept": 1003}[args.workload]
     case = maker(seed=seed0 + dist.rank, device=str(dev))
     if args.workload in ("forward", "vocab-split") and dist.world > 1:
         raise SystemExit(f"--workload {args.workload} runs on one GPU")
     if args.workload == "vocab-split":
         case["vocab_slices"] = 2
+    if args.workload == "kept":
+        case["keep"] = True
     st = Step(case, dev, dist)
     st.prepare_old_ref()
     torch.cuda.synchronize(dev)
@@ -635,6 +654,7 @@ def ours(args):
         "lse_combine": 12 * nsplit * T_L + 8 * T_L + 12 * st.T,
         "select_gather_fwd": 4 * T_L * st.d + 5 * st.T + 8 * T_L,
         "select_gather_bwd": 4 * T_L * st.d + 12 * st.T + 16 * T_L,
+        "form_g": 4 * T_L * st.V + 12 * T_L,   # kept form: E read, G written (bf16)
     }
     for name, k in kern.items():
         k["avg_ms"] = k["total_ms"] / k["launches"]

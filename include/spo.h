@@ -348,6 +348,40 @@ SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32
                                        int accumulate_dW, void* ws, size_t ws_bytes, void* stream);
 
 /* ---------------------------------------------------------------------------
+ * Kept-exponential form of a2 + a6: the forward also stores, for every kept
+ * token row r and vocabulary entry v, E[r][v] = exp(z - m) in bf16, m the
+ * row's largest logit in v's 256-entry vocabulary tile; the backward then forms
+ * G = inv_temp * g (onehot - E exp(m - lse)) from E instead of recomputing the
+ * logits, and E's buffer becomes G.  This trades T x V x 2 bytes of device
+ * memory (5 GB at T = 16384, V = 151936; small beside a GB300's 280 GB) for
+ * one of the four T x d x V products.  The default path (spo_logprobs_fwd,
+ * spo_policy_loss_bwd) keeps nothing: there the logits never reach memory.
+ *
+ * spo_logprobs_keep_size: bytes of E for T tokens and V entries (rows padded
+ *   to a multiple of 256, V bf16 each).
+ * spo_logprobs_fwd_keep: spo_logprobs_fwd plus E (16-byte aligned, >=
+ *   spo_logprobs_keep_size bytes); lse must be non-NULL.  E rows follow the
+ *   forward's compaction of kept tokens, which stays in `ws`.
+ * spo_policy_loss_bwd_kept: the backward of spo_policy_loss_bwd from the kept
+ *   forward: `keep` and `fwd_ws` exactly as that forward left them (same T,
+ *   d, V; E is overwritten with G), lse from it, g from spo_policy_loss_fwd,
+ *   W the same head.  dH bf16[T, d], dW fp32[V, d] (+= if accumulate_dW;
+ *   either may be NULL).  Accuracy as spo_policy_loss_bwd (E in bf16 adds one
+ *   bf16 rounding to G's).
+ * ------------------------------------------------------------------------- */
+SPO_API spo_status spo_logprobs_keep_size(int64_t T, int64_t V, size_t* bytes);
+SPO_API spo_status spo_logprobs_fwd_keep(const void* H, const void* W, const int32_t* tgt,
+                                         const uint8_t* mask, int64_t T, int64_t d, int64_t V,
+                                         float inv_temp, float* logp, float* entropy, float* lse,
+                                         void* keep, size_t keep_bytes, void* ws, size_t ws_bytes,
+                                         void* stream);
+SPO_API spo_status spo_policy_loss_bwd_kept(const void* W, const float* lse, const float* g,
+                                            int64_t T, int64_t d, int64_t V, float inv_temp,
+                                            void* keep, size_t keep_bytes, void* fwd_ws,
+                                            size_t fwd_ws_bytes, void* dH, float* dW,
+                                            int accumulate_dW, void* stream);
+
+/* ---------------------------------------------------------------------------
  * Vocabulary-split form of a2/a3 and a6-a8: the LM head's V rows split into
  * contiguous slices, one per GPU (tensor-parallel LM head).  The paper trains
  * on two GPUs (section 3, "Base Models") without describing this split; it is
@@ -450,7 +484,7 @@ SPO_API spo_status spo_policy_loss_fwd_noalloc(const float* logp, const float* o
  *   5 = forward row selection + gather, 6 = backward row selection + gather,
  *   7 = policy-loss forward (a5), 8 = group advantages (a4),
  *   9 = token selection (a1), 10 = reward composition, 11 = ranker,
- *   12 = merge of vocabulary-slice records.
+ *   12 = merge of vocabulary-slice records, 13 = G formed from a kept forward.
  * spo_launch_count: kernels launched by this library since it was loaded
  *   (host-side counter; every kernel launch adds one).
  * ------------------------------------------------------------------------- */

@@ -78,17 +78,24 @@ spo_status device_info(DevInfo* info) {
 }
 
 // Host-side shape checks shared by the forward and backward.
-spo_status check_hwv(const void* H, const void* W, const int32_t* tgt, int64_t T, int64_t d,
-                     int64_t V, float inv_temp) {
-  if (!H || !W || !tgt) return fail(SPO_ERR_INVALID_ARG, "H, W and tgt must be non-NULL");
+// Sizes and temperature shared by every call on the logits.
+spo_status check_dims(int64_t T, int64_t d, int64_t V, float inv_temp) {
   if (T < 1 || T > (1ll << 24)) return fail(SPO_ERR_SHAPE, "T = %lld outside [1, 2^24]", (long long)T);
   if (d < 64 || d > 65536 || d % 64 != 0)
     return fail(SPO_ERR_SHAPE, "d = %lld must be a multiple of 64 in [64, 65536]", (long long)d);
   if (V < 256 || V > (1ll << 24) || V % 8 != 0)
     return fail(SPO_ERR_SHAPE, "V = %lld must be a multiple of 8 in [256, 2^24]", (long long)V);
-  if (!aligned16(H) || !aligned16(W)) return fail(SPO_ERR_ALIGNMENT, "H and W must be 16-byte aligned");
   if (!(inv_temp > 0.f) || !isfinite(inv_temp))
     return fail(SPO_ERR_INVALID_ARG, "inv_temp must be finite and > 0");
+  return SPO_OK;
+}
+
+spo_status check_hwv(const void* H, const void* W, const int32_t* tgt, int64_t T, int64_t d,
+                     int64_t V, float inv_temp) {
+  if (!H || !W || !tgt) return fail(SPO_ERR_INVALID_ARG, "H, W and tgt must be non-NULL");
+  spo_status st = check_dims(T, d, V, inv_temp);
+  if (st != SPO_OK) return st;
+  if (!aligned16(H) || !aligned16(W)) return fail(SPO_ERR_ALIGNMENT, "H and W must be 16-byte aligned");
   return SPO_OK;
 }
 
@@ -252,13 +259,19 @@ enum TraceKind : int {
   kTraceReward = 10,
   kTraceRanker = 11,
   kTraceMergeSlices = 12,
+  kTraceFormG = 13,
 };
 
 // counters: the workspace's four tile counters (the one of this kind is
 // zeroed on the stream and used when the kind's dynamic-schedule bit is set).
-spo_status traced_gemm(int kind, bool a_mn, bool b_mn, const CUtensorMap& ta, const CUtensorMap& tb,
+// Launches GEMM epilogue `epi`.  Its schedule, tile counter and trace kind are
+// those of the product it computes (0 logits, 1 recompute, 2 dH, 3 dW): the
+// kept-exponential forward is the logits product.
+spo_status traced_gemm(int epi, bool a_mn, bool b_mn, const CUtensorMap& ta, const CUtensorMap& tb,
                        const CUtensorMap& tc, const spo::GemmArgs& args_in, int grid, cudaStream_t s,
                        int* counters) {
+  const int kind = epi == spo::EPI_LSE_KEEP ? spo::EPI_LSE : epi;
+  if (kind < 0 || kind > 3) return fail(SPO_ERR_INVALID_ARG, "GEMM kind %d", epi);
   spo::GemmArgs args = args_in;
   args.group_m = g_tune_group_m[kind];
   args.raster = g_tune_raster[kind];
@@ -268,7 +281,7 @@ spo_status traced_gemm(int kind, bool a_mn, bool b_mn, const CUtensorMap& ta, co
     SPO_CUDA(cudaMemsetAsync(args.tile_counter, 0, sizeof(int), s), "memset tile counter");
   }
   return traced(kind, s, "gemm launch", [&] {
-    return spo::launch_gemm(kind, a_mn, b_mn, g_tune_pair != 0, ta, tb, tc, args, grid, s);
+    return spo::launch_gemm(epi, a_mn, b_mn, g_tune_pair != 0, ta, tb, tc, args, grid, s);
   });
 }
 
@@ -300,7 +313,7 @@ uint32_t b_box_rows() { return static_cast<uint32_t>(spo::gemm_b_box_rows(g_tune
 spo_status logprobs_impl(const void* H, const void* W, const int32_t* tgt, const uint8_t* mask,
                          int64_t T, int64_t d, int64_t V, int64_t v_offset, float inv_temp,
                          float* logp, float* entropy, float* lse, float* rec, void* ws,
-                         cudaStream_t s) {
+                         cudaStream_t s, void* keep = nullptr) {
   spo_status st;
   DevInfo di;
   if ((st = device_info(&di)) != SPO_OK) return st;
@@ -330,10 +343,17 @@ spo_status logprobs_impl(const void* H, const void* W, const int32_t* tgt, const
   a.partials = w.partials;
   a.nsplit = w.nsplit;
   a.ztgt = w.ztgt;
-  if ((st = traced_gemm(spo::EPI_LSE, false, false, ta, tb, ta, a, grid_for(di, w.T_pad, V), s,
-                        w.counters)) !=
-      SPO_OK)
-    return st;
+  if (keep) {  // also keep E = 2^(t - tile max) in bf16 for spo_policy_loss_bwd_kept
+    CUtensorMap tk;
+    SPO_CUDA(spo::make_tmap_bf16(&tk, keep, V, w.T_pad, V * 2, 64, spo::kStoreBoxRows),
+             "tensor map E (store)");
+    st = traced_gemm(spo::EPI_LSE_KEEP, false, false, ta, tb, tk, a, grid_for(di, w.T_pad, V), s,
+                     w.counters);
+  } else {
+    st = traced_gemm(spo::EPI_LSE, false, false, ta, tb, ta, a, grid_for(di, w.T_pad, V), s,
+                     w.counters);
+  }
+  if (st != SPO_OK) return st;
   // a3: split-vocab combine, scattered back to token positions (skipped tokens read 0)
   if (rec) {
     SPO_CUDA(cudaMemsetAsync(rec, 0, sizeof(float) * 4 * T, s), "memset rec");
@@ -356,6 +376,71 @@ spo_status check_fwd_ws(int64_t T, int64_t d, int64_t V, const void* ws, size_t 
     return fail(SPO_ERR_WORKSPACE, "workspace needs %zu bytes, got %zu", need.bytes, ws_bytes);
   if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
     return fail(SPO_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
+  return SPO_OK;
+}
+
+// a6-a8 over vocabulary rows [v_offset, v_offset + V) (W points at row
+// v_offset); dH is bf16, or fp32 with dH_f32.  Arguments are validated by the caller.
+// a7 + a8 over a block of compacted rows [r0, r0 + rows): G holds them from
+// its first row (bf16, pitch ldG elements), Hc0 the same rows of the
+// compacted H, idx their token positions.  dH rows are scattered to token
+// rows (bf16, or fp32 with dH_f32); dW (+)= G^T Hc in passes of at most
+// g_tune_dw_split rows, the first pass adding into dW only when
+// accumulate_first.
+spo_status dh_dw_block(const DevInfo& di, const void* W, int64_t d, int64_t V,
+                       const __nv_bfloat16* G, long long ldG, long long rows,
+                       const __nv_bfloat16* Hc0, long long r0, const int* count, const int* idx,
+                       void* dH, bool dH_f32, float* dW, bool accumulate_first, int* counters,
+                       cudaStream_t s) {
+  spo_status st;
+  CUtensorMap tG_k, tW_mn;
+  SPO_CUDA(spo::make_tmap_bf16(&tG_k, G, V, rows, ldG * 2, spo::BK, spo::BM), "tensor map G");
+  SPO_CUDA(spo::make_tmap_bf16(&tW_mn, W, d, V, d * 2, 64, spo::BK), "tensor map W (MN)");
+  // a7: dH rows = G W, scattered to token rows
+  if (dH) {
+    spo::GemmArgs b = base_args(di);
+    b.m_count = count;
+    b.m_offset = static_cast<int>(r0);
+    b.m_cap = static_cast<int>(rows);
+    b.n = static_cast<int>(d);
+    b.k_static = static_cast<int>(V);
+    b.row_idx = idx + r0;
+    if (dH_f32)
+      b.out_f32 = static_cast<float*>(dH);
+    else
+      b.out_bf16 = static_cast<__nv_bfloat16*>(dH);
+    b.ld_out = d;
+    if ((st = traced_gemm(spo::EPI_DH, false, true, tG_k, tW_mn, tG_k, b, grid_for(di, rows, d), s,
+                          counters)) != SPO_OK)
+      return st;
+  }
+  // a8: dW (+)= G^T Hc over these rows, in passes of at most g_tune_dw_split
+  // rows (later passes reduce-add into dW)
+  if (dW) {
+    CUtensorMap tdW;
+    SPO_CUDA(spo::make_tmap_f32(&tdW, dW, d, V, d * 4, 32, spo::kStoreBoxRows), "tensor map dW");
+    const long long split = g_tune_dw_split > 0 ? g_tune_dw_split : rows;
+    for (long long q0 = 0; q0 < rows; q0 += split) {
+      const long long qrows = (rows - q0) < split ? (rows - q0) : split;
+      CUtensorMap tGq, tHq;
+      SPO_CUDA(spo::make_tmap_bf16(&tGq, G + q0 * ldG, V, qrows, ldG * 2, 64, spo::BK),
+               "tensor map G (MN)");
+      SPO_CUDA(spo::make_tmap_bf16(&tHq, Hc0 + q0 * d, d, qrows, d * 2, 64, spo::BK),
+               "tensor map Hc (MN)");
+      spo::GemmArgs b = base_args(di);
+      b.m_static = static_cast<int>(V);
+      b.n = static_cast<int>(d);
+      b.k_count = count;
+      b.k_offset = static_cast<int>(r0 + q0);
+      b.k_cap = static_cast<int>(qrows);
+      b.out_f32 = dW;
+      b.ld_out = d;
+      b.accumulate = (q0 == 0 && !accumulate_first) ? 0 : 1;
+      if ((st = traced_gemm(spo::EPI_DW, true, true, tGq, tHq, tdW, b, grid_for(di, V, d), s,
+                            counters)) != SPO_OK)
+        return st;
+    }
+  }
   return SPO_OK;
 }
 
@@ -384,27 +469,17 @@ spo_status bwd_impl(const void* H, const void* W, const int32_t* tgt, const floa
     SPO_CUDA(cudaMemsetAsync(dH, 0, (dH_f32 ? sizeof(float) : sizeof(uint16_t)) * T * d, s),
              "memset dH");
 
-  CUtensorMap tW_k, tW_mn, tG_k, tG_mn;  // operand maps
+  CUtensorMap tW_k, tG_store;
   SPO_CUDA(spo::make_tmap_bf16(&tW_k, W, d, V, d * 2, spo::BK, b_box_rows()), "tensor map W");
-  SPO_CUDA(spo::make_tmap_bf16(&tW_mn, W, d, V, d * 2, 64, spo::BK), "tensor map W (MN)");
-  SPO_CUDA(spo::make_tmap_bf16(&tG_k, w.G, V, w.chunk, V * 2, spo::BK, spo::BM), "tensor map G");
-  SPO_CUDA(spo::make_tmap_bf16(&tG_mn, w.G, V, w.chunk, V * 2, 64, spo::BK), "tensor map G (MN)");
-  CUtensorMap tG_store, tdW;
   SPO_CUDA(spo::make_tmap_bf16(&tG_store, w.G, V, w.chunk, V * 2, 64, spo::kStoreBoxRows),
            "tensor map G (store)");
-  if (dW)
-    SPO_CUDA(spo::make_tmap_f32(&tdW, dW, d, V, d * 4, 32, spo::kStoreBoxRows), "tensor map dW");
-  else
-    tdW = tG_store;
-
   const long long n_chunks = (w.T_pad + w.chunk - 1) / w.chunk;
   for (long long c = 0; c < n_chunks; ++c) {
     const long long r0 = c * w.chunk;
     const long long rows = (w.T_pad - r0) < w.chunk ? (w.T_pad - r0) : w.chunk;
     const __nv_bfloat16* Hc0 = w.Hc + r0 * d;
-    CUtensorMap tH_k, tH_mn;
+    CUtensorMap tH_k;
     SPO_CUDA(spo::make_tmap_bf16(&tH_k, Hc0, d, rows, d * 2, spo::BK, spo::BM), "tensor map Hc");
-    SPO_CUDA(spo::make_tmap_bf16(&tH_mn, Hc0, d, rows, d * 2, 64, spo::BK), "tensor map Hc (MN)");
 
     // a6: G = inv_temp * g * (onehot - softmax), logits recomputed
     spo::GemmArgs a = base_args(di);
@@ -419,54 +494,12 @@ spo_status bwd_impl(const void* H, const void* W, const int32_t* tgt, const floa
     a.gvec = w.g_c + r0;
     a.G = w.G;
     a.ldG = V;
-    if ((st = traced_gemm(spo::EPI_GRAD, false, false, tH_k, tW_k, tG_store, a, grid_for(di, rows, V), s,
-                          w.counters)) != SPO_OK)
+    if ((st = traced_gemm(spo::EPI_GRAD, false, false, tH_k, tW_k, tG_store, a,
+                          grid_for(di, rows, V), s, w.counters)) != SPO_OK)
       return st;
-    // a7: dH rows = G W, scattered to token rows
-    if (dH) {
-      spo::GemmArgs b = base_args(di);
-      b.m_count = w.count;
-      b.m_offset = static_cast<int>(r0);
-      b.m_cap = static_cast<int>(w.chunk);
-      b.n = static_cast<int>(d);
-      b.k_static = static_cast<int>(V);
-      b.row_idx = w.idx + r0;
-      if (dH_f32)
-        b.out_f32 = static_cast<float*>(dH);
-      else
-        b.out_bf16 = static_cast<__nv_bfloat16*>(dH);
-      b.ld_out = d;
-      if ((st = traced_gemm(spo::EPI_DH, false, true, tG_k, tW_mn, tG_k, b, grid_for(di, rows, d), s,
-                            w.counters)) != SPO_OK)
-        return st;
-    }
-    // a8: dW (+)= G^T Hc over this chunk's rows, in passes of at most
-    // g_tune_dw_split rows (later passes reduce-add into dW)
-    if (dW) {
-      const long long split = g_tune_dw_split > 0 ? g_tune_dw_split : rows;
-      for (long long q0 = 0; q0 < rows; q0 += split) {
-        const long long qrows = (rows - q0) < split ? (rows - q0) : split;
-        CUtensorMap tGq = tG_mn, tHq = tH_mn;
-        if (q0 > 0 || qrows < rows) {
-          SPO_CUDA(spo::make_tmap_bf16(&tGq, w.G + q0 * V, V, qrows, V * 2, 64, spo::BK),
-                   "tensor map G (MN, pass)");
-          SPO_CUDA(spo::make_tmap_bf16(&tHq, Hc0 + q0 * d, d, qrows, d * 2, 64, spo::BK),
-                   "tensor map Hc (MN, pass)");
-        }
-        spo::GemmArgs b = base_args(di);
-        b.m_static = static_cast<int>(V);
-        b.n = static_cast<int>(d);
-        b.k_count = w.count;
-        b.k_offset = static_cast<int>(r0 + q0);
-        b.k_cap = static_cast<int>(qrows);
-        b.out_f32 = dW;
-        b.ld_out = d;
-        b.accumulate = (c == 0 && q0 == 0) ? (accumulate_dW ? 1 : 0) : 1;
-        if ((st = traced_gemm(spo::EPI_DW, true, true, tGq, tHq, tdW, b, grid_for(di, V, d), s,
-                              w.counters)) != SPO_OK)
-          return st;
-      }
-    }
+    if ((st = dh_dw_block(di, W, d, V, w.G, V, rows, Hc0, r0, w.count, w.idx, dH, dH_f32, dW,
+                          c > 0 || accumulate_dW, w.counters, s)) != SPO_OK)
+      return st;
   }
   return ok();
 }
@@ -745,6 +778,66 @@ SPO_API spo_status spo_group_advantages_ws(const float* rewards, const int32_t* 
     return spo::launch_group_advantages_runs(rewards, group_id, n_seq, n_groups, std_mode, eps,
                                              adv, ws, s);
   });
+  return st == SPO_OK ? ok() : st;
+}
+
+SPO_API spo_status spo_logprobs_keep_size(int64_t T, int64_t V, size_t* bytes) {
+  if (!bytes) return fail(SPO_ERR_INVALID_ARG, "bytes must be non-NULL");
+  if (T < 1 || V < 1) return fail(SPO_ERR_SHAPE, "sizes must be positive");
+  *bytes = static_cast<size_t>(round_up(T, spo::kRowPad)) * static_cast<size_t>(V) * 2;
+  return ok();
+}
+
+SPO_API spo_status spo_logprobs_fwd_keep(const void* H, const void* W, const int32_t* tgt,
+                                         const uint8_t* mask, int64_t T, int64_t d, int64_t V,
+                                         float inv_temp, float* logp, float* entropy, float* lse,
+                                         void* keep, size_t keep_bytes, void* ws, size_t ws_bytes,
+                                         void* stream) {
+  spo_status st = check_hwv(H, W, tgt, T, d, V, inv_temp);
+  if (st != SPO_OK) return st;
+  if (!logp || !lse) return fail(SPO_ERR_INVALID_ARG, "logp and lse must be non-NULL");
+  const size_t need = static_cast<size_t>(round_up(T, spo::kRowPad)) * static_cast<size_t>(V) * 2;
+  if (!keep || keep_bytes < need)
+    return fail(SPO_ERR_WORKSPACE, "keep buffer needs %zu bytes, got %zu", need, keep_bytes);
+  if (!aligned16(keep)) return fail(SPO_ERR_ALIGNMENT, "keep buffer must be 16-byte aligned");
+  if ((st = check_fwd_ws(T, d, V, ws, ws_bytes)) != SPO_OK) return st;
+  return logprobs_impl(H, W, tgt, mask, T, d, V, 0, inv_temp, logp, entropy, lse, nullptr, ws,
+                       static_cast<cudaStream_t>(stream), keep);
+}
+
+SPO_API spo_status spo_policy_loss_bwd_kept(const void* W, const float* lse, const float* g,
+                                            int64_t T, int64_t d, int64_t V, float inv_temp,
+                                            void* keep, size_t keep_bytes, void* fwd_ws,
+                                            size_t fwd_ws_bytes, void* dH, float* dW,
+                                            int accumulate_dW, void* stream) {
+  // H and the targets come from the forward's workspace (compacted rows)
+  if (!W) return fail(SPO_ERR_INVALID_ARG, "W must be non-NULL");
+  spo_status st = check_dims(T, d, V, inv_temp);
+  if (st != SPO_OK) return st;
+  if (!aligned16(W)) return fail(SPO_ERR_ALIGNMENT, "W must be 16-byte aligned");
+  if (!lse || !g) return fail(SPO_ERR_INVALID_ARG, "lse and g must be non-NULL");
+  if (dH && !aligned16(dH)) return fail(SPO_ERR_ALIGNMENT, "dH must be 16-byte aligned");
+  if (dW && !aligned16(dW)) return fail(SPO_ERR_ALIGNMENT, "dW must be 16-byte aligned");
+  const size_t need = static_cast<size_t>(round_up(T, spo::kRowPad)) * static_cast<size_t>(V) * 2;
+  if (!keep || keep_bytes < need)
+    return fail(SPO_ERR_WORKSPACE, "keep buffer needs %zu bytes, got %zu", need, keep_bytes);
+  if (!aligned16(keep)) return fail(SPO_ERR_ALIGNMENT, "keep buffer must be 16-byte aligned");
+  if ((st = check_fwd_ws(T, d, V, fwd_ws, fwd_ws_bytes)) != SPO_OK) return st;
+  DevInfo di;
+  if ((st = device_info(&di)) != SPO_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (!dH && !dW) return ok();
+  const FwdWs w = carve_fwd(fwd_ws, T, d, V);
+  __nv_bfloat16* G = static_cast<__nv_bfloat16*>(keep);
+  // a6 without the recompute: G from E, in place
+  st = traced(kTraceFormG, s, "form G", [&] {
+    return spo::launch_form_g(G, V, static_cast<int>(V), static_cast<int>(w.T_pad), w.partials,
+                              w.nsplit, w.idx, w.count, w.tgt_c, lse, g, inv_temp, s);
+  });
+  if (st != SPO_OK) return st;
+  if (dH) SPO_CUDA(cudaMemsetAsync(dH, 0, sizeof(uint16_t) * T * d, s), "memset dH");
+  st = dh_dw_block(di, W, d, V, G, V, w.T_pad, w.Hc, 0, w.count, w.idx, dH, false, dW,
+                   accumulate_dW != 0, w.counters, s);
   return st == SPO_OK ? ok() : st;
 }
 

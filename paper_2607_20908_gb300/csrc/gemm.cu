@@ -261,17 +261,87 @@ __device__ __forceinline__ void epi_dw_tma(const GemmArgs& p, const CUtensorMap*
   }
 }
 
+// Forward that also keeps E[row][v] = 2^(t_v - m) in bf16 for the backward
+// (t = scale * z * log2 e, m the row's max over this vocabulary tile): one pass
+// over the accumulator for m, a second for the sums of epi_lse (now taken
+// against the final m) and for E, staged 64 columns at a time for the TMA
+// store.  Columns past n are staged as 0 and clipped by the store.
+__device__ __forceinline__ void epi_lse_keep(const GemmArgs& p, const CUtensorMap* tmC,
+                                             uint32_t taddr, int row, int row0, int M, int nb,
+                                             uint8_t* slots, int& slab, int lane) {
+  const bool row_ok = row < M;
+  const int y = row_ok ? p.tgt[row] : -1;
+  const float sc2 = p.scale * kLog2e;
+  const int col_base = nb * BN;
+  float mx = -INFINITY;
+#pragma unroll 1
+  for (int c = 0; c < BN / 32; ++c) {
+    const int c0 = col_base + c * 32;
+    if (c0 >= p.n) break;  // warp-uniform
+    float v[32];
+    tmem_ld32(taddr + c * 32, v);
+#pragma unroll
+    for (int j = 0; j < 32; ++j)
+      if (c0 + j < p.n) mx = fmaxf(mx, v[j]);
+  }
+  const float m2 = mx * sc2;  // scale > 0: the max of the scaled logits
+  float run_s = 0.f, run_e = 0.f, zt = 0.f;
+  bool hit = false;
+#pragma unroll 1
+  for (int c2 = 0; c2 < BN / 64; ++c2) {
+    const int c0 = col_base + c2 * 64;
+    if (c0 >= p.n) break;  // warp-uniform
+    uint32_t w[32];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      float v[32];
+      tmem_ld32(taddr + c2 * 64 + h * 32, v);
+      const int cb = c0 + h * 32;
+      if (y >= cb && y < cb + 32) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          if (cb + j == y) zt = v[j] * p.scale;
+        hit = true;
+      }
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const float ta = v[2 * j] * sc2, tb = v[2 * j + 1] * sc2;
+        const bool va = cb + 2 * j < p.n, vb = cb + 2 * j + 1 < p.n;
+        const float ea = va ? exp2f(ta - m2) : 0.f;
+        const float eb = vb ? exp2f(tb - m2) : 0.f;
+        run_s += ea;
+        run_e = fmaf(ea, ta, run_e);
+        run_s += eb;
+        run_e = fmaf(eb, tb, run_e);
+        w[h * 16 + j] = pack_bf16x2(ea, eb);
+      }
+    }
+    uint8_t* slot = acquire_slot(slots, slab, lane);
+    stage_row128(slot, lane, w);
+    flush_slot(tmC, slot, c0, row0, false, lane);
+    ++slab;
+  }
+  if (row_ok) {
+    float* q = p.partials + (static_cast<size_t>(row >> 5) * p.nsplit + nb) * kPartialBlock +
+               (row & 31);
+    q[0] = m2;
+    q[32] = run_s;
+    q[64] = run_e;
+    if (hit) p.ztgt[row] = zt;
+  }
+}
+
 // ------------------------------------------------------------ the kernel
 // Stage geometry.  Solo: one CTA stages A (128 x 64) and B (256 x 64).  Pair:
 // the two CTAs of a cluster compute one 256 x 256 tile with a shared
 // cta_group::2 MMA; each stages its own 128 rows of A and 128 of the 256 B
 // rows, so a stage is 32 KB and seven fit in shared memory (~2 us of MMA
 // work buffered against operand latency).
-// The G and dW epilogues store through TMA and need 32 KB of staging, so
+// The G, dW and kept-forward epilogues store through TMA and need 32 KB of staging, so
 // their pair-mode ring has six stages.
 template <bool PAIR, int EPI = EPI_LSE>
 struct Geo {
-  static constexpr bool kTmaStore = EPI == EPI_GRAD || EPI == EPI_DW;
+  static constexpr bool kTmaStore = EPI == EPI_GRAD || EPI == EPI_DW || EPI == EPI_LSE_KEEP;
   static constexpr int kStages = PAIR ? (kTmaStore ? 6 : 7) : 4;
   static constexpr uint32_t kEpiBytes = kTmaStore ? 4 * 2 * kEpiSlotBytes : 0;  // 4 warps x 2 slots
   static constexpr int kBRows = PAIR ? BN / 2 : BN;        // B rows staged per CTA
@@ -539,6 +609,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN);
       const int row0 = row - lane;  // first row of this warp
       if (EPI == EPI_LSE) epi_lse(p, taddr, row, M, nb);
+      if (EPI == EPI_LSE_KEEP) epi_lse_keep(p, &tmC, taddr, row, row0, M, nb, slots, slab, lane);
       if (EPI == EPI_GRAD) epi_grad_tma(p, &tmC, taddr, row, row0, M, nb, slots, slab, lane);
       if (EPI == EPI_DH) epi_dh(p, taddr, row, M, nb);
       if (EPI == EPI_DW) epi_dw_tma(p, &tmC, taddr, row0, nb, num_kb == 0, slots, slab, lane);
@@ -677,6 +748,7 @@ cudaError_t launch_gemm(int epi, bool a_mn, bool b_mn, bool pair, const CUtensor
     return pair ? launch_one<E, AM, BMN, true>(ta, tb, tc, args, grid, s)                \
                 : launch_one<E, AM, BMN, false>(ta, tb, tc, args, grid, s);
   SPO_GEMM_CASE(EPI_LSE, false, false)
+  SPO_GEMM_CASE(EPI_LSE_KEEP, false, false)
   SPO_GEMM_CASE(EPI_GRAD, false, false)
   SPO_GEMM_CASE(EPI_DH, false, true)
   SPO_GEMM_CASE(EPI_DW, true, true)

@@ -39,6 +39,7 @@ enum EpiKind : int {
   EPI_GRAD = 1,  // G = scale * g_row * (onehot - exp(scale*acc - lse_row)) -> bf16
   EPI_DH = 2,    // bf16 rows scattered to row_idx[row]
   EPI_DW = 3,    // fp32 rows, overwrite or accumulate
+  EPI_LSE_KEEP = 4,  // EPI_LSE, and E = 2^(t - tile max) kept in bf16 for the backward
 };
 
 struct GemmArgs {
@@ -95,10 +96,11 @@ cudaError_t make_tmap_bf16(CUtensorMap* tm, const void* base, uint64_t inner, ui
 cudaError_t make_tmap_f32(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer,
                           uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer);
 
-// Supported (epi, a_mn, b_mn): (LSE,0,0) (GRAD,0,0) (DH,0,1) (DW,1,1).  With
-// `pair` the grid must be even (clusters of two CTAs).  tc is the output's
-// tensor map for the TMA-store epilogues (GRAD: G as bf16, box 64 x 32; DW:
-// dW as fp32, box 32 x 32; both 128-byte swizzled); ignored by LSE and DH.
+// Supported (epi, a_mn, b_mn): (LSE,0,0) (LSE_KEEP,0,0) (GRAD,0,0) (DH,0,1)
+// (DW,1,1).  With `pair` the grid must be even (clusters of two CTAs).  tc is
+// the output's tensor map for the TMA-store epilogues (GRAD and LSE_KEEP: G or
+// E as bf16, box 64 x 32; DW: dW as fp32, box 32 x 32; all 128-byte swizzled);
+// ignored by LSE and DH.
 constexpr uint32_t kStoreBoxRows = 32;
 // One thread waits on a barrier nothing arrives on (bounded-wait self-test).
 cudaError_t launch_bounded_wait_selftest(int* err, cudaStream_t s);

@@ -35,6 +35,15 @@ cudaError_t launch_lse_combine(const float* partials, int nsplit,
                                int rows_cap, float* logp, float* entropy, float* lse,
                                const int* tgt_c, float4* rec, cudaStream_t s);
 
+// G from the kept forward, in place in E (bf16 [rows][ldE], V % 8 == 0):
+// rows r < *count of the forward's compaction (idx, compacted targets tgt_c),
+// lse and g at token positions, partials the forward's (first plane: the
+// per-tile max in log2 units).
+cudaError_t launch_form_g(__nv_bfloat16* E, long long ldE, int V, int rows_cap,
+                          const float* partials, int nsplit, const int* idx, const int* count,
+                          const int* tgt_c, const float* lse, const float* g, float inv_temp,
+                          cudaStream_t s);
+
 // Merges n_slices slice records per token, rec[k * T + t], into logp, entropy
 // and lse; a token whose records all have s == 0 (skipped) gets 0.
 cudaError_t launch_merge_slices(const float4* rec, int n_slices, long long T, float* logp,

@@ -15,6 +15,7 @@ constexpr int kCompactThreads = 256;
 constexpr int kCompactItems = 4;
 constexpr int kCompactTile = kCompactThreads * kCompactItems;  // tokens per block
 constexpr float kLn2 = 0.69314718055994531f;
+constexpr float kLog2e = 1.4426950408889634f;
 
 __device__ __forceinline__ bool selected(int kind, const uint8_t* mask, const int* tgt,
                                          const float* g, long long t) {
@@ -240,6 +241,41 @@ __global__ void merge_slices_kernel(const float4* rec, int n_slices, long long T
     logp[t] = 0.f;
     if (entropy) entropy[t] = 0.f;
     if (lse_out) lse_out[t] = 0.f;
+  }
+}
+
+// G from the kept forward, in place: for compacted row r < count and column v,
+//   G = inv_temp * g_t * (1[v == y_t] - E[r, v] * 2^(m[r, v / 256] - lse_t log2 e))
+// with E = 2^(t - m) kept by the forward and m its per-tile max (log2 units,
+// the partials' first plane).  Eight bf16 per thread (16-byte accesses).
+__global__ void form_g_kernel(__nv_bfloat16* E, long long ldE, int V, const float* partials,
+                              int nsplit, const int* idx, const int* count, const int* tgt_c,
+                              const float* lse, const float* g, float inv_temp) {
+  const int n = *count;
+  const int vec = V / 8;
+  const long long total = static_cast<long long>(n) * vec;
+  for (long long k = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x; k < total;
+       k += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const int r = static_cast<int>(k / vec);
+    const int v0 = static_cast<int>(k - static_cast<long long>(r) * vec) * 8;
+    const int t = idx[r];
+    const float coef = inv_temp * g[t];
+    const int y = tgt_c[r];
+    const float m = partials[(static_cast<size_t>(r >> 5) * nsplit + (v0 >> 8)) * kPartialBlock +
+                             (r & 31)];
+    const float scale = exp2f(m - lse[t] * kLog2e);   // 2^(m - lse log2 e)
+    uint4* p = reinterpret_cast<uint4*>(E + static_cast<size_t>(r) * ldE + v0);
+    uint4 w = *p;
+    __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&w);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float2 e = __bfloat1622float2(h[j]);
+      const int va = v0 + 2 * j;
+      const float ga = coef * ((va == y ? 1.f : 0.f) - e.x * scale);
+      const float gb = coef * ((va + 1 == y ? 1.f : 0.f) - e.y * scale);
+      h[j] = __floats2bfloat162_rn(ga, gb);
+    }
+    *p = w;
   }
 }
 
@@ -815,6 +851,18 @@ cudaError_t launch_lse_combine(const float* partials, int nsplit, const float* z
   const int blocks = (rows_cap + kCombineRows - 1) / kCombineRows;
   lse_combine_kernel<<<blocks, 256, 0, s>>>(partials, nsplit, ztgt, idx, count, logp, entropy, lse,
                                             tgt_c, rec);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_form_g(__nv_bfloat16* E, long long ldE, int V, int rows_cap,
+                          const float* partials, int nsplit, const int* idx, const int* count,
+                          const int* tgt_c, const float* lse, const float* g, float inv_temp,
+                          cudaStream_t s) {
+  const long long work = static_cast<long long>(rows_cap) * (V / 8);
+  const int blocks = static_cast<int>(max(1ll, min((work + 255) / 256, 16ll * sm_count())));
+  form_g_kernel<<<blocks, 256, 0, s>>>(E, ldE, V, partials, nsplit, idx, count, tgt_c, lse, g,
+                                       inv_temp);
   note_launches(1);
   return cudaGetLastError();
 }

@@ -64,6 +64,11 @@ _SIGS = {
     "spo_policy_loss_fwd_noalloc": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, _i32, _vp, _i64, _f32,
                                      _f32, ctypes.c_int, _vp, _vp, _vp, _vp], ctypes.c_int),
     "spo_selftest_bounded_wait": ([_vp], ctypes.c_int),
+    "spo_logprobs_keep_size": ([_i64, _i64, ctypes.POINTER(_c_size)], ctypes.c_int),
+    "spo_logprobs_fwd_keep": ([_vp, _vp, _vp, _vp, _i64, _i64, _i64, _f32, _vp, _vp, _vp, _vp,
+                               _c_size, _vp, _c_size, _vp], ctypes.c_int),
+    "spo_policy_loss_bwd_kept": ([_vp, _vp, _vp, _i64, _i64, _i64, _f32, _vp, _c_size, _vp,
+                                  _c_size, _vp, _vp, ctypes.c_int, _vp], ctypes.c_int),
     "spo_group_advantages_workspace_size": ([_i32, _i32, ctypes.POINTER(_c_size)], ctypes.c_int),
     "spo_group_advantages_ws": ([_vp, _vp, _i32, _i32, ctypes.c_int, _f32, _vp, _vp, _c_size, _vp],
                                 ctypes.c_int),
@@ -77,7 +82,7 @@ _SIGS = {
 TRACE_KINDS = {0: "logits_lse_fwd", 1: "logits_grad_recompute", 2: "gemm_dH", 3: "gemm_dW",
                4: "lse_combine", 5: "select_gather_fwd", 6: "select_gather_bwd",
                7: "policy_loss_fwd", 8: "group_advantages", 9: "token_select",
-               10: "reward_compose", 11: "ranker", 12: "merge_slices"}
+               10: "reward_compose", 11: "ranker", 12: "merge_slices", 13: "form_g"}
 
 
 class SpoError(RuntimeError):
@@ -203,6 +208,57 @@ def spo_logprobs_fwd(H, W, tgt, mask=None, inv_temp: float = 1.0, ws=None, want_
                                   float(inv_temp), _ptr(logp), _ptr(ent), _ptr(lse), _ptr(w),
                                   w.numel(), _stream(dev)))
     return logp, ent, lse
+
+
+def logprobs_keep_size(T: int, V: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().spo_logprobs_keep_size(T, V, ctypes.byref(n)))
+    return n.value
+
+
+def spo_logprobs_fwd_keep(H, W, tgt, mask=None, inv_temp: float = 1.0, keep=None, ws=None):
+    """Kept-exponential forward: returns (logp, entropy, lse, keep, ws); pass
+    keep and ws unchanged to spo_policy_loss_bwd_kept."""
+    dev = H.device
+    T, d = H.shape
+    V = W.shape[0]
+    _need(H, "H", torch.bfloat16, device=dev)
+    _need(W, "W", torch.bfloat16, device=dev)
+    _need(tgt, "tgt", torch.int32, T, dev)
+    if mask is not None:
+        _need(mask, "mask", torch.uint8, T, dev)
+    logp, ent, lse = (torch.empty(T, dtype=torch.float32, device=dev) for _ in range(3))
+    kb = logprobs_keep_size(T, V)
+    if keep is None:
+        keep = torch.empty(kb, dtype=torch.uint8, device=dev)
+    w = _workspace(logprobs_workspace_size(T, d, V), dev, ws)
+    _check(lib().spo_logprobs_fwd_keep(_ptr(H), _ptr(W), _ptr(tgt), _ptr(mask), T, d, V,
+                                       float(inv_temp), _ptr(logp), _ptr(ent), _ptr(lse),
+                                       _ptr(keep), keep.numel() * keep.element_size(), _ptr(w),
+                                       w.numel(), _stream(dev)))
+    return logp, ent, lse, keep, w
+
+
+def spo_policy_loss_bwd_kept(W, lse, g, keep, fwd_ws, T: int, d: int, inv_temp: float = 1.0,
+                             dH=None, dW=None, accumulate_dW: bool = False, want_dH=True,
+                             want_dW=True):
+    """Backward from a kept forward: returns (dH bf16[T, d] or None, dW fp32[V, d] or None)."""
+    dev = W.device
+    V = W.shape[0]
+    _need(W, "W", torch.bfloat16, device=dev)
+    _need(lse, "lse", torch.float32, T, dev)
+    _need(g, "g", torch.float32, T, dev)
+    if want_dH and dH is None:
+        dH = torch.empty((T, d), dtype=torch.bfloat16, device=dev)
+    if want_dW and dW is None:
+        dW = (torch.zeros if accumulate_dW else torch.empty)((V, d), dtype=torch.float32,
+                                                             device=dev)
+    _check(lib().spo_policy_loss_bwd_kept(_ptr(W), _ptr(lse), _ptr(g), T, d, V, float(inv_temp),
+                                          _ptr(keep), keep.numel() * keep.element_size(),
+                                          _ptr(fwd_ws), fwd_ws.numel() * fwd_ws.element_size(),
+                                          _ptr(dH), _ptr(dW), int(bool(accumulate_dW)),
+                                          _stream(dev)))
+    return dH, dW
 
 
 def spo_group_advantages(rewards, group_id, n_groups: int, std_mode: int = SPO_STD_UNBIASED,

@@ -122,3 +122,21 @@ def test_group_advantages_ws_host_validation(lib):
     assert f(p, p, 16, 4, 5, 1e-6, p, p, 1 << 20, nul) == 1
     assert f(p, nul, 16, 4, 0, 1e-6, p, p, 1 << 20, nul) == 1
     assert f(p, p, 0, 4, 0, 1e-6, p, p, 1 << 20, nul) == 2
+
+
+def test_kept_form_host_validation(lib):
+    from paper_2607_20908_gb300 import spo
+    p = ctypes.c_void_p(4096)
+    nul = ctypes.c_void_p(0)
+    assert spo.logprobs_keep_size(16384, 151936) == 16384 * 151936 * 2
+    assert spo.logprobs_keep_size(300, 4096) == 512 * 4096 * 2      # rows padded to 256
+    fk = lib.spo_logprobs_fwd_keep
+    ok_ws = 1 << 30
+    assert fk(p, p, p, nul, 256, 256, 4096, 1.0, p, nul, nul, p, 1 << 30, p, ok_ws, nul) == 1  # lse
+    assert fk(p, p, p, nul, 256, 256, 4096, 1.0, p, nul, p, p, 1024, p, ok_ws, nul) == 4      # keep
+    assert fk(p, p, p, nul, 256, 256, 4096, 1.0, p, nul, p, ctypes.c_void_p(4100), 1 << 30, p,
+              ok_ws, nul) == 3
+    bk = lib.spo_policy_loss_bwd_kept
+    assert bk(nul, p, p, 256, 256, 4096, 1.0, p, 1 << 30, p, ok_ws, p, p, 0, nul) == 1
+    assert bk(p, p, p, 256, 100, 4096, 1.0, p, 1 << 30, p, ok_ws, p, p, 0, nul) == 2
+    assert bk(p, p, p, 256, 256, 4096, 1.0, p, 1 << 30, p, 64, p, p, 0, nul) == 4            # fwd ws
