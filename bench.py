@@ -588,6 +588,8 @@ def config_block(case, T_L, world, workload="full"):
         cfg.update(clip_eps=case["clip_eps"], kl_beta=case["kl_beta"], window=case["window"])
     if case.get("vocab_slices"):
         cfg["vocab_slices"] = case["vocab_slices"]
+    if case.get("keep"):
+        cfg["kept_exponentials"] = "forward keeps exp(z - tile max) in bf16; backward forms G from it"
     cfg["l2"] = "inputs larger than L2 (W alone is 1.2-1.56 GB and is streamed every step)"
     cfg["parallelism"] = (f"dp{world}: whole groups per GPU, dW and loss all-reduced (NCCL) every step"
                           if world > 1 else "1 GPU")
@@ -613,7 +615,9 @@ def ours(args):
         raise SystemExit(f"--workload {args.workload} runs on one GPU")
     if args.workload == "vocab-split":
         case["vocab_slices"] = 2
-    if args.workload == "kept":
+    if args.workload == "kept" or args.keep:
+        if args.workload in ("forward", "vocab-split"):
+            raise SystemExit(f"--keep does not apply to --workload {args.workload}")
         case["keep"] = True
     st = Step(case, dev, dist)
     st.prepare_old_ref()
@@ -786,6 +790,9 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle timing")
+    ap.add_argument("--keep", action="store_true",
+                    help="kept-exponential form (spo_logprobs_fwd_keep / spo_policy_loss_bwd_kept) "
+                         "for a forward + backward workload")
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default="full",
                     help="supplementary workloads; the default is the one the metric is quoted on")
     args = ap.parse_args()
