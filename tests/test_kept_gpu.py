@@ -122,3 +122,31 @@ def test_full_workload_kept_backward_sampled(spo):
     assert P.rel_l2(dW.cpu().numpy(), dW_o) <= P.TOL_GRAD_REL
     del keep, fws, dW, dW1
     torch.cuda.empty_cache()
+
+
+def test_kept_backward_optional_outputs(spo):
+    """dW added into an existing buffer, dH or dW skipped, against the recompute
+    path's own accumulate and skip behaviour on the same inputs."""
+    c = _case(seed=1503)
+    dev = torch.device("cuda")
+    H, W, tgt, mask = (c[k].to(dev) for k in ("H", "W", "tgt", "mask"))
+    T, d, V, tau = c["T"], c["d"], c["V"], c["inv_temp"]
+    gen = torch.Generator().manual_seed(4)
+    g = (torch.randn(T, generator=gen) * 1e-2).float().to(dev)
+    base = torch.randn(V, d, generator=gen).float().to(dev)
+    # each kept backward overwrites E with G, so every call gets its own kept forward
+    _, _, lse, keep, fws = spo.spo_logprobs_fwd_keep(H, W, tgt, mask, tau)
+    dH, dW = spo.spo_policy_loss_bwd_kept(W, lse, g, keep, fws, T, d, tau, dW=base.clone(),
+                                          accumulate_dW=True)
+    _, _, lse, keep, fws = spo.spo_logprobs_fwd_keep(H, W, tgt, mask, tau)
+    dH2, none_w = spo.spo_policy_loss_bwd_kept(W, lse, g, keep, fws, T, d, tau, want_dW=False)
+    _, _, lse, keep, fws = spo.spo_logprobs_fwd_keep(H, W, tgt, mask, tau)
+    none_h, dW3 = spo.spo_policy_loss_bwd_kept(W, lse, g, keep, fws, T, d, tau, want_dH=False)
+    torch.cuda.synchronize()
+    assert none_w is None and none_h is None
+    assert torch.equal(dH.view(torch.int16), dH2.view(torch.int16))
+    torch.testing.assert_close(dW, base + dW3, rtol=1e-5, atol=1e-6)
+    lm = (mask == 1) & (tgt >= 0)
+    dH1, dW1 = spo.spo_policy_loss_bwd(H, W, tgt, lse, torch.where(lm, g, torch.zeros_like(g)), tau)
+    assert P.rel_l2(dW3.cpu().numpy(), dW1.cpu().numpy()) <= 1e-2
+    assert P.rel_l2(dH2.float().cpu().numpy(), dH1.float().cpu().numpy()) <= 1e-2
