@@ -83,6 +83,24 @@ def test_population_std_and_temperature():
     _compare(case, std_mode=O.STD_POPULATION)
 
 
+def test_lowest_sampling_temperature():
+    """tau = 0.2, the paper's lowest sampling temperature: logits scaled by 5."""
+    case = inputs.tiny_case(seed=1032)
+    case["inv_temp"] = 1.0 / 0.2
+    _compare(case)
+
+
+def test_peaked_softmax():
+    """Logits spread over about +-100 (W ~ N(0, 2^2) at d = 256): most
+    exponentials underflow, the softmax is nearly one-hot and the entropy is
+    near 0."""
+    case = inputs.tiny_case(seed=1033)
+    gen = torch.Generator().manual_seed(17)
+    case["W"] = (torch.randn(case["V"], case["d"], generator=gen) * 2.0).to(torch.bfloat16)
+    o, g = _compare(case)
+    assert np.median(o["entropy"]) < 0.5 and np.abs(g["entropy"] - o["entropy"]).max() <= P.TOL_LOGP
+
+
 def test_advantages_bit_exact_fp32_order():
     from paper_2607_20908_gb300 import spo
     rng = np.random.default_rng(3)
