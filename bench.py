@@ -216,7 +216,7 @@ class ClockSampler:
 class Step:
     """Device buffers + workspaces for one batch, driven through the C ABI."""
 
-    def __init__(self, case, dev, dist=None):
+    def __init__(self, case, dev, dist=None, own_inputs=False):
         from paper_2607_20908_gb300 import spo
         self.spo = spo
         self.forward_only = case.get("forward_only", "cu_seqlens" not in case)
@@ -229,7 +229,8 @@ class Step:
         self.case = case
         T, d, V = case["T"], case["d"], case["V"]
         self.T, self.d, self.V = T, d, V
-        to = lambda t: t.to(dev).contiguous()
+        # own_inputs: fresh device copies even where the case already sits on the device
+        to = lambda t: t.to(dev, copy=own_inputs).contiguous()
         self.H, self.W = to(case["H"]), to(case["W"])
         self.tgt, self.mask = to(case["tgt"]), to(case["mask"])
         f32 = dict(dtype=torch.float32, device=dev)
@@ -346,14 +347,27 @@ class Step:
 
 class HostIO:
     """End-to-end step from host buffers: every input copied host -> device and
-    every output copied device -> host, pipelined over two device buffer sets
-    so that the copies of one step overlap the compute of its neighbours
-    (H2D and D2H each on their own stream, compute on the step's stream)."""
+    every output copied device -> host, pipelined over `sets` device buffer
+    sets so that the copies of one step overlap the compute of its neighbours
+    (H2D and D2H each on their own stream, compute on the step's stream).  A
+    set is reused `sets` steps later, which is the time its copies have: host
+    copies on this platform stall for about 0.1 s every half second or so, and
+    four sets give a step's copies three steps of compute to land in."""
 
-    def __init__(self, st: "Step"):
-        self.sets = [st, Step(st.case, st.dev, st.dist)]
-        self.sets[1].old.copy_(st.old)
-        self.sets[1].ref.copy_(st.ref)
+    def __init__(self, st: "Step", sets: int = 4, set_bytes: int = 0):
+        # at most what fits in 70 % of the free device memory (a set of the large
+        # workload in the kept form holds ~60 GB), never fewer than two
+        if set_bytes > 0:
+            free, _ = torch.cuda.mem_get_info(st.dev)
+            sets = max(2, min(sets, 1 + int(0.7 * free) // set_bytes))
+        self.n = sets
+        # every set owns its inputs: a step's copies in must not land in a buffer
+        # another step's kernels are reading
+        self.sets = [st] + [Step(st.case, st.dev, st.dist, own_inputs=True)
+                            for _ in range(sets - 1)]
+        for x in self.sets[1:]:
+            x.old.copy_(st.old)
+            x.ref.copy_(st.ref)
         pinned = lambda t: torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
         if st.forward_only:
             ins = lambda x: (x.H, x.W, x.tgt, x.mask)
@@ -372,21 +386,21 @@ class HostIO:
         self.s_out = torch.cuda.Stream(st.dev)
         for x in self.sets:
             x.stream = self.compute
-        mk = lambda: [torch.cuda.Event() for _ in range(2)]
+        mk = lambda: [torch.cuda.Event() for _ in range(sets)]
         self.in_done, self.comp_done, self.out_done = mk(), mk(), mk()
         self.i = 0
 
     def step(self):
-        b = self.i & 1
+        b = self.i % self.n
         x = self.sets[b]
-        if self.i >= 2:
+        if self.i >= self.n:
             self.s_in.wait_event(self.comp_done[b])     # set b's inputs no longer read
         with torch.cuda.stream(self.s_in):
             for d, h in zip(self.dev_in[b], self.host_in):
                 d.copy_(h, non_blocking=True)
             self.in_done[b].record(self.s_in)
         self.compute.wait_event(self.in_done[b])
-        if self.i >= 2:
+        if self.i >= self.n:
             self.compute.wait_event(self.out_done[b])   # set b's outputs already copied out
         x.run()
         self.comp_done[b].record(self.compute)
@@ -619,7 +633,10 @@ def ours(args):
         if args.workload in ("forward", "vocab-split"):
             raise SystemExit(f"--keep does not apply to --workload {args.workload}")
         case["keep"] = True
+    base_bytes = torch.cuda.memory_allocated(dev)
     st = Step(case, dev, dist)
+    step_bytes = (torch.cuda.memory_allocated(dev) - base_bytes      # one buffer set:
+                  + sum(t.numel() * t.element_size() for t in (st.H, st.W)))  # + its own H, W
     st.prepare_old_ref()
     torch.cuda.synchronize(dev)
     T_L = int(st.loss_mask.sum().item())
@@ -702,16 +719,21 @@ def ours(args):
             k["frac_of_read_ceiling"] = k["gbs"] / k["read_ceiling_gbs"]
 
     # e2e: host buffers, H2D + step + D2H inside the timed region
-    hio = HostIO(st)
-    for _ in range(2):
+    hio = HostIO(st, sets=args.e2e_sets, set_bytes=step_bytes)
+    for _ in range(hio.n):
         hio.step()
     ms_e2e = timed_e2e(hio, args.steps, dist, dev)
     e2e = {"value": dist.world * T_L * args.steps / (ms_e2e / 1e3), "unit": UNIT,
            "h2d_bytes_per_step": hio.h2d, "d2h_bytes_per_step": hio.d2h,
            "ms_per_step": ms_e2e / args.steps,
-           "path": "pinned host -> device copies of every input (H, W, ids, masks, rewards, old/ref "
-                   "log-probs), the C-ABI calls, device -> host copies of loss, stats, logp, entropy, "
-                   "dH, dW; two buffer sets so copies overlap the neighbouring steps' compute"}
+           "path": ("pinned host -> device copies of every input (H, W, targets, mask), the C-ABI "
+                    "call, device -> host copies of logp, entropy, lse"
+                    if st.forward_only else
+                    "pinned host -> device copies of every input (H, W, ids, masks, rewards, old/ref "
+                    "log-probs), the C-ABI calls, device -> host copies of loss, stats, logp, "
+                    "entropy, dH, dW")
+                   + f"; {hio.n} buffer sets so a step's copies overlap the compute of the steps "
+                     "around it"}
 
     line = {
         "metric": METRIC_FWD if st.forward_only else METRIC, "value": tokens_s, "unit": UNIT,
@@ -790,6 +812,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle timing")
+    ap.add_argument("--e2e-sets", type=int, default=4,
+                    help="device buffer sets the end-to-end pipeline rotates through")
     ap.add_argument("--keep", action="store_true",
                     help="kept-exponential form (spo_logprobs_fwd_keep / spo_policy_loss_bwd_kept) "
                          "for a forward + backward workload")
