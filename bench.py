@@ -84,8 +84,8 @@ SAMPLE_SEQS, SAMPLE_TOKENS = 8, 8   # CPU sample: one group of 8 rollouts, first
 # `ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum` capture of this command
 # (profiles/launches_full_workload.md), valid only for the kernel sources they were taken on.
 TRAFFIC = {"sources_sha256_16": "229497a5c2c2001d",
-           "bytes": {"logits_lse_fwd": 6.887e9, "logits_grad_recompute": 13.462e9,
-                     "gemm_dH": 55.757e9, "gemm_dW": 14.148e9}}
+           "bytes": {"logits_lse_fwd": 6.859e9, "logits_grad_recompute": 13.466e9,
+                     "gemm_dH": 55.463e9, "gemm_dW": 13.860e9}}
 KERNEL_SOURCES = ["paper_2607_20908_gb300/csrc/gemm.cu", "paper_2607_20908_gb300/csrc/tc.cuh",
                   "paper_2607_20908_gb300/csrc/gemm.h"]
 

@@ -272,11 +272,12 @@ SPO_API spo_status spo_group_advantages(const float* rewards, const int32_t* gro
 /* spo_group_advantages_ws: the same advantages, bit for bit, in
  * O(n_seq + n_groups) work when each group's sequences are contiguous (one
  * run of equal group ids, the usual packing of rollouts), for batches far
- * beyond one step's few hundred sequences.  A first pass finds each group's
- * run; if some group has more than one run the call falls back to the
- * per-group scan of spo_group_advantages.  Arguments as there, plus
+ * beyond one step's few hundred sequences.  When the ids are non-decreasing
+ * one pass over ids and rewards does the whole job; otherwise a pass finds
+ * each group's run, and if some group has more than one run the call falls
+ * back to the per-group scan of spo_group_advantages.  Arguments as there, plus
  *   ws  >= spo_group_advantages_workspace_size(n_seq, n_groups) bytes,
- *       256-byte aligned (3 ints per group + 1).
+ *       256-byte aligned (3 ints per group + 2).
  * Sequences whose group id lies outside [0, n_groups) get no advantage
  * written, as in spo_group_advantages. */
 SPO_API spo_status spo_group_advantages_workspace_size(int32_t n_seq, int32_t n_groups,
@@ -308,10 +309,11 @@ SPO_API spo_status spo_group_advantages_ws(const float* rewards, const int32_t* 
  *   stats      fp32[4] out or NULL: {clip fraction, mean ratio, mean kl,
  *              number of loss tokens} over loss tokens
  *   ws         >= spo_policy_loss_workspace_size bytes
- * The reduction order is fixed: one warp per sequence sums its tokens in
- * fp32 (each lane its own tokens in order, then a fixed butterfly), and the
- * sums over sequences run in fp64 in two fixed stages whose split depends
- * only on n_seq, so results are deterministic run to run and across devices.
+ * The reduction order is fixed: a group of lanes per sequence (8 when the
+ * sequences average at most 256 tokens, else 32) sums its tokens in fp32
+ * (each lane its own tokens in order, then a fixed butterfly), and the sums
+ * over sequences run in fp64 in two fixed stages whose split depends only on
+ * n_seq, so results are deterministic run to run and across devices.
  * ------------------------------------------------------------------------- */
 SPO_API spo_status spo_policy_loss_workspace_size(int32_t n_seq, int32_t n_groups, size_t* bytes);
 SPO_API spo_status spo_policy_loss_fwd(const float* logp, const float* old_logp,

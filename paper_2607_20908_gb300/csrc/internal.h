@@ -95,12 +95,13 @@ cudaError_t launch_validate(const int* tgt, long long T, long long V, const int*
                             const float* ref_logp, const uint8_t* mask, int* counts, cudaStream_t s);
 
 struct LossWs {
+  unsigned long long* scal;  // [3]: non-empty groups, total loss tokens (token mean), ticket
   int* gsize;                // [n_groups]
   int* n_tok;                // [n_seq]
-  unsigned long long* scal;  // [2]: non-empty groups, total loss tokens
-  double* part;              // [n_seq][3]: sum c*l, sum rho, sum kl
+  float2* part_l;            // [n_seq]: c_i * sum of the sequence's l_t as a (hi, lo) pair
+  float2* part_rk;           // [n_seq]: sums of rho and of kl
   int* part_clip;            // [n_seq]
-  double* bpart;             // [64][4]: first-stage sums of the final reduction
+  void* bpart;               // [<= 1024]: first-stage sums of the final reduction
 };
 size_t loss_ws_bytes(int n_seq, int n_groups);
 LossWs carve_loss_ws(void* ws, int n_seq, int n_groups);

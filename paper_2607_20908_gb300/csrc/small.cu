@@ -364,10 +364,12 @@ __global__ void group_adv_kernel(const float* rewards, const int* gid, int n_seq
 }
 
 // Runs of equal group ids: the number of runs of each group and the start /
-// end of its run (meaningful when it has one).  The atomics' results are not
-// waited for.
+// end of its run (meaningful when it has one); raises *split when a group
+// has a second run (its members are not contiguous).  Runs only when the
+// sorted pass found the ids out of order.
 __global__ void adv_runs_kernel(const int* gid, int n_seq, int n_groups, int* runs, int* start,
-                                int* end) {
+                                int* end, int* split, const int* unsorted) {
+  if (!*unsorted) return;
   const int stride = gridDim.x * blockDim.x;
   for (int i0 = blockIdx.x * blockDim.x + threadIdx.x; i0 < n_seq; i0 += 4 * stride) {
     int gv[4], gp[4], gn[4];
@@ -384,21 +386,12 @@ __global__ void adv_runs_kernel(const int* gid, int n_seq, int n_groups, int* ru
       const int g = gv[u];
       if (i >= n_seq || g < 0 || g >= n_groups) continue;  // no group: no advantage
       if (i == 0 || gp[u] != g) {
-        atomicAdd(&runs[g], 1);
+        if (atomicAdd(&runs[g], 1) > 0) *split = 1;
         start[g] = i;
       }
       if (i == n_seq - 1 || gn[u] != g) end[g] = i + 1;
     }
   }
-}
-
-// Raises *split when some group has more than one run (its members are not
-// contiguous).
-__global__ void adv_split_kernel(const int* runs, int n_groups, int* split) {
-  bool multi = false;
-  for (int g = blockIdx.x * blockDim.x + threadIdx.x; g < n_groups; g += gridDim.x * blockDim.x)
-    multi |= runs[g] > 1;
-  if (__any_sync(0xffffffffu, multi) && (threadIdx.x & 31) == 0) atomicOr(split, 1);
 }
 
 // The same fold by one thread over a contiguous run [b, e): the identical
@@ -448,6 +441,44 @@ __device__ __forceinline__ void group_adv_thread(const float* src, int b, int e,
     dst[at(i)] = zero ? 0.f : __fdiv_rn(__fsub_rn(src[at(i)], mu), den);
 }
 
+// The same fold for a group of n <= N members held in registers: each member
+// is read once, and the three passes run over the registers (predicated on
+// u < n, in ascending order: the same operations as group_adv_thread).
+template <int N, class At>
+__device__ __forceinline__ void group_adv_regs(float* s, int b, int n, int std_mode, float eps,
+                                               At at) {
+  float r[N];
+#pragma unroll
+  for (int u = 0; u < N; ++u) r[u] = u < n ? s[at(b + u)] : 0.f;
+  float acc = 0.f, lo = INFINITY, hi = -INFINITY;
+#pragma unroll
+  for (int u = 0; u < N; ++u) {
+    if (u < n) {
+      acc = __fadd_rn(acc, r[u]);
+      lo = fminf(lo, r[u]);
+      hi = fmaxf(hi, r[u]);
+    }
+  }
+  const bool zero = n <= 1 || lo == hi;
+  float mu = 0.f, den = 1.f;
+  if (!zero) {
+    mu = __fdiv_rn(acc, static_cast<float>(n));
+    float ss = 0.f;
+#pragma unroll
+    for (int u = 0; u < N; ++u) {
+      if (u < n) {
+        const float dv = __fsub_rn(r[u], mu);
+        ss = __fadd_rn(ss, __fmul_rn(dv, dv));
+      }
+    }
+    const float var = __fdiv_rn(ss, static_cast<float>(std_mode == 0 ? n - 1 : n));
+    den = __fadd_rn(__fsqrt_rn(var), eps);
+  }
+#pragma unroll
+  for (int u = 0; u < N; ++u)
+    if (u < n) s[at(b + u)] = zero ? 0.f : __fdiv_rn(__fsub_rn(r[u], mu), den);
+}
+
 struct AtIdentity {
   __device__ int operator()(int i) const { return i; }
 };
@@ -468,8 +499,10 @@ constexpr int kAdvStage = 8192;
 
 __global__ void __launch_bounds__(256) group_adv_runs_kernel(
     const float* rewards, const int* gid, int n_seq, int n_groups, int std_mode, float eps,
-    const int* runs, const int* start, const int* end, const int* split, float* adv) {
+    const int* runs, const int* start, const int* end, const int* split, const int* unsorted,
+    float* adv) {
   __shared__ float st[kAdvStage + kAdvStage / 32];
+  if (!*unsorted) return;
   if (*split) {
     const int lane = threadIdx.x & 31;
     const int warps = (gridDim.x * blockDim.x) >> 5;
@@ -502,6 +535,128 @@ __global__ void __launch_bounds__(256) group_adv_runs_kernel(
     for (int k = threadIdx.x; k < hi - lo; k += blockDim.x) adv[lo + k] = st[at(k)];
     __syncthreads();
   }
+}
+
+// End of the run of group g that starts at b, for non-decreasing ids: the
+// first index past b whose id differs (or n).  Probes b + 1, b + 2, b + 4, ...
+// and then bisects, so a run of length L costs O(log L) loads.  On ids that
+// are not sorted it still returns an index in (b, n]; the caller's result is
+// then replaced by the run path.
+__device__ int adv_run_end(const int* gid, int b, int n, int g) {
+  int lo = b + 1, hi = n;  // gid[lo - 1] == g; the end lies in [lo, hi]
+  for (int step = 1;; step <<= 1) {
+    const long long p = static_cast<long long>(b) + step;
+    if (p < n && gid[p] == g) {
+      lo = static_cast<int>(p) + 1;
+    } else {
+      hi = static_cast<int>(p < n ? p : n);
+      break;
+    }
+  }
+  while (lo < hi) {
+    const int mid = lo + (hi - lo) / 2;
+    if (gid[mid] == g) lo = mid + 1;
+    else hi = mid;
+  }
+  return lo;
+}
+
+// Sorted pass of the run path: one block per chunk of kAdvChunk consecutive
+// sequences.  The block stages the chunk's rewards (padded, as in the run
+// kernel) and ids, plus the id before it and a halo of kAdvHalo sequences
+// after it, in shared memory with coalesced loads, and checks that every id
+// of the chunk is in [0, n_groups) and none is below its predecessor; if one
+// is, it raises *unsorted and the run path recomputes every advantage.
+// Otherwise each group is one run: the groups that start in the chunk are
+// found with ballots and a block scan, each is folded by one thread in
+// ascending index (group_adv_thread: the same bits), and the advantages go
+// back with coalesced stores.  The chunk's last group may run on past its
+// end: if it ends inside the halo it is folded there too, else it is folded
+// from memory.  Sequences before the chunk's first start belong to an
+// earlier block.  The block also clears its share of the run counters for
+// the run path.
+constexpr int kAdvChunk = 4096;
+constexpr int kAdvHalo = 256;  // one sequence per thread
+constexpr int kAdvStaged = kAdvChunk + kAdvHalo;
+
+__global__ void __launch_bounds__(256, 6) adv_sorted_kernel(const float* rewards, const int* gid,
+                                                         int n_seq, int n_groups, int std_mode,
+                                                         float eps, float* adv, int* runs,
+                                                         int* unsorted) {
+  __shared__ float st[kAdvStaged + kAdvStaged / 32];
+  __shared__ int sg[kAdvStaged + 1];  // ids of [c0 - 1, c1 + halo); then the list of group starts
+  __shared__ unsigned starts[kAdvChunk / 32];
+  __shared__ int tail_end;
+  const int tid = threadIdx.x;
+  for (int g = blockIdx.x * blockDim.x + tid; g < n_groups; g += gridDim.x * blockDim.x) runs[g] = 0;
+  const int c0 = blockIdx.x * kAdvChunk;
+  const int len = min(kAdvChunk, n_seq - c0);
+  const int staged = min(kAdvStaged, n_seq - c0);  // chunk + halo
+  const AtPadded at;
+#pragma unroll 8
+  for (int k = tid; k < staged; k += 256) {
+    sg[k + 1] = gid[c0 + k];
+    st[at(k)] = rewards[c0 + k];
+  }
+  if (tid == 0) {
+    sg[0] = c0 > 0 ? gid[c0 - 1] : -1;
+    tail_end = INT_MAX;
+  }
+  __syncthreads();
+  // bit k of the chunk's start mask: a group starts at c0 + k
+  bool bad = false;
+#pragma unroll
+  for (int j = 0; j < kAdvChunk / 256; ++j) {
+    const int k = j * 256 + tid;
+    const bool in = k < len;
+    const int g = in ? sg[k + 1] : 0, gp = in ? sg[k] : 0;
+    bad |= in && (g < 0 || g >= n_groups || (c0 + k > 0 && g < gp));
+    const unsigned m = __ballot_sync(0xffffffffu, in && g != gp);
+    if ((tid & 31) == 0) starts[j * 8 + (tid >> 5)] = m;
+  }
+  if (__syncthreads_or(bad)) {
+    if (tid == 0) atomicOr(unsorted, 1);
+    return;
+  }
+  // the last group runs on past the chunk when the next id is the same; its
+  // end is the first halo position with another id
+  const bool straddle = len < staged && sg[len] == sg[len + 1];
+  const int g_tail = sg[len];
+  if (straddle && len + tid < staged && sg[len + tid + 1] != g_tail) atomicMin(&tail_end, len + tid);
+  __syncthreads();
+  const unsigned word = tid < kAdvChunk / 32 ? starts[tid] : 0u;
+  int n_starts = 0;
+  int o = block_exclusive_scan(__popc(word), &n_starts);  // ends with a barrier: sg is free
+  // inside the halo, at the end of the data, or (-1) beyond the halo
+  const int e_tail = tail_end != INT_MAX ? tail_end : (c0 + staged == n_seq ? staged : -1);
+  int* list = sg;
+  for (unsigned w = word; w; w &= w - 1u) list[o++] = tid * 32 + __ffs(w) - 1;
+  __syncthreads();
+  for (int q0 = 0; q0 < n_starts; q0 += 256) {
+    // thread q0 + tid folds group q in shared memory, in registers when the
+    // largest group of its warp has at most 16 members; a last group that runs
+    // past the halo is folded from memory
+    const int q = q0 + tid;
+    const bool live = q < n_starts;
+    const int b = live ? list[q] : 0;
+    const int e = !live ? 0 : q + 1 < n_starts ? list[q + 1] : !straddle ? len : e_tail;
+    const bool from_memory = live && e < 0;
+    const int n = live && !from_memory ? e - b : 0;
+    const int n_max = __reduce_max_sync(0xffffffffu, n);
+    if (n_max <= 4) group_adv_regs<4>(st, b, n, std_mode, eps, at);
+    else if (n_max <= 8) group_adv_regs<8>(st, b, n, std_mode, eps, at);
+    else if (n_max <= 16) group_adv_regs<16>(st, b, n, std_mode, eps, at);
+    else if (n > 0) group_adv_thread(st, b, e, std_mode, eps, st, at);
+    if (from_memory) {
+      const int end = adv_run_end(gid, c0 + b, n_seq, g_tail);
+      group_adv_thread(rewards, c0 + b, end, std_mode, eps, adv, AtIdentity());
+    }
+  }
+  __syncthreads();
+  // the groups that start in this chunk, the last one into the halo when it ends there
+  const int wb_lo = n_starts > 0 ? list[0] : len;
+  const int wb_hi = !straddle || n_starts == 0 ? len : e_tail >= 0 ? e_tail : list[n_starts - 1];
+  for (int k = wb_lo + tid; k < wb_hi; k += 256) adv[c0 + k] = st[at(k)];
 }
 
 // Composite reward of one candidate: the piecewise verifiable reward
@@ -581,210 +736,348 @@ __global__ void validate_kernel(const int* tgt, long long T, long long V, const 
 // ---------------------------------------------------------------- policy loss
 constexpr int kLossThreads = 256;
 
-__device__ __forceinline__ double block_sum_d(double v, double* sh) {
-  // fixed-order tree over the block (deterministic for a fixed blockDim)
-  sh[threadIdx.x] = v;
-  __syncthreads();
-  for (int s = kLossThreads / 2; s > 0; s >>= 1) {
-    if (threadIdx.x < s) sh[threadIdx.x] += sh[threadIdx.x + s];
-    __syncthreads();
-  }
-  const double r = sh[0];
-  __syncthreads();
-  return r;
-}
-
 // One warp per sequence; the grid strides over sequences.
 __device__ __forceinline__ int warp_seq0() { return (blockIdx.x * blockDim.x + threadIdx.x) >> 5; }
 __device__ __forceinline__ int warp_seq_stride() { return (gridDim.x * blockDim.x) >> 5; }
 
-// Sum over a warp by a fixed xor butterfly: every lane ends with the same bits.
-__device__ __forceinline__ float warp_sum_f(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v = __fadd_rn(v, __shfl_xor_sync(0xffffffffu, v, o));
-  return v;
-}
 __device__ __forceinline__ long long warp_sum_ll(long long v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
   return v;
 }
 
-// (a) loss tokens per sequence and sequences per group (integers).
-__global__ void loss_count_kernel(const int* cu, const int* gid, const uint8_t* lm, int n_seq,
-                                  int n_groups, int* n_tok, int* gsize) {
-  const int lane = threadIdx.x & 31;
-  for (int i = warp_seq0(); i < n_seq; i += warp_seq_stride()) {
-    const int b = cu[i], e = cu[i + 1];
-    int c = 0;
-    for (int t0 = b + lane; t0 < e; t0 += 128) {
-      uint8_t m[4];
-#pragma unroll
-      for (int u = 0; u < 4; ++u) m[u] = t0 + 32 * u < e ? lm[t0 + 32 * u] : 0;
-#pragma unroll
-      for (int u = 0; u < 4; ++u) c += m[u] ? 1 : 0;
-    }
-    c = __reduce_add_sync(0xffffffffu, c);
-    if (lane == 0) {
-      n_tok[i] = c;
-      const int g = gid[i];
-      if (g >= 0 && g < n_groups) atomicAdd(&gsize[g], 1);
-    }
-  }
+// (a) sequences per group and the number of non-empty groups; for the token
+// mean also the number of loss tokens of [cu[0], cu[n_seq]) (integers; the
+// counters were cleared on the stream).
+__device__ __forceinline__ int nonzero_bytes(unsigned w) {
+  // high bit of each byte set iff the byte is non-zero (no carry crosses bytes)
+  return __popc((((w & 0x7f7f7f7fu) + 0x7f7f7f7fu) | w) & 0x80808080u);
 }
 
-// (b) number of non-empty groups and of loss tokens (integer sums; scal zeroed).
-__global__ void loss_scalars_kernel(const int* gsize, int n_groups, const int* n_tok, int n_seq,
-                                    unsigned long long* scal) {
-  long long ng = 0, nt = 0;
-  for (int k = blockIdx.x * blockDim.x + threadIdx.x; k < max(n_groups, n_seq);
-       k += gridDim.x * blockDim.x) {
-    if (k < n_groups) ng += gsize[k] > 0 ? 1 : 0;
-    if (k < n_seq) nt += n_tok[k];
+__global__ void loss_groups_kernel(const int* gid, int n_seq, int n_groups, const int* cu,
+                                   const uint8_t* lm, int agg, int* gsize,
+                                   unsigned long long* scal) {
+  const int stride = gridDim.x * blockDim.x;
+  const int tid = blockIdx.x * blockDim.x + threadIdx.x;
+  int first = 0;
+  for (int i = tid; i < n_seq; i += stride) {
+    const int g = gid[i];
+    if (g >= 0 && g < n_groups && atomicAdd(&gsize[g], 1) == 0) ++first;
   }
-  ng = warp_sum_ll(ng);
+  long long nt = 0;
+  if (agg == 1) {
+    const long long lo = cu[0], hi = cu[n_seq];
+    // bytes up to the first 16-byte-aligned address, then 16 at a time, then the tail
+    const long long lead = static_cast<long long>((16u - (reinterpret_cast<uintptr_t>(lm + lo) & 15u)) & 15u);
+    const long long a = min(hi, lo + lead);
+    const long long z = a + (hi - a) / 16 * 16;
+    for (long long t = lo + tid; t < a; t += stride) nt += lm[t] != 0;
+    const uint4* v = reinterpret_cast<const uint4*>(lm + a);
+    for (long long k = tid; k < (z - a) / 16; k += stride) {
+      const uint4 q = __ldcs(v + k);
+      nt += nonzero_bytes(q.x) + nonzero_bytes(q.y) + nonzero_bytes(q.z) + nonzero_bytes(q.w);
+    }
+    for (long long t = z + tid; t < hi; t += stride) nt += lm[t] != 0;
+  }
+  // one update of each counter per block (same-address atomics serialise)
+  __shared__ long long sf[kLossThreads / 32], st[kLossThreads / 32];
+  first = __reduce_add_sync(0xffffffffu, first);
   nt = warp_sum_ll(nt);
   if ((threadIdx.x & 31) == 0) {
-    if (ng) atomicAdd(&scal[0], static_cast<unsigned long long>(ng));
-    if (nt) atomicAdd(&scal[1], static_cast<unsigned long long>(nt));
+    sf[threadIdx.x >> 5] = first;
+    st[threadIdx.x >> 5] = nt;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    long long f = 0, n = 0;
+    for (int w = 0; w < kLossThreads / 32; ++w) {
+      f += sf[w];
+      n += st[w];
+    }
+    if (f) atomicAdd(&scal[0], static_cast<unsigned long long>(f));
+    if (n) atomicAdd(&scal[1], static_cast<unsigned long long>(n));
   }
 }
 
-// (c) per-token surrogate, KL, dL/dlogp; per-sequence fp64 partial sums (each
-// lane over tokens b + lane, b + lane + 32, ..., then the fixed butterfly).
-__global__ void loss_token_kernel(const float* logp, const float* old_logp, const float* ref_logp,
-                                  const float* adv, const int* cu, const int* gid, int n_seq,
-                                  int n_groups, const uint8_t* lm, float clip_eps, float kl_beta,
-                                  int agg, const int* n_tok, const int* gsize,
-                                  const unsigned long long* scal, float* g, double* part,
-                                  int* part_clip) {
+// (b) per-token surrogate, KL, dL/dlogp; per-sequence sums.  A group of LPS
+// lanes takes one sequence (LPS = 16 when sequences average at most 128
+// tokens, so a warp holds two at once; else the whole warp) in passes of
+// 8 tokens a lane: the group counts the sequence's loss tokens (n_i of c_t)
+// while the first pass's inputs stay in registers (a sequence of up to 8 LPS
+// tokens is read once), then lane l of the group sums its own tokens
+// b + l, b + l + LPS, ... in order in fp32 and the group's lanes are
+// combined by a fixed xor butterfly.  The next sequence's bounds, group and
+// advantage are loaded one sequence ahead.
+//
+// kl = e^delta - delta - 1 is taken from the Taylor series of e^delta for
+// |delta| <= 1/2: kl = delta^2 (1/2! + delta/3! + ... + delta^7/9!) (the
+// first omitted term is below 3e-9 of the sum), which also avoids the
+// cancellation of e^delta - 1 - delta near 0; beyond, e^delta - 1 - delta
+// directly.  e^delta - 1 = delta + kl in both cases.
+__device__ __forceinline__ float kl_k3(float delta, float* em1) {
+  float kl;
+  if (fabsf(delta) <= 0.5f) {
+    float p = 1.f / 362880.f;
+    p = fmaf(p, delta, 1.f / 40320.f);
+    p = fmaf(p, delta, 1.f / 5040.f);
+    p = fmaf(p, delta, 1.f / 720.f);
+    p = fmaf(p, delta, 1.f / 120.f);
+    p = fmaf(p, delta, 1.f / 24.f);
+    p = fmaf(p, delta, 1.f / 6.f);
+    p = fmaf(p, delta, 0.5f);
+    kl = delta * delta * p;
+    *em1 = delta + kl;
+  } else {
+    *em1 = expf(delta) - 1.f;
+    kl = *em1 - delta;
+  }
+  return kl;
+}
+
+struct LossTok {
+  float lo, hi, A, c, beta;
+  bool use_kl;
+  float s_l = 0.f, s_rho = 0.f, s_kl = 0.f;
+  int n_clip = 0;
+  __device__ __forceinline__ float token(float lp, float ol, float rf) {
+    const float rho = expf(lp - ol);
+    const float clipped = fminf(fmaxf(rho, lo), hi);
+    const float surr = fminf(rho * A, clipped * A);
+    const bool binds = (A > 0.f && rho > hi) || (A < 0.f && rho < lo);
+    float kl = 0.f, dkl = 0.f;
+    if (use_kl) {
+      float em1;
+      kl = kl_k3(rf - lp, &em1);
+      dkl = -em1;  // d kl / d logp = 1 - e^delta
+    }
+    s_l += -(surr - beta * kl);
+    s_rho += rho;
+    s_kl += kl;
+    n_clip += binds ? 1 : 0;
+    return c * ((binds ? 0.f : -A * rho) + (use_kl ? beta * dkl : 0.f));
+  }
+};
+
+// Fixed xor butterfly over the LPS lanes of a group (mask m): every lane of
+// the group ends with the same bits.
+template <int LPS>
+__device__ __forceinline__ float group_sum_f(float v, unsigned m) {
+#pragma unroll
+  for (int o = LPS / 2; o > 0; o >>= 1) v = __fadd_rn(v, __shfl_xor_sync(m, v, o));
+  return v;
+}
+
+template <int LPS>
+__global__ void __launch_bounds__(kLossThreads) loss_token_kernel(
+    const float* logp, const float* old_logp, const float* ref_logp, const float* adv,
+    const int* cu, const int* gid, int n_seq, int n_groups, const uint8_t* lm, float clip_eps,
+    float kl_beta, int agg, const int* gsize, const unsigned long long* scal, float* g,
+    float2* part_l, float2* part_rk, int* part_clip, int* n_tok) {
+  constexpr int kTpl = 8;            // tokens a lane has in flight in one pass
+  constexpr int kStep = kTpl * LPS;  // tokens of one pass of the group
   const int lane = threadIdx.x & 31;
+  const int sl = lane % LPS;
+  const unsigned gm = LPS == 32 ? 0xffffffffu : ((1u << LPS) - 1u) << (lane - sl);
   const bool use_kl = ref_logp != nullptr && kl_beta != 0.f;
-  const float lo = 1.f - clip_eps, hi = 1.f + clip_eps;
-  for (int i = warp_seq0(); i < n_seq; i += warp_seq_stride()) {
-    const int b = cu[i], e = cu[i + 1];
-    const int ni = n_tok[i];
+  const float ng = static_cast<float>(scal[0]);
+  const float c_tok = scal[1] > 0 ? __frcp_rn(static_cast<float>(scal[1])) : 0.f;
+  const int stride = warp_seq_stride() * (32 / LPS);
+  int i = warp_seq0() * (32 / LPS) + lane / LPS;
+  int b = 0, e = 0, gi = -1;
+  float A = 0.f;
+  if (i < n_seq) {
+    b = cu[i];
+    e = cu[i + 1];
+    gi = gid[i];
+    A = adv[i];
+  }
+  for (; i < n_seq; i += stride) {
+    const int in = i + stride;
+    int nb = 0, ne = 0, ngi = -1;
+    float nA = 0.f;
+    if (in < n_seq) {
+      nb = cu[in];
+      ne = cu[in + 1];
+      ngi = gid[in];
+      nA = adv[in];
+    }
+    const int gs = agg == 0 && gi >= 0 && gi < n_groups ? gsize[gi] : 0;
+    // the first pass's inputs stay in registers while the mask is counted
+    uint8_t mk[kTpl];
+    float lpv[kTpl], olv[kTpl], rfv[kTpl];
+#pragma unroll
+    for (int u = 0; u < kTpl; ++u) {
+      const int t = b + sl + LPS * u;
+      const bool inside = t < e;
+      mk[u] = inside ? lm[t] : 0;
+      lpv[u] = inside ? logp[t] : 0.f;
+      olv[u] = inside ? old_logp[t] : 0.f;
+      rfv[u] = inside && use_kl ? ref_logp[t] : 0.f;
+    }
+    int cnt = 0;
+#pragma unroll
+    for (int u = 0; u < kTpl; ++u) cnt += mk[u] != 0;
+    for (int t0 = b + kStep + sl; t0 < e; t0 += kStep) {
+#pragma unroll
+      for (int u = 0; u < kTpl; ++u) cnt += t0 + LPS * u < e && lm[t0 + LPS * u] != 0;
+    }
+    const int ni = __reduce_add_sync(gm, cnt);
     // c_t of Eq. 3's average; fp32 (GB300's fp64 unit is narrow, and every
-    // lane of the warp computes it)
-    float c = 0.f;
-    if (agg == 0) {
-      const unsigned long long ng = scal[0];
-      const int gi = gid[i];
-      if (ni > 0 && ng > 0 && gi >= 0 && gi < n_groups)
-        c = __frcp_rn(static_cast<float>(ng) * static_cast<float>(gsize[gi]) *
-                      static_cast<float>(ni));
-    } else {
-      const unsigned long long nt = scal[1];
-      if (nt > 0) c = __frcp_rn(static_cast<float>(nt));
-    }
-    const float A = adv[i];
-    // a lane sums its own tokens and the warp its lanes in fp32 (fixed
-    // butterfly); the sums over sequences are fp64
-    float s_l = 0.f, s_rho = 0.f, s_kl = 0.f;
-    int n_clip = 0;
-    // a lane's tokens b + lane, b + lane + 32, ... in order, four loads in flight
-    for (int t0 = b + lane; t0 < e; t0 += 128) {
-      uint8_t mk[4];
-      float lpv[4], olv[4], rfv[4];
+    // lane computes it)
+    float c = c_tok;
+    if (agg == 0)
+      c = ni > 0 && ng > 0.f && gs > 0
+              ? __frcp_rn(ng * static_cast<float>(gs) * static_cast<float>(ni))
+              : 0.f;
+    LossTok k{1.f - clip_eps, 1.f + clip_eps, A, c, kl_beta, use_kl};
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int t = t0 + 32 * u;
-        mk[u] = t < e ? lm[t] : 0;
-        lpv[u] = mk[u] ? logp[t] : 0.f;
-        olv[u] = mk[u] ? old_logp[t] : 0.f;
-        rfv[u] = mk[u] && use_kl ? ref_logp[t] : 0.f;
+    for (int u = 0; u < kTpl; ++u) {
+      const int t = b + sl + LPS * u;
+      if (t < e) g[t] = mk[u] ? k.token(lpv[u], olv[u], rfv[u]) : 0.f;
+    }
+    for (int t0 = b + kStep + sl; t0 < e; t0 += kStep) {
+#pragma unroll
+      for (int u = 0; u < kTpl; ++u) {
+        const int t = t0 + LPS * u;
+        const bool inside = t < e;
+        mk[u] = inside ? lm[t] : 0;
+        lpv[u] = inside ? logp[t] : 0.f;
+        olv[u] = inside ? old_logp[t] : 0.f;
+        rfv[u] = inside && use_kl ? ref_logp[t] : 0.f;
       }
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int t = t0 + 32 * u;
-        if (t >= e) break;
-        if (!mk[u]) {
-          g[t] = 0.f;
-          continue;
-        }
-        const float lp = lpv[u];
-        const float rho = expf(lp - olv[u]);
-        const float clipped = fminf(fmaxf(rho, lo), hi);
-        const float surr = fminf(rho * A, clipped * A);
-        const bool binds = (A > 0.f && rho > hi) || (A < 0.f && rho < lo);
-        float kl = 0.f, dkl = 0.f;
-        if (use_kl) {
-          const float delta = rfv[u] - lp;
-          const float em1 = expm1f(delta);
-          kl = em1 - delta;  // exp(delta) - delta - 1
-          dkl = -em1;        // 1 - exp(delta)
-        }
-        const float ell = -(surr - kl_beta * kl);
-        g[t] = c * ((binds ? 0.f : -A * rho) + (use_kl ? kl_beta * dkl : 0.f));
-        s_l += ell;
-        s_rho += rho;
-        s_kl += kl;
-        n_clip += binds ? 1 : 0;
+      for (int u = 0; u < kTpl; ++u) {
+        const int t = t0 + LPS * u;
+        if (t < e) g[t] = mk[u] ? k.token(lpv[u], olv[u], rfv[u]) : 0.f;
       }
     }
-    s_l = warp_sum_f(s_l);
-    s_rho = warp_sum_f(s_rho);
-    s_kl = warp_sum_f(s_kl);
-    n_clip = __reduce_add_sync(0xffffffffu, n_clip);
-    if (lane == 0) {
-      part[3 * i + 0] = static_cast<double>(s_l) * static_cast<double>(c);
-      part[3 * i + 1] = s_rho;
-      part[3 * i + 2] = s_kl;
+    const float s_l = group_sum_f<LPS>(k.s_l, gm);
+    const float s_rho = group_sum_f<LPS>(k.s_rho, gm);
+    const float s_kl = group_sum_f<LPS>(k.s_kl, gm);
+    const int n_clip = __reduce_add_sync(gm, k.n_clip);
+    if (sl == 0) {
+      const float hi = s_l * c;  // c * s_l as an unevaluated pair: hi + lo exactly
+      part_l[i] = make_float2(hi, fmaf(s_l, c, -hi));
+      part_rk[i] = make_float2(s_rho, s_kl);
       part_clip[i] = n_clip;
+      n_tok[i] = ni;
     }
+    b = nb;
+    e = ne;
+    gi = ngi;
+    A = nA;
   }
 }
 
-// (d) fixed-order sum over sequences in two stages: block k sums the
-// sequences of its contiguous chunk (thread-strided, then a fixed tree), and
-// one block sums the kLossFinalBlocks block results.  The split depends only
-// on n_seq, so the loss is the same bits on any device.
-constexpr int kLossFinalBlocks = 64;
+// (c) fixed-order sum over sequences in two stages: block k sums the
+// sequences of its contiguous chunk (one per thread at the usual sizes; then
+// each warp by a fixed butterfly and the block's warps in order), and the
+// last block to finish (a ticket taken after its sums are visible) sums the
+// block results the same way in block order.  The loss terms are carried as
+// unevaluated pairs of floats (hi + lo, about 48 significant bits) and added
+// with Knuth's TwoSum, so cancellation between the terms costs no accuracy
+// and GB300's narrow fp64 unit is not used; the ratio and KL statistics are
+// summed in fp32, the counts as integers.  The chunk size depends only on
+// n_seq, so the results are the same bits on any device.
+constexpr int kLossFinalMaxBlocks = 1024;
 
-__global__ void loss_final_partial_kernel(const double* part, const int* part_clip, int n_seq,
-                                          int chunk, double* bpart) {
-  __shared__ double sh[kLossThreads];
+// (a_hi + a_lo) + (b_hi + b_lo) as a normalised pair (TwoSum of the high
+// parts, the low parts added to its error term, then a fast renormalisation)
+__device__ __forceinline__ float2 pair_add(float2 a, float2 b) {
+  const float s = __fadd_rn(a.x, b.x);
+  const float v = __fsub_rn(s, a.x);
+  float err = __fadd_rn(__fsub_rn(a.x, __fsub_rn(s, v)), __fsub_rn(b.x, v));
+  err = __fadd_rn(err, __fadd_rn(a.y, b.y));
+  const float hi = __fadd_rn(s, err);
+  return make_float2(hi, __fsub_rn(err, __fsub_rn(hi, s)));
+}
+
+struct LossSums {
+  float2 l;
+  float r, k;
+  long long c, n;
+  __device__ __forceinline__ void zero() {
+    l = make_float2(0.f, 0.f);
+    r = k = 0.f;
+    c = n = 0;
+  }
+  __device__ __forceinline__ void add(const LossSums& o) {
+    l = pair_add(l, o.l);
+    r = __fadd_rn(r, o.r);
+    k = __fadd_rn(k, o.k);
+    c += o.c;
+    n += o.n;
+  }
+};
+
+__device__ __forceinline__ LossSums block_sums(LossSums v, LossSums* sh) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    LossSums w;
+    w.l.x = __shfl_xor_sync(0xffffffffu, v.l.x, o);
+    w.l.y = __shfl_xor_sync(0xffffffffu, v.l.y, o);
+    w.r = __shfl_xor_sync(0xffffffffu, v.r, o);
+    w.k = __shfl_xor_sync(0xffffffffu, v.k, o);
+    w.c = __shfl_xor_sync(0xffffffffu, v.c, o);
+    w.n = __shfl_xor_sync(0xffffffffu, v.n, o);
+    v.add(w);
+  }
+  if ((threadIdx.x & 31) == 0) sh[threadIdx.x >> 5] = v;
+  __syncthreads();
+  LossSums t = sh[0];
+  for (int w = 1; w < kLossThreads / 32; ++w) t.add(sh[w]);
+  __syncthreads();
+  return t;
+}
+
+__global__ void __launch_bounds__(kLossThreads) loss_final_kernel(
+    const float2* part_l, const float2* part_rk, const int* part_clip, const int* n_tok, int n_seq,
+    int chunk, LossSums* bpart, unsigned long long* ticket, float* loss, float* stats) {
+  __shared__ LossSums sh[kLossThreads / 32];
+  __shared__ bool last;
   const int i0 = blockIdx.x * chunk, i1 = min(n_seq, i0 + chunk);
-  double l = 0, r = 0, k = 0, c = 0;
+  LossSums v;
+  v.zero();
   for (int i = i0 + threadIdx.x; i < i1; i += kLossThreads) {
-    l += part[3 * i];
-    r += part[3 * i + 1];
-    k += part[3 * i + 2];
-    c += part_clip[i];
+    LossSums q;
+    q.l = part_l[i];
+    const float2 rk = part_rk[i];
+    q.r = rk.x;
+    q.k = rk.y;
+    q.c = part_clip[i];
+    q.n = n_tok[i];
+    v.add(q);
   }
-  l = block_sum_d(l, sh);
-  r = block_sum_d(r, sh);
-  k = block_sum_d(k, sh);
-  c = block_sum_d(c, sh);
+  v = block_sums(v, sh);
   if (threadIdx.x == 0) {
-    bpart[4 * blockIdx.x + 0] = l;
-    bpart[4 * blockIdx.x + 1] = r;
-    bpart[4 * blockIdx.x + 2] = k;
-    bpart[4 * blockIdx.x + 3] = c;
+    bpart[blockIdx.x] = v;
+    __threadfence();
+    last = atomicAdd(ticket, 1ull) == gridDim.x - 1;
   }
-}
-
-__global__ void loss_final_kernel(const double* bpart, int nb, const unsigned long long* scal,
-                                  float* loss, float* stats) {
-  __shared__ double sh[kLossThreads];
-  double l = 0, r = 0, k = 0, c = 0;
-  for (int j = threadIdx.x; j < nb; j += kLossThreads) {
-    l += bpart[4 * j];
-    r += bpart[4 * j + 1];
-    k += bpart[4 * j + 2];
-    c += bpart[4 * j + 3];
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  LossSums u;
+  u.zero();
+  for (int j = threadIdx.x; j < static_cast<int>(gridDim.x); j += kLossThreads) {
+    const volatile LossSums* q = bpart + j;
+    LossSums x;
+    x.l.x = q->l.x;
+    x.l.y = q->l.y;
+    x.r = q->r;
+    x.k = q->k;
+    x.c = q->c;
+    x.n = q->n;
+    u.add(x);
   }
-  l = block_sum_d(l, sh);
-  r = block_sum_d(r, sh);
-  k = block_sum_d(k, sh);
-  c = block_sum_d(c, sh);
+  u = block_sums(u, sh);
   if (threadIdx.x == 0) {
-    *loss = static_cast<float>(l);
+    *loss = __fadd_rn(u.l.x, u.l.y);
     if (stats) {
-      const double n = static_cast<double>(scal[1]);
-      stats[0] = n > 0 ? static_cast<float>(c / n) : 0.f;
-      stats[1] = n > 0 ? static_cast<float>(r / n) : 0.f;
-      stats[2] = n > 0 ? static_cast<float>(k / n) : 0.f;
+      const double n = static_cast<double>(u.n);
+      stats[0] = n > 0 ? static_cast<float>(static_cast<double>(u.c) / n) : 0.f;
+      stats[1] = n > 0 ? static_cast<float>(static_cast<double>(u.r) / n) : 0.f;
+      stats[2] = n > 0 ? static_cast<float>(static_cast<double>(u.k) / n) : 0.f;
       stats[3] = static_cast<float>(n);
     }
   }
@@ -896,7 +1189,7 @@ cudaError_t launch_group_advantages(const float* rewards, const int* group_id, i
   return cudaGetLastError();
 }
 
-size_t adv_ws_bytes(int n_groups) { return align256(sizeof(int) * (3 * static_cast<size_t>(n_groups) + 1)); }
+size_t adv_ws_bytes(int n_groups) { return align256(sizeof(int) * (3 * static_cast<size_t>(n_groups) + 2)); }
 
 cudaError_t launch_group_advantages_runs(const float* rewards, const int* group_id, int n_seq,
                                          int n_groups, int std_mode, float eps, float* adv,
@@ -904,19 +1197,20 @@ cudaError_t launch_group_advantages_runs(const float* rewards, const int* group_
   int* runs = static_cast<int*>(ws);
   int* start = runs + n_groups;
   int* end = start + n_groups;
-  int* split = end + n_groups;
-  cudaError_t e = cudaMemsetAsync(runs, 0, sizeof(int) * n_groups, s);
-  if (e == cudaSuccess) e = cudaMemsetAsync(split, 0, sizeof(int), s);
+  int* split = end + n_groups;  // [0]: some group has several runs; [1]: ids out of order
+  int* unsorted = split + 1;
+  cudaError_t e = cudaMemsetAsync(split, 0, 2 * sizeof(int), s);
   if (e != cudaSuccess) return e;
   const int sms = sm_count();
-  adv_runs_kernel<<<max(1, min((n_seq + 1023) / 1024, sms * 8)), 256, 0, s>>>(
-      group_id, n_seq, n_groups, runs, start, end);
-  adv_split_kernel<<<max(1, min((n_groups + 255) / 256, sms * 4)), 256, 0, s>>>(runs, n_groups,
-                                                                               split);
-  // enough warps for the per-group scan of the fallback, one thread per group otherwise
-  const int blocks2 = max(1, min((n_groups + 7) / 8, sms * 16));
+  adv_sorted_kernel<<<(n_seq + kAdvChunk - 1) / kAdvChunk, 256, 0, s>>>(
+      rewards, group_id, n_seq, n_groups, std_mode, eps, adv, runs, unsorted);
+  // the run path: each kernel returns at once when the sorted pass succeeded,
+  // so its grid is one block per SM (grid-stride loops)
+  adv_runs_kernel<<<max(1, min((n_seq + 1023) / 1024, sms)), 256, 0, s>>>(
+      group_id, n_seq, n_groups, runs, start, end, split, unsorted);
+  const int blocks2 = max(1, min((n_groups + 7) / 8, sms));
   group_adv_runs_kernel<<<blocks2, 256, 0, s>>>(rewards, group_id, n_seq, n_groups, std_mode, eps,
-                                                runs, start, end, split, adv);
+                                                runs, start, end, split, unsorted, adv);
   note_launches(3);
   return cudaGetLastError();
 }
@@ -974,25 +1268,28 @@ cudaError_t launch_validate(const int* tgt, long long T, long long V, const int*
 }
 
 size_t loss_ws_bytes(int n_seq, int n_groups) {
-  return align256(sizeof(int) * n_groups) + align256(sizeof(int) * n_seq) +
-         align256(2 * sizeof(long long)) + align256(3 * sizeof(double) * n_seq) +
-         align256(sizeof(int) * n_seq) + align256(4 * sizeof(double) * kLossFinalBlocks);
+  return align256(3 * sizeof(long long)) + align256(sizeof(int) * n_groups) +
+         align256(sizeof(int) * n_seq) + align256(sizeof(float2) * n_seq) +
+         align256(sizeof(float2) * n_seq) + align256(sizeof(int) * n_seq) +
+         align256(sizeof(LossSums) * kLossFinalMaxBlocks);
 }
 
 LossWs carve_loss_ws(void* ws, int n_seq, int n_groups) {
   char* p = static_cast<char*>(ws);
   LossWs w;
+  w.scal = reinterpret_cast<unsigned long long*>(p);  // cleared with gsize in one memset
+  p += align256(3 * sizeof(long long));
   w.gsize = reinterpret_cast<int*>(p);
   p += align256(sizeof(int) * n_groups);
   w.n_tok = reinterpret_cast<int*>(p);
   p += align256(sizeof(int) * n_seq);
-  w.scal = reinterpret_cast<unsigned long long*>(p);
-  p += align256(2 * sizeof(long long));
-  w.part = reinterpret_cast<double*>(p);
-  p += align256(3 * sizeof(double) * n_seq);
+  w.part_l = reinterpret_cast<float2*>(p);
+  p += align256(sizeof(float2) * n_seq);
+  w.part_rk = reinterpret_cast<float2*>(p);
+  p += align256(sizeof(float2) * n_seq);
   w.part_clip = reinterpret_cast<int*>(p);
   p += align256(sizeof(int) * n_seq);
-  w.bpart = reinterpret_cast<double*>(p);
+  w.bpart = p;
   return w;
 }
 
@@ -1001,28 +1298,45 @@ cudaError_t launch_policy_loss(const float* logp, const float* old_logp, const f
                                int n_seq, int n_groups, const uint8_t* loss_mask, long long T,
                                float clip_eps, float kl_beta, int agg, float* loss, float* g,
                                float* stats, const LossWs& w, cudaStream_t s) {
-  (void)T;
-  cudaError_t e = cudaMemsetAsync(w.gsize, 0, sizeof(int) * n_groups, s);
-  if (e == cudaSuccess) e = cudaMemsetAsync(w.scal, 0, 2 * sizeof(unsigned long long), s);
+  // scal (groups, tokens, ticket) and gsize are adjacent: one clear
+  cudaError_t e = cudaMemsetAsync(w.scal, 0,
+                                  reinterpret_cast<char*>(w.gsize + n_groups) -
+                                      reinterpret_cast<char*>(w.scal), s);
   if (e != cudaSuccess) return e;
   const int sms = sm_count();
-  const int per_block = kLossThreads / 32;  // sequences in flight per block
-  const int seq_blocks = max(1, min((n_seq + per_block - 1) / per_block, sms * 8));
-  loss_count_kernel<<<seq_blocks, kLossThreads, 0, s>>>(cu_seqlens, group_id, loss_mask, n_seq,
-                                                        n_groups, w.n_tok, w.gsize);
-  const int nmax = n_seq > n_groups ? n_seq : n_groups;
-  loss_scalars_kernel<<<max(1, min((nmax + kLossThreads - 1) / kLossThreads, sms * 4)), kLossThreads,
-                        0, s>>>(w.gsize, n_groups, w.n_tok, n_seq, w.scal);
-  loss_token_kernel<<<seq_blocks, kLossThreads, 0, s>>>(logp, old_logp, ref_logp, adv, cu_seqlens,
-                                                        group_id, n_seq, n_groups, loss_mask,
-                                                        clip_eps, kl_beta, agg, w.n_tok, w.gsize,
-                                                        w.scal, g, w.part, w.part_clip);
-  const int chunk = (n_seq + kLossFinalBlocks - 1) / kLossFinalBlocks;
+  const long long count_work = agg == 1 ? max(static_cast<long long>(n_seq), T / 16) : n_seq;
+  const int count_blocks =
+      static_cast<int>(max(1ll, min((count_work + kLossThreads - 1) / kLossThreads, sms * 4ll)));
+  loss_groups_kernel<<<count_blocks, kLossThreads, 0, s>>>(group_id, n_seq, n_groups, cu_seqlens,
+                                                           loss_mask, agg, w.gsize, w.scal);
+  // one wave of resident blocks striding over the sequences; a group of 16
+  // lanes per sequence when they are short
+  const bool short_seqs = T <= 128ll * n_seq;
+  static int resident[2] = {0, 0};
+  int& res = resident[short_seqs ? 0 : 1];
+  if (res == 0) {
+    int r = 0;
+    const cudaError_t q =
+        short_seqs ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&r, loss_token_kernel<16>, kLossThreads, 0)
+                   : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&r, loss_token_kernel<32>, kLossThreads, 0);
+    res = q == cudaSuccess && r > 0 ? r : 4;
+  }
+  const int per_block = (kLossThreads / 32) * (short_seqs ? 2 : 1);  // sequences in flight per block
+  const int seq_blocks = max(1, min((n_seq + per_block - 1) / per_block, sms * res));
+  if (short_seqs)
+    loss_token_kernel<16><<<seq_blocks, kLossThreads, 0, s>>>(
+        logp, old_logp, ref_logp, adv, cu_seqlens, group_id, n_seq, n_groups, loss_mask, clip_eps,
+        kl_beta, agg, w.gsize, w.scal, g, w.part_l, w.part_rk, w.part_clip, w.n_tok);
+  else
+    loss_token_kernel<32><<<seq_blocks, kLossThreads, 0, s>>>(
+        logp, old_logp, ref_logp, adv, cu_seqlens, group_id, n_seq, n_groups, loss_mask, clip_eps,
+        kl_beta, agg, w.gsize, w.scal, g, w.part_l, w.part_rk, w.part_clip, w.n_tok);
+  const int chunk = max(256, (n_seq + kLossFinalMaxBlocks - 1) / kLossFinalMaxBlocks);
   const int nb = (n_seq + chunk - 1) / chunk;
-  loss_final_partial_kernel<<<nb, kLossThreads, 0, s>>>(w.part, w.part_clip, n_seq, chunk,
-                                                        w.bpart);
-  loss_final_kernel<<<1, kLossThreads, 0, s>>>(w.bpart, nb, w.scal, loss, stats);
-  note_launches(5);
+  loss_final_kernel<<<nb, kLossThreads, 0, s>>>(w.part_l, w.part_rk, w.part_clip, w.n_tok, n_seq,
+                                                chunk, static_cast<LossSums*>(w.bpart), w.scal + 2,
+                                                loss, stats);
+  note_launches(3);
   return cudaGetLastError();
 }
 

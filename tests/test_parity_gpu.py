@@ -148,6 +148,99 @@ def test_advantages_run_path_bit_exact(layout):
     np.testing.assert_array_equal(got[ok].view(np.uint32), base.cpu().numpy()[ok].view(np.uint32))
 
 
+@pytest.mark.parametrize("layout", ["sorted", "reversed"])
+def test_advantages_sorted_pass_chunk_edges(layout):
+    """Group sizes around the sorted pass's chunks of 4096 sequences: groups
+    of one, groups that end exactly on a chunk edge or one before or after it,
+    and groups of 4097 and 10000 sequences that run on through two and three
+    chunks (one of them with all rewards equal).  "reversed" lays the same
+    groups out with their ids in descending order: still one run per group,
+    but not sorted, so the call takes the run path.  Bit-exact against the
+    fp32-order oracle either way."""
+    from paper_2607_20908_gb300 import spo
+    rng = np.random.default_rng(6)
+    sizes = np.array([4096, 1, 4095, 2, 4097, 16, 10000, 3, 1, 4094, 5000, 7000]
+                     + list(rng.integers(1, 40, 300)))
+    ng = sizes.size
+    ids = np.arange(ng) if layout == "sorted" else np.arange(ng)[::-1]
+    gid = np.repeat(ids, sizes).astype(np.int32)
+    r = rng.normal(0.3, 1.0, gid.size).astype(np.float32)
+    r[gid == ids[11]] = 2.5                      # 7000 equal rewards across chunk edges
+    want = O.group_advantages_f32(r, gid, ng)
+    adv = torch.full((gid.size,), 7.0, device="cuda")
+    got = spo.spo_group_advantages_ws(torch.from_numpy(r).cuda(), torch.from_numpy(gid).cuda(), ng,
+                                      adv=adv).cpu().numpy()
+    np.testing.assert_array_equal(got.view(np.uint32), want.view(np.uint32))
+    assert np.all(got[gid == ids[11]] == 0) and np.all(got[gid == ids[1]] == 0)
+
+
+def test_advantages_sorted_pass_large():
+    """2^22 rollouts in sorted groups of 4 to 16 (the enlarged benchmark
+    shape): 1025 chunks, every chunk edge inside some group.  The oracle runs
+    on 1500 sampled groups (groups are independent, so each sampled group is
+    its own small problem)."""
+    from paper_2607_20908_gb300 import spo
+    rng = np.random.default_rng(7)
+    sizes = rng.integers(4, 17, (1 << 22) // 10)
+    sizes = sizes[np.cumsum(sizes) <= (1 << 22) + 1000]
+    ng = sizes.size
+    gid = np.repeat(np.arange(ng), sizes).astype(np.int32)
+    r = rng.normal(0.3, 1.0, gid.size).astype(np.float32)
+    got = spo.spo_group_advantages_ws(torch.from_numpy(r).cuda(), torch.from_numpy(gid).cuda(),
+                                      ng).cpu().numpy()
+    starts = np.concatenate([[0], np.cumsum(sizes)])
+    for g in np.sort(rng.choice(ng, 1500, replace=False)):
+        seg = slice(starts[g], starts[g + 1])
+        want = O.group_advantages_f32(r[seg], np.zeros(sizes[g], dtype=np.int32), 1)
+        np.testing.assert_array_equal(got[seg].view(np.uint32), want.view(np.uint32))
+
+
+@pytest.mark.parametrize("agg", [0, 1])
+@pytest.mark.parametrize("max_len", [700, 120])
+def test_loss_long_sequences_and_unaligned_mask(agg, max_len):
+    """The loss forward on sequences of 1 to 700 tokens (a warp per sequence:
+    its first 128 tokens held in registers, the rest reloaded) or of 1 to 120
+    (eight lanes per sequence, 32 tokens a pass), groups with a sequence of
+    no loss tokens and an empty group, a mask that starts 3 bytes past a
+    16-byte boundary (the token mean counts it 16 bytes at a time after a
+    ragged head), KL arguments around the switch from the series, and
+    stand-in log-probs, against the fp64 oracle."""
+    from paper_2607_20908_gb300 import spo
+    rng = np.random.default_rng(8)
+    lens = rng.integers(1, max_len + 1, 41 if max_len > 256 else 160)
+    lens[[3, 17, 18, 19]] = [128, 129, 32, 33] if max_len > 256 else [31, 32, 33, 120]
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    T, n_seq = int(cu[-1]), lens.size
+    gid = np.minimum(np.arange(n_seq) // 4, 9).astype(np.int32)
+    gid[gid >= 5] += 1                                   # group 5 empty
+    ng = int(gid.max()) + 1
+    lm = (rng.random(T) < 0.7).astype(np.uint8)
+    lm[cu[6]:cu[7]] = 0                                  # a sequence with no loss tokens
+    lp = (-6.0 * rng.random(T)).astype(np.float32)
+    old = (lp + 0.2 * rng.normal(size=T)).astype(np.float32)
+    ref = (lp + 0.05 * rng.normal(size=T)).astype(np.float32)
+    # KL arguments on both sides of the series / direct switch at |delta| = 1/2, and far out
+    far = rng.choice(np.nonzero(lm)[0], 200, replace=False)
+    ref[far] = lp[far] + rng.choice([-0.5001, -0.4999, 0.4999, 0.5001, -3.0, 2.0, 6.0, 1e-4], 200)
+    adv = rng.normal(size=n_seq).astype(np.float32)
+    buf = torch.zeros(T + 3, dtype=torch.uint8, device="cuda")
+    mask = buf[3:]
+    mask.copy_(torch.from_numpy(lm))
+    dev = lambda a: torch.from_numpy(a).cuda()
+    loss, g, stats = spo.spo_policy_loss_fwd(dev(lp), dev(old), dev(ref), dev(adv), dev(cu),
+                                             dev(gid), ng, mask, 0.2, 0.04, agg)
+    loss_o, g_o, st_o = O.policy_loss(lp.astype(np.float64), old.astype(np.float64),
+                                      ref.astype(np.float64), adv.astype(np.float64), cu, gid, ng,
+                                      lm, 0.2, 0.04, agg)
+    assert abs(loss.item() - loss_o) <= 1e-5 * abs(loss_o)
+    assert P.rel_l2(g.cpu().numpy(), g_o) <= 1e-5
+    assert np.all(g.cpu().numpy()[lm == 0] == 0)
+    assert stats[3].item() == st_o["n_loss_tokens"]
+    assert abs(stats[0].item() - st_o["clip_frac"]) <= 1e-6
+    assert abs(stats[1].item() - st_o["mean_ratio"]) <= 1e-5 * st_o["mean_ratio"]
+    assert abs(stats[2].item() - st_o["mean_kl"]) <= 1e-5 * st_o["mean_kl"]
+
+
 def test_no_loss_tokens():
     """Every token masked: log-probs, loss, g, dH and dW are exactly zero."""
     case = inputs.tiny_case(seed=1041)
