@@ -2,11 +2,15 @@
 for ncu captures: the group advantages (spo_group_advantages_ws; 2^n
 rollouts in sorted contiguous groups of 16) and the loss forward
 (spo_policy_loss_fwd; 2^n tokens as sequences of 128, groups of 8, every
-token a loss token, KL on).  The inputs are the ones bench.py's `aux`
-measurement uses.
+token a loss token, KL on), with the inputs bench.py's `aux` measurement
+uses; or the forward at the full workload's T = 16384 and V = 151936 with a
+hidden size of 256 ("combine"), whose split-vocabulary combine reads the
+same 117 MB of partials as the full workload's while the device holds under
+1 GB.
 
     python -m paper_2607_20908_gb300.profile_aux --which adv --reps 6
     python -m paper_2607_20908_gb300.profile_aux --which loss --reps 6
+    python -m paper_2607_20908_gb300.profile_aux --which combine --reps 6
 
 Each rep follows a 256 MB write that evicts L2 and is timed with CUDA events;
 prints the sorted per-call times in microseconds.
@@ -25,7 +29,7 @@ if ROOT not in sys.path:
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--which", choices=["adv", "loss", "both"], default="both")
+    ap.add_argument("--which", choices=["adv", "loss", "both", "combine"], default="both")
     ap.add_argument("--log2n", type=int, default=24)
     ap.add_argument("--reps", type=int, default=6)
     a = ap.parse_args()
@@ -57,6 +61,13 @@ def main():
         ws2 = torch.empty(spo.policy_loss_workspace_size(ns, ng), dtype=torch.uint8, device=dev)
         calls["loss"] = lambda: spo.spo_policy_loss_fwd(lp, old, ref, a_seq, cu, gid2, ng, lm, 0.2,
                                                         0.04, ws=ws2)
+    if a.which == "combine":
+        T, d, V = 16384, 256, 151936
+        H = torch.randn(T, d, device=dev, generator=gen).to(torch.bfloat16)
+        W = (torch.randn(V, d, device=dev, generator=gen) * 0.02).to(torch.bfloat16)
+        tgt = torch.randint(0, V, (T,), device=dev, generator=gen, dtype=torch.int32)
+        ws3 = torch.empty(spo.logprobs_workspace_size(T, d, V), dtype=torch.uint8, device=dev)
+        calls["fwd_d256"] = lambda: spo.spo_logprobs_fwd(H, W, tgt, ws=ws3)
     for name, fn in calls.items():
         times = []
         for i in range(a.reps):
