@@ -562,9 +562,11 @@ def aux_measurements(dev, pk):
     ms = median_ms(lambda: spo.spo_group_advantages_ws(r, gid, groups, adv=adv, ws=ws))
     gbs = 12 * n / (ms / 1e3) / 1e9
     res["group_advantages"] = {"rollouts": n, "groups": groups, "ms": ms, "gbs": gbs,
-                               "frac_of_hbm": gbs / pk["hbm"], "bound": "hbm",
-                               "note": "enlarged synthetic size, contiguous groups of 16 "
-                                       "(spo_group_advantages_ws); a step has 128-640 sequences"}
+                               "frac_of_hbm": gbs / pk["hbm"], "bound": "issue",
+                               "note": "enlarged synthetic size, sorted contiguous groups of 16 "
+                                       "(spo_group_advantages_ws); instruction-issue-bound (one "
+                                       "correctly rounded divide per rollout for the bit-exact "
+                                       "fp32 order); a step has 128-640 sequences"}
     del gid, r, adv, ws
 
     # a5 at 2^24 loss tokens (131072 sequences of 128, groups of 8): per token
