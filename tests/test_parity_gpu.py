@@ -174,6 +174,27 @@ def test_advantages_sorted_pass_chunk_edges(layout):
     assert np.all(got[gid == ids[11]] == 0) and np.all(got[gid == ids[1]] == 0)
 
 
+@pytest.mark.parametrize("sizes", [
+    [4000, 196],            # the last group runs from chunk 0 to the end of the data, in the halo
+    [4000, 1000],           # ... past the halo to the end of the data (folded from memory)
+    [3, 4093, 4096, 1],     # groups ending exactly on chunk edges; a last group of one
+    [5, 17, 2000],          # one partial chunk
+    [1],                    # one sequence
+], ids=["tail_in_halo", "tail_past_halo", "exact_edges", "one_chunk", "single"])
+def test_advantages_sorted_pass_data_end(sizes):
+    """Where the sorted pass's last group meets the end of the data."""
+    from paper_2607_20908_gb300 import spo
+    rng = np.random.default_rng(9)
+    sizes = np.array(sizes)
+    gid = np.repeat(np.arange(sizes.size), sizes).astype(np.int32)
+    r = rng.normal(0.3, 1.0, gid.size).astype(np.float32)
+    want = O.group_advantages_f32(r, gid, sizes.size)
+    adv = torch.full((gid.size,), 7.0, device="cuda")
+    got = spo.spo_group_advantages_ws(torch.from_numpy(r).cuda(), torch.from_numpy(gid).cuda(),
+                                      sizes.size, adv=adv).cpu().numpy()
+    np.testing.assert_array_equal(got.view(np.uint32), want.view(np.uint32))
+
+
 def test_advantages_sorted_pass_large():
     """2^22 rollouts in sorted groups of 4 to 16 (the enlarged benchmark
     shape): 1025 chunks, every chunk edge inside some group.  The oracle runs
