@@ -59,7 +59,9 @@ spo_status device_info(DevInfo* info) {
   int dev = 0;
   SPO_CUDA(cudaGetDevice(&dev), "cudaGetDevice");
   static DevInfo cache[64];
+  static std::mutex cache_mu;  // calls may come from several host threads
   if (dev < 0 || dev >= 64) return fail(SPO_ERR_UNSUPPORTED, "device ordinal %d out of range", dev);
+  std::lock_guard<std::mutex> lock(cache_mu);
   DevInfo& c = cache[dev];
   if (c.dev != dev) {
     DevInfo n;

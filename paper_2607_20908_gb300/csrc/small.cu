@@ -1096,14 +1096,14 @@ std::atomic<long long> g_launches{0};
 int sm_count() {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
-  static int cache[64] = {0};
-  if (cache[dev] == 0) {
+  static std::atomic<int> cache[64] = {};  // racing first calls store the same value
+  int c = cache[dev].load(std::memory_order_relaxed);
+  if (c == 0) {
     int n = 0;
-    cache[dev] = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && n > 0
-                     ? n
-                     : 1;
+    c = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && n > 0 ? n : 1;
+    cache[dev].store(c, std::memory_order_relaxed);
   }
-  return cache[dev];
+  return c;
 }
 
 void note_launches(int n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
@@ -1312,14 +1312,17 @@ cudaError_t launch_policy_loss(const float* logp, const float* old_logp, const f
   // one wave of resident blocks striding over the sequences; a group of 16
   // lanes per sequence when they are short
   const bool short_seqs = T <= 128ll * n_seq;
-  static int resident[2] = {0, 0};
-  int& res = resident[short_seqs ? 0 : 1];
+  // resident blocks per SM of each variant (a property of the kernel and the
+  // architecture), looked up once; racing first calls store the same value
+  static std::atomic<int> resident[2] = {{0}, {0}};
+  int res = resident[short_seqs ? 0 : 1].load(std::memory_order_relaxed);
   if (res == 0) {
     int r = 0;
     const cudaError_t q =
         short_seqs ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&r, loss_token_kernel<16>, kLossThreads, 0)
                    : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&r, loss_token_kernel<32>, kLossThreads, 0);
     res = q == cudaSuccess && r > 0 ? r : 4;
+    resident[short_seqs ? 0 : 1].store(res, std::memory_order_relaxed);
   }
   const int per_block = (kLossThreads / 32) * (short_seqs ? 2 : 1);  // sequences in flight per block
   const int seq_blocks = max(1, min((n_seq + per_block - 1) / per_block, sms * res));

@@ -147,3 +147,42 @@ def test_two_streams_at_once_match_serial_runs(spo):
         _same_bits(alone_a, oa)
         _same_bits(alone_b, ob)
     assert spo.spo_device_error() == 0
+
+
+def test_host_threads_match_serial_runs(spo):
+    """Four host threads, each with its own batch, workspaces and stream,
+    call the whole step at the same time (ctypes releases the GIL around each
+    call): the library's per-device caches and launch paths are shared, and
+    every result is the same bits as a run alone."""
+    import threading
+    cases = [_tensors(spo, inputs.tiny_case(seed=1310 + k, T_per_seq=60 + 7 * k, n_groups=3,
+                                            rollouts=4, V=4096 + 512 * k)) for k in range(4)]
+    torch.cuda.synchronize()
+    alone = []
+    for t in cases:
+        alone.append({k: v.clone() for k, v in _step(spo, t).items()})
+    torch.cuda.synchronize()
+    outs, errors = [None] * 4, []
+
+    def work(k):
+        try:
+            s = torch.cuda.Stream()
+            with torch.cuda.stream(s):
+                res = [_step(spo, cases[k]) for _ in range(3)]
+                outs[k] = [{n: v.clone() for n, v in r.items()} for r in res]
+            s.synchronize()
+        except Exception as e:     # reported below, on the test's thread
+            errors.append(e)
+
+    threads = [threading.Thread(target=work, args=(k,)) for k in range(4)]
+    for th in threads:
+        th.start()
+    for th in threads:
+        th.join()
+    assert not errors, errors
+    torch.cuda.synchronize()
+    for k in range(4):
+        for r in outs[k]:
+            _same_bits(alone[k], r)
+    assert spo.spo_device_error() == 0
+
