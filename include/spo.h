@@ -247,7 +247,8 @@ SPO_API spo_status spo_validate_inputs(const int32_t* tgt, int64_t T, int64_t V,
 /* ---------------------------------------------------------------------------
  * x[i] *= alpha for i < n (alpha_dev: device fp32 scalar used instead of alpha
  * when non-NULL).  Used by the data-parallel step to weight a rank's loss and
- * dL/dlogp by its share of the global normaliser of Eq. 3's average.
+ * dL/dlogp by its share of the global normaliser of Eq. 3's average.  Any
+ * 4-byte-aligned x; n == 0 is a no-op (x may then be NULL).
  * ------------------------------------------------------------------------- */
 SPO_API spo_status spo_scale_f32(float* x, int64_t n, float alpha, const float* alpha_dev,
                                  void* stream);

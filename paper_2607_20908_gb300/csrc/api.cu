@@ -717,10 +717,10 @@ SPO_API spo_status spo_ranker_pair_loss(const float* phi, const float* mu, const
 
 SPO_API spo_status spo_scale_f32(float* x, int64_t n, float alpha, const float* alpha_dev,
                                  void* stream) {
-  if (!x) return fail(SPO_ERR_INVALID_ARG, "x must be non-NULL");
   if (n < 0 || n > (1ll << 40)) return fail(SPO_ERR_SHAPE, "n = %lld out of range", (long long)n);
   if (!alpha_dev && !isfinite(alpha)) return fail(SPO_ERR_INVALID_ARG, "alpha must be finite");
   if (n == 0) return ok();
+  if (!x) return fail(SPO_ERR_INVALID_ARG, "x must be non-NULL");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   SPO_CUDA(spo::launch_scale(x, n, alpha, alpha_dev, s), "scale launch");
   return ok();

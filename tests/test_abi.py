@@ -111,6 +111,16 @@ def test_vocab_split_host_validation_without_gpu(lib):
               nul) == 3
 
 
+def test_scale_host_validation(lib):
+    p = ctypes.c_void_p(4096)
+    nul = ctypes.c_void_p(0)
+    f = lib.spo_scale_f32
+    assert f(nul, 0, 2.0, nul, nul) == 0                    # nothing to scale: no launch
+    assert f(nul, 5, 2.0, nul, nul) == 1                    # data needed
+    assert f(p, -1, 2.0, nul, nul) == 2
+    assert f(p, 5, float("inf"), nul, nul) == 1             # host factor must be finite
+
+
 def test_group_advantages_ws_host_validation(lib):
     from paper_2607_20908_gb300 import spo
     p = ctypes.c_void_p(4096)
