@@ -589,6 +589,38 @@ def aux_measurements(dev, pk):
     res["policy_loss_fwd"] = {"tokens": n, "sequences": ns, "groups": ng, "ms": ms, "gbs": gbs,
                               "frac_of_hbm": gbs / pk["hbm"], "bound": "hbm",
                               "note": "enlarged synthetic size; a step has 16384-131072 tokens"}
+    del cu, gid, lp, old, ref, a_seq, lm, ws
+
+    # a3 at the large workload's 131072 rows x 594 vocabulary tiles (936 MB of partials), timed
+    # by the library's own events around the combine launch inside a forward at d = 256
+    T2, d2, V2 = 131072, 256, 151936
+    H2 = torch.randn(T2, d2, device=dev, generator=gen).to(torch.bfloat16)
+    W2 = (torch.randn(V2, d2, device=dev, generator=gen) * 0.02).to(torch.bfloat16)
+    tgt2 = torch.randint(0, V2, (T2,), device=dev, generator=gen, dtype=torch.int32)
+    ws2 = torch.empty(spo.logprobs_workspace_size(T2, d2, V2), dtype=torch.uint8, device=dev)
+    fwd = lambda: spo.spo_logprobs_fwd(H2, W2, tgt2, ws=ws2)
+    for _ in range(2):
+        fwd()
+    torch.cuda.synchronize(dev)
+    spo.spo_trace_read()
+    spo.spo_trace_enable(True)
+    try:
+        for i in range(6):
+            flush.fill_(i & 0xFF)
+            fwd()
+        torch.cuda.synchronize(dev)
+        recs = spo.spo_trace_read()
+    finally:
+        spo.spo_trace_enable(False)
+    comb = sorted(t for k, t in recs if KERNEL_NAMES.get(k) == "lse_combine")
+    ms = comb[len(comb) // 2]
+    nbytes = T2 * (12 * ((V2 + 255) // 256) + 20)
+    gbs = nbytes / (ms / 1e3) / 1e9
+    res["lse_combine"] = {"rows": T2, "vocab_tiles": (V2 + 255) // 256, "ms": ms, "gbs": gbs,
+                          "frac_of_hbm": gbs / pk["hbm"], "bound": "hbm",
+                          "note": "the large workload's row count (the full workload's 16384 rows "
+                                  "move 117 MB, where launch and ramp weigh); partials written by "
+                                  "the forward just before, so part of them may sit in L2"}
     return res
 
 
