@@ -124,8 +124,9 @@ SPO_API spo_status spo_selftest_bounded_wait(void* stream);
  *   tgt        int32[T]
  *   loss_mask  uint8[T]  out   1 for loss tokens, else 0
  *   n_tok      int32[n_seq] out number of loss tokens of each sequence (|o_i|)
- * Bit-exact (integer work).  cu_seqlens monotonicity is the caller's contract
- * (device data is not inspected on the host).
+ * 1 <= n_seq <= 2^24, 1 <= T <= 2^30.  Bit-exact (integer work).  cu_seqlens
+ * monotonicity is the caller's contract (device data is not inspected on the
+ * host).
  * ------------------------------------------------------------------------- */
 SPO_API spo_status spo_token_select(const int32_t* cu_seqlens, const uint8_t* mask,
                                     const int32_t* tgt, int32_t n_seq, int64_t T, int32_t window,
@@ -310,8 +311,9 @@ SPO_API spo_status spo_group_advantages_ws(const float* rewards, const int32_t* 
  *   stats      fp32[4] out or NULL: {clip fraction, mean ratio, mean kl,
  *              number of loss tokens} over loss tokens
  *   ws         >= spo_policy_loss_workspace_size bytes
- * The reduction order is fixed: a group of lanes per sequence (8 when the
- * sequences average at most 256 tokens, else 32) sums its tokens in fp32
+ *   1 <= n_seq, n_groups <= 2^24, 1 <= T <= 2^30
+ * The reduction order is fixed: a group of lanes per sequence (16 when the
+ * sequences average at most 128 tokens, else 32) sums its tokens in fp32
  * (each lane its own tokens in order, then a fixed butterfly), and the sums
  * over sequences run in fp64 in two fixed stages whose split depends only on
  * n_seq, so results are deterministic run to run and across devices.

@@ -593,7 +593,7 @@ SPO_API spo_status spo_token_select(const int32_t* cu_seqlens, const uint8_t* ma
   if (!cu_seqlens || !tgt || !loss_mask || !n_tok)
     return fail(SPO_ERR_INVALID_ARG, "cu_seqlens, tgt, loss_mask and n_tok must be non-NULL");
   if (n_seq < 1 || n_seq > (1 << 24)) return fail(SPO_ERR_SHAPE, "n_seq = %d outside [1, 2^24]", n_seq);
-  if (T < 1 || T > (1ll << 31) - 1) return fail(SPO_ERR_SHAPE, "T = %lld out of range", (long long)T);
+  if (T < 1 || T > (1ll << 30)) return fail(SPO_ERR_SHAPE, "T = %lld outside [1, 2^30]", (long long)T);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   spo_status st = traced(kTraceTokenSelect, s, "token_select launch", [&] {
     return spo::launch_token_select(cu_seqlens, mask, tgt, n_seq, window, loss_mask, n_tok, s);
@@ -861,7 +861,7 @@ SPO_API spo_status spo_policy_loss_fwd(const float* logp, const float* old_logp,
     return fail(SPO_ERR_INVALID_ARG, "a required pointer is NULL");
   if (n_seq < 1 || n_groups < 1 || n_seq > (1 << 24) || n_groups > (1 << 24))
     return fail(SPO_ERR_SHAPE, "n_seq = %d, n_groups = %d out of range", n_seq, n_groups);
-  if (T < 1 || T > (1ll << 31) - 1) return fail(SPO_ERR_SHAPE, "T = %lld out of range", (long long)T);
+  if (T < 1 || T > (1ll << 30)) return fail(SPO_ERR_SHAPE, "T = %lld outside [1, 2^30]", (long long)T);
   if (agg != SPO_AGG_SEQ_GROUP && agg != SPO_AGG_TOKEN)
     return fail(SPO_ERR_INVALID_ARG, "agg %d unknown", agg);
   if (!(clip_eps >= 0.f && clip_eps < 1.f)) return fail(SPO_ERR_INVALID_ARG, "clip_eps must be in [0, 1)");
@@ -1045,7 +1045,7 @@ SPO_API spo_status spo_policy_loss_fwd_noalloc(const float* logp, const float* o
     return fail(SPO_ERR_INVALID_ARG, "a required pointer is NULL");
   if (n_seq < 1 || n_groups < 1 || n_seq > (1 << 24) || n_groups > (1 << 24))
     return fail(SPO_ERR_SHAPE, "n_seq = %d, n_groups = %d out of range", n_seq, n_groups);
-  if (T < 1 || T > (1ll << 31) - 1) return fail(SPO_ERR_SHAPE, "T = %lld out of range", (long long)T);
+  if (T < 1 || T > (1ll << 30)) return fail(SPO_ERR_SHAPE, "T = %lld outside [1, 2^30]", (long long)T);
   if (agg != SPO_AGG_SEQ_GROUP && agg != SPO_AGG_TOKEN)
     return fail(SPO_ERR_INVALID_ARG, "agg %d unknown", agg);
   if (!(clip_eps >= 0.f && clip_eps < 1.f)) return fail(SPO_ERR_INVALID_ARG, "clip_eps must be in [0, 1)");

@@ -111,6 +111,15 @@ def test_vocab_split_host_validation_without_gpu(lib):
               nul) == 3
 
 
+def test_token_and_loss_size_limits(lib):
+    """T above 2^30 is refused on the host (the kernels index tokens in 32-bit)."""
+    p = ctypes.c_void_p(4096)
+    nul = ctypes.c_void_p(0)
+    assert lib.spo_token_select(p, nul, p, 4, (1 << 30) + 1, 1024, p, p, nul) == 2
+    assert lib.spo_policy_loss_fwd(p, p, nul, p, p, p, 4, 2, p, (1 << 30) + 1, 0.2, 0.0, 0, p, p,
+                                   nul, p, 1 << 20, nul) == 2
+
+
 def test_scale_host_validation(lib):
     p = ctypes.c_void_p(4096)
     nul = ctypes.c_void_p(0)
