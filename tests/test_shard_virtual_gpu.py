@@ -1,0 +1,144 @@
+"""Data-parallel sharding through the CUDA kernels, with virtual ranks on one
+GPU: ``shard.DataParallelStep`` runs unmodified with ``shard.SpoEngine``
+(libspo) as every rank's compute, one host thread and CUDA stream per rank,
+and its collectives served in-process (the threads meet at a barrier and add
+the ranks' tensors in rank order; nothing on the device waits for another
+rank).  The sharded step must give the unsharded step's loss, dW and, row by
+row, dH."""
+
+import threading
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2607_20908_gb300 import shard
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def spo():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    from paper_2607_20908_gb300 import build
+    build.build()
+    from paper_2607_20908_gb300 import spo as mod
+    return mod
+
+
+class ThreadCollectives:
+    """all_reduce(sum) across n host threads, each registered with its rank."""
+
+    def __init__(self, n):
+        self.n = n
+        self.bar = threading.Barrier(n, timeout=60)
+        self.slots = [None] * n
+        self.local = threading.local()
+
+    def all_reduce(self, t, group=None):
+        if t.is_cuda:
+            torch.cuda.current_stream().synchronize()
+        self.slots[self.local.rank] = t.detach().clone()
+        self.bar.wait()
+        total = self.slots[0].clone()
+        for x in self.slots[1:]:
+            total += x.to(total.device)
+        self.bar.wait()
+        t.copy_(total)
+
+
+def _batch(seed):
+    rng = np.random.default_rng(seed)
+    sizes = [3, 5, 2, 4, 6, 1, 8]                 # rollouts per group (variable G, a group of one)
+    lens, gid = [], []
+    for g, n in enumerate(sizes):
+        for _ in range(n):
+            lens.append(int(rng.integers(6, 90)))
+            gid.append(g)
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    T, d, V = int(cu[-1]), 256, 4096
+    gen = torch.Generator().manual_seed(seed)
+    return dict(H=torch.randn(T, d, generator=gen).to(torch.bfloat16),
+                W=(torch.randn(V, d, generator=gen) * 0.05).to(torch.bfloat16),
+                tgt=torch.randint(0, V, (T,), generator=gen, dtype=torch.int32),
+                mask=torch.from_numpy((rng.random(T) > 0.25).astype(np.uint8)),
+                cu=cu, gid=np.array(gid, dtype=np.int32), n_groups=len(sizes),
+                rewards=torch.from_numpy(rng.uniform(0, 3, len(lens)).astype(np.float32)),
+                old_noise=torch.from_numpy(rng.normal(0, 0.2, T).astype(np.float32)),
+                ref_noise=torch.from_numpy(rng.normal(0, 0.05, T).astype(np.float32)))
+
+
+def _rank_dict(spo, b, rb, old, ref):
+    dev = torch.device("cuda")
+    tok = torch.from_numpy(rb.token_index).long()
+    seq = torch.from_numpy(rb.seq_index).long()
+    return dict(H=b["H"][tok].contiguous().to(dev), W=b["W"].to(dev),
+                tgt=b["tgt"][tok].contiguous().to(dev), mask=b["mask"][tok].contiguous().to(dev),
+                cu_seqlens=torch.from_numpy(rb.cu_seqlens).to(dev),
+                group_id=torch.from_numpy(rb.group_id).to(dev), n_groups=rb.n_groups,
+                rewards=b["rewards"][seq].contiguous().to(dev),
+                old=old[tok].contiguous().to(dev), ref=ref[tok].contiguous().to(dev),
+                window=40, inv_temp=1.0, clip_eps=0.2, kl_beta=0.04)
+
+
+@pytest.mark.parametrize("world", [2, 3])
+@pytest.mark.parametrize("agg", [0, 1])
+def test_virtual_ranks_reproduce_the_unsharded_step(spo, monkeypatch, world, agg):
+    import torch.distributed as dist
+    b = _batch(40 + world)
+    T = b["H"].shape[0]
+    # old / ref log-probs around the current policy's, fixed before sharding
+    dev = torch.device("cuda")
+    lp, _, _ = spo.spo_logprobs_fwd(b["H"].to(dev), b["W"].to(dev), b["tgt"].to(dev))
+    old = (lp.cpu() + b["old_noise"]).contiguous()
+    ref = (lp.cpu() + b["ref_noise"]).contiguous()
+
+    coll = ThreadCollectives(1)
+    monkeypatch.setattr(dist, "all_reduce", coll.all_reduce)
+    coll.local.rank = 0
+    whole = shard.rank_batch(b["cu"], b["gid"], range(b["n_groups"]))
+    loss1, dH1, dW1 = shard.DataParallelStep(shard.SpoEngine(), agg).run(
+        _rank_dict(spo, b, whole, old, ref))
+    torch.cuda.synchronize()
+
+    tokens_per_group = [int(b["cu"][np.nonzero(b["gid"] == g)[0] + 1].sum()
+                            - b["cu"][np.nonzero(b["gid"] == g)[0]].sum())
+                        for g in range(b["n_groups"])]
+    groups = shard.shard_groups(tokens_per_group, world)
+    batches = [shard.rank_batch(b["cu"], b["gid"], groups[r]) for r in range(world)]
+    coll = ThreadCollectives(world)
+    monkeypatch.setattr(dist, "all_reduce", coll.all_reduce)
+    outs, errors = [None] * world, []
+
+    def rank(r):
+        try:
+            coll.local.rank = r
+            s = torch.cuda.Stream()
+            with torch.cuda.stream(s):
+                outs[r] = shard.DataParallelStep(shard.SpoEngine(), agg).run(
+                    _rank_dict(spo, b, batches[r], old, ref))
+            s.synchronize()
+        except Exception as e:     # reported on the test's thread
+            errors.append(e)
+            coll.bar.abort()
+
+    threads = [threading.Thread(target=rank, args=(r,)) for r in range(world)]
+    for th in threads:
+        th.start()
+    for th in threads:
+        th.join()
+    assert not errors, errors
+    torch.cuda.synchronize()
+
+    for r in range(world):
+        loss_r, dH_r, dW_r = outs[r]
+        assert abs(loss_r.item() - loss1.item()) <= 1e-5 * abs(loss1.item()) + 1e-7
+        rel = ((dW_r - dW1).double().norm() / dW1.double().norm()).item()
+        assert rel <= 2e-3, rel
+        tok = torch.from_numpy(batches[r].token_index).long().to(dev)
+        want = dH1[tok].double()
+        rel_h = ((dH_r.double() - want).norm() / want.norm()).item()
+        assert rel_h <= 2e-3, rel_h
+    assert sum(len(x.token_index) for x in batches) == T
+    assert spo.spo_device_error() == 0
