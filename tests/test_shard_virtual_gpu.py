@@ -1,10 +1,11 @@
-"""Data-parallel sharding through the CUDA kernels, with virtual ranks on one
-GPU: ``shard.DataParallelStep`` runs unmodified with ``shard.SpoEngine``
-(libspo) as every rank's compute, one host thread and CUDA stream per rank,
-and its collectives served in-process (the threads meet at a barrier and add
-the ranks' tensors in rank order; nothing on the device waits for another
-rank).  The sharded step must give the unsharded step's loss, dW and, row by
-row, dH."""
+"""The multi-GPU step forms through the CUDA kernels, with virtual ranks on
+one GPU: ``shard.DataParallelStep`` (whole groups per rank) with
+``shard.SpoEngine`` and ``shard.VocabParallelStep`` (W's rows split) with
+``shard.SpoVocabEngine`` run unmodified, libspo as every rank's compute, one
+host thread and CUDA stream per rank, and their collectives served in-process
+(the threads meet at a barrier and add or gather the ranks' tensors in rank
+order; nothing on the device waits for another rank).  Each must give the
+unsharded step's results."""
 
 import threading
 
@@ -35,6 +36,18 @@ class ThreadCollectives:
         self.bar = threading.Barrier(n, timeout=60)
         self.slots = [None] * n
         self.local = threading.local()
+
+    def get_world_size(self, group=None):
+        return self.n
+
+    def all_gather(self, parts, t, group=None):
+        if t.is_cuda:
+            torch.cuda.current_stream().synchronize()
+        self.slots[self.local.rank] = t.detach().clone()
+        self.bar.wait()
+        for r in range(self.n):
+            parts[r].copy_(self.slots[r])
+        self.bar.wait()
 
     def all_reduce(self, t, group=None):
         if t.is_cuda:
@@ -109,6 +122,22 @@ def test_virtual_ranks_reproduce_the_unsharded_step(spo, monkeypatch, world, agg
     batches = [shard.rank_batch(b["cu"], b["gid"], groups[r]) for r in range(world)]
     coll = ThreadCollectives(world)
     monkeypatch.setattr(dist, "all_reduce", coll.all_reduce)
+    outs = _run_ranks(coll, world, lambda r: shard.DataParallelStep(shard.SpoEngine(), agg).run(
+        _rank_dict(spo, b, batches[r], old, ref)))
+    for r in range(world):
+        loss_r, dH_r, dW_r = outs[r]
+        assert abs(loss_r.item() - loss1.item()) <= 1e-5 * abs(loss1.item()) + 1e-7
+        rel = ((dW_r - dW1).double().norm() / dW1.double().norm()).item()
+        assert rel <= 2e-3, rel
+        tok = torch.from_numpy(batches[r].token_index).long().to(dev)
+        want = dH1[tok].double()
+        rel_h = ((dH_r.double() - want).norm() / want.norm()).item()
+        assert rel_h <= 2e-3, rel_h
+    assert sum(len(x.token_index) for x in batches) == T
+    assert spo.spo_device_error() == 0
+
+
+def _run_ranks(coll, world, fn):
     outs, errors = [None] * world, []
 
     def rank(r):
@@ -116,8 +145,7 @@ def test_virtual_ranks_reproduce_the_unsharded_step(spo, monkeypatch, world, agg
             coll.local.rank = r
             s = torch.cuda.Stream()
             with torch.cuda.stream(s):
-                outs[r] = shard.DataParallelStep(shard.SpoEngine(), agg).run(
-                    _rank_dict(spo, b, batches[r], old, ref))
+                outs[r] = fn(r)
             s.synchronize()
         except Exception as e:     # reported on the test's thread
             errors.append(e)
@@ -130,15 +158,56 @@ def test_virtual_ranks_reproduce_the_unsharded_step(spo, monkeypatch, world, agg
         th.join()
     assert not errors, errors
     torch.cuda.synchronize()
+    return outs
 
-    for r in range(world):
-        loss_r, dH_r, dW_r = outs[r]
+
+@pytest.mark.parametrize("world", [2, 3])
+def test_virtual_vocab_ranks_reproduce_the_unsplit_step(spo, monkeypatch, world):
+    """W's 4096 rows as 2 or 3 slices (3: uneven, with a ragged vocabulary
+    tile inside a slice): every rank ends with the unsplit log-probs, loss and
+    dH, and its own rows of dW."""
+    import torch.distributed as dist
+    b = _batch(50 + world)
+    dev = torch.device("cuda")
+    H, W, tgt = b["H"].to(dev), b["W"].to(dev), b["tgt"].to(dev)
+    cu, gid = torch.from_numpy(b["cu"]).to(dev), torch.from_numpy(b["gid"]).to(dev)
+    mask, rewards = b["mask"].to(dev), b["rewards"].to(dev)
+    lp0, _, _ = spo.spo_logprobs_fwd(H, W, tgt)
+    old = (lp0 + b["old_noise"].to(dev)).contiguous()
+    ref = (lp0 + b["ref_noise"].to(dev)).contiguous()
+    # the unsplit step
+    lm, _ = spo.spo_token_select(cu, mask, tgt, 40)
+    logp1, _, lse1 = spo.spo_logprobs_fwd(H, W, tgt, lm)
+    adv = spo.spo_group_advantages(rewards, gid, b["n_groups"])
+    loss1, g1, _ = spo.spo_policy_loss_fwd(logp1, old, ref, adv, cu, gid, b["n_groups"], lm, 0.2,
+                                           0.04)
+    dH1, dW1 = spo.spo_policy_loss_bwd(H, W, tgt, lse1, g1)
+    torch.cuda.synchronize()
+
+    slices = shard.vocab_slices(W.shape[0], world)
+    coll = ThreadCollectives(world)
+    monkeypatch.setattr(dist, "all_reduce", coll.all_reduce)
+    monkeypatch.setattr(dist, "all_gather", coll.all_gather)
+    monkeypatch.setattr(dist, "get_world_size", coll.get_world_size)
+
+    def rank(r):
+        off, n = slices[r]
+        rb = dict(H=H, W_slice=W[off:off + n], v_offset=off, tgt=tgt, mask=mask, cu_seqlens=cu,
+                  group_id=gid, n_groups=b["n_groups"], rewards=rewards, old=old, ref=ref,
+                  window=40, inv_temp=1.0, clip_eps=0.2, kl_beta=0.04)
+        return shard.VocabParallelStep(shard.SpoVocabEngine(), 0).run(rb)
+
+    outs = _run_ranks(coll, world, rank)
+    for r, (loss_r, logp_r, dH_r, dW_r) in enumerate(outs):
+        assert torch.abs(logp_r - logp1).max().item() <= 1e-5
         assert abs(loss_r.item() - loss1.item()) <= 1e-5 * abs(loss1.item()) + 1e-7
-        rel = ((dW_r - dW1).double().norm() / dW1.double().norm()).item()
-        assert rel <= 2e-3, rel
-        tok = torch.from_numpy(batches[r].token_index).long().to(dev)
-        want = dH1[tok].double()
-        rel_h = ((dH_r.double() - want).norm() / want.norm()).item()
-        assert rel_h <= 2e-3, rel_h
-    assert sum(len(x.token_index) for x in batches) == T
+        want = dH1.double()
+        assert ((dH_r.double() - want).norm() / want.norm()).item() <= 3e-3
+        off, n = slices[r]
+        w_rows = dW1[off:off + n].double()
+        assert ((dW_r.double() - w_rows).norm() / w_rows.norm()).item() <= 2e-3
+    # every rank holds the same merged results
+    for loss_r, logp_r, dH_r, _ in outs[1:]:
+        assert torch.equal(logp_r, outs[0][1]) and torch.equal(dH_r, outs[0][2])
     assert spo.spo_device_error() == 0
+
