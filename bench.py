@@ -83,9 +83,9 @@ SAMPLE_SEQS, SAMPLE_TOKENS = 8, 8   # CPU sample: one group of 8 rollouts, first
 # DRAM bytes (read + write) per launch of each tensor-core kernel on this workload, from one
 # `ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum` capture of this command
 # (profiles/launches_full_workload.md), valid only for the kernel sources they were taken on.
-TRAFFIC = {"sources_sha256_16": "229497a5c2c2001d",
-           "bytes": {"logits_lse_fwd": 6.859e9, "logits_grad_recompute": 13.466e9,
-                     "gemm_dH": 55.463e9, "gemm_dW": 13.860e9}}
+TRAFFIC = {"sources_sha256_16": "a451e474f3cd76dc",
+           "bytes": {"logits_lse_fwd": 6.879e9, "logits_grad_recompute": 13.570e9,
+                     "gemm_dH": 52.128e9, "gemm_dW": 14.965e9}}
 KERNEL_SOURCES = ["paper_2607_20908_gb300/csrc/gemm.cu", "paper_2607_20908_gb300/csrc/tc.cuh",
                   "paper_2607_20908_gb300/csrc/gemm.h"]
 
