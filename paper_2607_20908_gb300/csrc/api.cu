@@ -467,9 +467,10 @@ spo_status bwd_impl(const void* H, const void* W, const int32_t* tgt, const floa
                               lse, w.lse_c, g, w.g_c, s);
   });
   if (st != SPO_OK) return st;
+  // rows the compaction skips get zero; the dH GEMM writes all the others
   if (dH)
-    SPO_CUDA(cudaMemsetAsync(dH, 0, (dH_f32 ? sizeof(float) : sizeof(uint16_t)) * T * d, s),
-             "memset dH");
+    SPO_CUDA(spo::launch_zero_skipped_rows(g, T, static_cast<int>((dH_f32 ? 4 : 2) * d), dH, s),
+             "zero skipped dH rows");
 
   CUtensorMap tW_k, tG_store;
   SPO_CUDA(spo::make_tmap_bf16(&tW_k, W, d, V, d * 2, spo::BK, b_box_rows()), "tensor map W");

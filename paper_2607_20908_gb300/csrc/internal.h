@@ -89,6 +89,11 @@ cudaError_t launch_ranker_pair_loss(const float* phi, const float* mu, const flo
 // x[i] *= alpha (alpha read from device memory when alpha_dev != NULL).
 cudaError_t launch_scale(float* x, long long n, float alpha, const float* alpha_dev, cudaStream_t s);
 
+// Zeroes row t of out (row_bytes per row, a multiple of 16; out 16-byte aligned)
+// for every t < T with g[t] == 0: the dH rows the backward's compaction skips.
+cudaError_t launch_zero_skipped_rows(const float* g, long long T, int row_bytes, void* out,
+                                     cudaStream_t s);
+
 // Counts of invalid device inputs into counts[6] (zeroed here first); see spo_validate_inputs.
 cudaError_t launch_validate(const int* tgt, long long T, long long V, const int* cu, int n_seq,
                             const int* gid, int n_groups, const float* rewards, const float* old_logp,

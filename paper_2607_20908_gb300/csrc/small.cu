@@ -708,6 +708,20 @@ __global__ void scale_kernel(float* x, long long n, float alpha, const float* al
     x[i] *= a;
 }
 
+// Rows of dH that the backward skips (g == 0, the complement of its row
+// compaction) are zeroed here, one warp per token row with 16-byte stores; the
+// dH GEMM writes every other row.
+__global__ void zero_skipped_rows_kernel(const float* g, long long T, int row_bytes, uint8_t* out) {
+  const int lane = threadIdx.x & 31;
+  const long long nw = (static_cast<long long>(gridDim.x) * blockDim.x) >> 5;
+  for (long long t = (blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x) >> 5; t < T;
+       t += nw) {
+    if (g[t] != 0.f) continue;  // the same test as the compaction; uniform across the warp
+    uint4* row = reinterpret_cast<uint4*>(out + t * row_bytes);
+    for (int k = lane; k < row_bytes / 16; k += 32) row[k] = make_uint4(0u, 0u, 0u, 0u);
+  }
+}
+
 // Input validation: one grid-stride pass, integer atomics (counts are exact).
 __global__ void validate_kernel(const int* tgt, long long T, long long V, const int* cu, int n_seq,
                                 const int* gid, int n_groups, const float* rewards,
@@ -1248,6 +1262,16 @@ cudaError_t launch_scale(float* x, long long n, float alpha, const float* alpha_
   const long long want = (n + 255) / 256;
   const int blocks = static_cast<int>(want < sms * 8 ? (want < 1 ? 1 : want) : sms * 8);
   scale_kernel<<<blocks, 256, 0, s>>>(x, n, alpha, alpha_dev);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_zero_skipped_rows(const float* g, long long T, int row_bytes, void* out,
+                                     cudaStream_t s) {
+  const int sms = sm_count();
+  const long long want = (T + 7) / 8;  // 8 rows (warps) per block
+  const int blocks = static_cast<int>(want < sms * 16ll ? (want < 1 ? 1 : want) : sms * 16ll);
+  zero_skipped_rows_kernel<<<blocks, 256, 0, s>>>(g, T, row_bytes, static_cast<uint8_t*>(out));
   note_launches(1);
   return cudaGetLastError();
 }
