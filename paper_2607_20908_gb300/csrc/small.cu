@@ -750,7 +750,8 @@ __global__ void validate_kernel(const int* tgt, long long T, long long V, const 
 // ---------------------------------------------------------------- policy loss
 constexpr int kLossThreads = 256;
 
-// One warp per sequence; the grid strides over sequences.
+// Global warp index and warp count of the grid (the loss kernels' sequence
+// groups are derived from them; the grid strides over sequences).
 __device__ __forceinline__ int warp_seq0() { return (blockIdx.x * blockDim.x + threadIdx.x) >> 5; }
 __device__ __forceinline__ int warp_seq_stride() { return (gridDim.x * blockDim.x) >> 5; }
 
