@@ -564,9 +564,9 @@ def aux_measurements(dev, pk):
     res["group_advantages"] = {"rollouts": n, "groups": groups, "ms": ms, "gbs": gbs,
                                "frac_of_hbm": gbs / pk["hbm"], "bound": "issue",
                                "note": "enlarged synthetic size, sorted contiguous groups of 16 "
-                                       "(spo_group_advantages_ws); instruction-issue-bound (one "
-                                       "correctly rounded divide per rollout for the bit-exact "
-                                       "fp32 order); a step has 128-640 sequences"}
+                                       "(spo_group_advantages_ws); issue- and latency-bound block "
+                                       "program (stage, search, fold in the fp32 order, store); "
+                                       "a step has 128-640 sequences"}
     del gid, r, adv, ws
 
     # a5 at 2^24 loss tokens (131072 sequences of 128, groups of 8): per token
