@@ -314,9 +314,12 @@ SPO_API spo_status spo_group_advantages_ws(const float* rewards, const int32_t* 
  *   1 <= n_seq, n_groups <= 2^24, 1 <= T <= 2^30
  * The reduction order is fixed: a group of lanes per sequence (16 when the
  * sequences average at most 128 tokens, else 32) sums its tokens in fp32
- * (each lane its own tokens in order, then a fixed butterfly), and the sums
- * over sequences run in fp64 in two fixed stages whose split depends only on
- * n_seq, so results are deterministic run to run and across devices.
+ * (each lane its own tokens in order, then a fixed butterfly); the sums over
+ * sequences run in two fixed stages whose split depends only on n_seq -- the
+ * loss as an unevaluated pair of floats added with TwoSum (about 48
+ * significant bits, so cancellation between groups costs no accuracy), the
+ * ratio and KL statistics in fp32, the counts as integers -- so results are
+ * deterministic run to run and across devices.
  * ------------------------------------------------------------------------- */
 SPO_API spo_status spo_policy_loss_workspace_size(int32_t n_seq, int32_t n_groups, size_t* bytes);
 SPO_API spo_status spo_policy_loss_fwd(const float* logp, const float* old_logp,
