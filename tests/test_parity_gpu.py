@@ -262,6 +262,56 @@ def test_loss_long_sequences_and_unaligned_mask(agg, max_len):
     assert abs(stats[2].item() - st_o["mean_kl"]) <= 1e-5 * st_o["mean_kl"]
 
 
+@pytest.mark.parametrize("window", [-1, 0, 1, 7, 1024])
+def test_token_select_windows_and_empty_sequences(window):
+    """Loss-token selection, bit-exact against the oracle, for no cap (window
+    <= 0), a cap of one token, a small and the paper's 1024-token cap, on
+    ragged sequences that include empty ones (equal consecutive cu_seqlens),
+    with prompt masks and ignored targets."""
+    from paper_2607_20908_gb300 import spo
+    rng = np.random.default_rng(10)
+    lens = rng.integers(0, 2000, 60)
+    lens[[0, 7, 8, 59]] = 0                           # empty sequences, one at each end
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    T = int(cu[-1])
+    mask = (rng.random(T) > 0.4).astype(np.uint8)
+    tgt = rng.integers(0, 5000, T).astype(np.int32)
+    tgt[rng.random(T) < 0.05] = -100
+    lm, n_tok = spo.spo_token_select(torch.from_numpy(cu).cuda(), torch.from_numpy(mask).cuda(),
+                                     torch.from_numpy(tgt).cuda(), window)
+    lm_o, n_o = O.token_select(cu, mask, tgt, window)
+    np.testing.assert_array_equal(lm.cpu().numpy(), lm_o)
+    np.testing.assert_array_equal(n_tok.cpu().numpy(), n_o)
+    assert np.all(n_tok.cpu().numpy()[lens == 0] == 0)
+
+
+@pytest.mark.parametrize("agg", [0, 1])
+def test_loss_with_empty_sequences(agg):
+    """Empty sequences (no tokens) still count in their group's size and add
+    nothing to the loss (reading R6); checked against the fp64 oracle."""
+    from paper_2607_20908_gb300 import spo
+    rng = np.random.default_rng(11)
+    lens = rng.integers(1, 300, 48)
+    lens[[0, 5, 6, 47]] = 0
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    T = int(cu[-1])
+    gid = (np.arange(48) // 4).astype(np.int32)
+    lm = (rng.random(T) < 0.8).astype(np.uint8)
+    lp = (-5.0 * rng.random(T)).astype(np.float32)
+    old = (lp + 0.1 * rng.normal(size=T)).astype(np.float32)
+    ref = (lp + 0.05 * rng.normal(size=T)).astype(np.float32)
+    adv = rng.normal(size=48).astype(np.float32)
+    dev = lambda a: torch.from_numpy(a).cuda()
+    loss, g, stats = spo.spo_policy_loss_fwd(dev(lp), dev(old), dev(ref), dev(adv), dev(cu),
+                                             dev(gid), 12, dev(lm), 0.2, 0.04, agg)
+    loss_o, g_o, st_o = O.policy_loss(lp.astype(np.float64), old.astype(np.float64),
+                                      ref.astype(np.float64), adv.astype(np.float64), cu, gid, 12,
+                                      lm, 0.2, 0.04, agg)
+    assert abs(loss.item() - loss_o) <= 1e-5 * abs(loss_o)
+    assert P.rel_l2(g.cpu().numpy(), g_o) <= 1e-5
+    assert stats[3].item() == st_o["n_loss_tokens"]
+
+
 def test_no_loss_tokens():
     """Every token masked: log-probs, loss, g, dH and dW are exactly zero."""
     case = inputs.tiny_case(seed=1041)
