@@ -1,0 +1,82 @@
+"""Seeded shape fuzzing of the whole path against the fp64 oracle: 64 random
+small configurations, each with its own T (ragged sequence lengths, some
+empty), d (a multiple of 64), V (any multiple of 8 from 256), group layout,
+mask density, ignored targets, window, temperature, clip, KL weight,
+aggregation and std mode.  The bars are the path's (|d logp| <= 2e-2, loss
+relative error <= 1e-3, g / dH / dW relative L2 <= 2e-2); the configurations
+are fixed by the seed, so a failure reproduces."""
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import spo_oracle as O
+from paper_2607_20908_gb300 import inputs
+from tests import pipeline as P
+
+pytestmark = pytest.mark.gpu
+
+N_CASES = 64
+
+
+def _config(k):
+    rng = np.random.default_rng(9000 + k)
+    n_groups = int(rng.integers(1, 7))
+    sizes = rng.integers(1, 6, n_groups)
+    lens = rng.integers(0, 160, int(sizes.sum()))
+    lens[0] = max(lens[0], 1)
+    d = 64 * int(rng.integers(1, 9))
+    V = 8 * int(rng.integers(32, 1200))
+    return dict(rng=rng, sizes=sizes, lens=lens, d=d, V=V,
+                mask_p=float(rng.choice([1.0, 0.9, 0.6])),
+                ignore_p=float(rng.choice([0.0, 0.03])),
+                window=int(rng.choice([0, 5, 40, 1024])),
+                inv_temp=float(rng.choice([1.0, 1.0 / 0.7, 1.0 / 0.2])),
+                clip_eps=float(rng.choice([0.1, 0.2, 0.3])),
+                kl_beta=float(rng.choice([0.0, 0.04, 0.2])),
+                agg=int(rng.integers(0, 2)), std_mode=int(rng.integers(0, 2)),
+                old_std=float(rng.choice([0.05, 0.3])))
+
+
+def _case(k):
+    c = _config(k)
+    rng = c["rng"]
+    lens = c["lens"]
+    T = int(lens.sum())
+    H, W = inputs._dense_H_W(T, c["d"], c["V"], 9100 + k, "cpu")
+    tgt = torch.from_numpy(rng.integers(0, c["V"], T).astype(np.int32))
+    tgt[torch.from_numpy(rng.random(T) < c["ignore_p"])] = -100
+    mask = torch.from_numpy((rng.random(T) < c["mask_p"]).astype(np.uint8))
+    cu = torch.from_numpy(np.concatenate([[0], np.cumsum(lens)]).astype(np.int32))
+    gid = torch.from_numpy(np.repeat(np.arange(c["sizes"].size), c["sizes"]).astype(np.int32))
+    return dict(name=f"fuzz{k}", T=T, d=c["d"], V=c["V"], H=H, W=W, tgt=tgt, mask=mask,
+                cu_seqlens=cu, group_id=gid, n_groups=int(c["sizes"].size),
+                rewards=torch.from_numpy(rng.uniform(0, 3, c["sizes"].sum()).astype(np.float32)),
+                old_noise=torch.from_numpy((rng.normal(0, c["old_std"], T)).astype(np.float32)),
+                ref_noise=torch.from_numpy((rng.normal(0, 0.05, T)).astype(np.float32)),
+                clip_eps=c["clip_eps"], kl_beta=c["kl_beta"], inv_temp=c["inv_temp"],
+                window=c["window"]), c
+
+
+@pytest.mark.parametrize("k", range(N_CASES))
+def test_random_configuration(k):
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    case, c = _case(k)
+    if case["T"] == 0:
+        pytest.skip("no tokens drawn")
+    o = P.run_oracle(case, agg=c["agg"], std_mode=c["std_mode"])
+    g = P.run_gpu(case, o["old"], o["ref"], agg=c["agg"], std_mode=c["std_mode"])
+    desc = {x: c[x] for x in ("d", "V", "window", "inv_temp", "clip_eps", "kl_beta", "agg",
+                              "std_mode", "mask_p", "ignore_p")}
+    np.testing.assert_array_equal(g["loss_mask"], o["loss_mask"], err_msg=str(desc))
+    for key in ("logp", "entropy", "lse"):
+        assert np.abs(g[key] - o[key]).max() <= P.TOL_LOGP, (key, desc)
+    # the loss's advantage-weighted terms cancel within groups, so beside the
+    # relative bar its error may reach the first-order propagation of the
+    # log-prob error through g = dL/dlogp
+    err_lp = np.abs(g["logp"] - o["logp"]).max()
+    bound = P.TOL_LOSS_REL * abs(o["loss"]) + 2.0 * np.abs(o["g"]).sum() * err_lp + 1e-9
+    assert abs(g["loss"] - o["loss"]) <= bound, desc
+    for key in ("g", "dH", "dW"):
+        assert P.rel_l2(g[key], o[key]) <= P.TOL_GRAD_REL, (key, desc)
