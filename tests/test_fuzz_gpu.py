@@ -2,9 +2,11 @@
 small configurations, each with its own T (ragged sequence lengths, some
 empty), d (a multiple of 64), V (any multiple of 8 from 256), group layout,
 mask density, ignored targets, window, temperature, clip, KL weight,
-aggregation and std mode.  The bars are the path's (|d logp| <= 2e-2, loss
-relative error <= 1e-3, g / dH / dW relative L2 <= 2e-2); the configurations
-are fixed by the seed, so a failure reproduces."""
+aggregation and std mode; the first 24 of them also through the
+kept-exponential form and through the vocabulary split (2-4 slices at random
+multiples of 8).  The bars are the path's (|d logp| <= 2e-2, loss relative
+error <= 1e-3, g / dH / dW relative L2 <= 2e-2); the configurations are fixed
+by the seed, so a failure reproduces."""
 
 import numpy as np
 import pytest
@@ -80,3 +82,78 @@ def test_random_configuration(k):
     assert abs(g["loss"] - o["loss"]) <= bound, desc
     for key in ("g", "dH", "dW"):
         assert P.rel_l2(g[key], o[key]) <= P.TOL_GRAD_REL, (key, desc)
+
+
+def _oracle_and_inputs(k):
+    case, c = _case(k)
+    if case["T"] == 0:
+        pytest.skip("no tokens drawn")
+    o = P.run_oracle(case, agg=c["agg"], std_mode=c["std_mode"])
+    dev = torch.device("cuda")
+    t = {n: case[n].to(dev) for n in ("H", "W", "tgt", "mask", "cu_seqlens", "group_id", "rewards")}
+    return case, c, o, t
+
+
+def _loss_and_g(spo, case, c, o, t, logp, lm):
+    dev = torch.device("cuda")
+    adv = spo.spo_group_advantages(t["rewards"], t["group_id"], case["n_groups"], c["std_mode"])
+    loss, g, _ = spo.spo_policy_loss_fwd(logp, torch.from_numpy(o["old"]).to(dev),
+                                         torch.from_numpy(o["ref"]).to(dev), adv,
+                                         t["cu_seqlens"], t["group_id"], case["n_groups"], lm,
+                                         case["clip_eps"], case["kl_beta"], c["agg"])
+    return loss, g
+
+
+@pytest.mark.parametrize("k", range(24))
+def test_random_configuration_kept_form(k):
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    from paper_2607_20908_gb300 import spo
+    case, c, o, t = _oracle_and_inputs(k)
+    lm, _ = spo.spo_token_select(t["cu_seqlens"], t["mask"], t["tgt"], case["window"])
+    logp, ent, lse, keep, fws = spo.spo_logprobs_fwd_keep(t["H"], t["W"], t["tgt"], lm,
+                                                         case["inv_temp"])
+    assert np.abs(logp.cpu().numpy() - o["logp"]).max() <= P.TOL_LOGP
+    loss, g = _loss_and_g(spo, case, c, o, t, logp, lm)
+    dH, dW = spo.spo_policy_loss_bwd_kept(t["W"], lse, g, keep, fws, case["T"], case["d"],
+                                         case["inv_temp"])
+    torch.cuda.synchronize()
+    assert P.rel_l2(g.cpu().numpy(), o["g"]) <= P.TOL_GRAD_REL
+    assert P.rel_l2(dH.float().cpu().numpy(), o["dH"]) <= P.TOL_GRAD_REL
+    assert P.rel_l2(dW.cpu().numpy(), o["dW"]) <= P.TOL_GRAD_REL
+    assert spo.spo_device_error() == 0
+
+
+@pytest.mark.parametrize("k", range(24))
+def test_random_configuration_vocab_split(k):
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    from paper_2607_20908_gb300 import spo
+    case, c, o, t = _oracle_and_inputs(k)
+    V = case["V"]
+    rng = np.random.default_rng(9500 + k)
+    n_sl = min(int(rng.integers(2, 5)), V // 256)    # each slice >= 256 rows (the call's minimum)
+    if n_sl < 2:
+        pytest.skip("vocabulary too small to split")
+    units = V // 8                                    # slice sizes are multiples of 8 rows
+    sizes = 32 + rng.multinomial(units - 32 * n_sl, np.ones(n_sl) / n_sl)
+    bounds = (8 * np.concatenate([[0], np.cumsum(sizes)])).tolist()
+    lm, _ = spo.spo_token_select(t["cu_seqlens"], t["mask"], t["tgt"], case["window"])
+    recs = [spo.spo_logprobs_fwd_slice(t["H"], t["W"][a:z], a, t["tgt"], lm, case["inv_temp"])
+            for a, z in zip(bounds[:-1], bounds[1:])]
+    logp, ent, lse = spo.spo_logprobs_merge_slices(torch.stack(recs))
+    assert np.abs(logp.cpu().numpy() - o["logp"]).max() <= P.TOL_LOGP
+    assert np.abs(ent.cpu().numpy() - o["entropy"]).max() <= P.TOL_LOGP
+    loss, g = _loss_and_g(spo, case, c, o, t, logp, lm)
+    dH = torch.zeros(case["T"], case["d"], device="cuda")
+    dWs = []
+    for a, z in zip(bounds[:-1], bounds[1:]):
+        part, dw = spo.spo_policy_loss_bwd_slice(t["H"], t["W"][a:z], a, t["tgt"], lse, g,
+                                                 case["inv_temp"])
+        dH += part
+        dWs.append(dw)
+    torch.cuda.synchronize()
+    assert P.rel_l2(dH.cpu().numpy(), o["dH"]) <= P.TOL_GRAD_REL
+    assert P.rel_l2(torch.cat(dWs).cpu().numpy(), o["dW"]) <= P.TOL_GRAD_REL
+    assert spo.spo_device_error() == 0
+
