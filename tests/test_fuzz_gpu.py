@@ -4,7 +4,8 @@ empty), d (a multiple of 64), V (any multiple of 8 from 256), group layout,
 mask density, ignored targets, window, temperature, clip, KL weight,
 aggregation and std mode; the first 24 of them also through the
 kept-exponential form and through the vocabulary split (2-4 slices at random
-multiples of 8).  The bars are the path's (|d logp| <= 2e-2, loss relative
+multiples of 8); and 32 random group layouts for both advantage calls,
+bit-exact.  The bars are the path's (|d logp| <= 2e-2, loss relative
 error <= 1e-3, g / dH / dW relative L2 <= 2e-2); the configurations are fixed
 by the seed, so a failure reproduces."""
 
@@ -157,3 +158,42 @@ def test_random_configuration_vocab_split(k):
     assert P.rel_l2(torch.cat(dWs).cpu().numpy(), o["dW"]) <= P.TOL_GRAD_REL
     assert spo.spo_device_error() == 0
 
+
+
+@pytest.mark.parametrize("k", range(32))
+def test_random_advantage_layouts(k):
+    """Both advantage calls, bit-exact against the fp32-order oracle, on random
+    group layouts: sorted runs, runs in shuffled order, scattered members,
+    and (some cases) ids outside [0, n_groups), whose advantages stay as the
+    caller left them."""
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    from paper_2607_20908_gb300 import spo
+    rng = np.random.default_rng(9700 + k)
+    ng = int(rng.integers(1, 400))
+    sizes = rng.integers(1, int(rng.choice([3, 17, 40])), ng)
+    gid = np.repeat(np.arange(ng), sizes).astype(np.int32)
+    layout = ("sorted", "shuffled_runs", "scattered")[k % 3]
+    if layout == "shuffled_runs":
+        order = rng.permutation(ng)
+        gid = np.repeat(order, sizes[order]).astype(np.int32)
+    elif layout == "scattered":
+        gid = gid[rng.permutation(gid.size)]
+    n = gid.size
+    r = rng.normal(0.5, 1.0, n).astype(np.float32)
+    r[gid == 0] = 2.0                                   # one zero-variance group
+    invalid = k % 4 == 3
+    if invalid:
+        gid[rng.choice(n, max(1, n // 50), replace=False)] = rng.choice([-1, ng, ng + 7])
+    ok = (gid >= 0) & (gid < ng)
+    std_mode = int(rng.integers(0, 2))
+    # ids outside the range go to one extra oracle group whose values are not compared
+    want = O.group_advantages_f32(r, np.where(ok, gid, ng), ng + 1, std_mode)
+    rd, gd = torch.from_numpy(r).cuda(), torch.from_numpy(gid).cuda()
+    scan = spo.spo_group_advantages(rd, gd, ng, std_mode).cpu().numpy()
+    runs = spo.spo_group_advantages_ws(rd, gd, ng, std_mode,
+                                       adv=torch.full((n,), 7.0, device="cuda")).cpu().numpy()
+    for name, got in (("scan", scan), ("runs", runs)):
+        np.testing.assert_array_equal(got[ok].view(np.uint32), want[ok].view(np.uint32),
+                                      err_msg=f"{name} {layout}")
+    assert np.all(runs[~ok] == 7.0)
