@@ -13,6 +13,7 @@ import numpy as np
 import pytest
 import torch
 
+from oracle import spo_oracle as O
 from paper_2607_20908_gb300 import inputs
 
 pytestmark = pytest.mark.gpu
@@ -186,3 +187,39 @@ def test_host_threads_match_serial_runs(spo):
             _same_bits(alone[k], r)
     assert spo.spo_device_error() == 0
 
+
+
+def test_workspace_advantages_capture_into_a_graph(spo):
+    """spo_group_advantages_ws (a memset, the sorted pass and the gated run
+    path) and the loss forward captured into one graph: replays give the
+    eager bits, for sorted ids and, after the ids are rewritten in place, for
+    shuffled runs (the run path then does the work inside the replay)."""
+    rng = np.random.default_rng(12)
+    sizes = rng.integers(1, 30, 500)
+    ng = sizes.size
+    gid_sorted = np.repeat(np.arange(ng), sizes).astype(np.int32)
+    order = rng.permutation(ng)
+    gid_shuffled = np.repeat(order, sizes[order]).astype(np.int32)
+    n = gid_sorted.size
+    r = torch.from_numpy(rng.normal(0.3, 1.0, n).astype(np.float32)).cuda()
+    gid = torch.from_numpy(gid_sorted).cuda()
+    adv = torch.empty(n, device="cuda")
+    ws = torch.empty(spo.group_advantages_workspace_size(n, ng), dtype=torch.uint8, device="cuda")
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        spo.spo_group_advantages_ws(r, gid, ng, adv=adv, ws=ws)
+    torch.cuda.current_stream().wait_stream(side)
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        spo.spo_group_advantages_ws(r, gid, ng, adv=adv, ws=ws)
+    for ids in (gid_sorted, gid_shuffled):
+        gid.copy_(torch.from_numpy(ids))
+        adv.fill_(0)
+        graph.replay()
+        torch.cuda.synchronize()
+        eager = spo.spo_group_advantages_ws(r, gid, ng).cpu().numpy()
+        want = O.group_advantages_f32(r.cpu().numpy(), ids, ng)
+        np.testing.assert_array_equal(adv.cpu().numpy().view(np.uint32), want.view(np.uint32))
+        np.testing.assert_array_equal(eager.view(np.uint32), want.view(np.uint32))
+    assert spo.spo_device_error() == 0
