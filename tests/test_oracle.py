@@ -184,6 +184,108 @@ def test_advantage_f32_matches_f64():
     np.testing.assert_allclose(a32, a64, atol=2e-6, rtol=0)
 
 
+# Exact IEEE binary32 rounding (to nearest, ties to even) of a rational, in
+# integer arithmetic: checks the fixture's steps without any float32 unit.
+def _b32(bits_hex):
+    from fractions import Fraction
+    b = int(bits_hex, 16)
+    sign = -1 if b >> 31 else 1
+    e, m = (b >> 23) & 0xFF, b & 0x7FFFFF
+    assert 0 < e < 255, "fixture holds normal numbers only"
+    return sign * Fraction((1 << 23) | m, 1 << 23) * Fraction(2) ** (e - 127)
+
+
+def _round_b32(x):
+    from fractions import Fraction
+    x = Fraction(x)
+    if x == 0:
+        return "00000000"
+    a = abs(x)
+    e = a.numerator.bit_length() - a.denominator.bit_length()
+    while Fraction(2) ** e > a:
+        e -= 1
+    while Fraction(2) ** (e + 1) <= a:
+        e += 1
+    sc = a / Fraction(2) ** (e - 23)                      # in [2^23, 2^24)
+    q, rem = divmod(sc.numerator, sc.denominator)
+    rem = Fraction(rem, sc.denominator)
+    if rem > Fraction(1, 2) or (rem == Fraction(1, 2) and q % 2 == 1):
+        q += 1
+    if q == 1 << 24:
+        q, e = 1 << 23, e + 1
+    assert -126 <= e <= 127
+    return f"{((1 if x < 0 else 0) << 31) | ((e + 127) << 23) | (q - (1 << 23)):08x}"
+
+
+def _sqrt_b32(bits_hex):
+    """Correctly rounded binary32 square root of a binary32, by integer isqrt."""
+    from fractions import Fraction
+    x = _b32(bits_hex)
+    e = x.numerator.bit_length() - x.denominator.bit_length()
+    while Fraction(2) ** e > x:
+        e -= 1
+    es = e // 2                                            # floor(log2(sqrt(x)))
+    N = x * Fraction(2) ** (46 - 2 * es + 16)             # 8 guard bits beyond the 24
+    assert N.denominator == 1
+    r = math.isqrt(N.numerator)
+    exact = r * r == N.numerator
+    q, low = r >> 8, r & 0xFF
+    if low > 0x80 or (low == 0x80 and (not exact or q % 2 == 1)):
+        q += 1
+    return _round_b32(q * Fraction(2) ** (es - 23))
+
+
+def test_advantage_f32_bit_patterns(golden_dir):
+    """group_advantages_f32 reproduces, bit for bit, advantages derived step by
+    step in the fixed binary32 order (tests/golden/advantage_f32_bits.json).
+    The fixture's own steps are first re-derived here in exact integer
+    arithmetic, each one rounding of the previous listed values."""
+    gold = _golden(golden_dir, "advantage_f32_bits.json")
+    eps = _b32(gold["eps_bits"])
+    assert _round_b32(__import__("fractions").Fraction(gold["eps"])) == gold["eps_bits"]
+    for case in gold["cases"]:
+        r = np.asarray(case["rewards"], dtype=np.float32)
+        n = r.size
+        for mode_name, mode in case["modes"].items():
+            # the fixture's derivation, one rounded operation at a time
+            assert [f"{int(b):08x}" for b in r.view(np.uint32)] == mode["rewards_bits"]
+            rv = [_b32(b) for b in mode["rewards_bits"]]
+            acc = 0
+            for k in range(n):
+                acc_hex = _round_b32(acc + rv[k])
+                assert acc_hex == mode["running_sum"][k]
+                acc = _b32(acc_hex)
+            assert mode["sum"] == mode["running_sum"][-1]
+            assert _round_b32(acc / n) == mode["mean"]
+            mu = _b32(mode["mean"])
+            ss = 0
+            for k in range(n):
+                assert _round_b32(rv[k] - mu) == mode["deviations"][k]
+                dv = _b32(mode["deviations"][k])
+                assert _round_b32(dv * dv) == mode["rounded_squares"][k]
+                ss = _b32(_round_b32(ss + _b32(mode["rounded_squares"][k])))
+            assert _round_b32(ss) == mode["sum_sq"]
+            dof = n - 1 if mode_name == "unbiased" else n
+            assert _round_b32(_b32(mode["sum_sq"]) / dof) == mode["var"]
+            assert _sqrt_b32(mode["var"]) == mode["std"]
+            assert _round_b32(_b32(mode["std"]) + eps) == mode["den"]
+            den = _b32(mode["den"])
+            assert [_round_b32(_b32(d) / den) for d in mode["deviations"]] == mode["adv"]
+            # the pin: the oracle's fp32-order advantages carry exactly these bits
+            std_mode = O.STD_UNBIASED if mode_name == "unbiased" else O.STD_POPULATION
+            a = O.group_advantages_f32(r, np.zeros(n, np.int64), 1, std_mode, gold["eps"])
+            assert a.dtype == np.float32
+            assert [f"{int(b):08x}" for b in a.view(np.uint32)] == mode["adv"], (case["name"],
+                                                                                mode_name)
+            # group order does not matter: the same members scattered among another group
+            gid = np.array([0, 1] * n)[: 2 * n]
+            rr = np.empty(2 * n, np.float32)
+            rr[0::2] = r
+            rr[1::2] = np.float32(7.0)
+            a2 = O.group_advantages_f32(rr, gid, 2, std_mode, gold["eps"])
+            assert [f"{int(b):08x}" for b in a2[0::2].view(np.uint32)] == mode["adv"]
+
+
 # ---------------------------------------------------------------- loss
 def _single_token(rho, adv, beta, logp=None, ref=None, eps=0.2):
     lp = np.log(rho) if logp is None else logp

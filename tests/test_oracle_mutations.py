@@ -36,6 +36,14 @@ MUTATIONS = [
      "        if rg.max() == rg.min():\n            continue\n        mu = rg.sum() / n",
      "        mu = rg.sum() / n"),
     ("advantage f32: wrong count in the mean", "mu = f(acc / f(n))", "mu = f(acc / f(n + 1))"),
+    ("advantage f32: pairwise sum (np.sum) for the sequential one",
+     "        acc = f(0.0)\n        for i in idx:\n            acc = f(acc + r[i])",
+     "        acc = f(np.sum(r[idx]))"),
+    ("advantage f32: members summed in descending index",
+     "        for i in idx:\n            acc = f(acc + r[i])",
+     "        for i in reversed(idx):\n            acc = f(acc + r[i])"),
+    ("advantage f32: fused multiply-add in the sum of squares", "ss = f(ss + f(dv * dv))",
+     "ss = f(float(ss) + float(dv) * float(dv))"),
     ("KL: sign of delta", "kl = np.exp(delta) - delta - 1.0", "kl = np.exp(delta) + delta - 1.0"),
     ("surrogate: max for min", "surr = np.minimum(rho * A, clipped * A)",
      "surr = np.maximum(rho * A, clipped * A)"),
