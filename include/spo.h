@@ -462,7 +462,10 @@ SPO_API spo_status spo_policy_loss_bwd_slice(const void* H, const void* W_slice,
  * 1 MiB (roughly n_seq <= 32000 for a few thousand groups); larger sizes are
  * rejected with SPO_ERR_WORKSPACE before anything is enqueued.
  * The first call on a device looks up the array's device address (with that
- * device current); make that first call before any stream capture.
+ * device current); make that first call before any stream capture.  The
+ * scratch used is the current device's copy, so `stream` must belong to the
+ * current device: a stream of another device is refused with
+ * SPO_ERR_INVALID_ARG.
  * Every call shares the one array, and what is left in it is overwritten or
  * cleared on the stream by the next call: calls that can overlap on the GPU
  * (different streams, or several host threads) race on it and must be

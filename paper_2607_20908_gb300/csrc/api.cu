@@ -1060,17 +1060,27 @@ SPO_API spo_status spo_policy_loss_fwd_noalloc(const float* logp, const float* o
   DevInfo di;
   spo_status st = device_info(&di);
   if (st != SPO_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // The scratch looked up below is the current device's copy of the array; a
+  // stream of another device would run the kernels against it.
+  int stream_dev = -1;
+  SPO_CUDA(cudaStreamGetDevice(s, &stream_dev), "cudaStreamGetDevice");
+  if (stream_dev != di.dev)
+    return fail(SPO_ERR_INVALID_ARG,
+                "stream belongs to device %d but device %d is current; make the stream's device "
+                "current before calling spo_policy_loss_fwd_noalloc",
+                stream_dev, di.dev);
   void* scratch = nullptr;
   if ((st = noalloc_scratch(di.dev, &scratch)) != SPO_OK) return st;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
   // carve_loss_ws lays out the same buffers as the workspace entry point; the
   // group-size counters are cleared on the stream by launch_policy_loss.
   const spo::LossWs w = spo::carve_loss_ws(scratch, n_seq, n_groups);
-  SPO_CUDA(spo::launch_policy_loss(logp, old_logp, ref_logp, adv, cu_seqlens, group_id, n_seq,
+  st = traced(kTracePolicyLoss, s, "policy loss launch", [&] {
+    return spo::launch_policy_loss(logp, old_logp, ref_logp, adv, cu_seqlens, group_id, n_seq,
                                    n_groups, loss_mask, T, clip_eps, kl_beta, agg, loss, g, stats,
-                                   w, s),
-           "policy loss launch");
-  return ok();
+                                   w, s);
+  });
+  return st == SPO_OK ? ok() : st;
 }
 
 }  // extern "C"

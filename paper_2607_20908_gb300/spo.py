@@ -478,10 +478,12 @@ def spo_policy_loss_fwd_noalloc(logp, old_logp, ref_logp, adv, cu_seqlens, group
     _need(g, "g", torch.float32, T, dev)
     if stats is not None:
         _need(stats, "stats", torch.float32, 4, dev)
-    _check(lib().spo_policy_loss_fwd_noalloc(
-        _ptr(logp), _ptr(old_logp), _ptr(ref_logp), _ptr(adv), _ptr(cu_seqlens), _ptr(group_id),
-        n_seq, int(n_groups), _ptr(loss_mask), T, float(clip_eps), float(kl_beta), int(agg),
-        _ptr(loss), _ptr(g), _ptr(stats), _stream(dev)))
+    # the library uses the current device's copy of its static scratch
+    with torch.cuda.device(dev):
+        _check(lib().spo_policy_loss_fwd_noalloc(
+            _ptr(logp), _ptr(old_logp), _ptr(ref_logp), _ptr(adv), _ptr(cu_seqlens),
+            _ptr(group_id), n_seq, int(n_groups), _ptr(loss_mask), T, float(clip_eps),
+            float(kl_beta), int(agg), _ptr(loss), _ptr(g), _ptr(stats), _stream(dev)))
 
 
 SPO_TUNE_PAIR_MMA = 0

@@ -1,10 +1,14 @@
 """spo_policy_loss_fwd_noalloc: the policy-loss forward for callers that cannot
 give the library device scratch memory (a framework pool that owns all device
 memory, or a host path that must not call cudaMalloc because it synchronises
-the device).  Its scratch is a static array inside libspo, so the check here
-is that, called twice in a row through the C ABI on different batches, it
-gives what the workspace entry point gives on the same inputs, and that it
-refuses sizes beyond its fixed scratch.  Collected last on purpose."""
+the device).  Its scratch is a static array inside libspo that every call
+reuses.  It runs the same three kernels in the same fixed order as the
+workspace entry point, so on the same inputs the two must agree bit for bit;
+here that is checked through the C ABI on three calls in a row, the later
+ones on smaller batches with fewer groups (stale group counters or partial
+sums left in the array by a larger call would show), and each result is also
+checked against the fp64 oracle.  The call must refuse sizes beyond its fixed
+scratch.  Collected last on purpose."""
 
 import ctypes
 
@@ -12,6 +16,7 @@ import numpy as np
 import pytest
 import torch
 
+from oracle import spo_oracle as O
 from tests import pipeline as P
 
 pytestmark = pytest.mark.gpu
@@ -53,22 +58,45 @@ def _c_call(spo, b, loss, g, stats, agg):
         b["n_groups"], p(b["mask"]), b["T"], 0.2, 0.04, agg, p(loss), p(g), p(stats), stream)
 
 
-def test_noalloc_matches_workspace_entry_on_two_calls(spo):
+def _oracle(b, agg):
+    c = lambda t: t.cpu().numpy()
+    return O.policy_loss(c(b["logp"]).astype(np.float64), c(b["old"]).astype(np.float64),
+                         c(b["ref"]).astype(np.float64), c(b["adv"]).astype(np.float64), c(b["cu"]),
+                         c(b["gid"]), b["n_groups"], c(b["mask"]), 0.2, 0.04, agg)
+
+
+def test_noalloc_matches_workspace_entry_on_consecutive_calls(spo):
     dev = torch.device("cuda")
-    batches = [(_batch(11, 16, 8, 128, dev), 0), (_batch(12, 5, 3, 300, dev), 1)]
-    for b, agg in batches:
-        want_loss, want_g, want_stats = spo.spo_policy_loss_fwd(
-            b["logp"], b["old"], b["ref"], b["adv"], b["cu"], b["gid"], b["n_groups"], b["mask"],
-            0.2, 0.04, agg)
-        loss = torch.full((1,), float("nan"), device=dev)
-        g = torch.full((b["T"],), float("nan"), device=dev)
-        stats = torch.full((4,), float("nan"), device=dev)
-        assert _c_call(spo, b, loss, g, stats, agg) == 0
-        torch.cuda.synchronize()
-        wl, gl = float(want_loss.item()), float(loss.item())
-        assert abs(gl - wl) <= P.TOL_LOSS_REL * max(abs(wl), 1e-12), (gl, wl)
-        assert P.rel_l2(g.cpu().numpy(), want_g.cpu().numpy()) <= P.TOL_GRAD_REL
-        np.testing.assert_allclose(stats.cpu().numpy(), want_stats.cpu().numpy(), rtol=1e-6)
+    # largest first: each later call has fewer groups and sequences than the one before
+    batches = [(_batch(11, 16, 8, 128, dev), 0), (_batch(12, 5, 3, 300, dev), 1),
+               (_batch(14, 2, 3, 40, dev), 0)]
+    spo.spo_trace_read()
+    spo.spo_trace_enable(True)
+    try:
+        for b, agg in batches:
+            want_loss, want_g, want_stats = spo.spo_policy_loss_fwd(
+                b["logp"], b["old"], b["ref"], b["adv"], b["cu"], b["gid"], b["n_groups"],
+                b["mask"], 0.2, 0.04, agg)
+            loss = torch.full((1,), float("nan"), device=dev)
+            g = torch.full((b["T"],), float("nan"), device=dev)
+            stats = torch.full((4,), float("nan"), device=dev)
+            assert _c_call(spo, b, loss, g, stats, agg) == 0
+            torch.cuda.synchronize()
+            # the same kernels in the same order on the same inputs: the same bits
+            assert torch.equal(loss, want_loss), (loss.item(), want_loss.item())
+            assert torch.equal(g, want_g)
+            assert torch.equal(stats, want_stats)
+            # and the definition of Eq. 3 in fp64
+            o_loss, o_g, o_st = _oracle(b, agg)
+            gl = float(loss.item())
+            assert abs(gl - o_loss) <= P.TOL_LOSS_REL * max(abs(o_loss), 1e-12), (gl, o_loss)
+            assert P.rel_l2(g.cpu().numpy(), o_g) <= P.TOL_GRAD_REL
+            assert int(stats[3].item()) == o_st["n_loss_tokens"]
+        recs = spo.spo_trace_read()
+    finally:
+        spo.spo_trace_enable(False)
+    # every loss forward, with or without a workspace, is traced as kind 7
+    assert [k for k, _ in recs].count(7) == 2 * len(batches)
     assert spo.spo_device_error() == 0
 
 
