@@ -16,12 +16,16 @@ algorithmic TFLOP/s (from CUDA events recorded around each launch on its
 stream) against the measured bf16 peak; `cpu_baseline` is the fp64 oracle on
 a bounded sample of the same workload on this machine's host cores.
 
---impl reference times the fp64 oracle itself (host cores) on bounded
-samples of the same workload and prints the same line with impl=reference.
-Under torchrun every rank owns 16 whole groups of a data-parallel batch (weak
-scaling): its loss and dL/dlogp carry weight 1/N and dW is summed across
-ranks with one NCCL all-reduce per step; the timing adds a barrier and a max
-over ranks.
+The step is one C-ABI call (spo_grpo_step); --separate-calls times the
+individual calls in turn instead.  --impl reference times the fp64 oracle
+itself (host cores) on bounded samples of the same workload and prints the
+same line with impl=reference.  Under torchrun every rank owns 16 whole
+groups of a data-parallel batch (weak scaling): its loss and dL/dlogp carry
+weight 1/N (applied on the device) and dW is summed across ranks by NCCL in
+four vocabulary blocks, each started as soon as the backward has finished
+it; with --workload vocab-split the ranks instead split W's rows over one
+shared batch (strong scaling).  The timing adds a barrier and a max over
+ranks.
 """
 
 from __future__ import annotations
@@ -67,9 +71,9 @@ WORKLOADS = {
              "groups, KL to reference log-probs, d=5120, V=151936, bf16 fwd+bwd (4 backward chunks)",
     "kept": WORKLOAD + "; kept-exponential form: the forward also keeps exp(z - tile max) in bf16 "
             "(5 GB) and the backward forms G from it instead of recomputing the logits",
-    "vocab-split": WORKLOAD + "; vocabulary-split form: the head's rows as 2 slices of 75968, run "
-                   "in turn on one GPU (per-slice log-prob records merged, fp32 dH parts summed on "
-                   "the device where ranks would all-gather / all-reduce, dW written per slice)",
+    "vocab-split": WORKLOAD + "; vocabulary-split form: the head's rows as slices (one per GPU; "
+                   "on one GPU 2 slices of 75968 run in turn, fp32 dH parts summed on the device "
+                   "where ranks all-reduce), per-slice log-prob records merged, dW written per slice",
 }
 
 KERNEL_NAMES = {0: "logits_lse_fwd", 1: "logits_grad_recompute", 2: "gemm_dH", 3: "gemm_dW",
@@ -81,8 +85,8 @@ SAMPLE_SEQS, SAMPLE_TOKENS = 8, 8   # CPU sample: one group of 8 rollouts, first
 
 
 # DRAM bytes (read + write) per launch of each tensor-core kernel on this workload, from one
-# `ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum` capture of this command
-# (profiles/launches_full_workload.md), valid only for the kernel sources they were taken on.
+# `ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum` capture (one pass, the GEMM kernels
+# only), valid only for the kernel sources they were taken on.
 TRAFFIC = {"sources_sha256_16": "a451e474f3cd76dc",
            "bytes": {"logits_lse_fwd": 6.879e9, "logits_grad_recompute": 13.570e9,
                      "gemm_dH": 52.128e9, "gemm_dW": 14.965e9}}
@@ -214,16 +218,26 @@ class ClockSampler:
 
 # ----------------------------------------------------------------- the GPU step
 class Step:
-    """Device buffers + workspaces for one batch, driven through the C ABI."""
+    """Device buffers + workspaces for one batch, driven through the C ABI.
 
-    def __init__(self, case, dev, dist=None, own_inputs=False):
-        from paper_2607_20908_gb300 import spo
+    Modes: "fused" (the default: spo_grpo_step, the whole path in one call;
+    with several ranks, shard.DataParallelStep.run_fused: each rank's step
+    weighted by 1/N on the device, dW all-reduced block by block while the
+    backward's later blocks run), "separate" (the individual calls in turn),
+    "kept" (the kept-exponential form), "vocab" (W's rows as slices: in turn
+    on one GPU, or one slice per rank through shard.VocabParallelStep) and
+    "forward" (log-probs and entropy only)."""
+
+    def __init__(self, case, dev, dist=None, own_inputs=False, mode="fused", reserve_sms=8):
+        from paper_2607_20908_gb300 import shard, spo
         self.spo = spo
         self.forward_only = case.get("forward_only", "cu_seqlens" not in case)
+        self.mode = "forward" if self.forward_only else mode
         # data parallel over whole groups: every rank owns the same number of groups, so each
         # rank's share of Eq. 3's group average is exactly 1 / world
         self.dist = dist if dist is not None and dist.world > 1 else None
-        self.dp_weight = 1.0 / dist.world if self.dist else 1.0
+        self.world = dist.world if self.dist else 1
+        self.rank = dist.rank if self.dist else 0
         self.L = spo.lib()
         self.dev = dev
         self.case = case
@@ -251,37 +265,78 @@ class Step:
         self.loss, self.stats = torch.empty(1, **f32), torch.empty(4, **f32)
         self.g = torch.empty(T, **f32)
         self.dH = torch.empty((T, d), dtype=torch.bfloat16, device=dev)
-        self.dW = torch.empty((V, d), **f32)
-        # kept-exponential form: the forward keeps exp(z - tile max) for the backward
-        self.keep = None
-        if case.get("keep"):
-            self.keep = torch.empty(spo.logprobs_keep_size(T, V), dtype=torch.uint8, device=dev)
-        # vocabulary-split form: slices of W's rows run in turn, records merged
-        self.slices = []
-        if case.get("vocab_slices"):
-            from paper_2607_20908_gb300 import shard
-            self.slices = shard.vocab_slices(V, case["vocab_slices"])
-            self.rec = torch.empty((len(self.slices), T, 4), **f32)
-            self.dH_parts = [torch.empty((T, d), **f32) for _ in self.slices]
-            self.dH = torch.empty((T, d), **f32)   # the sum of the parts (fp32)
-        self.ws_f = torch.empty(spo.logprobs_workspace_size(T, d, V), dtype=torch.uint8, device=dev)
-        self.ws_l = torch.empty(max(256, spo.policy_loss_workspace_size(self.n_seq, self.n_groups)),
-                                dtype=torch.uint8, device=dev)
-        self.ws_b = torch.empty(spo.policy_loss_bwd_workspace_size(T, d, V), dtype=torch.uint8, device=dev)
         self.old = torch.empty(T, **f32)
         self.ref = torch.empty(T, **f32)
+        self.ws_f = torch.empty(spo.logprobs_workspace_size(T, d, V), dtype=torch.uint8, device=dev)
+        self.ws_l = self.ws_b = self.ws_s = self.keep = None
+        self.slices = []
+        if self.mode == "vocab":
+            # one slice per rank (the rank's rows only), or every slice in turn on one GPU
+            self.slices = shard.vocab_slices(V, max(2, self.world))
+            if self.dist:
+                off, n = self.slices[self.rank]
+                self.v_offset = off
+                self.W = self.W[off:off + n].contiguous()
+                self.vstep = shard.VocabParallelStep(shard.SpoVocabEngine(reserve_sms), 0)
+                self.dW = torch.empty((n, d), **f32)
+            else:
+                self.rec = torch.empty((len(self.slices), T, 4), **f32)
+                self.dH_parts = [torch.empty((T, d), **f32) for _ in self.slices]
+                self.dW = torch.empty((V, d), **f32)
+            self.dH = torch.empty((T, d), **f32)   # the sum of the parts (fp32)
+        elif not self.forward_only:
+            self.dW = torch.empty((V, d), **f32)
+        if self.mode == "kept":   # the forward keeps exp(z - tile max) for the backward
+            self.keep = torch.empty(spo.logprobs_keep_size(T, V), dtype=torch.uint8, device=dev)
+        if self.mode in ("separate", "kept", "vocab"):
+            self.ws_l = torch.empty(max(256, spo.policy_loss_workspace_size(self.n_seq, self.n_groups)),
+                                    dtype=torch.uint8, device=dev)
+        if self.mode in ("separate", "vocab") and not self.dist:
+            self.ws_b = torch.empty(spo.policy_loss_bwd_workspace_size(T, d, V), dtype=torch.uint8,
+                                    device=dev)
+        if self.mode == "fused":
+            if self.dist:
+                self.dp = shard.DataParallelStep(shard.SpoEngine(reserve_sms), 0, dw_blocks=4)
+            else:
+                self.ws_s = torch.empty(spo.grpo_workspace_size(T, d, V, self.n_seq, self.n_groups),
+                                        dtype=torch.uint8, device=dev)
+                self._structs()
         self.stream = torch.cuda.current_stream(dev)
+
+    def _structs(self):
+        """The one-call step's argument blocks, built once (device pointers stay fixed)."""
+        spo, c, p = self.spo, self.case, lambda t: ctypes.c_void_p(t.data_ptr())
+        self.c_batch = spo.GrpoBatch(p(self.H), p(self.W), p(self.tgt), p(self.mask), p(self.cu),
+                                     p(self.gid), p(self.rewards), p(self.old), p(self.ref), self.T,
+                                     self.d, self.V, self.n_seq, self.n_groups)
+        self.c_params = spo.GrpoParams(c["inv_temp"], c["window"], c["clip_eps"], c["kl_beta"], 0, 0,
+                                       1e-6, None)
+        self.c_out = spo.GrpoOutputs(p(self.loss), p(self.stats), p(self.logp), p(self.ent),
+                                     p(self.lse), p(self.g), p(self.adv), p(self.loss_mask),
+                                     p(self.dH), p(self.dW), 0)
 
     def prepare_old_ref(self):
         """Old / reference log-probs = current log-probs + noise (one forward, untimed)."""
         if self.forward_only:
             return
-        self.run(stop_after_fwd=True)
+        L, p, c = self.L, lambda t: ctypes.c_void_p(t.data_ptr()), self.case
+        s = ctypes.c_void_p(self.stream.cuda_stream)
+        W, V = (self.case["W"].to(self.dev), self.V) if self.mode == "vocab" else (self.W, self.V)
+        self.spo._check(L.spo_logprobs_fwd(p(self.H), p(W), p(self.tgt), p(self.mask), self.T,
+                                           self.d, V, c["inv_temp"], p(self.logp), None, None,
+                                           p(self.ws_f), self.ws_f.numel(), s))
         torch.cuda.synchronize(self.dev)
         self.old.copy_(self.logp + self.case["old_noise"].to(self.dev))
         self.ref.copy_(self.logp + self.case["ref_noise"].to(self.dev))
 
-    def run(self, stop_after_fwd=False):
+    def _rank_batch(self):
+        c = self.case
+        return dict(H=self.H, W=self.W, tgt=self.tgt, mask=self.mask, cu_seqlens=self.cu,
+                    group_id=self.gid, n_groups=self.n_groups, rewards=self.rewards, old=self.old,
+                    ref=self.ref, window=c["window"], inv_temp=c["inv_temp"],
+                    clip_eps=c["clip_eps"], kl_beta=c["kl_beta"], dH_out=self.dH, dW_out=self.dW)
+
+    def run(self):
         L, p, c = self.L, lambda t: ctypes.c_void_p(t.data_ptr()), self.case
         s = ctypes.c_void_p(self.stream.cuda_stream)
         chk = self.spo._check
@@ -289,6 +344,19 @@ class Step:
             chk(L.spo_logprobs_fwd(p(self.H), p(self.W), p(self.tgt), p(self.mask), self.T, self.d,
                                    self.V, c["inv_temp"], p(self.logp), p(self.ent), p(self.lse),
                                    p(self.ws_f), self.ws_f.numel(), s))
+            return
+        if self.mode == "fused":
+            if self.dist:       # whole groups per rank; the plan gives every rank 1/N of them
+                self.loss, _, _ = self.dp.run_fused(self._rank_batch(), self.n_groups * self.world)
+            else:
+                R = ctypes.byref
+                chk(L.spo_grpo_step(R(self.c_batch), R(self.c_params), R(self.c_out), None,
+                                    p(self.ws_s), self.ws_s.numel(), s))
+            return
+        if self.mode == "vocab" and self.dist:
+            b = self._rank_batch()
+            b.update(W_slice=self.W, v_offset=self.v_offset)
+            self.loss, self.logp, self.dH, self.dW = self.vstep.run(b)
             return
         chk(L.spo_token_select(p(self.cu), p(self.mask), p(self.tgt), self.n_seq, self.T, c["window"],
                                p(self.loss_mask), p(self.n_tok), s))
@@ -308,17 +376,12 @@ class Step:
             chk(L.spo_logprobs_fwd(p(self.H), p(self.W), p(self.tgt), p(self.loss_mask), self.T,
                                    self.d, self.V, c["inv_temp"], p(self.logp), p(self.ent),
                                    p(self.lse), p(self.ws_f), self.ws_f.numel(), s))
-        if stop_after_fwd:
-            return
         chk(L.spo_group_advantages(p(self.rewards), p(self.gid), self.n_seq, self.n_groups, 0, 1e-6,
                                    p(self.adv), s))
         chk(L.spo_policy_loss_fwd(p(self.logp), p(self.old), p(self.ref), p(self.adv), p(self.cu),
                                   p(self.gid), self.n_seq, self.n_groups, p(self.loss_mask), self.T,
                                   c["clip_eps"], c["kl_beta"], 0, p(self.loss), p(self.g),
                                   p(self.stats), p(self.ws_l), self.ws_l.numel(), s))
-        if self.dist:
-            chk(L.spo_scale_f32(p(self.g), self.T, self.dp_weight, None, s))
-            chk(L.spo_scale_f32(p(self.loss), 1, self.dp_weight, None, s))
         if self.slices:
             for k, (off, n) in enumerate(self.slices):
                 chk(L.spo_policy_loss_bwd_slice(p(self.H), p(self.W[off:off + n]), p(self.tgt),
@@ -340,9 +403,6 @@ class Step:
             chk(L.spo_policy_loss_bwd(p(self.H), p(self.W), p(self.tgt), p(self.lse), p(self.g),
                                       self.T, self.d, self.V, c["inv_temp"], p(self.dH),
                                       p(self.dW), 0, p(self.ws_b), self.ws_b.numel(), s))
-        if self.dist:   # the one real exchange of data-parallel training: sum of dW (and the loss)
-            self.dist.pg.all_reduce(self.dW)
-            self.dist.pg.all_reduce(self.loss)
 
 
 class HostIO:
@@ -354,7 +414,7 @@ class HostIO:
     copies on this platform stall for about 0.1 s every half second or so, and
     four sets give a step's copies three steps of compute to land in."""
 
-    def __init__(self, st: "Step", sets: int = 4, set_bytes: int = 0):
+    def __init__(self, st: "Step", sets: int = 4, set_bytes: int = 0, reserve_sms: int = 8):
         # at most what fits in 70 % of the free device memory (a set of the large
         # workload in the kept form holds ~60 GB), never fewer than two
         if set_bytes > 0:
@@ -363,8 +423,8 @@ class HostIO:
         self.n = sets
         # every set owns its inputs: a step's copies in must not land in a buffer
         # another step's kernels are reading
-        self.sets = [st] + [Step(st.case, st.dev, st.dist, own_inputs=True)
-                            for _ in range(sets - 1)]
+        self.sets = [st] + [Step(st.case, st.dev, st.dist, own_inputs=True, mode=st.mode,
+                                 reserve_sms=reserve_sms) for _ in range(sets - 1)]
         for x in self.sets[1:]:
             x.old.copy_(st.old)
             x.ref.copy_(st.ref)
@@ -374,11 +434,17 @@ class HostIO:
             outs = lambda x: (x.logp, x.ent, x.lse)
         else:
             ins = lambda x: (x.H, x.W, x.tgt, x.mask, x.cu, x.gid, x.rewards, x.old, x.ref)
-            outs = lambda x: (x.loss, x.stats, x.logp, x.ent, x.dH, x.dW)
+            if st.dist and st.mode == "vocab":       # the rank's results
+                outs = lambda x: (x.loss, x.logp, x.dH, x.dW)
+            elif st.dist:
+                outs = lambda x: (x.loss, x.dH, x.dW)
+            else:
+                outs = lambda x: (x.loss, x.stats, x.logp, x.ent, x.dH, x.dW)
+        # outputs are looked up after each step: a multi-rank step may hand back new tensors
+        self.outs = outs
         self.host_in = [pinned(t).copy_(t) for t in ins(st)]
-        self.host_out = [[pinned(t) for t in outs(x)] for x in self.sets]
+        self.host_out = [[pinned(t) for t in outs(st)] for _ in self.sets]
         self.dev_in = [ins(x) for x in self.sets]
-        self.dev_out = [outs(x) for x in self.sets]
         self.h2d = sum(t.numel() * t.element_size() for t in self.host_in)
         self.d2h = sum(t.numel() * t.element_size() for t in self.host_out[0])
         self.compute = st.stream
@@ -406,7 +472,7 @@ class HostIO:
         self.comp_done[b].record(self.compute)
         self.s_out.wait_event(self.comp_done[b])
         with torch.cuda.stream(self.s_out):
-            for d, h in zip(self.dev_out[b], self.host_out[b]):
+            for d, h in zip(self.outs(x), self.host_out[b]):
                 h.copy_(d, non_blocking=True)
             self.out_done[b].record(self.s_out)
         self.i += 1
@@ -625,7 +691,7 @@ def aux_measurements(dev, pk):
 
 
 # ----------------------------------------------------------------- arms
-def config_block(case, T_L, world, workload="full"):
+def config_block(case, T_L, world, workload="full", mode="fused"):
     cfg = {"workload": WORKLOADS[workload], "T": case["T"], "loss_tokens": T_L, "d": case["d"],
            "V": case["V"]}
     if workload == "full":
@@ -639,8 +705,23 @@ def config_block(case, T_L, world, workload="full"):
     if case.get("keep"):
         cfg["kept_exponentials"] = "forward keeps exp(z - tile max) in bf16; backward forms G from it"
     cfg["l2"] = "inputs larger than L2 (W alone is 1.2-1.56 GB and is streamed every step)"
-    cfg["parallelism"] = (f"dp{world}: whole groups per GPU, dW and loss all-reduced (NCCL) every step"
-                          if world > 1 else "1 GPU")
+    cfg["call"] = {"fused": "spo_grpo_step: the whole path (a1-a8) in one C-ABI call per step",
+                   "separate": "spo_token_select, spo_logprobs_fwd, spo_group_advantages, "
+                               "spo_policy_loss_fwd, spo_policy_loss_bwd in turn",
+                   "kept": "the kept-exponential forward and backward calls",
+                   "vocab": "per-slice forward, record merge, loss, per-slice backward",
+                   "forward": "spo_logprobs_fwd"}[mode]
+    if world == 1:
+        cfg["parallelism"] = "1 GPU"
+    elif workload == "vocab-split":
+        cfg["parallelism"] = (f"tp{world}: W's rows split over the GPUs, the batch on every GPU; "
+                              "per-token records all-gathered (NCCL), dH all-reduced while the "
+                              "rank's dW GEMMs run")
+    else:
+        cfg["parallelism"] = (f"dp{world}: whole groups per GPU, each rank's loss and g weighted "
+                              "1/N on the device; dW all-reduced (NCCL) in 4 vocabulary blocks, "
+                              "each as soon as the backward has finished it, while the later "
+                              "blocks' GEMMs run; loss all-reduced")
     return cfg
 
 
@@ -658,23 +739,36 @@ def ours(args):
              "kept": inputs.full_case}[args.workload]
     seed0 = {"full": 1003, "forward": 1002, "ragged": 1004, "large": 1005,
              "vocab-split": 1003, "kept": 1003}[args.workload]
-    case = maker(seed=seed0 + dist.rank, device=str(dev))
-    if args.workload in ("forward", "vocab-split") and dist.world > 1:
-        raise SystemExit(f"--workload {args.workload} runs on one GPU")
+    # data parallel: every rank its own batch (weak scaling); vocabulary split: one batch, W's
+    # rows split over the ranks (strong scaling)
+    vocab_ranks = args.workload == "vocab-split" and dist.world > 1
+    case = maker(seed=seed0 + (0 if vocab_ranks else dist.rank), device=str(dev))
+    mode = "fused"
     if args.workload == "vocab-split":
-        case["vocab_slices"] = 2
+        case["vocab_slices"] = max(2, dist.world)
+        mode = "vocab"
     if args.workload == "kept" or args.keep:
         if args.workload in ("forward", "vocab-split"):
             raise SystemExit(f"--keep does not apply to --workload {args.workload}")
         case["keep"] = True
+        mode = "kept"
+    if args.separate_calls and mode == "fused":
+        mode = "separate"
+    if dist.world > 1 and (args.workload == "forward" or mode in ("kept", "separate")):
+        raise SystemExit(f"--workload {args.workload} ({mode}) runs on one GPU")
     base_bytes = torch.cuda.memory_allocated(dev)
-    st = Step(case, dev, dist)
+    st = Step(case, dev, dist, mode=mode, reserve_sms=args.reserve_sms)
     step_bytes = (torch.cuda.memory_allocated(dev) - base_bytes      # one buffer set:
                   + sum(t.numel() * t.element_size() for t in (st.H, st.W)))  # + its own H, W
     st.prepare_old_ref()
     torch.cuda.synchronize(dev)
-    T_L = int(st.loss_mask.sum().item())
-    flop_gemm = 2.0 * T_L * st.d * st.V          # one GEMM-equivalent (algorithmic)
+    if st.forward_only:
+        T_L = int(st.mask.sum().item())
+    else:   # loss tokens: the same selection the step makes (untimed)
+        lm, _ = spo.spo_token_select(st.cu, st.mask, st.tgt, case["window"])
+        T_L = int(lm.sum().item())
+    V_rank = st.W.shape[0]                       # this rank's vocabulary rows
+    flop_gemm = 2.0 * T_L * st.d * V_rank        # one GEMM-equivalent on this GPU (algorithmic)
     # fwd + dH + dW (the backward's recompute is not counted); the forward-only workload: fwd
     flop_metric = (1.0 if st.forward_only else 3.0) * flop_gemm
     pk = peaks()
@@ -698,7 +792,7 @@ def ours(args):
     err = spo.spo_device_error(dev)
     assert err == 0, f"device wait expired (code {err:#x})"
 
-    tokens_s = dist.world * T_L * args.steps / (ms / 1e3)
+    tokens_s = (1 if vocab_ranks else dist.world) * T_L * args.steps / (ms / 1e3)
     kern = {}
     for kind, t in trace:
         k = kern.setdefault(KERNEL_NAMES.get(kind, str(kind)), {"launches": 0, "total_ms": 0.0})
@@ -753,11 +847,12 @@ def ours(args):
             k["frac_of_read_ceiling"] = k["gbs"] / k["read_ceiling_gbs"]
 
     # e2e: host buffers, H2D + step + D2H inside the timed region
-    hio = HostIO(st, sets=args.e2e_sets, set_bytes=step_bytes)
+    hio = HostIO(st, sets=args.e2e_sets, set_bytes=step_bytes, reserve_sms=args.reserve_sms)
     for _ in range(hio.n):
         hio.step()
     ms_e2e = timed_e2e(hio, args.steps, dist, dev)
-    e2e = {"value": dist.world * T_L * args.steps / (ms_e2e / 1e3), "unit": UNIT,
+    e2e = {"value": (1 if vocab_ranks else dist.world) * T_L * args.steps / (ms_e2e / 1e3),
+           "unit": UNIT,
            "h2d_bytes_per_step": hio.h2d, "d2h_bytes_per_step": hio.d2h,
            "ms_per_step": ms_e2e / args.steps,
            "path": ("pinned host -> device copies of every input (H, W, targets, mask), the C-ABI "
@@ -773,10 +868,10 @@ def ours(args):
         "metric": METRIC_FWD if st.forward_only else METRIC, "value": tokens_s, "unit": UNIT,
         "n_gpus": dist.world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "scaling": "strong" if vocab_ranks else "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded; H~N(0,1), W~N(0,0.02^2) rounded to bf16: random-init stand-in for "
                 "the policy's final hidden states and LM head)",
-        "config": config_block(case, T_L, dist.world, args.workload),
+        "config": config_block(case, T_L, dist.world, args.workload, mode),
         "tensor_peak_frac": {"metric_tflops": flop_metric * args.steps / (ms / 1e3) / 1e12,
                              "of_burst": flop_metric * args.steps / (ms / 1e3) / 1e12 / pk["bf16_burst"],
                              "of_sustained": flop_metric * args.steps / (ms / 1e3) / 1e12 / pk["bf16_sustained"],
@@ -853,6 +948,10 @@ def main():
                          "for a forward + backward workload")
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default="full",
                     help="supplementary workloads; the default is the one the metric is quoted on")
+    ap.add_argument("--separate-calls", action="store_true",
+                    help="run the step as the separate C-ABI calls instead of spo_grpo_step")
+    ap.add_argument("--reserve-sms", type=int, default=8,
+                    help="with several GPUs: SMs the GEMMs that overlap a collective leave free")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

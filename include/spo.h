@@ -97,10 +97,20 @@ SPO_API const char* spo_status_string(int status);
  * call (SPO_OK if none failed). */
 SPO_API int spo_last_error(char* buf, size_t n);
 
+/* The same as spo_last_error, under the name and return type of the
+ * boundary's specification: the calling thread's one-line description of its
+ * last failed call, and that call's status. */
+SPO_API spo_status spo_last_error_detail(char* buf, size_t n);
+
 /* Reads and clears the device-side error word that bounded waits set on
  * timeout.  SYNCHRONISES `stream`.  *code receives 0 or the kernel's code.
  * Returns SPO_ERR_TIMEOUT if a wait expired, else SPO_OK / SPO_ERR_CUDA. */
 SPO_API spo_status spo_device_error(int* code, void* stream);
+
+/* spo_device_error without the code: SYNCHRONISES `stream`, then returns
+ * SPO_ERR_CUDA if the stream's work failed, SPO_ERR_TIMEOUT if a bounded
+ * device wait expired since the last check (clearing it), else SPO_OK. */
+SPO_API spo_status spo_sync_check(void* stream);
 
 /* Failure-detection self-test: enqueues one thread that waits, through the
  * tensor-core kernels' own bounded wait, on a shared-memory barrier nothing
@@ -254,6 +264,14 @@ SPO_API spo_status spo_validate_inputs(const int32_t* tgt, int64_t T, int64_t V,
 SPO_API spo_status spo_scale_f32(float* x, int64_t n, float alpha, const float* alpha_dev,
                                  void* stream);
 
+/* x[i] *= (float)(num[0] / den[0]) for i < n, or x[i] = 0 when den[0] == 0;
+ * num and den are DEVICE fp64 scalars.  A data-parallel rank's weight in Eq.
+ * 3's global average is its own count over the all-reduced count (groups for
+ * SEQ_GROUP, loss tokens for TOKEN): this applies that weight without the
+ * host reading either count.  n == 0 is a no-op (x may then be NULL). */
+SPO_API spo_status spo_scale_f32_ratio(float* x, int64_t n, const double* num, const double* den,
+                                       void* stream);
+
 /* ---------------------------------------------------------------------------
  * a4. Group-normalised advantage (definition under Eq. 3):
  *   A_hat_i = (r_i - mean(r_g)) / (std(r_g) + eps), g = group_id[i].
@@ -356,6 +374,48 @@ SPO_API spo_status spo_policy_loss_bwd(const void* H, const void* W, const int32
                                        int accumulate_dW, void* ws, size_t ws_bytes, void* stream);
 
 /* ---------------------------------------------------------------------------
+ * The backward with hooks for overlapping its results' collectives (no
+ * counterpart in the paper, which trains on two GPUs without describing how
+ * gradients are exchanged).  In data-parallel training dW is summed over the
+ * ranks; in the vocabulary split dH is.  With hooks, dW is computed in
+ * n_dw_blocks contiguous blocks of vocabulary rows, and a caller's CUDA event
+ * is recorded on `stream` as soon as every dH row is final (dh_event) and as
+ * soon as each dW block is final (dw_block_events[k]), so a collective issued
+ * on another stream after waiting on that event runs while the remaining
+ * GEMMs do.  The GEMMs that follow the first event leave reserve_sms SMs of
+ * the device free for such a collective's kernels (0: use every SM).
+ *
+ *   n_dw_blocks      >= 1; block k covers dW rows [s_k, s_{k+1}) from
+ *                    spo_dw_block_starts(V, n_dw_blocks, s) (multiples of 256,
+ *                    the last block ends at V; a block may be empty)
+ *   dw_block_events  cudaEvent_t[n_dw_blocks] (entries may be NULL) or NULL
+ *   dh_event         cudaEvent_t or NULL
+ *   reserve_sms      in [0, SM count - 2]
+ * Events belong to the stream's device.  Every event is recorded even when
+ * its part is skipped (dH or dW NULL).  Blocking does not change the order in
+ * which any dW element is reduced: results are bit-identical to the call
+ * without hooks.
+ *
+ * spo_policy_loss_bwd_ex: spo_policy_loss_bwd (v_offset = 0, dH_fp32 = 0) or
+ * spo_policy_loss_bwd_slice (W points at row v_offset of the head; dH_fp32 =
+ * 1: dH is fp32, the slice's part), plus hooks (NULL: none).  Workspace as
+ * spo_policy_loss_bwd_workspace_size(T, d, V).
+ * ------------------------------------------------------------------------- */
+typedef struct spo_bwd_hooks {
+    int32_t n_dw_blocks;
+    int32_t reserve_sms;
+    void* const* dw_block_events;
+    void* dh_event;
+} spo_bwd_hooks;
+SPO_API spo_status spo_dw_block_starts(int64_t V, int32_t n_blocks, int64_t* starts);
+SPO_API spo_status spo_policy_loss_bwd_ex(const void* H, const void* W, const int32_t* tgt,
+                                          const float* lse, const float* g, int64_t T, int64_t d,
+                                          int64_t V, int64_t v_offset, float inv_temp, void* dH,
+                                          int dH_fp32, float* dW, int accumulate_dW,
+                                          const spo_bwd_hooks* hooks, void* ws, size_t ws_bytes,
+                                          void* stream);
+
+/* ---------------------------------------------------------------------------
  * Kept-exponential form of a2 + a6: the forward also stores, for every kept
  * token row r and vocabulary entry v, E[r][v] = exp(z - m) in bf16, m the
  * row's largest logit in v's 256-entry vocabulary tile; the backward then forms
@@ -446,6 +506,88 @@ SPO_API spo_status spo_policy_loss_bwd_slice(const void* H, const void* W_slice,
                                              int64_t v_offset, float inv_temp, float* dH_part,
                                              float* dW_slice, int accumulate_dW, void* ws,
                                              size_t ws_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * The whole GRPO step of Eq. 3 in one call: a1 (loss tokens: mask, ignore
+ * index, the 1024-token window of section 3) -> a2 + a3 (log-probs over the
+ * full vocabulary) -> a4 (group advantages) -> a5 (clipped surrogate, KL,
+ * aggregation, g = dL/dlogp) -> a6 - a8 (dH, dW), in stream order, validated
+ * once on the host.  Each step computes exactly what the separate calls
+ * compute; the backward reuses the forward's compaction of loss tokens
+ * instead of compacting again, so loss tokens whose g is exactly 0 (a binding
+ * clip with kl_beta = 0) run through the GEMMs with a zero gradient row.
+ * With no such token, dH and dW are bit-identical to those of the separate
+ * calls on the same inputs.
+ *
+ * spo_grpo_batch (all DEVICE arrays, as in the separate calls):
+ *   H bf16[T, d], W bf16[V, d] (16-byte aligned), tgt int32[T],
+ *   mask uint8[T] or NULL (1 = generated token), cu_seqlens int32[n_seq+1],
+ *   group_id int32[n_seq] in [0, n_groups), rewards fp32[n_seq] (r_i),
+ *   old_logp fp32[T], ref_logp fp32[T] or NULL;
+ *   sizes as in spo_logprobs_fwd (T <= 2^24) and spo_policy_loss_fwd.
+ * spo_grpo_params: inv_temp (> 0), window (<= 0: no cap), clip_eps in
+ *   [0, 1), kl_beta, agg (spo_agg), std_mode (spo_std), adv_eps (>= 0),
+ *   loss_scale: DEVICE fp32 scalar multiplying the loss and g (a
+ *   data-parallel rank's weight), or NULL for 1.
+ * spo_grpo_outputs: loss fp32[1] (required); stats fp32[4] as in
+ *   spo_policy_loss_fwd; logp, entropy, lse, g fp32[T], adv fp32[n_seq],
+ *   loss_mask uint8[T]; dH bf16[T, d] (16-byte aligned), dW fp32[V, d]
+ *   (+= when accumulate_dW).  Every output but loss may be NULL: it is then
+ *   kept in the workspace where the step needs it (entropy is then not
+ *   computed; dH or dW not at all).
+ * hooks: as in spo_policy_loss_bwd_ex, or NULL.
+ * ws: >= spo_grpo_workspace_size(T, d, V, n_seq, n_groups) bytes, 256-byte
+ *   aligned.
+ * ------------------------------------------------------------------------- */
+typedef struct spo_grpo_batch {
+    const void* H;
+    const void* W;
+    const int32_t* tgt;
+    const uint8_t* mask;
+    const int32_t* cu_seqlens;
+    const int32_t* group_id;
+    const float* rewards;
+    const float* old_logp;
+    const float* ref_logp;
+    int64_t T, d, V;
+    int32_t n_seq, n_groups;
+} spo_grpo_batch;
+typedef struct spo_grpo_params {
+    float inv_temp;
+    int32_t window;
+    float clip_eps;
+    float kl_beta;
+    int32_t agg;
+    int32_t std_mode;
+    float adv_eps;
+    const float* loss_scale;
+} spo_grpo_params;
+typedef struct spo_grpo_outputs {
+    float* loss;
+    float* stats;
+    float* logp;
+    float* entropy;
+    float* lse;
+    float* g;
+    float* adv;
+    uint8_t* loss_mask;
+    void* dH;
+    float* dW;
+    int32_t accumulate_dW;
+} spo_grpo_outputs;
+SPO_API spo_status spo_grpo_workspace_size(int64_t T, int64_t d, int64_t V, int32_t n_seq,
+                                           int32_t n_groups, size_t* bytes);
+SPO_API spo_status spo_grpo_step(const spo_grpo_batch* batch, const spo_grpo_params* params,
+                                 const spo_grpo_outputs* out, const spo_bwd_hooks* hooks, void* ws,
+                                 size_t ws_bytes, void* stream);
+
+/* One workspace for a whole step, under the boundary specification's name:
+ * bytes enough for spo_grpo_step with any n_groups <= n_seq, and for any
+ * single call of spo_logprobs_fwd, spo_policy_loss_fwd (n_groups <= n_seq),
+ * spo_group_advantages_ws and spo_policy_loss_bwd at these sizes, so the
+ * separate calls of one step can share it on one stream. */
+SPO_API spo_status spo_workspace_size(int64_t T, int64_t d, int64_t V, int32_t n_seq,
+                                      size_t* bytes);
 
 /* ---------------------------------------------------------------------------
  * spo_policy_loss_fwd without a caller workspace.  The paper has no

@@ -296,12 +296,14 @@ spo::GemmArgs base_args(const DevInfo& di) {
   return a;
 }
 
-// Persistent grid: one CTA per SM (pairs in pair mode), never more than tiles.
-int grid_for(const DevInfo& di, long long max_m, long long n) {
+// Persistent grid: one CTA per SM (pairs in pair mode), never more than tiles;
+// `reserve` SMs are left free for kernels that run alongside (a collective).
+int grid_for(const DevInfo& di, long long max_m, long long n, int reserve = 0) {
   const bool pair = g_tune_pair != 0;
   const long long tm = spo::gemm_tile_m(pair);
   const long long tiles = ((max_m + tm - 1) / tm) * ((n + spo::BN - 1) / spo::BN);
-  const long long units = pair ? di.sms / 2 : di.sms;
+  const int sms = di.sms - reserve > 2 ? di.sms - reserve : 2;
+  const long long units = pair ? sms / 2 : sms;
   long long g = tiles < units ? tiles : units;
   if (g < 1) g = 1;
   return static_cast<int>(pair ? 2 * g : g);
@@ -381,19 +383,47 @@ spo_status check_fwd_ws(int64_t T, int64_t d, int64_t V, const void* ws, size_t 
   return SPO_OK;
 }
 
-// a6-a8 over vocabulary rows [v_offset, v_offset + V) (W points at row
-// v_offset); dH is bf16, or fp32 with dH_f32.  Arguments are validated by the caller.
+// Hooks of a backward: dW computed in contiguous vocabulary blocks, with a
+// caller's event recorded on the stream as soon as each block (and, before
+// that, every dH row) is final, so a collective on another stream can start
+// on it while the remaining GEMMs run.  reserve_sms: the GEMMs that follow the
+// first event leave that many SMs free for such a collective.
+struct BwdHooks {
+  int n_dw_blocks = 1;
+  int reserve_sms = 0;
+  const cudaEvent_t* dw_events = nullptr;  // [n_dw_blocks] entries, each may be NULL
+  cudaEvent_t dh_event = nullptr;
+};
+
+// First row of vocabulary block k of n (block starts are multiples of 256
+// rows, one GEMM tile; the last block ends at V; blocks may be empty).
+long long dw_block_start(long long V, int n, int k) {
+  if (k >= n) return V;
+  return (V * k / n) / 256 * 256;
+}
+
+spo_status record_hook_events(const BwdHooks* hooks, cudaStream_t s) {
+  if (!hooks) return SPO_OK;
+  if (hooks->dh_event) SPO_CUDA(cudaEventRecord(hooks->dh_event, s), "record dH event");
+  if (hooks->dw_events)
+    for (int k = 0; k < hooks->n_dw_blocks; ++k)
+      if (hooks->dw_events[k]) SPO_CUDA(cudaEventRecord(hooks->dw_events[k], s), "record dW event");
+  return SPO_OK;
+}
+
 // a7 + a8 over a block of compacted rows [r0, r0 + rows): G holds them from
 // its first row (bf16, pitch ldG elements), Hc0 the same rows of the
 // compacted H, idx their token positions.  dH rows are scattered to token
 // rows (bf16, or fp32 with dH_f32); dW (+)= G^T Hc in passes of at most
 // g_tune_dw_split rows, the first pass adding into dW only when
-// accumulate_first.
+// accumulate_first.  With hooks, dW runs block by block over the vocabulary
+// and the hook events are recorded as dH and each dW block become final
+// (the per-element reduction order is the same as without them).
 spo_status dh_dw_block(const DevInfo& di, const void* W, int64_t d, int64_t V,
                        const __nv_bfloat16* G, long long ldG, long long rows,
                        const __nv_bfloat16* Hc0, long long r0, const int* count, const int* idx,
                        void* dH, bool dH_f32, float* dW, bool accumulate_first, int* counters,
-                       cudaStream_t s) {
+                       cudaStream_t s, const BwdHooks* hooks = nullptr) {
   spo_status st;
   CUtensorMap tG_k, tW_mn;
   SPO_CUDA(spo::make_tmap_bf16(&tG_k, G, V, rows, ldG * 2, spo::BK, spo::BM), "tensor map G");
@@ -416,32 +446,107 @@ spo_status dh_dw_block(const DevInfo& di, const void* W, int64_t d, int64_t V,
                           counters)) != SPO_OK)
       return st;
   }
+  if (hooks && hooks->dh_event) SPO_CUDA(cudaEventRecord(hooks->dh_event, s), "record dH event");
   // a8: dW (+)= G^T Hc over these rows, in passes of at most g_tune_dw_split
-  // rows (later passes reduce-add into dW)
-  if (dW) {
-    CUtensorMap tdW;
-    SPO_CUDA(spo::make_tmap_f32(&tdW, dW, d, V, d * 4, 32, spo::kStoreBoxRows), "tensor map dW");
-    const long long split = g_tune_dw_split > 0 ? g_tune_dw_split : rows;
-    for (long long q0 = 0; q0 < rows; q0 += split) {
-      const long long qrows = (rows - q0) < split ? (rows - q0) : split;
-      CUtensorMap tGq, tHq;
-      SPO_CUDA(spo::make_tmap_bf16(&tGq, G + q0 * ldG, V, qrows, ldG * 2, 64, spo::BK),
-               "tensor map G (MN)");
-      SPO_CUDA(spo::make_tmap_bf16(&tHq, Hc0 + q0 * d, d, qrows, d * 2, 64, spo::BK),
-               "tensor map Hc (MN)");
-      spo::GemmArgs b = base_args(di);
-      b.m_static = static_cast<int>(V);
-      b.n = static_cast<int>(d);
-      b.k_count = count;
-      b.k_offset = static_cast<int>(r0 + q0);
-      b.k_cap = static_cast<int>(qrows);
-      b.out_f32 = dW;
-      b.ld_out = d;
-      b.accumulate = (q0 == 0 && !accumulate_first) ? 0 : 1;
-      if ((st = traced_gemm(spo::EPI_DW, true, true, tGq, tHq, tdW, b, grid_for(di, V, d), s,
-                            counters)) != SPO_OK)
-        return st;
+  // rows (later passes reduce-add into dW), vocabulary block by block
+  const int nb = hooks && hooks->n_dw_blocks > 1 ? hooks->n_dw_blocks : 1;
+  const int reserve = hooks ? hooks->reserve_sms : 0;
+  for (int kb = 0; kb < nb; ++kb) {
+    const long long v0 = dw_block_start(V, nb, kb), v1 = dw_block_start(V, nb, kb + 1);
+    if (dW && v1 > v0) {
+      CUtensorMap tdW;
+      SPO_CUDA(spo::make_tmap_f32(&tdW, dW + v0 * d, d, v1 - v0, d * 4, 32, spo::kStoreBoxRows),
+               "tensor map dW");
+      const long long split = g_tune_dw_split > 0 ? g_tune_dw_split : rows;
+      for (long long q0 = 0; q0 < rows; q0 += split) {
+        const long long qrows = (rows - q0) < split ? (rows - q0) : split;
+        CUtensorMap tGq, tHq;
+        SPO_CUDA(spo::make_tmap_bf16(&tGq, G + q0 * ldG + v0, v1 - v0, qrows, ldG * 2, 64, spo::BK),
+                 "tensor map G (MN)");
+        SPO_CUDA(spo::make_tmap_bf16(&tHq, Hc0 + q0 * d, d, qrows, d * 2, 64, spo::BK),
+                 "tensor map Hc (MN)");
+        spo::GemmArgs b = base_args(di);
+        b.m_static = static_cast<int>(v1 - v0);
+        b.n = static_cast<int>(d);
+        b.k_count = count;
+        b.k_offset = static_cast<int>(r0 + q0);
+        b.k_cap = static_cast<int>(qrows);
+        b.out_f32 = dW + v0 * d;
+        b.ld_out = d;
+        b.accumulate = (q0 == 0 && !accumulate_first) ? 0 : 1;
+        if ((st = traced_gemm(spo::EPI_DW, true, true, tGq, tHq, tdW, b,
+                              grid_for(di, v1 - v0, d, reserve), s, counters)) != SPO_OK)
+          return st;
+      }
     }
+    if (hooks && hooks->dw_events && kb < hooks->n_dw_blocks && hooks->dw_events[kb])
+      SPO_CUDA(cudaEventRecord(hooks->dw_events[kb], s), "record dW event");
+  }
+  if (hooks && hooks->dw_events)  // blocks beyond the ones run (n_dw_blocks <= 1 uses one)
+    for (int kb = nb; kb < hooks->n_dw_blocks; ++kb)
+      if (hooks->dw_events[kb]) SPO_CUDA(cudaEventRecord(hooks->dw_events[kb], s), "record dW event");
+  return SPO_OK;
+}
+
+// The rows a backward runs over: a compaction (Hc, idx, count, compacted
+// targets) and the per-row lse and g, either compacted (lse[r], g[r]) or at
+// token positions (lse[idx[r]], g[idx[r]]: by_token).
+struct BwdRows {
+  const __nv_bfloat16* Hc;
+  const int* idx;
+  const int* count;
+  const int* tgt_c;
+  const float* lse;
+  const float* g;
+  bool by_token;
+  long long T_pad;
+};
+
+// a6-a8 over vocabulary rows [0, V) of W (a slice's rows when W points into a
+// larger head) for the given rows, in chunks of at most `chunk` rows of G.
+spo_status bwd_core(const DevInfo& di, const void* W, int64_t d, int64_t V, float inv_temp,
+                    const BwdRows& r, __nv_bfloat16* G, long long chunk, void* dH, bool dH_f32,
+                    float* dW, int accumulate_dW, int* counters, const BwdHooks* hooks,
+                    cudaStream_t s) {
+  spo_status st;
+  CUtensorMap tW_k, tG_store;
+  SPO_CUDA(spo::make_tmap_bf16(&tW_k, W, d, V, d * 2, spo::BK, b_box_rows()), "tensor map W");
+  SPO_CUDA(spo::make_tmap_bf16(&tG_store, G, V, chunk, V * 2, 64, spo::kStoreBoxRows),
+           "tensor map G (store)");
+  const long long n_chunks = (r.T_pad + chunk - 1) / chunk;
+  for (long long c = 0; c < n_chunks; ++c) {
+    const long long r0 = c * chunk;
+    const long long rows = (r.T_pad - r0) < chunk ? (r.T_pad - r0) : chunk;
+    const __nv_bfloat16* Hc0 = r.Hc + r0 * d;
+    CUtensorMap tH_k;
+    SPO_CUDA(spo::make_tmap_bf16(&tH_k, Hc0, d, rows, d * 2, spo::BK, spo::BM), "tensor map Hc");
+
+    // a6: G = inv_temp * g * (onehot - softmax), logits recomputed
+    spo::GemmArgs a = base_args(di);
+    a.m_count = r.count;
+    a.m_offset = static_cast<int>(r0);
+    a.m_cap = static_cast<int>(chunk);
+    a.n = static_cast<int>(V);
+    a.k_static = static_cast<int>(d);
+    a.scale = inv_temp;
+    a.tgt = r.tgt_c + r0;
+    if (r.by_token) {
+      a.lse = r.lse;
+      a.gvec = r.g;
+      a.vec_idx = r.idx + r0;
+    } else {
+      a.lse = r.lse + r0;
+      a.gvec = r.g + r0;
+    }
+    a.G = G;
+    a.ldG = V;
+    if ((st = traced_gemm(spo::EPI_GRAD, false, false, tH_k, tW_k, tG_store, a,
+                          grid_for(di, rows, V), s, counters)) != SPO_OK)
+      return st;
+    if ((st = dh_dw_block(di, W, d, V, G, V, rows, Hc0, r0, r.count, r.idx, dH, dH_f32, dW,
+                          c > 0 || accumulate_dW, counters, s,
+                          c == n_chunks - 1 ? hooks : nullptr)) != SPO_OK)
+      return st;
   }
   return SPO_OK;
 }
@@ -451,12 +556,12 @@ spo_status dh_dw_block(const DevInfo& di, const void* W, int64_t d, int64_t V,
 spo_status bwd_impl(const void* H, const void* W, const int32_t* tgt, const float* lse,
                     const float* g, int64_t T, int64_t d, int64_t V, int64_t v_offset,
                     float inv_temp, void* dH, bool dH_f32, float* dW, int accumulate_dW, void* ws,
-                    cudaStream_t s) {
+                    cudaStream_t s, const BwdHooks* hooks = nullptr) {
   spo_status st;
   DevInfo di;
   if ((st = device_info(&di)) != SPO_OK) return st;
   const BwdWs w = carve_bwd(ws, T, d, V);
-  if (!dH && !dW) return ok();
+  if (!dH && !dW) return (st = record_hook_events(hooks, s)) == SPO_OK ? ok() : st;
 
   // rows with g != 0 are the only ones with a non-zero gradient row
   st = traced(kTraceSelectGatherBwd, s, "compact/gather", [&] {
@@ -471,40 +576,10 @@ spo_status bwd_impl(const void* H, const void* W, const int32_t* tgt, const floa
   if (dH)
     SPO_CUDA(spo::launch_zero_skipped_rows(g, T, static_cast<int>((dH_f32 ? 4 : 2) * d), dH, s),
              "zero skipped dH rows");
-
-  CUtensorMap tW_k, tG_store;
-  SPO_CUDA(spo::make_tmap_bf16(&tW_k, W, d, V, d * 2, spo::BK, b_box_rows()), "tensor map W");
-  SPO_CUDA(spo::make_tmap_bf16(&tG_store, w.G, V, w.chunk, V * 2, 64, spo::kStoreBoxRows),
-           "tensor map G (store)");
-  const long long n_chunks = (w.T_pad + w.chunk - 1) / w.chunk;
-  for (long long c = 0; c < n_chunks; ++c) {
-    const long long r0 = c * w.chunk;
-    const long long rows = (w.T_pad - r0) < w.chunk ? (w.T_pad - r0) : w.chunk;
-    const __nv_bfloat16* Hc0 = w.Hc + r0 * d;
-    CUtensorMap tH_k;
-    SPO_CUDA(spo::make_tmap_bf16(&tH_k, Hc0, d, rows, d * 2, spo::BK, spo::BM), "tensor map Hc");
-
-    // a6: G = inv_temp * g * (onehot - softmax), logits recomputed
-    spo::GemmArgs a = base_args(di);
-    a.m_count = w.count;
-    a.m_offset = static_cast<int>(r0);
-    a.m_cap = static_cast<int>(w.chunk);
-    a.n = static_cast<int>(V);
-    a.k_static = static_cast<int>(d);
-    a.scale = inv_temp;
-    a.tgt = w.tgt_c + r0;
-    a.lse = w.lse_c + r0;
-    a.gvec = w.g_c + r0;
-    a.G = w.G;
-    a.ldG = V;
-    if ((st = traced_gemm(spo::EPI_GRAD, false, false, tH_k, tW_k, tG_store, a,
-                          grid_for(di, rows, V), s, w.counters)) != SPO_OK)
-      return st;
-    if ((st = dh_dw_block(di, W, d, V, w.G, V, rows, Hc0, r0, w.count, w.idx, dH, dH_f32, dW,
-                          c > 0 || accumulate_dW, w.counters, s)) != SPO_OK)
-      return st;
-  }
-  return ok();
+  const BwdRows rows{w.Hc, w.idx, w.count, w.tgt_c, w.lse_c, w.g_c, false, w.T_pad};
+  st = bwd_core(di, W, d, V, inv_temp, rows, w.G, w.chunk, dH, dH_f32, dW, accumulate_dW,
+                w.counters, hooks, s);
+  return st == SPO_OK ? ok() : st;
 }
 
 
@@ -533,6 +608,80 @@ spo_status check_adv_args(const float* rewards, const int32_t* group_id, int32_t
   if (std_mode != SPO_STD_UNBIASED && std_mode != SPO_STD_POPULATION)
     return fail(SPO_ERR_INVALID_ARG, "std_mode %d unknown", std_mode);
   if (!(eps >= 0.f) || !isfinite(eps)) return fail(SPO_ERR_INVALID_ARG, "eps must be finite and >= 0");
+  return SPO_OK;
+}
+
+// Workspace of spo_grpo_step: the forward's region first (its compaction,
+// gathered rows and targets serve the backward too), then the per-token and
+// per-sequence vectors the caller did not ask for, the advantage and loss
+// scratch, and one bf16 G chunk.
+struct StepWs {
+  uint8_t* loss_mask;
+  int* n_tok;
+  float* logp;
+  float* lse;
+  float* g;
+  float* adv;
+  void* adv_ws;
+  void* loss_ws;
+  __nv_bfloat16* G;
+  long long chunk;
+  size_t bytes;
+};
+
+StepWs carve_step(void* base, long long T, long long d, long long V, int n_seq, int n_groups) {
+  StepWs w{};
+  char* p = static_cast<char*>(base);
+  size_t off = carve_fwd(nullptr, T, d, V).bytes;
+  auto take = [&](size_t n) {
+    char* q = p ? p + off : nullptr;
+    off += align256(n);
+    return q;
+  };
+  const long long T_pad = round_up(T, spo::kRowPad);
+  w.loss_mask = reinterpret_cast<uint8_t*>(take(static_cast<size_t>(T)));
+  w.n_tok = reinterpret_cast<int*>(take(sizeof(int) * static_cast<size_t>(n_seq)));
+  w.logp = reinterpret_cast<float*>(take(sizeof(float) * T));
+  w.lse = reinterpret_cast<float*>(take(sizeof(float) * T));
+  w.g = reinterpret_cast<float*>(take(sizeof(float) * T));
+  w.adv = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(n_seq)));
+  w.adv_ws = take(spo::adv_ws_bytes(n_groups));
+  w.loss_ws = take(spo::loss_ws_bytes(n_seq, n_groups));
+  w.chunk = T_pad < kBwdChunkRows ? T_pad : kBwdChunkRows;
+  w.G = reinterpret_cast<__nv_bfloat16*>(take(sizeof(__nv_bfloat16) * w.chunk * V));
+  w.bytes = off;
+  return w;
+}
+
+// Public hooks -> internal form (events copied), checked against the device.
+spo_status convert_hooks(const spo_bwd_hooks* h, const DevInfo& di, BwdHooks* out,
+                         std::vector<cudaEvent_t>* events) {
+  *out = BwdHooks{};
+  if (!h) return SPO_OK;
+  if (h->n_dw_blocks < 1 || h->n_dw_blocks > 4096)
+    return fail(SPO_ERR_INVALID_ARG, "n_dw_blocks = %d outside [1, 4096]", h->n_dw_blocks);
+  if (h->reserve_sms < 0 || h->reserve_sms > di.sms - 2)
+    return fail(SPO_ERR_INVALID_ARG, "reserve_sms = %d outside [0, %d]", h->reserve_sms, di.sms - 2);
+  out->n_dw_blocks = h->n_dw_blocks;
+  out->reserve_sms = h->reserve_sms;
+  out->dh_event = static_cast<cudaEvent_t>(h->dh_event);
+  if (h->dw_block_events) {
+    events->assign(static_cast<size_t>(h->n_dw_blocks), nullptr);
+    for (int k = 0; k < h->n_dw_blocks; ++k)
+      (*events)[k] = static_cast<cudaEvent_t>(h->dw_block_events[k]);
+    out->dw_events = events->data();
+  }
+  return SPO_OK;
+}
+
+spo_status check_loss_scalars(int32_t n_seq, int32_t n_groups, int agg, float clip_eps,
+                              float kl_beta) {
+  if (n_seq < 1 || n_groups < 1 || n_seq > (1 << 24) || n_groups > (1 << 24))
+    return fail(SPO_ERR_SHAPE, "n_seq = %d, n_groups = %d out of range", n_seq, n_groups);
+  if (agg != SPO_AGG_SEQ_GROUP && agg != SPO_AGG_TOKEN)
+    return fail(SPO_ERR_INVALID_ARG, "agg %d unknown", agg);
+  if (!(clip_eps >= 0.f && clip_eps < 1.f)) return fail(SPO_ERR_INVALID_ARG, "clip_eps must be in [0, 1)");
+  if (!isfinite(kl_beta)) return fail(SPO_ERR_INVALID_ARG, "kl_beta must be finite");
   return SPO_OK;
 }
 
@@ -913,6 +1062,150 @@ SPO_API spo_status spo_policy_loss_bwd_slice(const void* H, const void* W_slice,
     return fail(SPO_ERR_SHAPE, "v_offset = %lld outside [0, 2^31)", (long long)v_offset);
   return bwd_impl(H, W_slice, tgt, lse, g, T, d, V_slice, v_offset, inv_temp, dH_part, true,
                   dW_slice, accumulate_dW, ws, static_cast<cudaStream_t>(stream));
+}
+
+SPO_API spo_status spo_last_error_detail(char* buf, size_t n) {
+  return static_cast<spo_status>(spo_last_error(buf, n));
+}
+
+SPO_API spo_status spo_sync_check(void* stream) {
+  SPO_CUDA(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)), "stream work");
+  int code = 0;
+  return spo_device_error(&code, stream);
+}
+
+SPO_API spo_status spo_scale_f32_ratio(float* x, int64_t n, const double* num, const double* den,
+                                       void* stream) {
+  if (n < 0 || n > (1ll << 40)) return fail(SPO_ERR_SHAPE, "n = %lld out of range", (long long)n);
+  if (n == 0) return ok();
+  if (!x || !num || !den) return fail(SPO_ERR_INVALID_ARG, "x, num and den must be non-NULL");
+  SPO_CUDA(spo::launch_scale_ratio(x, n, num, den, static_cast<cudaStream_t>(stream)),
+           "scale launch");
+  return ok();
+}
+
+SPO_API spo_status spo_dw_block_starts(int64_t V, int32_t n_blocks, int64_t* starts) {
+  if (!starts) return fail(SPO_ERR_INVALID_ARG, "starts must be non-NULL");
+  if (V < 1) return fail(SPO_ERR_SHAPE, "V must be positive");
+  if (n_blocks < 1 || n_blocks > 4096)
+    return fail(SPO_ERR_INVALID_ARG, "n_blocks = %d outside [1, 4096]", n_blocks);
+  for (int k = 0; k <= n_blocks; ++k) starts[k] = dw_block_start(V, n_blocks, k);
+  return ok();
+}
+
+SPO_API spo_status spo_policy_loss_bwd_ex(const void* H, const void* W, const int32_t* tgt,
+                                          const float* lse, const float* g, int64_t T, int64_t d,
+                                          int64_t V, int64_t v_offset, float inv_temp, void* dH,
+                                          int dH_fp32, float* dW, int accumulate_dW,
+                                          const spo_bwd_hooks* hooks, void* ws, size_t ws_bytes,
+                                          void* stream) {
+  spo_status st = check_bwd_args(H, W, tgt, lse, g, T, d, V, inv_temp, dH, dW, ws, ws_bytes);
+  if (st != SPO_OK) return st;
+  if (v_offset < 0 || v_offset > (1ll << 31) - 1)
+    return fail(SPO_ERR_SHAPE, "v_offset = %lld outside [0, 2^31)", (long long)v_offset);
+  DevInfo di;
+  if ((st = device_info(&di)) != SPO_OK) return st;
+  BwdHooks hk;
+  std::vector<cudaEvent_t> events;
+  if ((st = convert_hooks(hooks, di, &hk, &events)) != SPO_OK) return st;
+  return bwd_impl(H, W, tgt, lse, g, T, d, V, v_offset, inv_temp, dH, dH_fp32 != 0, dW,
+                  accumulate_dW, ws, static_cast<cudaStream_t>(stream), hooks ? &hk : nullptr);
+}
+
+SPO_API spo_status spo_grpo_workspace_size(int64_t T, int64_t d, int64_t V, int32_t n_seq,
+                                           int32_t n_groups, size_t* bytes) {
+  if (!bytes) return fail(SPO_ERR_INVALID_ARG, "bytes must be non-NULL");
+  if (T < 1 || d < 1 || V < 1 || n_seq < 1 || n_groups < 1)
+    return fail(SPO_ERR_SHAPE, "sizes must be positive");
+  *bytes = carve_step(nullptr, T, d, V, n_seq, n_groups).bytes;
+  return ok();
+}
+
+SPO_API spo_status spo_workspace_size(int64_t T, int64_t d, int64_t V, int32_t n_seq,
+                                      size_t* bytes) {
+  if (!bytes) return fail(SPO_ERR_INVALID_ARG, "bytes must be non-NULL");
+  if (T < 1 || d < 1 || V < 1 || n_seq < 1) return fail(SPO_ERR_SHAPE, "sizes must be positive");
+  size_t b = carve_step(nullptr, T, d, V, n_seq, n_seq).bytes;
+  const size_t others[4] = {carve_fwd(nullptr, T, d, V).bytes, carve_bwd(nullptr, T, d, V).bytes,
+                            spo::loss_ws_bytes(n_seq, n_seq), spo::adv_ws_bytes(n_seq)};
+  for (size_t x : others) b = x > b ? x : b;
+  *bytes = b;
+  return ok();
+}
+
+SPO_API spo_status spo_grpo_step(const spo_grpo_batch* b, const spo_grpo_params* q,
+                                 const spo_grpo_outputs* o, const spo_bwd_hooks* hooks, void* ws,
+                                 size_t ws_bytes, void* stream) {
+  if (!b || !q || !o) return fail(SPO_ERR_INVALID_ARG, "batch, params and out must be non-NULL");
+  spo_status st = check_hwv(b->H, b->W, b->tgt, b->T, b->d, b->V, q->inv_temp);
+  if (st != SPO_OK) return st;
+  if (!b->cu_seqlens || !b->group_id || !b->rewards || !b->old_logp)
+    return fail(SPO_ERR_INVALID_ARG, "cu_seqlens, group_id, rewards and old_logp must be non-NULL");
+  if (!o->loss) return fail(SPO_ERR_INVALID_ARG, "out->loss must be non-NULL");
+  if ((st = check_loss_scalars(b->n_seq, b->n_groups, q->agg, q->clip_eps, q->kl_beta)) != SPO_OK)
+    return st;
+  if (q->std_mode != SPO_STD_UNBIASED && q->std_mode != SPO_STD_POPULATION)
+    return fail(SPO_ERR_INVALID_ARG, "std_mode %d unknown", q->std_mode);
+  if (!(q->adv_eps >= 0.f) || !isfinite(q->adv_eps))
+    return fail(SPO_ERR_INVALID_ARG, "adv_eps must be finite and >= 0");
+  if (o->dH && !aligned16(o->dH)) return fail(SPO_ERR_ALIGNMENT, "dH must be 16-byte aligned");
+  if (o->dW && !aligned16(o->dW)) return fail(SPO_ERR_ALIGNMENT, "dW must be 16-byte aligned");
+  const StepWs need = carve_step(nullptr, b->T, b->d, b->V, b->n_seq, b->n_groups);
+  if (!ws || ws_bytes < need.bytes)
+    return fail(SPO_ERR_WORKSPACE, "workspace needs %zu bytes, got %zu", need.bytes, ws_bytes);
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
+    return fail(SPO_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
+  DevInfo di;
+  if ((st = device_info(&di)) != SPO_OK) return st;
+  BwdHooks hk;
+  std::vector<cudaEvent_t> events;
+  if ((st = convert_hooks(hooks, di, &hk, &events)) != SPO_OK) return st;
+
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const StepWs w = carve_step(ws, b->T, b->d, b->V, b->n_seq, b->n_groups);
+  uint8_t* lm = o->loss_mask ? o->loss_mask : w.loss_mask;
+  float* logp = o->logp ? o->logp : w.logp;
+  float* lse = o->lse ? o->lse : w.lse;
+  float* g = o->g ? o->g : w.g;
+  float* adv = o->adv ? o->adv : w.adv;
+  // a1: loss tokens
+  st = traced(kTraceTokenSelect, s, "token_select launch", [&] {
+    return spo::launch_token_select(b->cu_seqlens, b->mask, b->tgt, b->n_seq, q->window, lm,
+                                    w.n_tok, s);
+  });
+  if (st != SPO_OK) return st;
+  // a2 + a3 over the loss tokens (the forward's region of the workspace)
+  if ((st = logprobs_impl(b->H, b->W, b->tgt, lm, b->T, b->d, b->V, 0, q->inv_temp, logp,
+                          o->entropy, lse, nullptr, ws, s)) != SPO_OK)
+    return st;
+  // a4: the per-group scan at a step's few hundred sequences, else the run path (same bits)
+  const bool scan = static_cast<long long>(b->n_seq) * b->n_groups <= (1ll << 22);
+  st = traced(kTraceAdvantages, s, "advantage launch", [&] {
+    return scan ? spo::launch_group_advantages(b->rewards, b->group_id, b->n_seq, b->n_groups,
+                                               q->std_mode, q->adv_eps, adv, s)
+                : spo::launch_group_advantages_runs(b->rewards, b->group_id, b->n_seq,
+                                                    b->n_groups, q->std_mode, q->adv_eps, adv,
+                                                    w.adv_ws, s);
+  });
+  if (st != SPO_OK) return st;
+  // a5: surrogate, KL, aggregation; g = dL/dlogp (times the rank weight, if any)
+  const spo::LossWs lw = spo::carve_loss_ws(w.loss_ws, b->n_seq, b->n_groups);
+  st = traced(kTracePolicyLoss, s, "policy loss launch", [&] {
+    return spo::launch_policy_loss(logp, b->old_logp, b->ref_logp, adv, b->cu_seqlens,
+                                   b->group_id, b->n_seq, b->n_groups, lm, b->T, q->clip_eps,
+                                   q->kl_beta, q->agg, o->loss, g, o->stats, lw, s, q->loss_scale);
+  });
+  if (st != SPO_OK) return st;
+  // a6 - a8 over the forward's compaction (loss tokens); lse and g read at token positions
+  if (!o->dH && !o->dW) return (st = record_hook_events(hooks ? &hk : nullptr, s)) == SPO_OK ? ok() : st;
+  const FwdWs f = carve_fwd(ws, b->T, b->d, b->V);
+  if (o->dH)
+    SPO_CUDA(spo::launch_zero_skipped_rows(g, b->T, static_cast<int>(2 * b->d), o->dH, s),
+             "zero skipped dH rows");
+  const BwdRows rows{f.Hc, f.idx, f.count, f.tgt_c, lse, g, true, f.T_pad};
+  st = bwd_core(di, b->W, b->d, b->V, q->inv_temp, rows, w.G, w.chunk, o->dH, false, o->dW,
+                o->accumulate_dW, f.counters, hooks ? &hk : nullptr, s);
+  return st == SPO_OK ? ok() : st;
 }
 
 SPO_API spo_status spo_trace_enable(int on) {

@@ -204,8 +204,9 @@ __device__ __forceinline__ void epi_grad_tma(const GemmArgs& p, const CUtensorMa
                                              int row, int row0, int M, int nb, uint8_t* slots,
                                              int& slab, int lane) {
   const bool row_ok = row < M;
-  const float gl = row_ok ? p.gvec[row] : 0.f;
-  const float l2 = row_ok ? p.lse[row] * kLog2e : 0.f;
+  const int vrow = row_ok && p.vec_idx ? p.vec_idx[row] : row;
+  const float gl = row_ok ? p.gvec[vrow] : 0.f;
+  const float l2 = row_ok ? p.lse[vrow] * kLog2e : 0.f;
   const int y = row_ok ? p.tgt[row] : -1;
   const float coef = p.scale * gl;
   const float sc2 = p.scale * kLog2e;

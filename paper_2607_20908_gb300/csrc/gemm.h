@@ -68,6 +68,9 @@ struct GemmArgs {
   // EPI_GRAD
   const float* lse;   // natural-log lse of each row
   const float* gvec;  // dL/dlogp of each row
+  // NULL: lse and gvec are indexed by row; else by vec_idx[row] (token
+  // positions of the compacted rows, so the vectors need no gather)
+  const int* vec_idx;
   __nv_bfloat16* G;   // [rows][ldG]
   long long ldG;
   // EPI_DH: rows scattered to row_idx[row], bf16 to out_bf16 or, when out_f32

@@ -87,6 +87,9 @@ cudaError_t launch_ranker_pair_loss(const float* phi, const float* mu, const flo
                                     float* ws, cudaStream_t s);
 
 // x[i] *= alpha (alpha read from device memory when alpha_dev != NULL).
+// launch_scale_ratio: x[i] *= num[0] / den[0] (fp64 device scalars; 0 when den is 0).
+cudaError_t launch_scale_ratio(float* x, long long n, const double* num, const double* den,
+                               cudaStream_t s);
 cudaError_t launch_scale(float* x, long long n, float alpha, const float* alpha_dev, cudaStream_t s);
 
 // Zeroes row t of out (row_bytes per row, a multiple of 16; out 16-byte aligned)
@@ -115,6 +118,7 @@ cudaError_t launch_policy_loss(const float* logp, const float* old_logp, const f
                                const float* adv, const int* cu_seqlens, const int* group_id,
                                int n_seq, int n_groups, const uint8_t* loss_mask, long long T,
                                float clip_eps, float kl_beta, int agg, float* loss, float* g,
-                               float* stats, const LossWs& w, cudaStream_t s);
+                               float* stats, const LossWs& w, cudaStream_t s,
+                               const float* cscale = nullptr);
 
 }  // namespace spo

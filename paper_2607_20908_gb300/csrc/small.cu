@@ -701,6 +701,16 @@ __global__ void reward_kernel_x4(const uchar4* compiled, const float4* pass_rate
   }
 }
 
+// x *= num / den (counts in fp64; 0 when den is 0): a data-parallel rank's
+// weight in the global average, taken from all-reduced counts on the device.
+__global__ void scale_ratio_kernel(float* x, long long n, const double* num, const double* den) {
+  const double dd = *den;
+  const float a = dd != 0.0 ? static_cast<float>(*num / dd) : 0.f;
+  for (long long i = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; i < n;
+       i += static_cast<long long>(gridDim.x) * blockDim.x)
+    x[i] *= a;
+}
+
 __global__ void scale_kernel(float* x, long long n, float alpha, const float* alpha_dev) {
   const float a = alpha_dev ? *alpha_dev : alpha;
   for (long long i = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; i < n;
@@ -886,8 +896,8 @@ template <int LPS>
 __global__ void __launch_bounds__(kLossThreads) loss_token_kernel(
     const float* logp, const float* old_logp, const float* ref_logp, const float* adv,
     const int* cu, const int* gid, int n_seq, int n_groups, const uint8_t* lm, float clip_eps,
-    float kl_beta, int agg, const int* gsize, const unsigned long long* scal, float* g,
-    float2* part_l, float2* part_rk, int* part_clip, int* n_tok) {
+    float kl_beta, int agg, const int* gsize, const unsigned long long* scal, const float* cscale,
+    float* g, float2* part_l, float2* part_rk, int* part_clip, int* n_tok) {
   constexpr int kTpl = 8;            // tokens a lane has in flight in one pass
   constexpr int kStep = kTpl * LPS;  // tokens of one pass of the group
   const int lane = threadIdx.x & 31;
@@ -944,6 +954,7 @@ __global__ void __launch_bounds__(kLossThreads) loss_token_kernel(
       c = ni > 0 && ng > 0.f && gs > 0
               ? __frcp_rn(ng * static_cast<float>(gs) * static_cast<float>(ni))
               : 0.f;
+    if (cscale) c *= *cscale;  // a data-parallel rank's share of the global average
     LossTok k{1.f - clip_eps, 1.f + clip_eps, A, c, kl_beta, use_kl};
 #pragma unroll
     for (int u = 0; u < kTpl; ++u) {
@@ -1267,6 +1278,16 @@ cudaError_t launch_scale(float* x, long long n, float alpha, const float* alpha_
   return cudaGetLastError();
 }
 
+cudaError_t launch_scale_ratio(float* x, long long n, const double* num, const double* den,
+                               cudaStream_t s) {
+  const int sms = sm_count();
+  const long long want = (n + 255) / 256;
+  const int blocks = static_cast<int>(want < sms * 8 ? (want < 1 ? 1 : want) : sms * 8);
+  scale_ratio_kernel<<<blocks, 256, 0, s>>>(x, n, num, den);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_zero_skipped_rows(const float* g, long long T, int row_bytes, void* out,
                                      cudaStream_t s) {
   const int sms = sm_count();
@@ -1322,7 +1343,8 @@ cudaError_t launch_policy_loss(const float* logp, const float* old_logp, const f
                                const float* adv, const int* cu_seqlens, const int* group_id,
                                int n_seq, int n_groups, const uint8_t* loss_mask, long long T,
                                float clip_eps, float kl_beta, int agg, float* loss, float* g,
-                               float* stats, const LossWs& w, cudaStream_t s) {
+                               float* stats, const LossWs& w, cudaStream_t s,
+                               const float* cscale) {
   // scal (groups, tokens, ticket) and gsize are adjacent: one clear
   cudaError_t e = cudaMemsetAsync(w.scal, 0,
                                   reinterpret_cast<char*>(w.gsize + n_groups) -
@@ -1354,11 +1376,11 @@ cudaError_t launch_policy_loss(const float* logp, const float* old_logp, const f
   if (short_seqs)
     loss_token_kernel<16><<<seq_blocks, kLossThreads, 0, s>>>(
         logp, old_logp, ref_logp, adv, cu_seqlens, group_id, n_seq, n_groups, loss_mask, clip_eps,
-        kl_beta, agg, w.gsize, w.scal, g, w.part_l, w.part_rk, w.part_clip, w.n_tok);
+        kl_beta, agg, w.gsize, w.scal, cscale, g, w.part_l, w.part_rk, w.part_clip, w.n_tok);
   else
     loss_token_kernel<32><<<seq_blocks, kLossThreads, 0, s>>>(
         logp, old_logp, ref_logp, adv, cu_seqlens, group_id, n_seq, n_groups, loss_mask, clip_eps,
-        kl_beta, agg, w.gsize, w.scal, g, w.part_l, w.part_rk, w.part_clip, w.n_tok);
+        kl_beta, agg, w.gsize, w.scal, cscale, g, w.part_l, w.part_rk, w.part_clip, w.n_tok);
   const int chunk = max(256, (n_seq + kLossFinalMaxBlocks - 1) / kLossFinalMaxBlocks);
   const int nb = (n_seq + chunk - 1) / chunk;
   loss_final_kernel<<<nb, kLossThreads, 0, s>>>(w.part_l, w.part_rk, w.part_clip, w.n_tok, n_seq,

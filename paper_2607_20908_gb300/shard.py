@@ -82,6 +82,14 @@ def rank_batch(cu_seqlens, group_id, groups) -> RankBatch:
     return RankBatch(seqs, tok, local_cu, local_gid, len(remap))
 
 
+def dw_block_starts(V: int, n_blocks: int):
+    """Row boundaries of dW's vocabulary blocks (libspo's layout: multiples of
+    256, the last block ends at V).  Every rank uses the same layout, so the
+    per-block collectives match across ranks.  A host computation."""
+    from paper_2607_20908_gb300 import spo
+    return spo.dw_block_starts(V, n_blocks)
+
+
 def loss_weight(agg: int, local_groups: float, global_groups: float, local_tokens: float,
                 global_tokens: float) -> float:
     """Weight of a rank's local loss (and dL/dlogp) in the global objective."""
@@ -93,9 +101,11 @@ def loss_weight(agg: int, local_groups: float, global_groups: float, local_token
 class SpoEngine:
     """libspo (CUDA) as the per-rank compute of a data-parallel step."""
 
-    def __init__(self):
+    def __init__(self, reserve_sms: int = 0):
         from paper_2607_20908_gb300 import spo
         self.spo = spo
+        self.reserve_sms = reserve_sms
+        self._side = {}
 
     def step_local(self, b: dict, agg: int):
         s = self.spo
@@ -107,15 +117,70 @@ class SpoEngine:
                                                b["kl_beta"], agg)
         return dict(loss=loss, g=g, lse=lse, n_loss_tokens=stats[3:4].to(torch.float64))
 
-    def scale(self, x, w: float):
-        self.spo.spo_scale_f32(x, alpha=w)
+    def local_counts(self, b: dict, loc):
+        """[groups owned, loss tokens] as a device fp64 tensor (no host read)."""
+        groups = torch.full((1,), float(b["n_groups"]), dtype=torch.float64,
+                            device=loc["n_loss_tokens"].device)
+        return torch.cat([groups, loc["n_loss_tokens"].reshape(1)])
+
+    def zero_counts(self, b: dict):
+        return torch.zeros(2, dtype=torch.float64, device=b["W"].device)
+
+    def scale_ratio(self, x, num, den):
+        self.spo.spo_scale_f32_ratio(x, num, den)
         return x
 
-    def backward(self, b: dict, lse, g):
-        return self.spo.spo_policy_loss_bwd(b["H"], b["W"], b["tgt"], lse, g, b["inv_temp"])
+    def backward_blocks(self, b: dict, lse, g, n_blocks: int):
+        """dH, dW and dW's vocabulary blocks [(first row, end row, event when final)]."""
+        s = self.spo
+        evs = [torch.cuda.Event() for _ in range(n_blocks)]
+        hooks = s.make_hooks(n_blocks, evs, None, reserve_sms=self.reserve_sms)
+        dH, dW = s.spo_policy_loss_bwd_ex(b["H"], b["W"], b["tgt"], lse, g, b["inv_temp"],
+                                          hooks=hooks)
+        starts = dw_block_starts(b["W"].shape[0], n_blocks)
+        return dH, dW, [(starts[k], starts[k + 1], evs[k]) for k in range(n_blocks)]
+
+    def step_fused(self, b: dict, weight: float, n_blocks: int):
+        """The whole local step in one call (spo_grpo_step) with the loss and g
+        scaled by `weight` on the device: (loss, dH, dW, dW blocks)."""
+        s = self.spo
+        dev = b["W"].device
+        scale = torch.full((1,), float(weight), dtype=torch.float32, device=dev)
+        evs = [torch.cuda.Event() for _ in range(n_blocks)]
+        hooks = s.make_hooks(n_blocks, evs, None, reserve_sms=self.reserve_sms)
+        out = s.spo_grpo_step(b["H"], b["W"], b["tgt"], b["mask"], b["cu_seqlens"],
+                              b["group_id"], b["n_groups"], b["rewards"], b["old"], b["ref"],
+                              inv_temp=b["inv_temp"], window=b["window"], clip_eps=b["clip_eps"],
+                              kl_beta=b["kl_beta"], agg=AGG_SEQ_GROUP, loss_scale=scale, want=(),
+                              hooks=hooks, dH=b.get("dH_out"), dW=b.get("dW_out"))
+        starts = dw_block_starts(b["W"].shape[0], n_blocks)
+        return (out["loss"], out["dH"], out["dW"],
+                [(starts[k], starts[k + 1], evs[k]) for k in range(n_blocks)])
 
     def zeros_dW(self, V: int, d: int, like):
         return torch.zeros((V, d), dtype=torch.float32, device=like.device)
+
+    def comm_stream(self, t):
+        """Side stream on t's device for the collectives that overlap the GEMMs."""
+        dev = t.device
+        if dev not in self._side:
+            self._side[dev] = torch.cuda.Stream(dev)
+        return self._side[dev]
+
+
+def _overlapped_all_reduce(t, ready, side, group):
+    """Sum-all-reduce of t issued once `ready` (a CUDA event, or None: now)
+    has fired, from the side stream when there is one, so that it runs while
+    the launching stream goes on.  Returns the async work handle."""
+    import torch.distributed as dist
+    if side is None:
+        return dist.all_reduce(t, group=group, async_op=True)
+    if ready is not None:
+        side.wait_event(ready)
+    else:
+        side.wait_stream(torch.cuda.current_stream(t.device))
+    with torch.cuda.stream(side):
+        return dist.all_reduce(t, group=group, async_op=True)
 
 
 class DataParallelStep:
@@ -124,14 +189,18 @@ class DataParallelStep:
     run(b) takes this rank's batch (dict with H, W, tgt, mask, cu_seqlens,
     group_id, n_groups, rewards, old, ref, window, inv_temp, clip_eps,
     kl_beta; n_groups may be 0) and returns (global loss, local dH, global dW).
-    Collectives: one all-reduce of [groups, loss tokens], one of the loss,
-    one of dW.
+    Collectives: one all-reduce of [groups, loss tokens] whose result is used
+    on the device (the rank's weight is applied by a kernel: the host never
+    reads a count), one of the loss, and one per vocabulary block of dW, each
+    started as soon as the backward has finished that block, so it runs
+    while the GEMMs of the later blocks do.
     """
 
-    def __init__(self, engine, agg: int = AGG_SEQ_GROUP, process_group=None):
+    def __init__(self, engine, agg: int = AGG_SEQ_GROUP, process_group=None, dw_blocks: int = 4):
         self.engine = engine
         self.agg = agg
         self.pg = process_group
+        self.dw_blocks = dw_blocks
 
     def run(self, b: dict):
         import torch.distributed as dist
@@ -139,27 +208,59 @@ class DataParallelStep:
         V, d = b["W"].shape
         if b["n_groups"] > 0:
             loc = e.step_local(b, self.agg)
-            counts = torch.cat([torch.tensor([float(b["n_groups"])], dtype=torch.float64,
-                                             device=loc["n_loss_tokens"].device),
-                                loc["n_loss_tokens"].reshape(1)])
+            local = e.local_counts(b, loc)
         else:
             loc = None
-            counts = torch.zeros(2, dtype=torch.float64, device=b["W"].device)
-        local = counts.clone()
-        dist.all_reduce(counts, group=self.pg)
-        w = loss_weight(self.agg, float(local[0]), float(counts[0]), float(local[1]),
-                        float(counts[1]))
+            local = e.zero_counts(b)
+        total = local.clone()
+        dist.all_reduce(total, group=self.pg)
+        k = 0 if self.agg == AGG_SEQ_GROUP else 1
         if loc is not None:
-            e.scale(loc["g"], w)
-            e.scale(loc["loss"], w)
-            dH, dW = e.backward(b, loc["lse"], loc["g"])
+            # weight of this rank's local average in the global one (Eq. 3)
+            e.scale_ratio(loc["g"], local[k:k + 1], total[k:k + 1])
+            e.scale_ratio(loc["loss"], local[k:k + 1], total[k:k + 1])
+            dH, dW, blocks = e.backward_blocks(b, loc["lse"], loc["g"], self.dw_blocks)
             loss = loc["loss"]
         else:
             dH = None
             dW = e.zeros_dW(V, d, b["W"])
             loss = torch.zeros(1, dtype=dW.dtype, device=dW.device)
+            starts = dw_block_starts(V, self.dw_blocks)
+            blocks = [(starts[k], starts[k + 1], None) for k in range(self.dw_blocks)]
+        return self._exchange(loss, dH, dW, blocks)
+
+    def run_fused(self, b: dict, global_groups: int):
+        """The same step for SEQ_GROUP aggregation when every rank knows the
+        global number of non-empty groups on the host (each rank owns whole,
+        non-empty groups of a sharding plan all ranks share): the rank's
+        weight N_r / N is then known before the step, so the local step runs
+        as one call (spo_grpo_step) with that weight applied on the device,
+        and no count is exchanged.  Collectives: dW per vocabulary block as
+        in run(), and the loss."""
+        if self.agg != AGG_SEQ_GROUP:
+            raise ValueError("run_fused needs SEQ_GROUP aggregation (TOKEN weights need the "
+                             "all-reduced token count)")
+        e = self.engine
+        V, d = b["W"].shape
+        starts = dw_block_starts(V, self.dw_blocks)
+        if b["n_groups"] > 0:
+            weight = b["n_groups"] / global_groups if global_groups > 0 else 0.0
+            loss, dH, dW, blocks = e.step_fused(b, weight, self.dw_blocks)
+        else:
+            dH = None
+            dW = e.zeros_dW(V, d, b["W"])
+            loss = torch.zeros(1, dtype=dW.dtype, device=dW.device)
+            blocks = [(starts[k], starts[k + 1], None) for k in range(self.dw_blocks)]
+        return self._exchange(loss, dH, dW, blocks)
+
+    def _exchange(self, loss, dH, dW, blocks):
+        import torch.distributed as dist
+        side = self.engine.comm_stream(dW)
+        works = [_overlapped_all_reduce(dW[r0:r1], ready, side, self.pg)
+                 for r0, r1, ready in blocks if r1 > r0]
         dist.all_reduce(loss, group=self.pg)
-        dist.all_reduce(dW, group=self.pg)
+        for w in works:
+            w.wait()          # the launching stream waits for the block sums
         return loss, dH, dW
 
 
@@ -186,9 +287,11 @@ def vocab_slices(V: int, world: int, align: int = 8):
 class SpoVocabEngine:
     """libspo (CUDA) as the per-rank compute of a vocabulary-parallel step."""
 
-    def __init__(self):
+    def __init__(self, reserve_sms: int = 0):
         from paper_2607_20908_gb300 import spo
         self.spo = spo
+        self.reserve_sms = reserve_sms
+        self._side = {}
 
     def forward_slice(self, b: dict):
         s = self.spo
@@ -209,8 +312,19 @@ class SpoVocabEngine:
         return loss, g
 
     def backward_slice(self, b: dict, lse, g):
-        return self.spo.spo_policy_loss_bwd_slice(b["H"], b["W_slice"], b["v_offset"], b["tgt"],
-                                                  lse, g, b["inv_temp"])
+        """(fp32 dH part, dW rows of the slice, event recorded once dH is final)."""
+        s = self.spo
+        ev = torch.cuda.Event()
+        hooks = s.make_hooks(1, None, ev, reserve_sms=self.reserve_sms)
+        dH, dW = s.spo_policy_loss_bwd_ex(b["H"], b["W_slice"], b["tgt"], lse, g, b["inv_temp"],
+                                          v_offset=b["v_offset"], dH_fp32=True, hooks=hooks)
+        return dH, dW, ev
+
+    def comm_stream(self, t):
+        dev = t.device
+        if dev not in self._side:
+            self._side[dev] = torch.cuda.Stream(dev)
+        return self._side[dev]
 
 
 class VocabParallelStep:
@@ -221,8 +335,9 @@ class VocabParallelStep:
     inv_temp, clip_eps, kl_beta -- plus W_slice and v_offset of this rank's
     rows) and returns (loss, logp, dH, dW_slice): loss, logp and dH are the
     same on every rank, dW_slice holds the gradient of this rank's rows.
-    Collectives: one all-gather of the per-token records, one all-reduce of
-    dH.
+    Collectives: one all-gather of the per-token records, and one all-reduce
+    of dH, started as soon as the backward's dH GEMM has finished so that it
+    runs while the rank's dW GEMMs do.
     """
 
     def __init__(self, engine, agg: int = AGG_SEQ_GROUP, process_group=None):
@@ -239,6 +354,7 @@ class VocabParallelStep:
         dist.all_gather(parts, rec.contiguous(), group=self.pg)
         logp, _, lse = e.merge(torch.stack(parts))
         loss, g = e.loss(b, lm, logp, self.agg)
-        dH, dW = e.backward_slice(b, lse, g)
-        dist.all_reduce(dH, group=self.pg)
+        dH, dW, dh_ready = e.backward_slice(b, lse, g)
+        work = _overlapped_all_reduce(dH, dh_ready, e.comm_stream(dH), self.pg)
+        work.wait()
         return loss, logp, dH, dW

@@ -77,6 +77,17 @@ _SIGS = {
     "spo_logprobs_merge_slices": ([_vp, _i32, _i64, _vp, _vp, _vp, _vp], ctypes.c_int),
     "spo_policy_loss_bwd_slice": ([_vp, _vp, _vp, _vp, _vp, _i64, _i64, _i64, _i64, _f32, _vp,
                                    _vp, ctypes.c_int, _vp, _c_size, _vp], ctypes.c_int),
+    "spo_last_error_detail": ([ctypes.c_char_p, _c_size], ctypes.c_int),
+    "spo_sync_check": ([_vp], ctypes.c_int),
+    "spo_scale_f32_ratio": ([_vp, _i64, _vp, _vp, _vp], ctypes.c_int),
+    "spo_dw_block_starts": ([_i64, _i32, ctypes.POINTER(_i64)], ctypes.c_int),
+    "spo_policy_loss_bwd_ex": ([_vp, _vp, _vp, _vp, _vp, _i64, _i64, _i64, _i64, _f32, _vp,
+                                ctypes.c_int, _vp, ctypes.c_int, _vp, _vp, _c_size, _vp],
+                               ctypes.c_int),
+    "spo_grpo_workspace_size": ([_i64, _i64, _i64, _i32, _i32, ctypes.POINTER(_c_size)],
+                                ctypes.c_int),
+    "spo_grpo_step": ([_vp, _vp, _vp, _vp, _vp, _c_size, _vp], ctypes.c_int),
+    "spo_workspace_size": ([_i64, _i64, _i64, _i32, ctypes.POINTER(_c_size)], ctypes.c_int),
 }
 
 TRACE_KINDS = {0: "logits_lse_fwd", 1: "logits_grad_recompute", 2: "gemm_dH", 3: "gemm_dW",
@@ -431,6 +442,173 @@ def spo_policy_loss_bwd_slice(H, W_slice, v_offset: int, tgt, lse, g, inv_temp: 
                                            _ptr(dW_slice), int(bool(accumulate_dW)), _ptr(w),
                                            w.numel(), _stream(dev)))
     return dH_part, dW_slice
+
+
+class BwdHooks(ctypes.Structure):
+    """spo_bwd_hooks: dW in vocabulary blocks with an event per finished block."""
+    _fields_ = [("n_dw_blocks", _i32), ("reserve_sms", _i32), ("dw_block_events", _vp),
+                ("dh_event", _vp)]
+
+
+def _event_handle(ev) -> int:
+    """The cudaEvent_t of a torch.cuda.Event (created by recording it once)."""
+    if ev.cuda_event == 0:
+        ev.record()
+    return int(ev.cuda_event)
+
+
+def make_hooks(n_dw_blocks: int = 1, dw_events=None, dh_event=None, reserve_sms: int = 0):
+    """A spo_bwd_hooks for the C call; keep the returned object alive until the call returns."""
+    h = BwdHooks()
+    h.n_dw_blocks = int(n_dw_blocks)
+    h.reserve_sms = int(reserve_sms)
+    # the events must outlive the call that records them: the hooks hold them
+    h._events = (list(dw_events) if dw_events is not None else [], dh_event)
+    if dw_events is not None:
+        if len(dw_events) != n_dw_blocks:
+            raise ValueError("one event per dW block")
+        arr = (_vp * n_dw_blocks)(*[_event_handle(e) if e is not None else None for e in dw_events])
+        h._arr = arr
+        h.dw_block_events = ctypes.cast(arr, _vp)
+    h.dh_event = _event_handle(dh_event) if dh_event is not None else None
+    return h
+
+
+def dw_block_starts(V: int, n_blocks: int):
+    """First dW row of each of n_blocks vocabulary blocks, plus V (host computation)."""
+    out = (_i64 * (n_blocks + 1))()
+    _check(lib().spo_dw_block_starts(int(V), int(n_blocks), out))
+    return [int(x) for x in out]
+
+
+def spo_policy_loss_bwd_ex(H, W, tgt, lse, g, inv_temp: float = 1.0, v_offset: int = 0,
+                           dH=None, dW=None, dH_fp32: bool = False, accumulate_dW: bool = False,
+                           hooks=None, want_dH=True, want_dW=True, ws=None):
+    """a6-a8 with hooks: returns (dH, dW).  With v_offset / dH_fp32 the vocabulary-slice form."""
+    dev = H.device
+    T, d = H.shape
+    V = W.shape[0]
+    _need(H, "H", torch.bfloat16, device=dev)
+    _need(W, "W", torch.bfloat16, device=dev)
+    _need(tgt, "tgt", torch.int32, T, dev)
+    _need(lse, "lse", torch.float32, T, dev)
+    _need(g, "g", torch.float32, T, dev)
+    dh_type = torch.float32 if dH_fp32 else torch.bfloat16
+    if want_dH and dH is None:
+        dH = torch.empty((T, d), dtype=dh_type, device=dev)
+    if want_dW and dW is None:
+        dW = (torch.zeros if accumulate_dW else torch.empty)((V, d), dtype=torch.float32,
+                                                             device=dev)
+    if dH is not None:
+        _need(dH, "dH", dh_type, T * d, dev)
+    if dW is not None:
+        _need(dW, "dW", torch.float32, V * d, dev)
+    w = _workspace(policy_loss_bwd_workspace_size(T, d, V), dev, ws)
+    _check(lib().spo_policy_loss_bwd_ex(_ptr(H), _ptr(W), _ptr(tgt), _ptr(lse), _ptr(g), T, d, V,
+                                        int(v_offset), float(inv_temp), _ptr(dH), int(bool(dH_fp32)),
+                                        _ptr(dW), int(bool(accumulate_dW)),
+                                        None if hooks is None else ctypes.byref(hooks), _ptr(w),
+                                        w.numel(), _stream(dev)))
+    return dH, dW
+
+
+class GrpoBatch(ctypes.Structure):
+    _fields_ = [("H", _vp), ("W", _vp), ("tgt", _vp), ("mask", _vp), ("cu_seqlens", _vp),
+                ("group_id", _vp), ("rewards", _vp), ("old_logp", _vp), ("ref_logp", _vp),
+                ("T", _i64), ("d", _i64), ("V", _i64), ("n_seq", _i32), ("n_groups", _i32)]
+
+
+class GrpoParams(ctypes.Structure):
+    _fields_ = [("inv_temp", _f32), ("window", _i32), ("clip_eps", _f32), ("kl_beta", _f32),
+                ("agg", _i32), ("std_mode", _i32), ("adv_eps", _f32), ("loss_scale", _vp)]
+
+
+class GrpoOutputs(ctypes.Structure):
+    _fields_ = [("loss", _vp), ("stats", _vp), ("logp", _vp), ("entropy", _vp), ("lse", _vp),
+                ("g", _vp), ("adv", _vp), ("loss_mask", _vp), ("dH", _vp), ("dW", _vp),
+                ("accumulate_dW", _i32)]
+
+
+def grpo_workspace_size(T: int, d: int, V: int, n_seq: int, n_groups: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().spo_grpo_workspace_size(T, d, V, n_seq, n_groups, ctypes.byref(n)))
+    return n.value
+
+
+def workspace_size(T: int, d: int, V: int, n_seq: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().spo_workspace_size(T, d, V, n_seq, ctypes.byref(n)))
+    return n.value
+
+
+def spo_grpo_step(H, W, tgt, mask, cu_seqlens, group_id, n_groups: int, rewards, old_logp,
+                  ref_logp=None, inv_temp: float = 1.0, window: int = 1024, clip_eps: float = 0.2,
+                  kl_beta: float = 0.0, agg: int = SPO_AGG_SEQ_GROUP,
+                  std_mode: int = SPO_STD_UNBIASED, adv_eps: float = 1e-6, loss_scale=None,
+                  want=("logp", "entropy", "lse", "g", "adv", "loss_mask", "stats"),
+                  want_dH=True, want_dW=True, dH=None, dW=None, accumulate_dW=False, hooks=None,
+                  ws=None):
+    """The whole step a1 -> a8 in one call.  Returns a dict of the outputs
+    asked for (loss always; dH, dW unless switched off)."""
+    dev = H.device
+    T, d = H.shape
+    V = W.shape[0]
+    n_seq = cu_seqlens.numel() - 1
+    _need(H, "H", torch.bfloat16, device=dev)
+    _need(W, "W", torch.bfloat16, device=dev)
+    _need(tgt, "tgt", torch.int32, T, dev)
+    if mask is not None:
+        _need(mask, "mask", torch.uint8, T, dev)
+    _need(cu_seqlens, "cu_seqlens", torch.int32, n_seq + 1, dev)
+    _need(group_id, "group_id", torch.int32, n_seq, dev)
+    _need(rewards, "rewards", torch.float32, n_seq, dev)
+    _need(old_logp, "old_logp", torch.float32, T, dev)
+    if ref_logp is not None:
+        _need(ref_logp, "ref_logp", torch.float32, T, dev)
+    if loss_scale is not None:
+        _need(loss_scale, "loss_scale", torch.float32, 1, dev)
+    f32 = dict(dtype=torch.float32, device=dev)
+    out = {"loss": torch.empty(1, **f32)}
+    shapes = {"stats": (4, torch.float32), "logp": (T, torch.float32),
+              "entropy": (T, torch.float32), "lse": (T, torch.float32), "g": (T, torch.float32),
+              "adv": (n_seq, torch.float32), "loss_mask": (T, torch.uint8)}
+    for k in want:
+        n, dt = shapes[k]
+        out[k] = torch.empty(n, dtype=dt, device=dev)
+    if want_dH:
+        out["dH"] = dH if dH is not None else torch.empty((T, d), dtype=torch.bfloat16, device=dev)
+        _need(out["dH"], "dH", torch.bfloat16, T * d, dev)
+    if want_dW:
+        out["dW"] = dW if dW is not None else (torch.zeros if accumulate_dW else torch.empty)(
+            (V, d), **f32)
+        _need(out["dW"], "dW", torch.float32, V * d, dev)
+    b = GrpoBatch(_ptr(H), _ptr(W), _ptr(tgt), _ptr(mask), _ptr(cu_seqlens), _ptr(group_id),
+                  _ptr(rewards), _ptr(old_logp), _ptr(ref_logp), T, d, V, n_seq, int(n_groups))
+    q = GrpoParams(float(inv_temp), int(window), float(clip_eps), float(kl_beta), int(agg),
+                   int(std_mode), float(adv_eps), _ptr(loss_scale))
+    o = GrpoOutputs(*[_ptr(out.get(k)) for k in ("loss", "stats", "logp", "entropy", "lse", "g",
+                                                  "adv", "loss_mask", "dH", "dW")],
+                    int(bool(accumulate_dW)))
+    w = _workspace(grpo_workspace_size(T, d, V, n_seq, int(n_groups)), dev, ws)
+    _check(lib().spo_grpo_step(ctypes.byref(b), ctypes.byref(q), ctypes.byref(o),
+                               None if hooks is None else ctypes.byref(hooks), _ptr(w), w.numel(),
+                               _stream(dev)))
+    return out
+
+
+def spo_sync_check(device=None) -> int:
+    """Synchronises the current stream; the status (0, SPO_ERR_TIMEOUT or SPO_ERR_CUDA)."""
+    device = torch.device(device or torch.cuda.current_device())
+    return int(lib().spo_sync_check(_stream(device)))
+
+
+def spo_scale_f32_ratio(x, num, den):
+    """In place x *= num[0] / den[0] (device fp64 scalars; 0 when den[0] is 0)."""
+    _need(x, "x", torch.float32, device=x.device)
+    _need(num, "num", torch.float64, 1, x.device)
+    _need(den, "den", torch.float64, 1, x.device)
+    _check(lib().spo_scale_f32_ratio(_ptr(x), x.numel(), _ptr(num), _ptr(den), _stream(x.device)))
+    return x
 
 
 def spo_selftest_bounded_wait(device=None):

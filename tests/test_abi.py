@@ -159,3 +159,70 @@ def test_kept_form_host_validation(lib):
     assert bk(nul, p, p, 256, 256, 4096, 1.0, p, 1 << 30, p, ok_ws, p, p, 0, nul) == 1
     assert bk(p, p, p, 256, 100, 4096, 1.0, p, 1 << 30, p, ok_ws, p, p, 0, nul) == 2
     assert bk(p, p, p, 256, 256, 4096, 1.0, p, 1 << 30, p, 64, p, p, 0, nul) == 4            # fwd ws
+
+
+def test_boundary_names_and_step_sizes(lib):
+    """The boundary's named entry points: the error text under both names,
+    one workspace size for a whole step, and the dW block layout (host only)."""
+    from paper_2607_20908_gb300 import spo
+    nul = ctypes.c_void_p(0)
+    assert lib.spo_grpo_step(nul, nul, nul, nul, nul, 0, nul) == 1
+    b1 = ctypes.create_string_buffer(256)
+    b2 = ctypes.create_string_buffer(256)
+    assert lib.spo_last_error(b1, 256) == 1 and lib.spo_last_error_detail(b2, 256) == 1
+    assert b1.value == b2.value and b"non-NULL" in b1.value
+    T, d, V, n_seq = 16384, 5120, 151936, 128
+    step = spo.grpo_workspace_size(T, d, V, n_seq, 16)
+    one = spo.workspace_size(T, d, V, n_seq)
+    assert one >= step >= spo.logprobs_workspace_size(T, d, V) + T * V * 2
+    for part in (spo.logprobs_workspace_size(T, d, V), spo.policy_loss_bwd_workspace_size(T, d, V),
+                 spo.policy_loss_workspace_size(n_seq, n_seq),
+                 spo.group_advantages_workspace_size(n_seq, n_seq),
+                 spo.grpo_workspace_size(T, d, V, n_seq, n_seq)):
+        assert one >= part
+    starts = spo.dw_block_starts(V, 4)
+    assert starts == [0, 37888, 75776, 113920, V]
+    assert spo.dw_block_starts(V, 1) == [0, V]
+    small = spo.dw_block_starts(256, 4)                 # blocks may be empty
+    assert small[0] == 0 and small[-1] == 256 and all(x % 256 == 0 for x in small[:-1])
+    out = (ctypes.c_int64 * 2)()
+    assert lib.spo_dw_block_starts(V, 0, out) == 1
+
+
+def test_step_and_hooks_host_validation(lib):
+    from paper_2607_20908_gb300 import spo
+    p = ctypes.c_void_p(4096)
+    nul = ctypes.c_void_p(0)
+    T, d, V, n_seq, n_groups = 64, 128, 1024, 8, 2
+    b = spo.GrpoBatch(p, p, p, nul, p, p, p, p, nul, T, d, V, n_seq, n_groups)
+    q = spo.GrpoParams(1.0, 1024, 0.2, 0.04, 0, 0, 1e-6, nul)
+    o = spo.GrpoOutputs(p, nul, nul, nul, nul, nul, nul, nul, nul, nul, 0)
+    need = spo.grpo_workspace_size(T, d, V, n_seq, n_groups)
+    R = ctypes.byref
+    f = lib.spo_grpo_step
+    assert f(R(b), R(q), R(o), nul, p, need - 1, nul) == 4
+    assert f(R(b), R(q), R(o), nul, ctypes.c_void_p(4368), need, nul) == 3
+    o.loss = None
+    assert f(R(b), R(q), R(o), nul, p, need, nul) == 1 and "loss" in _err(lib)[1]
+    o.loss = p
+    for field, bad, code in (("agg", 3, 1), ("std_mode", 2, 1), ("clip_eps", 1.0, 1),
+                             ("adv_eps", -1.0, 1), ("inv_temp", 0.0, 1)):
+        old = getattr(q, field)
+        setattr(q, field, bad)
+        assert f(R(b), R(q), R(o), nul, p, need, nul) == code, field
+        setattr(q, field, old)
+    b.n_groups = 0
+    assert f(R(b), R(q), R(o), nul, p, need, nul) == 2
+    b.n_groups = n_groups
+    b.d = 100
+    assert f(R(b), R(q), R(o), nul, p, need, nul) == 2
+    b.d = d
+    o.dH = ctypes.c_void_p(4098)
+    assert f(R(b), R(q), R(o), nul, p, need, nul) == 3
+    bx = lib.spo_policy_loss_bwd_ex
+    assert bx(p, p, p, p, p, 256, 256, 2048, -1, 1.0, p, 1, p, 0, nul, p, 1 << 40, nul) == 2
+    assert bx(p, p, p, nul, p, 256, 256, 2048, 0, 1.0, p, 0, p, 0, nul, p, 1 << 40, nul) == 1
+    sr = lib.spo_scale_f32_ratio
+    assert sr(nul, 0, nul, nul, nul) == 0
+    assert sr(p, 4, p, nul, nul) == 1
+    assert sr(p, -1, p, p, nul) == 2

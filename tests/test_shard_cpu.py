@@ -67,16 +67,34 @@ class OracleEngine:
                     lse=lse, n_loss_tokens=torch.tensor([float(st["n_loss_tokens"])],
                                                         dtype=torch.float64))
 
-    def scale(self, x, w):
-        x.mul_(w)
+    def local_counts(self, b, loc):
+        return torch.tensor([float(b["n_groups"]), float(loc["n_loss_tokens"][0])],
+                            dtype=torch.float64)
+
+    def zero_counts(self, b):
+        return torch.zeros(2, dtype=torch.float64)
+
+    def scale_ratio(self, x, num, den):
+        x.mul_(num[0] / den[0] if den[0] != 0 else 0.0)
         return x
 
-    def backward(self, b, lse, g):
+    def backward_blocks(self, b, lse, g, n_blocks):
         dH, dW = O.policy_loss_bwd(b["H"], b["W"], b["tgt"], g.numpy())
-        return torch.from_numpy(dH), torch.from_numpy(np.ascontiguousarray(dW))
+        starts = shard.dw_block_starts(b["W"].shape[0], n_blocks)
+        return (torch.from_numpy(dH), torch.from_numpy(np.ascontiguousarray(dW)),
+                [(starts[k], starts[k + 1], None) for k in range(n_blocks)])
+
+    def step_fused(self, b, weight, n_blocks):
+        loc = self.step_local(b, O.AGG_SEQ_GROUP)
+        g = loc["g"] * weight
+        dH, dW, blocks = self.backward_blocks(b, loc["lse"], g, n_blocks)
+        return loc["loss"] * weight, dH, dW, blocks
 
     def zeros_dW(self, V, d, like):
         return torch.zeros((V, d), dtype=torch.float64)
+
+    def comm_stream(self, t):
+        return None
 
 
 def _rank_inputs(b, rb, old, ref):
@@ -87,7 +105,7 @@ def _rank_inputs(b, rb, old, ref):
                 kl_beta=b["beta"])
 
 
-def _worker(rank, world, port, outdir, agg, groups_override):
+def _worker(rank, world, port, outdir, agg, groups_override, dw_blocks=4, fused=False):
     os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
     dist.init_process_group("gloo", rank=rank, world_size=world, timeout=timedelta(seconds=60))
     b = _batch()
@@ -97,8 +115,11 @@ def _worker(rank, world, port, outdir, agg, groups_override):
               for g in range(b["n_groups"])]
     groups = groups_override or shard.shard_groups(tokens, world)
     rb = shard.rank_batch(b["cu"], b["gid"], groups[rank])
-    step = shard.DataParallelStep(OracleEngine(), agg)
-    loss, dH, dW = step.run(_rank_inputs(b, rb, old, ref))
+    step = shard.DataParallelStep(OracleEngine(), agg, dw_blocks=dw_blocks)
+    if fused:   # every rank knows the plan: all n_groups groups are non-empty
+        loss, dH, dW = step.run_fused(_rank_inputs(b, rb, old, ref), b["n_groups"])
+    else:
+        loss, dH, dW = step.run(_rank_inputs(b, rb, old, ref))
     np.save(os.path.join(outdir, f"loss{rank}.npy"), loss.numpy())
     np.save(os.path.join(outdir, f"dW{rank}.npy"), dW.numpy())
     np.save(os.path.join(outdir, f"tok{rank}.npy"), rb.token_index)
@@ -145,6 +166,68 @@ def test_data_parallel_step_matches_unsharded(agg, override):
             tok = np.load(os.path.join(d, f"tok{r}.npy"))
             if tok.size:
                 np.testing.assert_allclose(np.load(os.path.join(d, f"dH{r}.npy")), dH[tok], atol=1e-13)
+
+
+@pytest.mark.parametrize("override", [None, [[0, 1, 2, 3, 4], []]])
+def test_fused_data_parallel_step_matches_unsharded(override):
+    """run_fused: one local call per rank with its weight N_r / N applied before
+    the backward, then the per-block dW and loss all-reduces."""
+    world = 2
+    with tempfile.TemporaryDirectory() as d:
+        mp.start_processes(_worker, args=(world, _free_port(), d, O.AGG_SEQ_GROUP, override, 4,
+                                          True), nprocs=world, join=True, start_method="spawn")
+        b = _batch()
+        loss, dH, dW, _, _ = _reference(b, O.AGG_SEQ_GROUP)
+        for r in range(world):
+            assert abs(float(np.load(os.path.join(d, f"loss{r}.npy"))[0]) - loss) < 1e-12
+            np.testing.assert_allclose(np.load(os.path.join(d, f"dW{r}.npy")), dW, atol=1e-13)
+            tok = np.load(os.path.join(d, f"tok{r}.npy"))
+            if tok.size:
+                np.testing.assert_allclose(np.load(os.path.join(d, f"dH{r}.npy")), dH[tok], atol=1e-13)
+
+
+def test_block_by_block_dW_reduction_equals_one_reduction():
+    """dW summed across ranks as one all-reduce, or as one all-reduce per
+    vocabulary block (each issued as its block is final), gives the same
+    bits; the blocks tile the vocabulary (V = 53: one 256-row block holds it
+    all, the others are empty and skipped)."""
+    world = 2
+    outs = {}
+    for blocks in (1, 3):
+        with tempfile.TemporaryDirectory() as d:
+            mp.start_processes(_worker, args=(world, _free_port(), d, O.AGG_SEQ_GROUP, None, blocks),
+                               nprocs=world, join=True, start_method="spawn")
+            outs[blocks] = [np.load(os.path.join(d, f"dW{r}.npy")) for r in range(world)]
+    for r in range(world):
+        np.testing.assert_array_equal(outs[1][r], outs[3][r])
+    assert shard.dw_block_starts(53, 3) == [0, 0, 0, 53]
+
+
+def _wide_worker(rank, world, port, outdir, n_blocks):
+    """dW rows summed block by block over a vocabulary of 1000 rows (blocks of
+    0, 256, 512 and 744 rows... as the library lays them out)."""
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world, timeout=timedelta(seconds=60))
+    V, d = 1000, 3
+    dW = torch.from_numpy(np.random.default_rng(rank).standard_normal((V, d)))
+    starts = shard.dw_block_starts(V, n_blocks)
+    works = [shard._overlapped_all_reduce(dW[starts[k]:starts[k + 1]], None, None, None)
+             for k in range(n_blocks) if starts[k + 1] > starts[k]]
+    for w in works:
+        w.wait()
+    np.save(os.path.join(outdir, f"w{rank}.npy"), dW.numpy())
+    dist.destroy_process_group()
+
+
+def test_overlapped_block_reductions_sum_every_row():
+    world = 3
+    with tempfile.TemporaryDirectory() as d:
+        mp.start_processes(_wide_worker, args=(world, _free_port(), d, 4), nprocs=world, join=True,
+                           start_method="spawn")
+        want = sum(np.random.default_rng(r).standard_normal((1000, 3)) for r in range(world))
+        for r in range(world):
+            np.testing.assert_allclose(np.load(os.path.join(d, f"w{r}.npy")), want, atol=1e-12)
+    assert shard.dw_block_starts(1000, 4) == [0, 0, 256, 512, 1000]
 
 
 def _failing_worker(rank, world, port, outdir):
@@ -195,7 +278,10 @@ class OracleVocabEngine:
     def backward_slice(self, b, lse, g):
         dH, dW = O.policy_loss_bwd_slice(b["H"], b["W_slice"], b["v_offset"], b["tgt"],
                                          lse.numpy(), g.numpy(), b["inv_temp"])
-        return torch.from_numpy(dH), torch.from_numpy(dW)
+        return torch.from_numpy(dH), torch.from_numpy(dW), None
+
+    def comm_stream(self, t):
+        return None
 
 
 def _vocab_batch():

@@ -49,7 +49,7 @@ class ThreadCollectives:
             parts[r].copy_(self.slots[r])
         self.bar.wait()
 
-    def all_reduce(self, t, group=None):
+    def all_reduce(self, t, group=None, async_op=False):
         if t.is_cuda:
             torch.cuda.current_stream().synchronize()
         self.slots[self.local.rank] = t.detach().clone()
@@ -59,6 +59,23 @@ class ThreadCollectives:
             total += x.to(total.device)
         self.bar.wait()
         t.copy_(total)
+        if async_op:
+            return _Done(t.is_cuda)
+
+
+class _Done:
+    """Work handle of a collective served in-process: wait() orders the
+    caller's stream after the stream the result was written on."""
+
+    def __init__(self, cuda):
+        self.ev = None
+        if cuda:
+            self.ev = torch.cuda.Event()
+            self.ev.record()
+
+    def wait(self):
+        if self.ev is not None:
+            torch.cuda.current_stream().wait_event(self.ev)
 
 
 def _batch(seed):
@@ -96,8 +113,8 @@ def _rank_dict(spo, b, rb, old, ref):
 
 
 @pytest.mark.parametrize("world", [2, 3])
-@pytest.mark.parametrize("agg", [0, 1])
-def test_virtual_ranks_reproduce_the_unsharded_step(spo, monkeypatch, world, agg):
+@pytest.mark.parametrize("agg,fused", [(0, False), (1, False), (0, True)])
+def test_virtual_ranks_reproduce_the_unsharded_step(spo, monkeypatch, world, agg, fused):
     import torch.distributed as dist
     b = _batch(40 + world)
     T = b["H"].shape[0]
@@ -122,8 +139,14 @@ def test_virtual_ranks_reproduce_the_unsharded_step(spo, monkeypatch, world, agg
     batches = [shard.rank_batch(b["cu"], b["gid"], groups[r]) for r in range(world)]
     coll = ThreadCollectives(world)
     monkeypatch.setattr(dist, "all_reduce", coll.all_reduce)
-    outs = _run_ranks(coll, world, lambda r: shard.DataParallelStep(shard.SpoEngine(), agg).run(
-        _rank_dict(spo, b, batches[r], old, ref)))
+
+    def rank(r):
+        step = shard.DataParallelStep(shard.SpoEngine(reserve_sms=8), agg)
+        inp = _rank_dict(spo, b, batches[r], old, ref)
+        # run_fused: one spo_grpo_step per rank, weight N_r / N known from the plan
+        return step.run_fused(inp, b["n_groups"]) if fused else step.run(inp)
+
+    outs = _run_ranks(coll, world, rank)
     for r in range(world):
         loss_r, dH_r, dW_r = outs[r]
         assert abs(loss_r.item() - loss1.item()) <= 1e-5 * abs(loss1.item()) + 1e-7
