@@ -691,7 +691,7 @@ def aux_measurements(dev, pk):
 
 
 # ----------------------------------------------------------------- arms
-def config_block(case, T_L, world, workload="full", mode="fused"):
+def config_block(case, T_L, world, workload="full", mode="fused", tunings=()):
     cfg = {"workload": WORKLOADS[workload], "T": case["T"], "loss_tokens": T_L, "d": case["d"],
            "V": case["V"]}
     if workload == "full":
@@ -705,6 +705,8 @@ def config_block(case, T_L, world, workload="full", mode="fused"):
     if case.get("keep"):
         cfg["kept_exponentials"] = "forward keeps exp(z - tile max) in bf16; backward forms G from it"
     cfg["l2"] = "inputs larger than L2 (W alone is 1.2-1.56 GB and is streamed every step)"
+    if tunings:
+        cfg["tunings"] = {str(k): v for k, v in tunings}
     cfg["call"] = {"fused": "spo_grpo_step: the whole path (a1-a8) in one C-ABI call per step",
                    "separate": "spo_token_select, spo_logprobs_fwd, spo_group_advantages, "
                                "spo_policy_loss_fwd, spo_policy_loss_bwd in turn",
@@ -756,6 +758,9 @@ def ours(args):
         mode = "separate"
     if dist.world > 1 and (args.workload == "forward" or mode in ("kept", "separate")):
         raise SystemExit(f"--workload {args.workload} ({mode}) runs on one GPU")
+    tunings = [tuple(int(x) for x in kv.split("=")) for kv in args.tune.split(",") if kv]
+    for key, value in tunings:
+        spo.spo_set_tuning(key, value)
     base_bytes = torch.cuda.memory_allocated(dev)
     st = Step(case, dev, dist, mode=mode, reserve_sms=args.reserve_sms)
     step_bytes = (torch.cuda.memory_allocated(dev) - base_bytes      # one buffer set:
@@ -871,7 +876,7 @@ def ours(args):
         "scaling": "strong" if vocab_ranks else "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded; H~N(0,1), W~N(0,0.02^2) rounded to bf16: random-init stand-in for "
                 "the policy's final hidden states and LM head)",
-        "config": config_block(case, T_L, dist.world, args.workload, mode),
+        "config": config_block(case, T_L, dist.world, args.workload, mode, tunings),
         "tensor_peak_frac": {"metric_tflops": flop_metric * args.steps / (ms / 1e3) / 1e12,
                              "of_burst": flop_metric * args.steps / (ms / 1e3) / 1e12 / pk["bf16_burst"],
                              "of_sustained": flop_metric * args.steps / (ms / 1e3) / 1e12 / pk["bf16_sustained"],
@@ -950,6 +955,9 @@ def main():
                     help="supplementary workloads; the default is the one the metric is quoted on")
     ap.add_argument("--separate-calls", action="store_true",
                     help="run the step as the separate C-ABI calls instead of spo_grpo_step")
+    ap.add_argument("--tune", type=str, default="",
+                    help="launch tunings applied first, 'key=value' pairs (spo_tune_key numbers) "
+                         "separated by ','; results do not depend on them")
     ap.add_argument("--reserve-sms", type=int, default=8,
                     help="with several GPUs: SMs the GEMMs that overlap a collective leave free")
     args = ap.parse_args()

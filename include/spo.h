@@ -657,6 +657,13 @@ SPO_API spo_status spo_policy_loss_fwd_noalloc(const float* logp, const float* o
  *   SPO_TUNE_DW_SPLIT_ROWS (default 8192; multiple of 256, 0 = off): dW =
  *     G^T H is reduced over at most this many token rows per pass, later
  *     passes adding into dW (smaller operand slabs stay in L2).
+ *   SPO_TUNE_KSYNC_FWD / _GRAD / _DH / _DW (default 0 = off): a k-progress
+ *     throttle for one GEMM kind: each CTA pair publishes the k-blocks (64
+ *     elements of the reduction) it has issued and does not run more than
+ *     this many ahead of the slowest pair, so the pairs whose tiles share an
+ *     operand slab read it close together in time (from L2).  The waits are
+ *     bounded (20 us); results do not depend on the setting.
+ *   SPO_TUNE_KSYNC_EPOCH (default 16): k-blocks between two throttle checks.
  *   SPO_TUNE_DEFAULTS (value ignored): every setting back to its default.
  * Results do not depend on any setting beyond fp32 summation order. */
 typedef enum spo_tune_key {
@@ -673,7 +680,12 @@ typedef enum spo_tune_key {
     SPO_TUNE_RASTER_GRAD = 10,
     SPO_TUNE_RASTER_DH = 11,
     SPO_TUNE_RASTER_DW = 12,
-    SPO_TUNE_DEFAULTS = 13
+    SPO_TUNE_DEFAULTS = 13,
+    SPO_TUNE_KSYNC_FWD = 14,
+    SPO_TUNE_KSYNC_GRAD = 15,
+    SPO_TUNE_KSYNC_DH = 16,
+    SPO_TUNE_KSYNC_DW = 17,
+    SPO_TUNE_KSYNC_EPOCH = 18
 } spo_tune_key;
 SPO_API spo_status spo_set_tuning(int key, int64_t value);
 

@@ -105,7 +105,7 @@ spo_status check_hwv(const void* H, const void* W, const int32_t* tgt, int64_t T
 struct FwdWs {
   int* idx;
   int* count;
-  int* counters;  // tile counter of the dynamic schedule
+  int* counters;  // tile counters of the dynamic schedule (4), then the throttle's progress slots
   int* scratch;
   int* tgt_c;
   float* ztgt;
@@ -130,7 +130,7 @@ FwdWs carve_fwd(void* base, long long T, long long d, long long V) {
   };
   w.idx = reinterpret_cast<int*>(take(sizeof(int) * w.T_pad));
   w.count = reinterpret_cast<int*>(take(sizeof(int)));
-  w.counters = reinterpret_cast<int*>(take(sizeof(int) * 4));
+  w.counters = reinterpret_cast<int*>(take(sizeof(int) * (4 + spo::kKsyncSlots)));
   w.scratch = reinterpret_cast<int*>(take(sizeof(int) * 2 * nb));
   w.tgt_c = reinterpret_cast<int*>(take(sizeof(int) * w.T_pad));
   w.ztgt = reinterpret_cast<float*>(take(sizeof(float) * w.T_pad));
@@ -146,7 +146,7 @@ constexpr long long kBwdChunkRows = 32768;  // G scratch rows per chunk (multipl
 struct BwdWs {
   int* idx;
   int* count;
-  int* counters;  // tile counters of the dynamic schedule, one per GEMM kind
+  int* counters;  // tile counters of the dynamic schedule (4), then the throttle's progress slots
   int* scratch;
   int* tgt_c;
   float* lse_c;
@@ -172,7 +172,7 @@ BwdWs carve_bwd(void* base, long long T, long long d, long long V) {
   };
   w.idx = reinterpret_cast<int*>(take(sizeof(int) * w.T_pad));
   w.count = reinterpret_cast<int*>(take(sizeof(int)));
-  w.counters = reinterpret_cast<int*>(take(sizeof(int) * 4));
+  w.counters = reinterpret_cast<int*>(take(sizeof(int) * (4 + spo::kKsyncSlots)));
   w.scratch = reinterpret_cast<int*>(take(sizeof(int) * 2 * nb));
   w.tgt_c = reinterpret_cast<int*>(take(sizeof(int) * w.T_pad));
   w.lse_c = reinterpret_cast<float*>(take(sizeof(float) * w.T_pad));
@@ -198,6 +198,11 @@ int g_tune_dynamic_mask = spo::kDefaultDynamicMask;
 // dW = G^T H runs as passes over at most this many token rows (0: one pass
 // per chunk): smaller operand slabs keep a wave's working set inside L2.
 int g_tune_dw_split = spo::kDefaultDwSplitRows;
+// k-progress throttle per GEMM kind: window in k-blocks (0 = off), and the
+// k-blocks between two checks.
+int g_tune_ksync[4] = {spo::kDefaultKsync[0], spo::kDefaultKsync[1], spo::kDefaultKsync[2],
+                       spo::kDefaultKsync[3]};
+int g_tune_ksync_epoch = spo::kDefaultKsyncEpoch;
 
 // ------------------------------------------------------------ tracing
 // When enabled, a start/stop CUDA event pair is recorded on the launch stream
@@ -281,6 +286,14 @@ spo_status traced_gemm(int epi, bool a_mn, bool b_mn, const CUtensorMap& ta, con
   if (counters && ((g_tune_dynamic_mask >> kind) & 1)) {
     args.tile_counter = counters + kind;
     SPO_CUDA(cudaMemsetAsync(args.tile_counter, 0, sizeof(int), s), "memset tile counter");
+  }
+  args.kprog = nullptr;
+  if (counters && g_tune_ksync[kind] > 0) {
+    args.kprog = counters + 4;
+    args.ksync_window = g_tune_ksync[kind];
+    args.ksync_epoch = g_tune_ksync_epoch;
+    SPO_CUDA(cudaMemsetAsync(args.kprog, 0, sizeof(int) * spo::kKsyncSlots, s),
+             "memset progress slots");
   }
   return traced(kind, s, "gemm launch", [&] {
     return spo::launch_gemm(epi, a_mn, b_mn, g_tune_pair != 0, ta, tb, tc, args, grid, s);
@@ -1278,12 +1291,27 @@ SPO_API spo_status spo_set_tuning(int key, int64_t value) {
       if (value != 0 && value != 1) return fail(SPO_ERR_INVALID_ARG, "raster must be 0 or 1");
       g_tune_raster[key - SPO_TUNE_RASTER_FWD] = static_cast<int>(value);
       return ok();
+    case SPO_TUNE_KSYNC_FWD:
+    case SPO_TUNE_KSYNC_GRAD:
+    case SPO_TUNE_KSYNC_DH:
+    case SPO_TUNE_KSYNC_DW:
+      if (value < 0 || value > (1 << 20))
+        return fail(SPO_ERR_INVALID_ARG, "throttle window must be in [0, 2^20] k-blocks");
+      g_tune_ksync[key - SPO_TUNE_KSYNC_FWD] = static_cast<int>(value);
+      return ok();
+    case SPO_TUNE_KSYNC_EPOCH:
+      if (value < 1 || value > 4096)
+        return fail(SPO_ERR_INVALID_ARG, "throttle epoch must be in [1, 4096] k-blocks");
+      g_tune_ksync_epoch = static_cast<int>(value);
+      return ok();
     case SPO_TUNE_DEFAULTS:
       g_tune_pair = 1;
       for (int k = 0; k < 4; ++k) {
         g_tune_group_m[k] = kDefaultGroupM[k];
         g_tune_raster[k] = kDefaultRaster[k];
+        g_tune_ksync[k] = spo::kDefaultKsync[k];
       }
+      g_tune_ksync_epoch = spo::kDefaultKsyncEpoch;
       g_tune_dynamic_mask = spo::kDefaultDynamicMask;
       g_tune_dw_split = spo::kDefaultDwSplitRows;
       return ok();

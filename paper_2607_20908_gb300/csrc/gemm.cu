@@ -58,6 +58,27 @@ __device__ __forceinline__ void tile_coords(int tile, int mt, int nt, int gm, in
   nb = raster ? o : i;
 }
 
+// The k-progress throttle.  kstate[0] holds the k-blocks issued so far by the
+// units (CTA pairs, or CTAs) that are running, kstate[1] how many are running.
+// A unit adds its progress every `epoch` k-blocks and waits (bounded) while
+// it is more than `window` k-blocks ahead of the running units' average, so
+// the units whose tiles share operand slabs read them close together in time,
+// from L2 instead of DRAM.  One fire-and-forget add and two loads per check.
+// A wait gives up after kKsyncMaxWaitNs (a unit not yet resident, another
+// kernel on the SMs): results never depend on the throttle.
+constexpr unsigned long long kKsyncMaxWaitNs = 20000ull;  // 20 us
+
+__device__ __forceinline__ void ksync_wait(unsigned long long* kstate, long long prog, int window) {
+  const unsigned long long t0 = globaltimer();
+  for (;;) {
+    const long long sum = static_cast<long long>(ld_relaxed_gpu_u64(kstate));
+    const long long active = static_cast<long long>(ld_relaxed_gpu_u64(kstate + 1));
+    if (active <= 0 || prog * active <= sum + static_cast<long long>(window) * active) return;
+    if (globaltimer() - t0 > kKsyncMaxWaitNs) return;
+    __nanosleep(128);
+  }
+}
+
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&h);
@@ -474,6 +495,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       uint32_t phase = 0;
       int issued = 0;
       bool ok = true;
+      // the throttle runs on the pair's leader (the follower's loads feed the same MMAs)
+      const bool throttle = p.kprog != nullptr && rank == 0;
+      unsigned long long* kstate = reinterpret_cast<unsigned long long*>(p.kprog);
+      const int epoch = max(1, p.ksync_epoch);
+      long long prog = 0, published = 0;
+      // state loaded at the previous check: decided on one epoch later, so the
+      // producer never waits for these loads to land
+      unsigned long long seen_sum = 0, seen_active = 0;
       for (int i = 0; ok; ++i) {
         const int tile = !dyn ? static_tile(i)
                               : (rank == 0 ? publish(i, ok) : take(i, ok, kErrWaitProducer));
@@ -483,6 +512,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         const int a_row = mb * G::kTileM + static_cast<int>(rank) * BM;
         const int b_row = nb * BN + static_cast<int>(rank) * G::kBRows;
         for (int kb = 0; kb < num_kb; ++kb) {
+          if (throttle && prog % epoch == 0) {
+            if (prog == 0) {
+              red_add_gpu_u64(kstate + 1, 1ull);  // this unit is running
+            } else {
+              red_add_gpu_u64(kstate, static_cast<unsigned long long>(prog - published));
+              published = prog;
+              const long long act = static_cast<long long>(seen_active);
+              if (act > 0 && prog * act > static_cast<long long>(seen_sum) +
+                                              static_cast<long long>(p.ksync_window) * act)
+                ksync_wait(kstate, prog, p.ksync_window);  // ahead a epoch ago: wait on fresh state
+            }
+            seen_sum = ld_relaxed_gpu_u64(kstate);
+            seen_active = ld_relaxed_gpu_u64(kstate + 1);
+          }
+          ++prog;
           if (!mbar_wait(&empty_bar[stage], phase ^ 1u, abort_flag, p.err, kErrWaitProducer)) {
             ok = false;
             break;
@@ -516,6 +560,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             phase ^= 1u;
           }
         }
+      }
+      if (throttle && prog > 0) {  // done: its progress leaves the running average
+        red_add_gpu_u64(kstate, static_cast<unsigned long long>(-published));
+        red_add_gpu_u64(kstate + 1, static_cast<unsigned long long>(-1ll));
       }
       if (!ok && (!PAIR || rank == 0)) {
         // Aborted: let the copies already in flight land before the CTA exits.

@@ -32,6 +32,11 @@ constexpr int kDefaultGroupM[4] = {16, 16, 4, 8};
 constexpr int kDefaultRaster[4] = {0, 0, 0, 1};
 constexpr int kDefaultDynamicMask = 0xF;
 constexpr int kDefaultDwSplitRows = 8192;
+// Ints of workspace reserved for the k-progress throttle's state (two u64), its
+// default window per GEMM kind in k-blocks (0 = off) and its check interval.
+constexpr int kKsyncSlots = 4;
+constexpr int kDefaultKsync[4] = {0, 0, 0, 0};
+constexpr int kDefaultKsyncEpoch = 16;
 
 // What the epilogue does with a finished 128 x 256 fp32 accumulator tile.
 enum EpiKind : int {
@@ -57,6 +62,13 @@ struct GemmArgs {
   int group_m;  // tile rows (raster 0) or columns (raster 1) walked together
   int raster;   // 0: groups of tile rows, 1: groups of tile columns
   int* tile_counter;  // zeroed int: tiles are taken in raster order from it; NULL = static
+  // k-progress throttle (NULL = off): 16 zeroed, 8-byte aligned bytes holding
+  // the running units' summed k-block progress and their count; a unit stays
+  // at most ksync_window k-blocks ahead of the average (bounded wait), checked
+  // every ksync_epoch k-blocks.  Affects timing and L2 reuse only.
+  int* kprog;
+  int ksync_window;
+  int ksync_epoch;
   float scale;  // inv_temp for EPI_LSE / EPI_GRAD
   // EPI_LSE
   const int* tgt;     // target id of each row

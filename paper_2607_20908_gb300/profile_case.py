@@ -10,7 +10,9 @@ sweeps.
 either "pair,group,raster[,dynamic_mask[,dw_split_rows]]" applied to every
 GEMM, or '|'-separated "key=value" settings (spo_tune_key numbers, e.g.
 "7=4|11=0" for dH's raster group and direction) applied after the defaults;
-each is run for --iters iterations of fwd + bwd.  The default reduced size keeps the reduction lengths of the full workload
+each is run for --iters iterations of fwd + bwd.  --no-dW leaves dW out, so a
+case with the full vocabulary and a reduced token count (e.g. --T 8192) holds
+a few GB on the device.  The default reduced size keeps the reduction lengths of the full workload
 (K = d = 5120 for the logits and their recompute, K = T = 16384 tokens for
 dW) with a vocabulary cut to 8192, so one launch takes about a millisecond
 and the device holds about 1 GB; the streamed operands of dW (G = 268 MB,
@@ -36,6 +38,8 @@ def main():
     ap.add_argument("--V", type=int, default=8192)
     ap.add_argument("--iters", type=int, default=3)
     ap.add_argument("--configs", type=str, default="", help='e.g. "1,16,0;0,16,0"')
+    ap.add_argument("--no-dW", action="store_true",
+                    help="backward without dW (the forward, the recompute and dH only)")
     a = ap.parse_args()
     from paper_2607_20908_gb300 import spo
     dev = torch.device("cuda")
@@ -48,7 +52,7 @@ def main():
     ws_b = torch.empty(spo.policy_loss_bwd_workspace_size(a.T, a.d, a.V), dtype=torch.uint8,
                        device=dev)
     dH = torch.empty(a.T, a.d, dtype=torch.bfloat16, device=dev)
-    dW = torch.empty(a.V, a.d, dtype=torch.float32, device=dev)
+    dW = None if a.no_dW else torch.empty(a.V, a.d, dtype=torch.float32, device=dev)
     configs = [c if "=" in c else tuple(int(x) for x in c.split(","))
                for c in a.configs.split(";") if c] or [None]
     for cfg in configs:
@@ -69,7 +73,8 @@ def main():
         for i in range(a.iters):
             spo.spo_trace_enable(i == a.iters - 1)
             _, _, lse = spo.spo_logprobs_fwd(H, W, tgt, ws=ws_f)
-            spo.spo_policy_loss_bwd(H, W, tgt, lse, gl, dH=dH, dW=dW, ws=ws_b)
+            spo.spo_policy_loss_bwd(H, W, tgt, lse, gl, dH=dH, dW=dW, ws=ws_b,
+                                    want_dW=dW is not None)
         torch.cuda.synchronize()
         label = ("default" if cfg is None else cfg if isinstance(cfg, str)
                  else "pair,group,raster,dynamic=" + ",".join(map(str, cfg)))

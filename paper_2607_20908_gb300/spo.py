@@ -672,6 +672,8 @@ SPO_TUNE_DW_SPLIT_ROWS = 4
 SPO_TUNE_GROUP_M_FWD, SPO_TUNE_GROUP_M_GRAD, SPO_TUNE_GROUP_M_DH, SPO_TUNE_GROUP_M_DW = 5, 6, 7, 8
 SPO_TUNE_RASTER_FWD, SPO_TUNE_RASTER_GRAD, SPO_TUNE_RASTER_DH, SPO_TUNE_RASTER_DW = 9, 10, 11, 12
 SPO_TUNE_DEFAULTS = 13
+SPO_TUNE_KSYNC_FWD, SPO_TUNE_KSYNC_GRAD, SPO_TUNE_KSYNC_DH, SPO_TUNE_KSYNC_DW = 14, 15, 16, 17
+SPO_TUNE_KSYNC_EPOCH = 18
 
 
 def spo_set_tuning(key: int, value: int):

@@ -223,3 +223,26 @@ def test_scale_ratio_and_sync_check(spo):
     spo.spo_selftest_bounded_wait()
     assert spo.spo_sync_check() == 7
     assert spo.spo_sync_check() == 0
+
+
+def test_k_progress_throttle_changes_no_bit(spo):
+    """The k-progress throttle only delays operand loads: with every GEMM kind
+    throttled to a tight window the outputs are the same bits."""
+    case = inputs.tiny_case(seed=1061, d=512, V=8192, T_per_seq=64)
+    o = P.run_oracle(case)
+    b = _dev(case, o["old"], o["ref"])
+    want = _separate(spo, case, b)
+    try:
+        for key in (spo.SPO_TUNE_KSYNC_FWD, spo.SPO_TUNE_KSYNC_GRAD, spo.SPO_TUNE_KSYNC_DH,
+                    spo.SPO_TUNE_KSYNC_DW):
+            spo.spo_set_tuning(key, 2)
+        spo.spo_set_tuning(spo.SPO_TUNE_KSYNC_EPOCH, 1)
+        got = _separate(spo, case, b)
+        fused = _fused(spo, case, b)
+        torch.cuda.synchronize()
+    finally:
+        spo.spo_set_tuning(spo.SPO_TUNE_DEFAULTS, 0)
+    for k in ("logp", "entropy", "lse", "loss", "g", "dH", "dW"):
+        assert torch.equal(got[k], want[k]), k
+        assert torch.equal(fused[k], want[k]), k
+    assert spo.spo_device_error() == 0
