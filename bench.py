@@ -84,12 +84,19 @@ GEMM_KINDS = ("logits_lse_fwd", "logits_grad_recompute", "gemm_dH", "gemm_dW")
 SAMPLE_SEQS, SAMPLE_TOKENS = 8, 8   # CPU sample: one group of 8 rollouts, first 8 tokens each
 
 
-# DRAM bytes (read + write) per launch of each tensor-core kernel on this workload, from one
-# `ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum` capture (one pass, the GEMM kernels
-# only), valid only for the kernel sources they were taken on.
-TRAFFIC = {"sources_sha256_16": "a451e474f3cd76dc",
-           "bytes": {"logits_lse_fwd": 6.879e9, "logits_grad_recompute": 13.570e9,
-                     "gemm_dH": 52.128e9, "gemm_dW": 14.965e9}}
+# DRAM bytes (read + write) per launch of each tensor-core kernel at this workload, valid only for
+# the kernel sources they were taken on.  Derived from one-pass ncu captures
+# (dram__bytes_read.sum + dram__bytes_write.sum, the GEMM kernels only) of two reduced cases of the
+# same kernels, scaled by the units a launch processes: 8192 tokens with the full vocabulary and no
+# dW (the logits GEMMs and dH: x 2 tokens) and the full 16384 tokens with 8192 vocabulary rows (dW:
+# x 151936 / 8192 rows, the mean of its two passes).  The logits GEMMs' traffic is proportional to
+# the tokens (checked against full-size captures: 6.88 and 13.57 GB); dH's grows faster than its
+# waves (its CTA pairs drift further apart over more waves), so its figure is a lower estimate.
+TRAFFIC = {"sources_sha256_16": "fd2c248a3911b49e",
+           "bytes": {"logits_lse_fwd": 6.844e9, "logits_grad_recompute": 13.394e9,
+                     "gemm_dH": 35.11e9, "gemm_dW": 17.25e9},
+           "derivation": "reduced-case captures scaled by tokens (T = 8192 -> 16384) or vocabulary "
+                         "rows (V = 8192 -> 151936); dH a lower estimate"}
 KERNEL_SOURCES = ["paper_2607_20908_gb300/csrc/gemm.cu", "paper_2607_20908_gb300/csrc/tc.cuh",
                   "paper_2607_20908_gb300/csrc/gemm.h"]
 
@@ -834,6 +841,7 @@ def ours(args):
                 "frac_of_burst": achieved / pk["bf16_burst"],
                 "flop_per_launch": dom["flop_per_launch"], "traffic": kernel_traffic(dom_name),
                 "traffic_unit": "bytes per launch (ncu dram__bytes_read.sum + dram__bytes_write.sum)",
+                "traffic_source": TRAFFIC["derivation"],
                 "algorithmic_bytes": None}
     alg = {"logits_lse_fwd": 2 * T_L * st.d + 2 * st.V * st.d + 12 * T_L * ((st.V + 255) // 256),
            "logits_grad_recompute": 2 * T_L * st.d + 2 * st.V * st.d + 2 * T_L * st.V,

@@ -3,7 +3,10 @@
  * checks closed forms that need no reference implementation:
  *   - with H = 0 every logit is 0, so logp = -ln V and entropy = ln V;
  *   - log-probs are <= 0 and the loss is finite;
- *   - every status is SPO_OK and no device wait expired.
+ *   - every status is SPO_OK and no device wait expired;
+ *   - the one-call step (spo_grpo_step, workspace from spo_workspace_size)
+ *     gives the same bits as the separate calls, and a bad argument is
+ *     reported through spo_last_error_detail.
  * Build: cc -std=c99 abi_demo.c -I include -I <cuda>/include -L <lib> -lspo
  *        -L <cuda>/lib64 -lcudart -Wl,-rpath,<lib>
  * Exit status 0 on success. */
@@ -114,6 +117,29 @@ int main(void) {
   int code = 0;
   if (check(spo_device_error(&code, NULL), "device_error")) return 1;
 
+  /* the same step as one call, with one workspace sized for the whole step */
+  size_t ws_all = 0;
+  if (check(spo_workspace_size(T, D, V, NSEQ, &ws_all), "workspace_size")) return 1;
+  void* wall = dev_alloc(ws_all);
+  float* loss2 = (float*)dev_alloc(sizeof(float));
+  float* logp2 = (float*)dev_alloc(T * sizeof(float));
+  float* dW2 = (float*)dev_alloc((size_t)V * D * sizeof(float));
+  spo_grpo_batch batch = {H, W, tgt, mask, cu, gid, rew, old, NULL, T, D, V, NSEQ, NGROUPS};
+  spo_grpo_params prm = {1.0f, 1024, 0.2f, 0.0f, SPO_AGG_SEQ_GROUP, SPO_STD_UNBIASED, 1e-6f, NULL};
+  spo_grpo_outputs out;
+  memset(&out, 0, sizeof(out));
+  out.loss = loss2;
+  out.logp = logp2;
+  out.dW = dW2;
+  if (check(spo_grpo_step(&batch, &prm, &out, NULL, wall, ws_all, NULL), "grpo_step") ||
+      check(spo_sync_check(NULL), "sync_check"))
+    return 1;
+  /* an argument error is reported, with its text, under the boundary's name */
+  char why[256];
+  if (spo_grpo_step(NULL, &prm, &out, NULL, wall, ws_all, NULL) != SPO_ERR_INVALID_ARG ||
+      spo_last_error_detail(why, sizeof(why)) != SPO_ERR_INVALID_ARG || why[0] == '\0')
+    ++bad;
+
   float h_logp[T], h_ent[T], h_loss;
   cudaMemcpy(h_logp, logp, sizeof(h_logp), cudaMemcpyDeviceToHost);
   cudaMemcpy(h_ent, ent, sizeof(h_ent), cudaMemcpyDeviceToHost);
@@ -123,6 +149,18 @@ int main(void) {
     if (fabsf(h_logp[i] + lnV) > 1e-4f || fabsf(h_ent[i] - lnV) > 1e-4f) ++bad;
   }
   if (!isfinite(h_loss)) ++bad;
+  {
+    /* g has no zero on the loss tokens here, so the one-call step gives the same bits */
+    static float h_logp2[T], h_dW[64], h_dW2[64];
+    float h_loss2;
+    cudaMemcpy(h_logp2, logp2, sizeof(h_logp2), cudaMemcpyDeviceToHost);
+    cudaMemcpy(&h_loss2, loss2, sizeof(float), cudaMemcpyDeviceToHost);
+    cudaMemcpy(h_dW, dW, sizeof(h_dW), cudaMemcpyDeviceToHost);
+    cudaMemcpy(h_dW2, dW2, sizeof(h_dW2), cudaMemcpyDeviceToHost);
+    if (memcmp(h_logp, h_logp2, sizeof(h_logp2)) != 0 || memcmp(&h_loss, &h_loss2, sizeof(float)) != 0 ||
+        memcmp(h_dW, h_dW2, sizeof(h_dW)) != 0)
+      ++bad;
+  }
   printf("libspo %d.%d from C: logp[0]=%.6f (-ln V=%.6f) entropy[0]=%.6f loss=%.6g bad=%d\n",
          spo_version() >> 16, spo_version() & 0xffff, h_logp[0], -lnV, h_ent[0], h_loss, bad);
   return bad ? 1 : 0;

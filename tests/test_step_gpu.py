@@ -246,3 +246,28 @@ def test_k_progress_throttle_changes_no_bit(spo):
         assert torch.equal(got[k], want[k]), k
         assert torch.equal(fused[k], want[k]), k
     assert spo.spo_device_error() == 0
+
+
+def test_step_ragged_workload_two_chunks_equals_separate_calls(spo):
+    """The ragged multi-turn workload (65536 packed tokens, ~40% masked, about
+    39k loss tokens): the backward runs in two chunks of the forward's
+    compaction, reading lse and g at token positions through each chunk's
+    offset.  The one-call step equals the separate calls bit for bit."""
+    case = inputs.ragged_case(device="cuda")
+    dev = torch.device("cuda")
+    b = dict(H=case["H"], W=case["W"], tgt=case["tgt"].to(dev), mask=case["mask"].to(dev),
+             cu=case["cu_seqlens"].to(dev), gid=case["group_id"].to(dev),
+             rewards=case["rewards"].to(dev))
+    lm, _ = spo.spo_token_select(b["cu"], b["mask"], b["tgt"], case["window"])
+    assert int(lm.sum().item()) > 32768            # more than one backward chunk
+    logp, _, _ = spo.spo_logprobs_fwd(b["H"], b["W"], b["tgt"], lm)
+    b["old"] = logp + case["old_noise"].to(dev)
+    b["ref"] = logp + case["ref_noise"].to(dev)
+    want = _separate(spo, case, b)
+    want = {k: want[k] for k in ("loss", "g", "logp", "dH", "dW")}
+    torch.cuda.synchronize()
+    got = _fused(spo, case, b, want=("g", "logp"))
+    torch.cuda.synchronize()
+    for k in ("loss", "g", "logp", "dH", "dW"):
+        assert torch.equal(got[k], want[k]), k
+    assert spo.spo_sync_check() == 0
