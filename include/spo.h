@@ -18,12 +18,18 @@
  *   spo_policy_loss_bwd    dH = G W, dW = G^T H with
  *                          G = tau^-1 g (onehot - softmax), logits recomputed
  *
+ * or all of it as one call, spo_grpo_step, with one workspace
+ * (spo_workspace_size).  spo_policy_loss_bwd_ex adds hooks for overlapping the
+ * multi-GPU exchanges (dW per vocabulary block, dH) with the GEMMs that follow.
+ *
  * Conventions shared by every call
  *   - Every array argument is a DEVICE pointer owned by the caller unless the
  *     comment says otherwise.  The library never allocates device memory,
  *     never frees, and never synchronises the stream (except
- *     spo_device_error, which says so).  Scratch memory comes only from the
- *     caller's `ws` buffer, sized by the matching *_workspace_size call.
+ *     spo_device_error and spo_sync_check, which say so).  Scratch memory
+ *     comes only from the caller's `ws` buffer, sized by the matching
+ *     *_workspace_size call (spo_policy_loss_fwd_noalloc, which has none,
+ *     says where its scratch lives).
  *   - `stream` is a cudaStream_t (NULL = legacy default stream).  Work is
  *     enqueued asynchronously in stream order.  Calls on distinct workspaces
  *     may run concurrently on different streams.

@@ -893,7 +893,7 @@ __device__ __forceinline__ float group_sum_f(float v, unsigned m) {
 }
 
 template <int LPS>
-__global__ void __launch_bounds__(kLossThreads) loss_token_kernel(
+__global__ void __launch_bounds__(kLossThreads, 4) loss_token_kernel(
     const float* logp, const float* old_logp, const float* ref_logp, const float* adv,
     const int* cu, const int* gid, int n_seq, int n_groups, const uint8_t* lm, float clip_eps,
     float kl_beta, int agg, const int* gsize, const unsigned long long* scal, const float* cscale,
