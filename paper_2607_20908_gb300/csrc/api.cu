@@ -1034,12 +1034,15 @@ SPO_API spo_status spo_policy_loss_fwd(const float* logp, const float* old_logp,
     return fail(SPO_ERR_WORKSPACE, "workspace needs %zu bytes, got %zu", need, ws_bytes);
   if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
     return fail(SPO_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
+  DevInfo di;
+  spo_status st = device_info(&di);
+  if (st != SPO_OK) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const spo::LossWs w = spo::carve_loss_ws(ws, n_seq, n_groups);
-  spo_status st = traced(kTracePolicyLoss, s, "policy loss launch", [&] {
+  st = traced(kTracePolicyLoss, s, "policy loss launch", [&] {
     return spo::launch_policy_loss(logp, old_logp, ref_logp, adv, cu_seqlens, group_id, n_seq,
                                    n_groups, loss_mask, T, clip_eps, kl_beta, agg, loss, g, stats,
-                                   w, s);
+                                   w, s, di.err);
   });
   return st == SPO_OK ? ok() : st;
 }
@@ -1191,22 +1194,25 @@ SPO_API spo_status spo_grpo_step(const spo_grpo_batch* b, const spo_grpo_params*
   if ((st = logprobs_impl(b->H, b->W, b->tgt, lm, b->T, b->d, b->V, 0, q->inv_temp, logp,
                           o->entropy, lse, nullptr, ws, s)) != SPO_OK)
     return st;
-  // a4: the per-group scan at a step's few hundred sequences, else the run path (same bits)
+  // a4 + a5.  At a step's few hundred sequences the per-group scan of the
+  // advantages runs inside the loss launch (its first phase, with the group
+  // counts); otherwise the run path first (same bits), then the loss.
+  // g = dL/dlogp, times the rank weight if any.
   const bool scan = static_cast<long long>(b->n_seq) * b->n_groups <= (1ll << 22);
-  st = traced(kTraceAdvantages, s, "advantage launch", [&] {
-    return scan ? spo::launch_group_advantages(b->rewards, b->group_id, b->n_seq, b->n_groups,
-                                               q->std_mode, q->adv_eps, adv, s)
-                : spo::launch_group_advantages_runs(b->rewards, b->group_id, b->n_seq,
-                                                    b->n_groups, q->std_mode, q->adv_eps, adv,
-                                                    w.adv_ws, s);
-  });
-  if (st != SPO_OK) return st;
-  // a5: surrogate, KL, aggregation; g = dL/dlogp (times the rank weight, if any)
+  if (!scan) {
+    st = traced(kTraceAdvantages, s, "advantage launch", [&] {
+      return spo::launch_group_advantages_runs(b->rewards, b->group_id, b->n_seq, b->n_groups,
+                                               q->std_mode, q->adv_eps, adv, w.adv_ws, s);
+    });
+    if (st != SPO_OK) return st;
+  }
   const spo::LossWs lw = spo::carve_loss_ws(w.loss_ws, b->n_seq, b->n_groups);
   st = traced(kTracePolicyLoss, s, "policy loss launch", [&] {
     return spo::launch_policy_loss(logp, b->old_logp, b->ref_logp, adv, b->cu_seqlens,
                                    b->group_id, b->n_seq, b->n_groups, lm, b->T, q->clip_eps,
-                                   q->kl_beta, q->agg, o->loss, g, o->stats, lw, s, q->loss_scale);
+                                   q->kl_beta, q->agg, o->loss, g, o->stats, lw, s, di.err,
+                                   q->loss_scale, scan ? b->rewards : nullptr, q->std_mode,
+                                   q->adv_eps, scan ? adv : nullptr);
   });
   if (st != SPO_OK) return st;
   // a6 - a8 over the forward's compaction (loss tokens); lse and g read at token positions
@@ -1399,7 +1405,7 @@ SPO_API spo_status spo_policy_loss_fwd_noalloc(const float* logp, const float* o
   st = traced(kTracePolicyLoss, s, "policy loss launch", [&] {
     return spo::launch_policy_loss(logp, old_logp, ref_logp, adv, cu_seqlens, group_id, n_seq,
                                    n_groups, loss_mask, T, clip_eps, kl_beta, agg, loss, g, stats,
-                                   w, s);
+                                   w, s, di.err);
   });
   return st == SPO_OK ? ok() : st;
 }

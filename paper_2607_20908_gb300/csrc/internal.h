@@ -103,7 +103,8 @@ cudaError_t launch_validate(const int* tgt, long long T, long long V, const int*
                             const float* ref_logp, const uint8_t* mask, int* counts, cudaStream_t s);
 
 struct LossWs {
-  unsigned long long* scal;  // [3]: non-empty groups, total loss tokens (token mean), ticket
+  unsigned long long* scal;  // [4]: non-empty groups, total loss tokens (token mean), ticket,
+                             // grid-barrier arrivals
   int* gsize;                // [n_groups]
   int* n_tok;                // [n_seq]
   float2* part_l;            // [n_seq]: c_i * sum of the sequence's l_t as a (hi, lo) pair
@@ -114,11 +115,18 @@ struct LossWs {
 size_t loss_ws_bytes(int n_seq, int n_groups);
 LossWs carve_loss_ws(void* ws, int n_seq, int n_groups);
 
+// The loss forward (group counts, token pass, fixed-order sum) as one
+// cooperative launch; err is the device error word (a grid barrier that
+// expires records its code there).  cscale (device scalar or NULL)
+// multiplies every c_t.  With `rewards` non-NULL the launch first computes the
+// group advantages into adv_out (the per-group scan of
+// launch_group_advantages, the same bits) and uses them; `adv` is then unused.
 cudaError_t launch_policy_loss(const float* logp, const float* old_logp, const float* ref_logp,
                                const float* adv, const int* cu_seqlens, const int* group_id,
                                int n_seq, int n_groups, const uint8_t* loss_mask, long long T,
                                float clip_eps, float kl_beta, int agg, float* loss, float* g,
-                               float* stats, const LossWs& w, cudaStream_t s,
-                               const float* cscale = nullptr);
+                               float* stats, const LossWs& w, cudaStream_t s, int* err,
+                               const float* cscale = nullptr, const float* rewards = nullptr,
+                               int std_mode = 0, float adv_eps = 0.f, float* adv_out = nullptr);
 
 }  // namespace spo

@@ -6,6 +6,7 @@
 #include <atomic>
 
 #include "internal.h"
+#include "tc.cuh"
 
 namespace spo {
 
@@ -306,9 +307,9 @@ __global__ void token_select_kernel(const int* cu, const uint8_t* mask, const in
 // operation in a fixed order, so the result is reproducible bit for bit (the
 // _rn intrinsics also keep the compiler from contracting into fused
 // multiply-adds).
-__device__ __forceinline__ void group_adv_warp(const float* rewards, const int* gid, int g, int b,
-                                               int e, bool check_gid, int std_mode, float eps,
-                                               float* adv, int lane) {
+__device__ __forceinline__ int group_adv_warp(const float* rewards, const int* gid, int g, int b,
+                                              int e, bool check_gid, int std_mode, float eps,
+                                              float* adv, int lane) {
   float acc = 0.f, lo = INFINITY, hi = -INFINITY;
   int n = 0;
   for (int base = b; base < e; base += 32) {
@@ -351,6 +352,7 @@ __device__ __forceinline__ void group_adv_warp(const float* rewards, const int* 
     if (i < e && (!check_gid || gid[i] == g))
       adv[i] = zero ? 0.f : __fdiv_rn(__fsub_rn(rewards[i], mu), den);
   }
+  return n;  // the group's member count (the same in every lane)
 }
 
 // One warp per group, scanning every sequence: O(n_groups * n_seq) reads, no
@@ -773,40 +775,44 @@ __device__ __forceinline__ long long warp_sum_ll(long long v) {
 
 // (a) sequences per group and the number of non-empty groups; for the token
 // mean also the number of loss tokens of [cu[0], cu[n_seq]) (integers; the
-// counters were cleared on the stream).
+// counters were cleared on the stream).  Each phase of the launch strides over
+// the whole grid.
 __device__ __forceinline__ int nonzero_bytes(unsigned w) {
   // high bit of each byte set iff the byte is non-zero (no carry crosses bytes)
   return __popc((((w & 0x7f7f7f7fu) + 0x7f7f7f7fu) | w) & 0x80808080u);
 }
 
-__global__ void loss_groups_kernel(const int* gid, int n_seq, int n_groups, const int* cu,
-                                   const uint8_t* lm, int agg, int* gsize,
-                                   unsigned long long* scal) {
-  const int stride = gridDim.x * blockDim.x;
-  const int tid = blockIdx.x * blockDim.x + threadIdx.x;
-  int first = 0;
-  for (int i = tid; i < n_seq; i += stride) {
-    const int g = gid[i];
-    if (g >= 0 && g < n_groups && atomicAdd(&gsize[g], 1) == 0) ++first;
-  }
+__device__ __forceinline__ long long grid_tid() {
+  return static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+}
+__device__ __forceinline__ long long grid_threads() {
+  return static_cast<long long>(gridDim.x) * blockDim.x;
+}
+
+// Loss tokens of [cu[0], cu[n_seq]) counted by this thread: bytes up to the
+// first 16-byte-aligned address, then 16 at a time, then the tail.
+__device__ __forceinline__ long long count_loss_tokens(const int* cu, int n_seq, const uint8_t* lm) {
+  const long long tid = grid_tid(), stride = grid_threads();
   long long nt = 0;
-  if (agg == 1) {
-    const long long lo = cu[0], hi = cu[n_seq];
-    // bytes up to the first 16-byte-aligned address, then 16 at a time, then the tail
-    const long long lead = static_cast<long long>((16u - (reinterpret_cast<uintptr_t>(lm + lo) & 15u)) & 15u);
-    const long long a = min(hi, lo + lead);
-    const long long z = a + (hi - a) / 16 * 16;
-    for (long long t = lo + tid; t < a; t += stride) nt += lm[t] != 0;
-    const uint4* v = reinterpret_cast<const uint4*>(lm + a);
-    for (long long k = tid; k < (z - a) / 16; k += stride) {
-      const uint4 q = __ldcs(v + k);
-      nt += nonzero_bytes(q.x) + nonzero_bytes(q.y) + nonzero_bytes(q.z) + nonzero_bytes(q.w);
-    }
-    for (long long t = z + tid; t < hi; t += stride) nt += lm[t] != 0;
+  const long long lo = cu[0], hi = cu[n_seq];
+  const long long lead = static_cast<long long>((16u - (reinterpret_cast<uintptr_t>(lm + lo) & 15u)) & 15u);
+  const long long a = min(hi, lo + lead);
+  const long long z = a + (hi - a) / 16 * 16;
+  for (long long t = lo + tid; t < a; t += stride) nt += lm[t] != 0;
+  const uint4* v = reinterpret_cast<const uint4*>(lm + a);
+  for (long long k = tid; k < (z - a) / 16; k += stride) {
+    const uint4 q = __ldcs(v + k);
+    nt += nonzero_bytes(q.x) + nonzero_bytes(q.y) + nonzero_bytes(q.z) + nonzero_bytes(q.w);
   }
-  // one update of each counter per block (same-address atomics serialise)
+  for (long long t = z + tid; t < hi; t += stride) nt += lm[t] != 0;
+  return nt;
+}
+
+// One update of each counter per block (same-address atomics serialise).
+__device__ __forceinline__ void add_block_counts(long long first, long long nt,
+                                                 unsigned long long* scal) {
   __shared__ long long sf[kLossThreads / 32], st[kLossThreads / 32];
-  first = __reduce_add_sync(0xffffffffu, first);
+  first = warp_sum_ll(first);
   nt = warp_sum_ll(nt);
   if ((threadIdx.x & 31) == 0) {
     sf[threadIdx.x >> 5] = first;
@@ -822,6 +828,40 @@ __global__ void loss_groups_kernel(const int* gid, int n_seq, int n_groups, cons
     if (f) atomicAdd(&scal[0], static_cast<unsigned long long>(f));
     if (n) atomicAdd(&scal[1], static_cast<unsigned long long>(n));
   }
+}
+
+__device__ __forceinline__ void loss_group_counts(const int* gid, int n_seq, int n_groups,
+                                                  const int* cu, const uint8_t* lm, int agg,
+                                                  int* gsize, unsigned long long* scal) {
+  const long long tid = grid_tid(), stride = grid_threads();
+  long long first = 0;
+  for (long long i = tid; i < n_seq; i += stride) {
+    const int g = gid[i];
+    if (g >= 0 && g < n_groups && atomicAdd(&gsize[g], 1) == 0) ++first;
+  }
+  add_block_counts(first, agg == 1 ? count_loss_tokens(cu, n_seq, lm) : 0, scal);
+}
+
+// The same counts together with the group advantages (a4), for a step's few
+// hundred sequences: warp w of the grid folds groups w, w + warps, ... with
+// group_adv_warp (the per-group scan of spo_group_advantages: the same bits)
+// and records each group's size, so the sizes need no atomics.
+__device__ __forceinline__ void adv_and_group_counts(const float* rewards, const int* gid,
+                                                     int n_seq, int n_groups, int std_mode,
+                                                     float eps, float* adv, const int* cu,
+                                                     const uint8_t* lm, int agg, int* gsize,
+                                                     unsigned long long* scal) {
+  const int lane = threadIdx.x & 31;
+  const int warps = static_cast<int>(grid_threads() >> 5);
+  long long first = 0;
+  for (int g = static_cast<int>(grid_tid() >> 5); g < n_groups; g += warps) {
+    const int n = group_adv_warp(rewards, gid, g, 0, n_seq, true, std_mode, eps, adv, lane);
+    if (lane == 0) {
+      gsize[g] = n;
+      first += n > 0;
+    }
+  }
+  add_block_counts(first, agg == 1 ? count_loss_tokens(cu, n_seq, lm) : 0, scal);
 }
 
 // (b) per-token surrogate, KL, dL/dlogp; per-sequence sums.  A group of LPS
@@ -892,8 +932,11 @@ __device__ __forceinline__ float group_sum_f(float v, unsigned m) {
   return v;
 }
 
-template <int LPS>
-__global__ void __launch_bounds__(kLossThreads, 4) loss_token_kernel(
+// ld(p): a load of a count or advantage; with IN_LAUNCH (phases of one
+// launch) they were written by other blocks earlier in the same launch, so the
+// load goes to L2, past this SM's L1.
+template <int LPS, bool IN_LAUNCH>
+__device__ __forceinline__ void loss_token_pass(
     const float* logp, const float* old_logp, const float* ref_logp, const float* adv,
     const int* cu, const int* gid, int n_seq, int n_groups, const uint8_t* lm, float clip_eps,
     float kl_beta, int agg, const int* gsize, const unsigned long long* scal, const float* cscale,
@@ -904,8 +947,10 @@ __global__ void __launch_bounds__(kLossThreads, 4) loss_token_kernel(
   const int sl = lane % LPS;
   const unsigned gm = LPS == 32 ? 0xffffffffu : ((1u << LPS) - 1u) << (lane - sl);
   const bool use_kl = ref_logp != nullptr && kl_beta != 0.f;
-  const float ng = static_cast<float>(scal[0]);
-  const float c_tok = scal[1] > 0 ? __frcp_rn(static_cast<float>(scal[1])) : 0.f;
+  auto ld = [](const auto* p) { return IN_LAUNCH ? __ldcg(p) : *p; };
+  const unsigned long long n_nonempty = ld(scal), n_loss = ld(scal + 1);
+  const float ng = static_cast<float>(n_nonempty);
+  const float c_tok = n_loss > 0 ? __frcp_rn(static_cast<float>(n_loss)) : 0.f;
   const int stride = warp_seq_stride() * (32 / LPS);
   int i = warp_seq0() * (32 / LPS) + lane / LPS;
   int b = 0, e = 0, gi = -1;
@@ -914,7 +959,7 @@ __global__ void __launch_bounds__(kLossThreads, 4) loss_token_kernel(
     b = cu[i];
     e = cu[i + 1];
     gi = gid[i];
-    A = adv[i];
+    A = ld(adv + i);
   }
   for (; i < n_seq; i += stride) {
     const int in = i + stride;
@@ -924,9 +969,9 @@ __global__ void __launch_bounds__(kLossThreads, 4) loss_token_kernel(
       nb = cu[in];
       ne = cu[in + 1];
       ngi = gid[in];
-      nA = adv[in];
+      nA = ld(adv + in);
     }
-    const int gs = agg == 0 && gi >= 0 && gi < n_groups ? gsize[gi] : 0;
+    const int gs = agg == 0 && gi >= 0 && gi < n_groups ? ld(gsize + gi) : 0;
     // the first pass's inputs stay in registers while the mask is counted
     uint8_t mk[kTpl];
     float lpv[kTpl], olv[kTpl], rfv[kTpl];
@@ -1056,27 +1101,36 @@ __device__ __forceinline__ LossSums block_sums(LossSums v, LossSums* sh) {
   return t;
 }
 
-__global__ void __launch_bounds__(kLossThreads) loss_final_kernel(
-    const float2* part_l, const float2* part_rk, const int* part_clip, const int* n_tok, int n_seq,
-    int chunk, LossSums* bpart, unsigned long long* ticket, float* loss, float* stats) {
+// Chunk c of the sequences (fixed split: chunk sequences each, depending only
+// on n_seq) summed by the block in a fixed order, then the last block to
+// finish (a ticket taken after its sums are visible) sums the chunks' results
+// in chunk order.  Per-sequence partials written by other blocks earlier in
+// the launch are read through L2.
+__device__ __forceinline__ void loss_final_phase(const float2* part_l, const float2* part_rk,
+                                                 const int* part_clip, const int* n_tok,
+                                                 int n_seq, int chunk, int nb, LossSums* bpart,
+                                                 unsigned long long* ticket, float* loss,
+                                                 float* stats) {
   __shared__ LossSums sh[kLossThreads / 32];
   __shared__ bool last;
-  const int i0 = blockIdx.x * chunk, i1 = min(n_seq, i0 + chunk);
-  LossSums v;
-  v.zero();
-  for (int i = i0 + threadIdx.x; i < i1; i += kLossThreads) {
-    LossSums q;
-    q.l = part_l[i];
-    const float2 rk = part_rk[i];
-    q.r = rk.x;
-    q.k = rk.y;
-    q.c = part_clip[i];
-    q.n = n_tok[i];
-    v.add(q);
+  for (int c = blockIdx.x; c < nb; c += gridDim.x) {
+    const int i0 = c * chunk, i1 = min(n_seq, i0 + chunk);
+    LossSums v;
+    v.zero();
+    for (int i = i0 + threadIdx.x; i < i1; i += kLossThreads) {
+      LossSums q;
+      q.l = __ldcg(part_l + i);
+      const float2 rk = __ldcg(part_rk + i);
+      q.r = rk.x;
+      q.k = rk.y;
+      q.c = __ldcg(part_clip + i);
+      q.n = __ldcg(n_tok + i);
+      v.add(q);
+    }
+    v = block_sums(v, sh);
+    if (threadIdx.x == 0) bpart[c] = v;
   }
-  v = block_sums(v, sh);
   if (threadIdx.x == 0) {
-    bpart[blockIdx.x] = v;
     __threadfence();
     last = atomicAdd(ticket, 1ull) == gridDim.x - 1;
   }
@@ -1085,7 +1139,7 @@ __global__ void __launch_bounds__(kLossThreads) loss_final_kernel(
   __threadfence();
   LossSums u;
   u.zero();
-  for (int j = threadIdx.x; j < static_cast<int>(gridDim.x); j += kLossThreads) {
+  for (int j = threadIdx.x; j < nb; j += kLossThreads) {
     const volatile LossSums* q = bpart + j;
     LossSums x;
     x.l.x = q->l.x;
@@ -1108,6 +1162,110 @@ __global__ void __launch_bounds__(kLossThreads) loss_final_kernel(
     }
   }
 }
+
+// Grid-wide barrier of a cooperative launch (every block resident): each
+// block arrives once on *count and waits until `target` arrivals.  The wait
+// is bounded: past kWaitTimeoutNs the block records kErrWaitGridBarrier in the
+// device error word and the caller returns (its outputs are then undefined,
+// and spo_device_error / spo_sync_check report the timeout).
+__device__ __forceinline__ bool grid_barrier(unsigned long long* count, unsigned long long target,
+                                             int* err) {
+  __shared__ int ok_s;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    atomicAdd(count, 1ull);
+    const unsigned long long t0 = globaltimer();
+    int ok = 1;
+    while (ld_relaxed_gpu_u64(count) < target) {
+      if (globaltimer() - t0 > kWaitTimeoutNs) {
+        ok = 0;
+        if (err) atomicCAS(err, 0, kErrWaitGridBarrier);
+        break;
+      }
+      __nanosleep(32);
+    }
+    __threadfence();
+    ok_s = ok;
+  }
+  __syncthreads();
+  return ok_s != 0;
+}
+
+// The loss forward as one cooperative launch: (a) group sizes and counts --
+// with the group advantages too when WITH_ADV -- then (b) the token pass,
+// then (c) the fixed-order sum, a grid barrier between phases.  The phases
+// compute exactly what separate launches of them would.
+struct LossLaunch {
+  const float* logp;
+  const float* old_logp;
+  const float* ref_logp;
+  const float* adv;      // in, or (WITH_ADV) written by phase (a)
+  float* adv_out;
+  const float* rewards;  // WITH_ADV
+  int std_mode;
+  float adv_eps;
+  const int* cu;
+  const int* gid;
+  int n_seq;
+  int n_groups;
+  const uint8_t* lm;
+  float clip_eps;
+  float kl_beta;
+  int agg;
+  const float* cscale;
+  float* loss;
+  float* g;
+  float* stats;
+  LossWs w;
+  int chunk;
+  int nb;
+  int* err;
+};
+
+template <int LPS, bool WITH_ADV>
+__global__ void __launch_bounds__(kLossThreads) loss_fused_kernel(const LossLaunch a) {
+  unsigned long long* bar = a.w.scal + 3;
+  if (WITH_ADV)
+    adv_and_group_counts(a.rewards, a.gid, a.n_seq, a.n_groups, a.std_mode, a.adv_eps, a.adv_out,
+                         a.cu, a.lm, a.agg, a.w.gsize, a.w.scal);
+  else
+    loss_group_counts(a.gid, a.n_seq, a.n_groups, a.cu, a.lm, a.agg, a.w.gsize, a.w.scal);
+  if (!grid_barrier(bar, gridDim.x, a.err)) return;
+  loss_token_pass<LPS, true>(a.logp, a.old_logp, a.ref_logp, a.adv, a.cu, a.gid, a.n_seq,
+                             a.n_groups, a.lm, a.clip_eps, a.kl_beta, a.agg, a.w.gsize, a.w.scal,
+                             a.cscale, a.g, a.w.part_l, a.w.part_rk, a.w.part_clip, a.w.n_tok);
+  if (!grid_barrier(bar, 2ull * gridDim.x, a.err)) return;
+  loss_final_phase(a.w.part_l, a.w.part_rk, a.w.part_clip, a.w.n_tok, a.n_seq, a.chunk, a.nb,
+                   static_cast<LossSums*>(a.w.bpart), a.w.scal + 2, a.loss, a.stats);
+}
+
+// The same three phases as separate launches, for batches of more sequences
+// than a cooperative launch is worth (the phases then fill the device
+// independently and nothing waits at a grid barrier).
+template <bool WITH_ADV>
+__global__ void __launch_bounds__(kLossThreads) loss_counts_kernel(const LossLaunch a) {
+  if (WITH_ADV)
+    adv_and_group_counts(a.rewards, a.gid, a.n_seq, a.n_groups, a.std_mode, a.adv_eps, a.adv_out,
+                         a.cu, a.lm, a.agg, a.w.gsize, a.w.scal);
+  else
+    loss_group_counts(a.gid, a.n_seq, a.n_groups, a.cu, a.lm, a.agg, a.w.gsize, a.w.scal);
+}
+
+template <int LPS>
+__global__ void __launch_bounds__(kLossThreads, 4) loss_token_kernel(const LossLaunch a) {
+  loss_token_pass<LPS, false>(a.logp, a.old_logp, a.ref_logp, a.adv, a.cu, a.gid, a.n_seq,
+                              a.n_groups, a.lm, a.clip_eps, a.kl_beta, a.agg, a.w.gsize, a.w.scal,
+                              a.cscale, a.g, a.w.part_l, a.w.part_rk, a.w.part_clip, a.w.n_tok);
+}
+
+__global__ void __launch_bounds__(kLossThreads) loss_final_kernel(const LossLaunch a) {
+  loss_final_phase(a.w.part_l, a.w.part_rk, a.w.part_clip, a.w.n_tok, a.n_seq, a.chunk, a.nb,
+                   static_cast<LossSums*>(a.w.bpart), a.w.scal + 2, a.loss, a.stats);
+}
+
+// Sequences up to which the loss forward is one cooperative launch.
+constexpr int kLossFusedMaxSeq = 16384;
 
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
@@ -1314,7 +1472,7 @@ cudaError_t launch_validate(const int* tgt, long long T, long long V, const int*
 }
 
 size_t loss_ws_bytes(int n_seq, int n_groups) {
-  return align256(3 * sizeof(long long)) + align256(sizeof(int) * n_groups) +
+  return align256(4 * sizeof(long long)) + align256(sizeof(int) * n_groups) +
          align256(sizeof(int) * n_seq) + align256(sizeof(float2) * n_seq) +
          align256(sizeof(float2) * n_seq) + align256(sizeof(int) * n_seq) +
          align256(sizeof(LossSums) * kLossFinalMaxBlocks);
@@ -1324,7 +1482,7 @@ LossWs carve_loss_ws(void* ws, int n_seq, int n_groups) {
   char* p = static_cast<char*>(ws);
   LossWs w;
   w.scal = reinterpret_cast<unsigned long long*>(p);  // cleared with gsize in one memset
-  p += align256(3 * sizeof(long long));
+  p += align256(4 * sizeof(long long));
   w.gsize = reinterpret_cast<int*>(p);
   p += align256(sizeof(int) * n_groups);
   w.n_tok = reinterpret_cast<int*>(p);
@@ -1339,53 +1497,116 @@ LossWs carve_loss_ws(void* ws, int n_seq, int n_groups) {
   return w;
 }
 
+// Resident blocks per SM of a kernel (a property of the kernel and the
+// architecture), looked up once per kernel; racing first calls store the same value.
+template <class K>
+int resident_blocks(K kernel, std::atomic<int>& cache) {
+  int res = cache.load(std::memory_order_relaxed);
+  if (res == 0) {
+    int r = 0;
+    res = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&r, kernel, kLossThreads, 0) == cudaSuccess &&
+                  r > 0
+              ? r
+              : 1;
+    cache.store(res, std::memory_order_relaxed);
+  }
+  return res;
+}
+
 cudaError_t launch_policy_loss(const float* logp, const float* old_logp, const float* ref_logp,
                                const float* adv, const int* cu_seqlens, const int* group_id,
                                int n_seq, int n_groups, const uint8_t* loss_mask, long long T,
                                float clip_eps, float kl_beta, int agg, float* loss, float* g,
-                               float* stats, const LossWs& w, cudaStream_t s,
-                               const float* cscale) {
-  // scal (groups, tokens, ticket) and gsize are adjacent: one clear
+                               float* stats, const LossWs& w, cudaStream_t s, int* err,
+                               const float* cscale, const float* rewards, int std_mode,
+                               float adv_eps, float* adv_out) {
+  // scal (groups, tokens, ticket, barrier) and gsize are adjacent: one clear
   cudaError_t e = cudaMemsetAsync(w.scal, 0,
                                   reinterpret_cast<char*>(w.gsize + n_groups) -
                                       reinterpret_cast<char*>(w.scal), s);
   if (e != cudaSuccess) return e;
   const int sms = sm_count();
-  const long long count_work = agg == 1 ? max(static_cast<long long>(n_seq), T / 16) : n_seq;
-  const int count_blocks =
-      static_cast<int>(max(1ll, min((count_work + kLossThreads - 1) / kLossThreads, sms * 4ll)));
-  loss_groups_kernel<<<count_blocks, kLossThreads, 0, s>>>(group_id, n_seq, n_groups, cu_seqlens,
-                                                           loss_mask, agg, w.gsize, w.scal);
-  // one wave of resident blocks striding over the sequences; a group of 16
-  // lanes per sequence when they are short
+  // a group of 16 lanes per sequence when they are short, else a warp
   const bool short_seqs = T <= 128ll * n_seq;
-  // resident blocks per SM of each variant (a property of the kernel and the
-  // architecture), looked up once; racing first calls store the same value
-  static std::atomic<int> resident[2] = {{0}, {0}};
-  int res = resident[short_seqs ? 0 : 1].load(std::memory_order_relaxed);
-  if (res == 0) {
-    int r = 0;
-    const cudaError_t q =
-        short_seqs ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&r, loss_token_kernel<16>, kLossThreads, 0)
-                   : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&r, loss_token_kernel<32>, kLossThreads, 0);
-    res = q == cudaSuccess && r > 0 ? r : 4;
-    resident[short_seqs ? 0 : 1].store(res, std::memory_order_relaxed);
-  }
-  const int per_block = (kLossThreads / 32) * (short_seqs ? 2 : 1);  // sequences in flight per block
-  const int seq_blocks = max(1, min((n_seq + per_block - 1) / per_block, sms * res));
-  if (short_seqs)
-    loss_token_kernel<16><<<seq_blocks, kLossThreads, 0, s>>>(
-        logp, old_logp, ref_logp, adv, cu_seqlens, group_id, n_seq, n_groups, loss_mask, clip_eps,
-        kl_beta, agg, w.gsize, w.scal, cscale, g, w.part_l, w.part_rk, w.part_clip, w.n_tok);
-  else
-    loss_token_kernel<32><<<seq_blocks, kLossThreads, 0, s>>>(
-        logp, old_logp, ref_logp, adv, cu_seqlens, group_id, n_seq, n_groups, loss_mask, clip_eps,
-        kl_beta, agg, w.gsize, w.scal, cscale, g, w.part_l, w.part_rk, w.part_clip, w.n_tok);
+  const bool with_adv = rewards != nullptr;
+  // the final sum's chunks depend only on n_seq (fixed order on any device)
   const int chunk = max(256, (n_seq + kLossFinalMaxBlocks - 1) / kLossFinalMaxBlocks);
   const int nb = (n_seq + chunk - 1) / chunk;
-  loss_final_kernel<<<nb, kLossThreads, 0, s>>>(w.part_l, w.part_rk, w.part_clip, w.n_tok, n_seq,
-                                                chunk, static_cast<LossSums*>(w.bpart), w.scal + 2,
-                                                loss, stats);
+  const int per_block = (kLossThreads / 32) * (short_seqs ? 2 : 1);  // sequences in flight per block
+  const long long seq_blocks = (n_seq + per_block - 1) / per_block;
+  const long long group_blocks =
+      with_adv ? (static_cast<long long>(n_groups) + kLossThreads / 32 - 1) / (kLossThreads / 32) : 1;
+  const long long count_blocks = agg == 1 ? max(1ll, min(T / 16 / kLossThreads, 4ll * sms)) : 1;
+
+  LossLaunch a;
+  a.logp = logp;
+  a.old_logp = old_logp;
+  a.ref_logp = ref_logp;
+  a.adv = with_adv ? adv_out : adv;
+  a.adv_out = adv_out;
+  a.rewards = rewards;
+  a.std_mode = std_mode;
+  a.adv_eps = adv_eps;
+  a.cu = cu_seqlens;
+  a.gid = group_id;
+  a.n_seq = n_seq;
+  a.n_groups = n_groups;
+  a.lm = loss_mask;
+  a.clip_eps = clip_eps;
+  a.kl_beta = kl_beta;
+  a.agg = agg;
+  a.cscale = cscale;
+  a.loss = loss;
+  a.g = g;
+  a.stats = stats;
+  a.w = w;
+  a.chunk = chunk;
+  a.nb = nb;
+  a.err = err;
+
+  if (n_seq <= kLossFusedMaxSeq) {
+    // one cooperative launch: enough blocks for each phase, never more than
+    // can be resident at once (every phase strides over the grid)
+    using Kernel = void (*)(const LossLaunch);
+    static const Kernel kernels[4] = {loss_fused_kernel<16, false>, loss_fused_kernel<32, false>,
+                                      loss_fused_kernel<16, true>, loss_fused_kernel<32, true>};
+    static std::atomic<int> resident[4] = {{0}, {0}, {0}, {0}};
+    const int variant = (short_seqs ? 0 : 1) + (with_adv ? 2 : 0);
+    const int res = resident_blocks(kernels[variant], resident[variant]);
+    const long long want =
+        max(max(seq_blocks, group_blocks), max(static_cast<long long>(nb), count_blocks));
+    const int grid = static_cast<int>(max(1ll, min(want, static_cast<long long>(sms) * res)));
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(grid), 1, 1);
+    cfg.blockDim = dim3(kLossThreads, 1, 1);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, kernels[variant], a);
+    note_launches(1);
+    if (e != cudaSuccess) return e;
+    return cudaGetLastError();
+  }
+  // three launches
+  const int cblocks = static_cast<int>(max(1ll, min(max(max(group_blocks, count_blocks),
+                                                        (n_seq + kLossThreads - 1ll) / kLossThreads),
+                                                    4ll * sms)));
+  if (with_adv)
+    loss_counts_kernel<true><<<cblocks, kLossThreads, 0, s>>>(a);
+  else
+    loss_counts_kernel<false><<<cblocks, kLossThreads, 0, s>>>(a);
+  static std::atomic<int> resident_tok[2] = {{0}, {0}};
+  const int res = short_seqs ? resident_blocks(loss_token_kernel<16>, resident_tok[0])
+                             : resident_blocks(loss_token_kernel<32>, resident_tok[1]);
+  const int tblocks = static_cast<int>(max(1ll, min(seq_blocks, static_cast<long long>(sms) * res)));
+  if (short_seqs)
+    loss_token_kernel<16><<<tblocks, kLossThreads, 0, s>>>(a);
+  else
+    loss_token_kernel<32><<<tblocks, kLossThreads, 0, s>>>(a);
+  loss_final_kernel<<<nb, kLossThreads, 0, s>>>(a);
   note_launches(3);
   return cudaGetLastError();
 }

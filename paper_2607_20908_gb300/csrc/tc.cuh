@@ -20,6 +20,7 @@ enum DevErr : int {
   kErrWaitMma = 0x102,
   kErrWaitEpilogue = 0x103,
   kErrWaitDrain = 0x104,
+  kErrWaitGridBarrier = 0x105,  // a grid barrier of a cooperative launch
   kErrWaitSelftest = 0x1ff,  // the self-test's wait on a barrier nothing arrives on
 };
 

@@ -271,3 +271,43 @@ def test_step_ragged_workload_two_chunks_equals_separate_calls(spo):
     for k in ("loss", "g", "logp", "dH", "dW"):
         assert torch.equal(got[k], want[k]), k
     assert spo.spo_sync_check() == 0
+
+
+def test_loss_launch_forms_agree_across_the_sequence_threshold(spo):
+    """Up to 16384 sequences the loss forward is one cooperative launch (grid
+    barriers between its phases); beyond, three launches of the same phases.
+    With TOKEN aggregation an empty sequence changes nothing, so the batch of
+    16384 sequences and the same batch plus one empty sequence give the same
+    bits across the two forms; both match the oracle."""
+    dev = torch.device("cuda")
+    g = torch.Generator().manual_seed(71)
+    n = 16384
+    lens = torch.randint(1, 7, (n,), generator=g)
+    T = int(lens.sum())
+    cu = torch.zeros(n + 2, dtype=torch.int32)
+    cu[1:n + 1] = torch.cumsum(lens, 0).to(torch.int32)
+    cu[n + 1] = T                                   # the extra sequence is empty
+    gid = torch.arange(n + 1, dtype=torch.int32) // 8
+    gid[n] = 0
+    lp = -torch.rand(T, generator=g) * 6
+    old = lp + torch.randn(T, generator=g) * 0.2
+    ref = lp + torch.randn(T, generator=g) * 0.05
+    adv = torch.randn(n + 1, generator=g)
+    lm = (torch.rand(T, generator=g) > 0.2).to(torch.uint8)
+    d = lambda t: t.to(dev).contiguous()
+    outs = []
+    for k in (n, n + 1):
+        loss, gg, st = spo.spo_policy_loss_fwd(d(lp), d(old), d(ref), d(adv[:k]), d(cu[:k + 1]),
+                                               d(gid[:k]), n // 8, d(lm), 0.2, 0.04, 1)
+        torch.cuda.synchronize()
+        outs.append((loss, gg, st))
+    assert torch.equal(outs[0][0], outs[1][0]) and torch.equal(outs[0][1], outs[1][1])
+    assert torch.equal(outs[0][2], outs[1][2])
+    o_loss, o_g, o_st = O.policy_loss(lp.double().numpy(), old.double().numpy(),
+                                      ref.double().numpy(), adv[:n].double().numpy(),
+                                      cu[:n + 1].numpy(), gid[:n].numpy(), n // 8, lm.numpy(),
+                                      0.2, 0.04, 1)
+    assert abs(outs[0][0].item() - o_loss) <= P.TOL_LOSS_REL * abs(o_loss)
+    assert P.rel_l2(outs[0][1].cpu().numpy(), o_g) <= P.TOL_GRAD_REL
+    assert int(outs[0][2][3].item()) == o_st["n_loss_tokens"]
+    assert spo.spo_sync_check() == 0
