@@ -223,3 +223,39 @@ def test_workspace_advantages_capture_into_a_graph(spo):
         np.testing.assert_array_equal(adv.cpu().numpy().view(np.uint32), want.view(np.uint32))
         np.testing.assert_array_equal(eager.view(np.uint32), want.view(np.uint32))
     assert spo.spo_device_error() == 0
+
+
+def test_one_call_step_captures_into_a_cuda_graph(spo):
+    """spo_grpo_step (selection, forward, the cooperative loss launch with the
+    advantages, the backward) captured into one graph: replays give the eager
+    bits, and re-read rewards written in place."""
+    t = _tensors(spo, _medium_case())
+    ws = torch.empty(spo.grpo_workspace_size(t["H"].shape[0], t["H"].shape[1], t["W"].shape[0],
+                                             t["cu"].numel() - 1, t["n_groups"]),
+                     dtype=torch.uint8, device="cuda")
+
+    def step():
+        return spo.spo_grpo_step(t["H"], t["W"], t["tgt"], t["mask"], t["cu"], t["gid"],
+                                 t["n_groups"], t["rewards"], t["old"], t["ref"],
+                                 inv_temp=t["inv_temp"], window=t["window"],
+                                 clip_eps=t["clip_eps"], kl_beta=t["kl_beta"], ws=ws)
+
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        step()
+    torch.cuda.current_stream().wait_stream(side)
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        out = step()
+    graph.replay()
+    torch.cuda.synchronize()
+    _same_bits({k: v.clone() for k, v in step().items()}, out)
+    gen = torch.Generator().manual_seed(6)
+    t["rewards"].copy_(torch.rand(t["rewards"].numel(), generator=gen) * 3.0)
+    graph.replay()
+    torch.cuda.synchronize()
+    eager = step()
+    torch.cuda.synchronize()
+    _same_bits(eager, out)
+    assert spo.spo_sync_check() == 0
