@@ -92,9 +92,9 @@ SAMPLE_SEQS, SAMPLE_TOKENS = 8, 8   # CPU sample: one group of 8 rollouts, first
 # x 151936 / 8192 rows, the mean of its two passes).  The logits GEMMs' traffic is proportional to
 # the tokens (checked against full-size captures: 6.88 and 13.57 GB); dH's grows faster than its
 # waves (its CTA pairs drift further apart over more waves), so its figure is a lower estimate.
-TRAFFIC = {"sources_sha256_16": "fd2c248a3911b49e",
-           "bytes": {"logits_lse_fwd": 6.844e9, "logits_grad_recompute": 13.394e9,
-                     "gemm_dH": 35.11e9, "gemm_dW": 17.25e9},
+TRAFFIC = {"sources_sha256_16": "46f508fca6425566",
+           "bytes": {"logits_lse_fwd": 6.810e9, "logits_grad_recompute": 13.789e9,
+                     "gemm_dH": 39.73e9, "gemm_dW": 17.00e9},
            "derivation": "reduced-case captures scaled by tokens (T = 8192 -> 16384) or vocabulary "
                          "rows (V = 8192 -> 151936); dH a lower estimate"}
 KERNEL_SOURCES = ["paper_2607_20908_gb300/csrc/gemm.cu", "paper_2607_20908_gb300/csrc/tc.cuh",
@@ -810,7 +810,7 @@ def ours(args):
         k = kern.setdefault(KERNEL_NAMES.get(kind, str(kind)), {"launches": 0, "total_ms": 0.0})
         k["launches"] += 1
         k["total_ms"] += t
-    nsplit = (st.V + 255) // 256
+    nsplit = (V_rank + 255) // 256
     hbm_bytes = {   # algorithmic bytes per call of the HBM-bound steps
         "lse_combine": 12 * nsplit * T_L + 8 * T_L + 12 * st.T,
         "select_gather_fwd": 4 * T_L * st.d + 5 * st.T + 8 * T_L,
@@ -843,10 +843,11 @@ def ours(args):
                 "traffic_unit": "bytes per launch (ncu dram__bytes_read.sum + dram__bytes_write.sum)",
                 "traffic_source": TRAFFIC["derivation"],
                 "algorithmic_bytes": None}
-    alg = {"logits_lse_fwd": 2 * T_L * st.d + 2 * st.V * st.d + 12 * T_L * ((st.V + 255) // 256),
-           "logits_grad_recompute": 2 * T_L * st.d + 2 * st.V * st.d + 2 * T_L * st.V,
-           "gemm_dH": 2 * T_L * st.V + 2 * st.V * st.d + 2 * T_L * st.d,
-           "gemm_dW": 2 * T_L * st.V + 2 * T_L * st.d + 4 * st.V * st.d}
+    Vr = V_rank   # the vocabulary rows this GPU's GEMMs cover
+    alg = {"logits_lse_fwd": 2 * T_L * st.d + 2 * Vr * st.d + 12 * T_L * nsplit,
+           "logits_grad_recompute": 2 * T_L * st.d + 2 * Vr * st.d + 2 * T_L * Vr,
+           "gemm_dH": 2 * T_L * Vr + 2 * Vr * st.d + 2 * T_L * st.d,
+           "gemm_dW": 2 * T_L * Vr + 2 * T_L * st.d + 4 * Vr * st.d}
     # per launch: a step's operand and output bytes spread over its launches of that GEMM
     roofline["algorithmic_bytes"] = alg[dom_name] / dom["launches_per_step"]
     for name, k in kern.items():
