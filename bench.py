@@ -309,6 +309,7 @@ class Step:
                                         dtype=torch.uint8, device=dev)
                 self._structs()
         self.stream = torch.cuda.current_stream(dev)
+        self.c_hooks = None   # spo_bwd_hooks for the one-call step (set by the end-to-end pipeline)
 
     def _structs(self):
         """The one-call step's argument blocks, built once (device pointers stay fixed)."""
@@ -357,7 +358,8 @@ class Step:
                 self.loss, _, _ = self.dp.run_fused(self._rank_batch(), self.n_groups * self.world)
             else:
                 R = ctypes.byref
-                chk(L.spo_grpo_step(R(self.c_batch), R(self.c_params), R(self.c_out), None,
+                hooks = R(self.c_hooks) if self.c_hooks is not None else None
+                chk(L.spo_grpo_step(R(self.c_batch), R(self.c_params), R(self.c_out), hooks,
                                     p(self.ws_s), self.ws_s.numel(), s))
             return
         if self.mode == "vocab" and self.dist:
@@ -418,10 +420,13 @@ class HostIO:
     sets so that the copies of one step overlap the compute of its neighbours
     (H2D and D2H each on their own stream, compute on the step's stream).  A
     set is reused `sets` steps later, which is the time its copies have: host
-    copies on this platform stall for about 0.1 s every half second or so, and
-    four sets give a step's copies three steps of compute to land in."""
+    copies on this platform stall now and then for tens of milliseconds, and
+    four sets give a step's copies three steps of compute to land in.  With
+    the one-call step on one GPU, dH and each dW vocabulary block leave as soon
+    as the step's hook events mark them final."""
 
-    def __init__(self, st: "Step", sets: int = 4, set_bytes: int = 0, reserve_sms: int = 8):
+    def __init__(self, st: "Step", sets: int = 4, set_bytes: int = 0, reserve_sms: int = 8,
+                 dw_blocks: int = 4):
         # at most what fits in 70 % of the free device memory (a set of the large
         # workload in the kept form holds ~60 GB), never fewer than two
         if set_bytes > 0:
@@ -462,6 +467,19 @@ class HostIO:
         mk = lambda: [torch.cuda.Event() for _ in range(sets)]
         self.in_done, self.comp_done, self.out_done = mk(), mk(), mk()
         self.i = 0
+        # One GPU, one-call step: the step records an event when dH is final and
+        # one per vocabulary block of dW (spo_bwd_hooks), and each slice is copied
+        # out as soon as its event fires, while the rest of the backward runs.
+        # Only the last block's copy is left after the last step's compute.
+        self.blocks = None
+        if st.mode == "fused" and not st.dist and not st.forward_only and dw_blocks > 0:
+            spo = st.spo
+            self.starts = spo.dw_block_starts(st.V, dw_blocks)
+            self.blocks = []
+            for x in self.sets:
+                dh_ev, dw_ev = torch.cuda.Event(), [torch.cuda.Event() for _ in range(dw_blocks)]
+                x.c_hooks = spo.make_hooks(dw_blocks, dw_ev, dh_ev, reserve_sms=0)
+                self.blocks.append((dh_ev, dw_ev))
 
     def step(self):
         b = self.i % self.n
@@ -477,9 +495,20 @@ class HostIO:
             self.compute.wait_event(self.out_done[b])   # set b's outputs already copied out
         x.run()
         self.comp_done[b].record(self.compute)
-        self.s_out.wait_event(self.comp_done[b])
+        outs, host = self.outs(x), self.host_out[b]
         with torch.cuda.stream(self.s_out):
-            for d, h in zip(self.outs(x), self.host_out[b]):
+            if self.blocks is not None:   # (loss, stats, logp, ent, dH, dW): dH and dW early
+                dh_ev, dw_ev = self.blocks[b]
+                self.s_out.wait_event(dh_ev)
+                host[4].copy_(outs[4], non_blocking=True)
+                for k, ev in enumerate(dw_ev):
+                    v0, v1 = self.starts[k], self.starts[k + 1]
+                    if v1 > v0:
+                        self.s_out.wait_event(ev)
+                        host[5][v0:v1].copy_(outs[5][v0:v1], non_blocking=True)
+                outs, host = outs[:4], host[:4]
+            self.s_out.wait_event(self.comp_done[b])
+            for d, h in zip(outs, host):
                 h.copy_(d, non_blocking=True)
             self.out_done[b].record(self.s_out)
         self.i += 1
@@ -861,7 +890,8 @@ def ours(args):
             k["frac_of_read_ceiling"] = k["gbs"] / k["read_ceiling_gbs"]
 
     # e2e: host buffers, H2D + step + D2H inside the timed region
-    hio = HostIO(st, sets=args.e2e_sets, set_bytes=step_bytes, reserve_sms=args.reserve_sms)
+    hio = HostIO(st, sets=args.e2e_sets, set_bytes=step_bytes, reserve_sms=args.reserve_sms,
+                 dw_blocks=args.e2e_dw_blocks)
     for _ in range(hio.n):
         hio.step()
     ms_e2e = timed_e2e(hio, args.steps, dist, dev)
@@ -876,7 +906,10 @@ def ours(args):
                     "log-probs), the C-ABI calls, device -> host copies of loss, stats, logp, "
                     "entropy, dH, dW")
                    + f"; {hio.n} buffer sets so a step's copies overlap the compute of the steps "
-                     "around it"}
+                     "around it"
+                   + (f"; dH and each of {len(hio.starts) - 1} vocabulary blocks of dW copied out "
+                      "as soon as the step's hook events mark them final"
+                      if hio.blocks is not None else "")}
 
     line = {
         "metric": METRIC_FWD if st.forward_only else METRIC, "value": tokens_s, "unit": UNIT,
@@ -957,6 +990,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle timing")
     ap.add_argument("--e2e-sets", type=int, default=4,
                     help="device buffer sets the end-to-end pipeline rotates through")
+    ap.add_argument("--e2e-dw-blocks", type=int, default=4,
+                    help="one GPU, one-call step: vocabulary blocks of dW copied out as each becomes "
+                         "final (spo_bwd_hooks events); 0 = every output after the step")
     ap.add_argument("--keep", action="store_true",
                     help="kept-exponential form (spo_logprobs_fwd_keep / spo_policy_loss_bwd_kept) "
                          "for a forward + backward workload")

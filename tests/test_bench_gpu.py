@@ -65,3 +65,34 @@ def test_data_parallel_bench_step_on_two_identical_ranks(spo, monkeypatch):
     starts = spo.dw_block_starts(case["V"], 4)
     assert calls == [(b - a) * case["d"] for a, b in zip(starts[:-1], starts[1:]) if b > a] + [1]
     assert spo.spo_sync_check() == 0
+
+
+def test_end_to_end_pipeline_copies_each_output_after_its_event(spo):
+    """bench.py's end-to-end pipeline copies dH and each dW vocabulary block
+    out when the step's hook event marks it final.  Every step first poisons
+    dH and dW with NaN on the compute stream, so a copy that ran ahead of its
+    event would bring back NaN or a partial block."""
+    import bench
+    dev = torch.device("cuda")
+    case = inputs.tiny_case(seed=1402, d=320, V=5000, T_per_seq=40)
+    st = bench.Step(case, dev, None, mode="fused")
+    st.prepare_old_ref()
+    st.run()
+    torch.cuda.synchronize()
+    names = ("loss", "stats", "logp", "ent", "dH", "dW")
+    want = {k: getattr(st, k).cpu() for k in names}
+    hio = bench.HostIO(st, sets=2, dw_blocks=4)
+    assert hio.blocks is not None and len(hio.starts) == 5
+    for x in hio.sets:
+        def poisoned(x=x, run=x.run):
+            x.dW.fill_(float("nan"))
+            x.dH.fill_(float("nan"))
+            run()
+        x.run = poisoned
+    for _ in range(5):
+        hio.step()
+    torch.cuda.synchronize()
+    for host in hio.host_out:
+        for k, h in zip(names, host):
+            assert torch.equal(h, want[k]), k
+    assert spo.spo_sync_check() == 0
