@@ -653,7 +653,7 @@ SPO_API spo_status spo_policy_loss_fwd_noalloc(const float* logp, const float* o
  *   SPO_TUNE_GROUP_M: tile rows (or columns) walked together by the
  *     persistent raster (L2 reuse of the streamed operand), for every GEMM;
  *     SPO_TUNE_GROUP_M_FWD / _GRAD / _DH / _DW set one GEMM (trace kinds 0-3;
- *     defaults 16, 16, 4, 8).
+ *     defaults 16, 16, 8, 8).
  *   SPO_TUNE_RASTER: 0 = groups of tile rows, 1 = groups of tile columns, for
  *     every GEMM; SPO_TUNE_RASTER_FWD / _GRAD / _DH / _DW one GEMM (defaults
  *     0, 0, 0, 1).
@@ -670,6 +670,13 @@ SPO_API spo_status spo_policy_loss_fwd_noalloc(const float* logp, const float* o
  *     operand slab read it close together in time (from L2).  The waits are
  *     bounded (20 us); results do not depend on the setting.
  *   SPO_TUNE_KSYNC_EPOCH (default 16): k-blocks between two throttle checks.
+ *   SPO_TUNE_DH_WIDE (default 1): dH with 256 x 512 output tiles per CTA
+ *     pair (two N = 256 MMAs per k-step into both TMEM accumulators; the
+ *     tiles of the last round split into 256-column halves), pair mode only:
+ *     0 = never (256 x 256), 1 = when V >= 32768 (long reductions, where the
+ *     epilogue no longer overlapping the next tile's MMAs costs nothing),
+ *     2 = always.  A wave reads G's row slabs half as often.  Results are
+ *     bit-identical either way.
  *   SPO_TUNE_DEFAULTS (value ignored): every setting back to its default.
  * Results do not depend on any setting beyond fp32 summation order. */
 typedef enum spo_tune_key {
@@ -691,7 +698,8 @@ typedef enum spo_tune_key {
     SPO_TUNE_KSYNC_GRAD = 15,
     SPO_TUNE_KSYNC_DH = 16,
     SPO_TUNE_KSYNC_DW = 17,
-    SPO_TUNE_KSYNC_EPOCH = 18
+    SPO_TUNE_KSYNC_EPOCH = 18,
+    SPO_TUNE_DH_WIDE = 19
 } spo_tune_key;
 SPO_API spo_status spo_set_tuning(int key, int64_t value);
 

@@ -203,6 +203,9 @@ int g_tune_dw_split = spo::kDefaultDwSplitRows;
 int g_tune_ksync[4] = {spo::kDefaultKsync[0], spo::kDefaultKsync[1], spo::kDefaultKsync[2],
                        spo::kDefaultKsync[3]};
 int g_tune_ksync_epoch = spo::kDefaultKsyncEpoch;
+// dH with 256 x 512 tiles per CTA pair (pair mode only): 0 never, 1 for
+// reductions of at least spo::kDhWideMinK vocabulary rows, 2 always.
+int g_tune_dh_wide = spo::kDefaultDhWide;
 
 // ------------------------------------------------------------ tracing
 // When enabled, a start/stop CUDA event pair is recorded on the launch stream
@@ -295,8 +298,10 @@ spo_status traced_gemm(int epi, bool a_mn, bool b_mn, const CUtensorMap& ta, con
     SPO_CUDA(cudaMemsetAsync(args.kprog, 0, sizeof(int) * spo::kKsyncSlots, s),
              "memset progress slots");
   }
+  const bool wide = kind == spo::EPI_DH &&
+                    (g_tune_dh_wide == 2 || (g_tune_dh_wide == 1 && args.k_static >= spo::kDhWideMinK));
   return traced(kind, s, "gemm launch", [&] {
-    return spo::launch_gemm(epi, a_mn, b_mn, g_tune_pair != 0, ta, tb, tc, args, grid, s);
+    return spo::launch_gemm(epi, a_mn, b_mn, g_tune_pair != 0, ta, tb, tc, args, grid, s, wide);
   });
 }
 
@@ -1310,6 +1315,10 @@ SPO_API spo_status spo_set_tuning(int key, int64_t value) {
         return fail(SPO_ERR_INVALID_ARG, "throttle epoch must be in [1, 4096] k-blocks");
       g_tune_ksync_epoch = static_cast<int>(value);
       return ok();
+    case SPO_TUNE_DH_WIDE:
+      if (value < 0 || value > 2) return fail(SPO_ERR_INVALID_ARG, "dH wide must be 0, 1 or 2");
+      g_tune_dh_wide = static_cast<int>(value);
+      return ok();
     case SPO_TUNE_DEFAULTS:
       g_tune_pair = 1;
       for (int k = 0; k < 4; ++k) {
@@ -1320,6 +1329,7 @@ SPO_API spo_status spo_set_tuning(int key, int64_t value) {
       g_tune_ksync_epoch = spo::kDefaultKsyncEpoch;
       g_tune_dynamic_mask = spo::kDefaultDynamicMask;
       g_tune_dw_split = spo::kDefaultDwSplitRows;
+      g_tune_dh_wide = spo::kDefaultDhWide;
       return ok();
     case SPO_TUNE_RASTER:
       if (value != 0 && value != 1) return fail(SPO_ERR_INVALID_ARG, "raster must be 0 or 1");

@@ -152,15 +152,16 @@ __device__ __forceinline__ void epi_lse(const GemmArgs& p, uint32_t taddr, int r
   }
 }
 
-__device__ __forceinline__ void epi_dh(const GemmArgs& p, uint32_t taddr, int row, int M, int nb) {
+// Columns [col_base, col_base + ncols) of the tile, TMEM columns from taddr.
+__device__ __forceinline__ void epi_dh(const GemmArgs& p, uint32_t taddr, int row, int M, int col_base,
+                                       int ncols) {
   const bool row_ok = row < M;
   const int out_row = row_ok ? (p.row_idx ? p.row_idx[row] : row) : 0;
   const size_t off = static_cast<size_t>(out_row) * p.ld_out;
   __nv_bfloat16* dst = p.out_f32 ? nullptr : p.out_bf16 + off;
   float* dst32 = p.out_f32 ? p.out_f32 + off : nullptr;
-  const int col_base = nb * BN;
 #pragma unroll 1
-  for (int c = 0; c < BN / 32; ++c) {
+  for (int c = 0; c < ncols / 32; ++c) {
     const int c0 = col_base + c * 32;
     if (c0 >= p.n) break;
     float v[32];
@@ -361,25 +362,34 @@ __device__ __forceinline__ void epi_lse_keep(const GemmArgs& p, const CUtensorMa
 // work buffered against operand latency).
 // The G, dW and kept-forward epilogues store through TMA and need 32 KB of staging, so
 // their pair-mode ring has six stages.
-template <bool PAIR, int EPI = EPI_LSE>
+// WIDE (dH, pair mode): a tile is 256 x 512, two N = 256 MMAs per k-step into
+// both TMEM accumulators (so no accumulator double-buffering: at K = V one tile
+// is ~1.5 ms of MMA against a few us of epilogue).  Each CTA stages A and two
+// B halves, 48 KB a stage, four stages.  Twice the columns per tile halve the
+// G row slabs a wave reads from DRAM.
+template <bool PAIR, int EPI = EPI_LSE, bool WIDE = false>
 struct Geo {
   static constexpr bool kTmaStore = EPI == EPI_GRAD || EPI == EPI_DW || EPI == EPI_LSE_KEEP;
-  static constexpr int kStages = PAIR ? (kTmaStore ? 6 : 7) : 4;
+  static constexpr int kHalves = WIDE ? 2 : 1;              // N = 256 MMAs per k-step
+  static constexpr int kStages = WIDE ? 4 : (PAIR ? (kTmaStore ? 6 : 7) : 4);
   static constexpr uint32_t kEpiBytes = kTmaStore ? 4 * 2 * kEpiSlotBytes : 0;  // 4 warps x 2 slots
-  static constexpr int kBRows = PAIR ? BN / 2 : BN;        // B rows staged per CTA
+  static constexpr int kBRows = PAIR ? BN / 2 : BN;        // B rows staged per CTA and MMA
   static constexpr uint32_t kABytes = BM * BK * 2;         // 16 KB
-  static constexpr uint32_t kBBytes = kBRows * BK * 2;     // 16 or 32 KB
+  static constexpr uint32_t kBHalfBytes = kBRows * BK * 2;  // 16 or 32 KB
+  static constexpr uint32_t kBBytes = kHalves * kBHalfBytes;
   static constexpr uint32_t kStageBytes = kABytes + kBBytes;
   static constexpr int kTileM = PAIR ? 2 * BM : BM;         // output rows per tile
-  static constexpr uint32_t kTxBytes = PAIR ? 2 * kStageBytes : kStageBytes;  // per full barrier
+  static constexpr int kTileN = kHalves * BN;               // output columns per tile
   static constexpr size_t kSmem = 1024 + kStages * kStageBytes + kEpiBytes + 512;
+  static_assert(!WIDE || (PAIR && EPI == EPI_DH), "wide tiles: dH in pair mode only");
+  static_assert(kSmem <= 232448, "shared memory per CTA");
 };
 
-template <int EPI, bool A_MN, bool B_MN, bool PAIR>
+template <int EPI, bool A_MN, bool B_MN, bool PAIR, bool WIDE = false>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                 const __grid_constant__ CUtensorMap tmC, const GemmArgs p) {
-  using G = Geo<PAIR, EPI>;
+  using G = Geo<PAIR, EPI, WIDE>;
   constexpr int S = G::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -411,10 +421,26 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const int M = p.m_count ? clampi(*p.m_count - p.m_offset, 0, p.m_cap) : p.m_static;
   const int K = p.k_count ? clampi(*p.k_count - p.k_offset, 0, p.k_cap) : p.k_static;
   const int mt = (M + G::kTileM - 1) / G::kTileM;
-  const int nt = (p.n + BN - 1) / BN;
-  const int num_tiles = mt * nt;
+  const int nt = (p.n + G::kTileN - 1) / G::kTileN;
+  // Work items.  WIDE: whole tiles for the rounds in which every unit gets
+  // one, then the remaining tiles as two 256-column halves each, so the last
+  // round is as balanced as with 256 x 256 tiles throughout.
+  const int whole = WIDE ? (mt * nt / n_units) * n_units : mt * nt;
+  const int num_tiles = WIDE ? whole + 2 * (mt * nt - whole) : mt * nt;
   const int num_kb = (K + BK - 1) / BK;
   const int gm = max(1, p.group_m);
+  // item -> tile row, first output column and the N = 256 halves it covers
+  auto decode = [&](int item, int& mb, int& col0, int& halves) {
+    int tile = item, half = -1;
+    if (WIDE && item >= whole) {
+      tile = whole + (item - whole) / 2;
+      half = (item - whole) & 1;
+    }
+    int nb;
+    tile_coords(tile, mt, nt, gm, p.raster, mb, nb);
+    col0 = nb * G::kTileN + (half > 0 ? BN : 0);
+    halves = half < 0 ? G::kHalves : 1;
+  };
   // dW += (empty chunk): nothing to add.  Uniform across the cluster, before any setup.
   if (EPI == EPI_DW && num_kb == 0 && p.accumulate) return;
 
@@ -507,10 +533,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         const int tile = !dyn ? static_tile(i)
                               : (rank == 0 ? publish(i, ok) : take(i, ok, kErrWaitProducer));
         if (tile < 0) break;
-        int mb, nb;
-        tile_coords(tile, mt, nt, gm, p.raster, mb, nb);
+        int mb, col0, halves;
+        decode(tile, mb, col0, halves);
         const int a_row = mb * G::kTileM + static_cast<int>(rank) * BM;
-        const int b_row = nb * BN + static_cast<int>(rank) * G::kBRows;
+        const int b_row = col0 + static_cast<int>(rank) * G::kBRows;  // half h: + h * BN
+        const uint32_t tx = PAIR ? 2 * (G::kABytes + halves * G::kBHalfBytes)
+                                 : G::kABytes + halves * G::kBHalfBytes;
         for (int kb = 0; kb < num_kb; ++kb) {
           if (throttle && prog % epoch == 0) {
             if (prog == 0) {
@@ -533,7 +561,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
           uint8_t* a_dst = sA + stage * G::kABytes;
           uint8_t* b_dst = sB + stage * G::kBBytes;
-          if (!PAIR || rank == 0) mbar_arrive_expect_tx(&full_bar[stage], G::kTxBytes);
+          if (!PAIR || rank == 0) mbar_arrive_expect_tx(&full_bar[stage], tx);
           const uint32_t bar = PAIR ? mapa_shared(smem_u32(&full_bar[stage]), 0) : 0u;
           auto load = [&](uint8_t* dst, const CUtensorMap* tm, int x, int y) {
             if (PAIR)
@@ -547,12 +575,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           } else {
             load(a_dst, &tmA, kb * BK, a_row);
           }
-          if (B_MN) {
+          for (int h = 0; h < halves; ++h) {
+            uint8_t* bh = b_dst + h * G::kBHalfBytes;
+            if (B_MN) {
 #pragma unroll
-            for (int j = 0; j < G::kBRows / 64; ++j)
-              load(b_dst + j * MN_BLOCK_BYTES, &tmB, b_row + j * 64, kb * BK);
-          } else {
-            load(b_dst, &tmB, kb * BK, b_row);
+              for (int j = 0; j < G::kBRows / 64; ++j)
+                load(bh + j * MN_BLOCK_BYTES, &tmB, b_row + h * BN + j * 64, kb * BK);
+            } else {
+              load(bh, &tmB, kb * BK, b_row + h * BN);
+            }
           }
           ++issued;
           if (++stage == S) {
@@ -588,8 +619,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       for (int local = 0;; ++local) {
         const int tile = dyn ? take(local, ok, kErrWaitMma) : static_tile(local);
         if (tile < 0) break;
-        const int acc = local & 1;
-        const uint32_t acc_phase = (local >> 1) & 1;
+        // two accumulators used in turn; WIDE: both belong to every tile
+        const int acc = WIDE ? 0 : local & 1;
+        const uint32_t acc_phase = WIDE ? local & 1 : (local >> 1) & 1;
+        int mb, col0, halves;
+        decode(tile, mb, col0, halves);
         if (!mbar_wait(&tempty_bar[acc], acc_phase ^ 1u, abort_flag, p.err, kErrWaitMma)) {
           ok = false;
           break;
@@ -608,9 +642,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           for (int k = 0; k < BK / 16; ++k) {
             const uint64_t ad = A_MN ? sdesc_sw128(a0 + k * 2048, MN_BLOCK_BYTES, 1024)
                                      : sdesc_sw128(a0 + k * 32, 16, 1024);
-            const uint64_t bd = B_MN ? sdesc_sw128(b0 + k * 2048, MN_BLOCK_BYTES, 1024)
-                                     : sdesc_sw128(b0 + k * 32, 16, 1024);
-            umma_bf16<PAIR>(d_tmem, ad, bd, kIdesc, (kb | k) != 0 ? 1u : 0u);
+#pragma unroll
+            for (int h = 0; h < G::kHalves; ++h) {
+              if (h >= halves) break;
+              const uint32_t bh = b0 + h * G::kBHalfBytes;
+              const uint64_t bd = B_MN ? sdesc_sw128(bh + k * 2048, MN_BLOCK_BYTES, 1024)
+                                       : sdesc_sw128(bh + k * 32, 16, 1024);
+              umma_bf16<PAIR>(d_tmem + static_cast<uint32_t>(h * BN), ad, bd, kIdesc,
+                              (kb | k) != 0 ? 1u : 0u);
+            }
           }
           umma_commit<PAIR>(&empty_bar[stage]);  // frees the stage (in both CTAs) when done
           if (++stage == S) {
@@ -646,10 +686,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         tile = static_tile(local);
       }
       if (tile < 0) break;
-      const int acc = local & 1;
-      const uint32_t acc_phase = (local >> 1) & 1;
-      int mb, nb;
-      tile_coords(tile, mt, nt, gm, p.raster, mb, nb);
+      const int acc = WIDE ? 0 : local & 1;
+      const uint32_t acc_phase = WIDE ? local & 1 : (local >> 1) & 1;
+      int mb, col0, halves;
+      decode(tile, mb, col0, halves);
+      const int nb = col0 / BN;  // 256-column tile index (every epilogue but WIDE dH)
       const bool ok = mbar_wait(&tfull_bar[acc], acc_phase, abort_flag, p.err, kErrWaitEpilogue);
       if (!__all_sync(0xffffffffu, ok)) break;
       tc_fence_after();
@@ -660,7 +701,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       if (EPI == EPI_LSE) epi_lse(p, taddr, row, M, nb);
       if (EPI == EPI_LSE_KEEP) epi_lse_keep(p, &tmC, taddr, row, row0, M, nb, slots, slab, lane);
       if (EPI == EPI_GRAD) epi_grad_tma(p, &tmC, taddr, row, row0, M, nb, slots, slab, lane);
-      if (EPI == EPI_DH) epi_dh(p, taddr, row, M, nb);
+      if (EPI == EPI_DH) epi_dh(p, taddr, row, M, col0, halves * BN);
       if (EPI == EPI_DW) epi_dw_tma(p, &tmC, taddr, row0, nb, num_kb == 0, slots, slab, lane);
       tc_fence_before();
       __syncwarp();
@@ -709,11 +750,11 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-template <int EPI, bool A_MN, bool B_MN, bool PAIR>
+template <int EPI, bool A_MN, bool B_MN, bool PAIR, bool WIDE = false>
 cudaError_t launch_one(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc,
                        const GemmArgs& args, int grid, cudaStream_t s) {
-  auto k = gemm_kernel<EPI, A_MN, B_MN, PAIR>;
-  const size_t smem = Geo<PAIR, EPI>::kSmem;
+  auto k = gemm_kernel<EPI, A_MN, B_MN, PAIR, WIDE>;
+  const size_t smem = Geo<PAIR, EPI, WIDE>::kSmem;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
@@ -792,7 +833,9 @@ cudaError_t launch_bounded_wait_selftest(int* err, cudaStream_t s) {
 
 cudaError_t launch_gemm(int epi, bool a_mn, bool b_mn, bool pair, const CUtensorMap& ta,
                         const CUtensorMap& tb, const CUtensorMap& tc, const GemmArgs& args, int grid,
-                        cudaStream_t s) {
+                        cudaStream_t s, bool wide) {
+  if (wide && pair && epi == EPI_DH && !a_mn && b_mn)
+    return launch_one<EPI_DH, false, true, true, true>(ta, tb, tc, args, grid, s);
 #define SPO_GEMM_CASE(E, AM, BMN)                                                        \
   if (epi == E && a_mn == AM && b_mn == BMN)                                             \
     return pair ? launch_one<E, AM, BMN, true>(ta, tb, tc, args, grid, s)                \

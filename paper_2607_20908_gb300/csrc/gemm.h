@@ -23,12 +23,11 @@ constexpr int kRowPad = 256;
 constexpr int kPartialBlock = 96;
 
 // Default launch schedule per GEMM kind (0 logits + logsumexp, 1 recompute
-// -> G, 2 dH, 3 dW), from DRAM-traffic sweeps at the full workload: the
-// logits GEMMs walk 16 tile rows together, dH (whose tiles reduce over the
-// whole vocabulary) re-reads least with 4, dW with groups of 8 tile columns;
-// every GEMM takes its tiles from an atomic counter; dW reduces over passes
-// of at most 8192 token rows.
-constexpr int kDefaultGroupM[4] = {16, 16, 4, 8};
+// -> G, 2 dH, 3 dW), from DRAM-traffic sweeps: the logits GEMMs walk 16 tile
+// rows together, dH (whose 256 x 512 tiles reduce over the whole vocabulary)
+// 8, dW groups of 8 tile columns; every GEMM takes its tiles from an atomic
+// counter; dW reduces over passes of at most 8192 token rows.
+constexpr int kDefaultGroupM[4] = {16, 16, 8, 8};
 constexpr int kDefaultRaster[4] = {0, 0, 0, 1};
 constexpr int kDefaultDynamicMask = 0xF;
 constexpr int kDefaultDwSplitRows = 8192;
@@ -37,6 +36,12 @@ constexpr int kDefaultDwSplitRows = 8192;
 constexpr int kKsyncSlots = 4;
 constexpr int kDefaultKsync[4] = {0, 0, 0, 0};
 constexpr int kDefaultKsyncEpoch = 16;
+// dH with 256 x 512 tiles per CTA pair: 0 never, 1 when the reduction (the
+// vocabulary rows) is at least kDhWideMinK, 2 always.  A wide tile holds both
+// TMEM accumulators, so its epilogue no longer overlaps the next tile's MMAs:
+// negligible at K = 151936 (1.5 ms of MMA per tile), a few % at K = 8192.
+constexpr int kDefaultDhWide = 1;
+constexpr int kDhWideMinK = 32768;
 
 // What the epilogue does with a finished 128 x 256 fp32 accumulator tile.
 enum EpiKind : int {
@@ -120,8 +125,10 @@ constexpr uint32_t kStoreBoxRows = 32;
 // One thread waits on a barrier nothing arrives on (bounded-wait self-test).
 cudaError_t launch_bounded_wait_selftest(int* err, cudaStream_t s);
 
+// wide: dH (EPI_DH, MN-major B) in pair mode with 256 x 512 tiles (the last
+// round's tiles split in 256-column halves); ignored for every other case.
 cudaError_t launch_gemm(int epi, bool a_mn, bool b_mn, bool pair, const CUtensorMap& ta,
                         const CUtensorMap& tb, const CUtensorMap& tc, const GemmArgs& args, int grid,
-                        cudaStream_t s);
+                        cudaStream_t s, bool wide = false);
 
 }  // namespace spo

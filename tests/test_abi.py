@@ -226,3 +226,21 @@ def test_step_and_hooks_host_validation(lib):
     assert sr(nul, 0, nul, nul, nul) == 0
     assert sr(p, 4, p, nul, nul) == 1
     assert sr(p, -1, p, p, nul) == 2
+
+
+def test_tuning_keys_host_validation(lib):
+    """spo_set_tuning checks each value on the host (no device involved)."""
+    from paper_2607_20908_gb300 import spo
+    ok = [(spo.SPO_TUNE_DH_WIDE, 0), (spo.SPO_TUNE_DH_WIDE, 1), (spo.SPO_TUNE_DH_WIDE, 2),
+          (spo.SPO_TUNE_PAIR_MMA, 0), (spo.SPO_TUNE_GROUP_M_DH, 8), (spo.SPO_TUNE_KSYNC_DH, 64),
+          (spo.SPO_TUNE_DW_SPLIT_ROWS, 4096)]
+    bad = [(spo.SPO_TUNE_DH_WIDE, 3), (spo.SPO_TUNE_DH_WIDE, -1), (spo.SPO_TUNE_PAIR_MMA, 2),
+           (spo.SPO_TUNE_GROUP_M_DH, 0), (spo.SPO_TUNE_DW_SPLIT_ROWS, 100),
+           (spo.SPO_TUNE_KSYNC_EPOCH, 0), (99, 0)]
+    try:
+        for key, value in ok:
+            assert lib.spo_set_tuning(key, value) == 0, (key, value)
+        for key, value in bad:
+            assert lib.spo_set_tuning(key, value) == 1, (key, value)   # SPO_ERR_INVALID_ARG
+    finally:
+        assert lib.spo_set_tuning(spo.SPO_TUNE_DEFAULTS, 0) == 0
