@@ -677,6 +677,11 @@ SPO_API spo_status spo_policy_loss_fwd_noalloc(const float* logp, const float* o
  *     epilogue no longer overlapping the next tile's MMAs costs nothing),
  *     2 = always.  A wave reads G's row slabs half as often.  Results are
  *     bit-identical either way.
+ *   SPO_TUNE_LOGITS_WIDE (default 2): the logits GEMMs with 256 x 512 tiles,
+ *     bit 0 the forward (logits + logsumexp), bit 1 the backward's recompute
+ *     (G); pair mode only.  The two accumulator halves are drained one after
+ *     the other while MMAs fill the other half.  Results are bit-identical
+ *     either way.
  *   SPO_TUNE_DEFAULTS (value ignored): every setting back to its default.
  * Results do not depend on any setting beyond fp32 summation order. */
 typedef enum spo_tune_key {
@@ -699,7 +704,8 @@ typedef enum spo_tune_key {
     SPO_TUNE_KSYNC_DH = 16,
     SPO_TUNE_KSYNC_DW = 17,
     SPO_TUNE_KSYNC_EPOCH = 18,
-    SPO_TUNE_DH_WIDE = 19
+    SPO_TUNE_DH_WIDE = 19,
+    SPO_TUNE_LOGITS_WIDE = 20
 } spo_tune_key;
 SPO_API spo_status spo_set_tuning(int key, int64_t value);
 

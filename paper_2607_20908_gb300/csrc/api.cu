@@ -206,6 +206,8 @@ int g_tune_ksync_epoch = spo::kDefaultKsyncEpoch;
 // dH with 256 x 512 tiles per CTA pair (pair mode only): 0 never, 1 for
 // reductions of at least spo::kDhWideMinK vocabulary rows, 2 always.
 int g_tune_dh_wide = spo::kDefaultDhWide;
+// The logits GEMMs with 256 x 512 tiles: bit 0 the forward, bit 1 the recompute.
+int g_tune_logits_wide = spo::kDefaultLogitsWide;
 
 // ------------------------------------------------------------ tracing
 // When enabled, a start/stop CUDA event pair is recorded on the launch stream
@@ -298,8 +300,10 @@ spo_status traced_gemm(int epi, bool a_mn, bool b_mn, const CUtensorMap& ta, con
     SPO_CUDA(cudaMemsetAsync(args.kprog, 0, sizeof(int) * spo::kKsyncSlots, s),
              "memset progress slots");
   }
-  const bool wide = kind == spo::EPI_DH &&
-                    (g_tune_dh_wide == 2 || (g_tune_dh_wide == 1 && args.k_static >= spo::kDhWideMinK));
+  const bool wide = (kind == spo::EPI_DH &&
+                     (g_tune_dh_wide == 2 || (g_tune_dh_wide == 1 && args.k_static >= spo::kDhWideMinK))) ||
+                    (epi == spo::EPI_LSE && (g_tune_logits_wide & 1)) ||
+                    (epi == spo::EPI_GRAD && (g_tune_logits_wide & 2));
   return traced(kind, s, "gemm launch", [&] {
     return spo::launch_gemm(epi, a_mn, b_mn, g_tune_pair != 0, ta, tb, tc, args, grid, s, wide);
   });
@@ -1319,6 +1323,10 @@ SPO_API spo_status spo_set_tuning(int key, int64_t value) {
       if (value < 0 || value > 2) return fail(SPO_ERR_INVALID_ARG, "dH wide must be 0, 1 or 2");
       g_tune_dh_wide = static_cast<int>(value);
       return ok();
+    case SPO_TUNE_LOGITS_WIDE:
+      if (value < 0 || value > 3) return fail(SPO_ERR_INVALID_ARG, "logits wide must be in [0, 3]");
+      g_tune_logits_wide = static_cast<int>(value);
+      return ok();
     case SPO_TUNE_DEFAULTS:
       g_tune_pair = 1;
       for (int k = 0; k < 4; ++k) {
@@ -1330,6 +1338,7 @@ SPO_API spo_status spo_set_tuning(int key, int64_t value) {
       g_tune_dynamic_mask = spo::kDefaultDynamicMask;
       g_tune_dw_split = spo::kDefaultDwSplitRows;
       g_tune_dh_wide = spo::kDefaultDhWide;
+      g_tune_logits_wide = spo::kDefaultLogitsWide;
       return ok();
     case SPO_TUNE_RASTER:
       if (value != 0 && value != 1) return fail(SPO_ERR_INVALID_ARG, "raster must be 0 or 1");

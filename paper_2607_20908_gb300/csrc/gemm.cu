@@ -68,6 +68,11 @@ __device__ __forceinline__ void tile_coords(int tile, int mt, int nt, int gm, in
 // kernel on the SMs): results never depend on the throttle.
 constexpr unsigned long long kKsyncMaxWaitNs = 20000ull;  // 20 us
 
+// Wide tiles: k-blocks at each end of a tile whose two accumulator halves are
+// issued one after the other, so each half's drain overlaps MMAs (fewer than
+// the four stages of a wide ring, which hold them meanwhile).
+constexpr int kWideOverlap = 2;
+
 __device__ __forceinline__ void ksync_wait(unsigned long long* kstate, long long prog, int window) {
   const unsigned long long t0 = globaltimer();
   for (;;) {
@@ -381,7 +386,8 @@ struct Geo {
   static constexpr int kTileM = PAIR ? 2 * BM : BM;         // output rows per tile
   static constexpr int kTileN = kHalves * BN;               // output columns per tile
   static constexpr size_t kSmem = 1024 + kStages * kStageBytes + kEpiBytes + 512;
-  static_assert(!WIDE || (PAIR && EPI == EPI_DH), "wide tiles: dH in pair mode only");
+  static_assert(!WIDE || (PAIR && (EPI == EPI_DH || EPI == EPI_LSE || EPI == EPI_GRAD)),
+                "wide tiles: dH and the logits GEMMs in pair mode only");
   static_assert(kSmem <= 232448, "shared memory per CTA");
 };
 
@@ -616,54 +622,163 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true;
-      for (int local = 0;; ++local) {
-        const int tile = dyn ? take(local, ok, kErrWaitMma) : static_tile(local);
-        if (tile < 0) break;
-        // two accumulators used in turn; WIDE: both belong to every tile
-        const int acc = WIDE ? 0 : local & 1;
-        const uint32_t acc_phase = WIDE ? local & 1 : (local >> 1) & 1;
-        int mb, col0, halves;
-        decode(tile, mb, col0, halves);
-        if (!mbar_wait(&tempty_bar[acc], acc_phase ^ 1u, abort_flag, p.err, kErrWaitMma)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
-        for (int kb = 0; kb < num_kb; ++kb) {
-          if (!mbar_wait(&full_bar[stage], phase, abort_flag, p.err, kErrWaitMma)) {
-            ok = false;
-            break;
+      if constexpr (WIDE) {
+        // Each 256-column half h of the accumulator (TMEM columns h * 256 on)
+        // has its own barrier pair tfull / tempty [h].  The last kWideOverlap
+        // k-blocks of a tile issue their first-half MMAs first, so the
+        // epilogue drains that half while the second-half MMAs finish; the
+        // first kWideOverlap k-blocks of the next tile go into the drained
+        // first half while the second is drained.  Those k-blocks' stages
+        // are freed once both halves have used them.
+        uint32_t use0 = 0, use1 = 0;  // tiles that have used each half so far
+        auto next = [&](int& st, uint32_t& ph) {
+          if (++st == S) {
+            st = 0;
+            ph ^= 1u;
           }
+        };
+        auto wait_full = [&](int st, uint32_t ph) {
+          if (!mbar_wait(&full_bar[st], ph, abort_flag, p.err, kErrWaitMma)) return false;
           tc_fence_after();
-          const uint32_t a0 = smem_u32(sA + stage * G::kABytes);
-          const uint32_t b0 = smem_u32(sB + stage * G::kBBytes);
+          return true;
+        };
+        // the four K-steps of stage st into half h
+        auto issue_half = [&](int st, int h, int kb) {
+          const uint32_t a0 = smem_u32(sA + st * G::kABytes);
+          const uint32_t bh = smem_u32(sB + st * G::kBBytes) + h * G::kBHalfBytes;
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k) {
             const uint64_t ad = A_MN ? sdesc_sw128(a0 + k * 2048, MN_BLOCK_BYTES, 1024)
                                      : sdesc_sw128(a0 + k * 32, 16, 1024);
-#pragma unroll
-            for (int h = 0; h < G::kHalves; ++h) {
-              if (h >= halves) break;
-              const uint32_t bh = b0 + h * G::kBHalfBytes;
-              const uint64_t bd = B_MN ? sdesc_sw128(bh + k * 2048, MN_BLOCK_BYTES, 1024)
-                                       : sdesc_sw128(bh + k * 32, 16, 1024);
-              umma_bf16<PAIR>(d_tmem + static_cast<uint32_t>(h * BN), ad, bd, kIdesc,
-                              (kb | k) != 0 ? 1u : 0u);
+            const uint64_t bd = B_MN ? sdesc_sw128(bh + k * 2048, MN_BLOCK_BYTES, 1024)
+                                     : sdesc_sw128(bh + k * 32, 16, 1024);
+            umma_bf16<PAIR>(tmem_base + static_cast<uint32_t>(h * BN), ad, bd, kIdesc,
+                            (kb | k) != 0 ? 1u : 0u);
+          }
+        };
+        auto full_without_mma = [&](int h) {  // K == 0: nothing to wait for
+          mbar_arrive(&tfull_bar[h]);
+          if (PAIR) mbar_arrive_cluster(mapa_shared(smem_u32(&tfull_bar[h]), 1));
+        };
+        for (int local = 0; ok; ++local) {
+          const int tile = dyn ? take(local, ok, kErrWaitMma) : static_tile(local);
+          if (tile < 0) break;
+          int mb, col0, halves;
+          decode(tile, mb, col0, halves);
+          const bool both = halves == 2;
+          const int head = both ? min(kWideOverlap, num_kb) : 0;
+          const int tail = both ? min(kWideOverlap, num_kb - head) : 0;
+          if (!mbar_wait(&tempty_bar[0], (use0 & 1) ^ 1u, abort_flag, p.err, kErrWaitMma)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          // head: the first half of the first k-blocks, stages kept
+          int st = stage;
+          uint32_t ph = phase;
+          for (int kb = 0; kb < head; ++kb) {
+            if (!wait_full(st, ph)) {
+              ok = false;
+              break;
+            }
+            issue_half(st, 0, kb);
+            next(st, ph);
+          }
+          if (!ok) break;
+          if (both) {
+            if (tail == 0 && num_kb > 0) umma_commit<PAIR>(&tfull_bar[0]);  // first half complete
+            if (!mbar_wait(&tempty_bar[1], (use1 & 1) ^ 1u, abort_flag, p.err, kErrWaitMma)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            for (int kb = 0; kb < head; ++kb) {  // their second half; then the stages are free
+              issue_half(stage, 1, kb);
+              umma_commit<PAIR>(&empty_bar[stage]);
+              next(stage, phase);
             }
           }
-          umma_commit<PAIR>(&empty_bar[stage]);  // frees the stage (in both CTAs) when done
-          if (++stage == S) {
-            stage = 0;
-            phase ^= 1u;
+          // both halves (or a half tile's one half) k-block by k-block
+          for (int kb = head; kb < num_kb - tail; ++kb) {
+            if (!wait_full(stage, phase)) {
+              ok = false;
+              break;
+            }
+            issue_half(stage, 0, kb);
+            if (both) issue_half(stage, 1, kb);
+            umma_commit<PAIR>(&empty_bar[stage]);
+            next(stage, phase);
           }
+          if (!ok) break;
+          if (!both && num_kb > 0) umma_commit<PAIR>(&tfull_bar[0]);
+          // tail: the first half of the last k-blocks, then their second half
+          st = stage;
+          ph = phase;
+          for (int kb = num_kb - tail; kb < num_kb; ++kb) {
+            if (!wait_full(st, ph)) {
+              ok = false;
+              break;
+            }
+            issue_half(st, 0, kb);
+            next(st, ph);
+          }
+          if (!ok) break;
+          if (tail > 0) umma_commit<PAIR>(&tfull_bar[0]);
+          for (int kb = num_kb - tail; kb < num_kb; ++kb) {
+            issue_half(stage, 1, kb);
+            umma_commit<PAIR>(&empty_bar[stage]);
+            next(stage, phase);
+          }
+          if (both && num_kb > 0) umma_commit<PAIR>(&tfull_bar[1]);
+          if (num_kb == 0) {
+            full_without_mma(0);
+            if (both) full_without_mma(1);
+          }
+          ++use0;
+          if (both) ++use1;
         }
-        if (!ok) break;
-        if (num_kb > 0) {
-          umma_commit<PAIR>(&tfull_bar[acc]);  // accumulator complete (both CTAs)
-        } else {                               // K == 0: nothing to wait for
-          mbar_arrive(&tfull_bar[acc]);
-          if (PAIR) mbar_arrive_cluster(mapa_shared(smem_u32(&tfull_bar[acc]), 1));
+      } else {
+        for (int local = 0;; ++local) {
+          const int tile = dyn ? take(local, ok, kErrWaitMma) : static_tile(local);
+          if (tile < 0) break;
+          // two accumulators used in turn
+          const int acc = local & 1;
+          const uint32_t acc_phase = (local >> 1) & 1;
+          if (!mbar_wait(&tempty_bar[acc], acc_phase ^ 1u, abort_flag, p.err, kErrWaitMma)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
+          for (int kb = 0; kb < num_kb; ++kb) {
+            if (!mbar_wait(&full_bar[stage], phase, abort_flag, p.err, kErrWaitMma)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t a0 = smem_u32(sA + stage * G::kABytes);
+            const uint32_t b0 = smem_u32(sB + stage * G::kBBytes);
+#pragma unroll
+            for (int k = 0; k < BK / 16; ++k) {
+              const uint64_t ad = A_MN ? sdesc_sw128(a0 + k * 2048, MN_BLOCK_BYTES, 1024)
+                                       : sdesc_sw128(a0 + k * 32, 16, 1024);
+              const uint64_t bd = B_MN ? sdesc_sw128(b0 + k * 2048, MN_BLOCK_BYTES, 1024)
+                                       : sdesc_sw128(b0 + k * 32, 16, 1024);
+              umma_bf16<PAIR>(d_tmem, ad, bd, kIdesc, (kb | k) != 0 ? 1u : 0u);
+            }
+            umma_commit<PAIR>(&empty_bar[stage]);  // frees the stage (in both CTAs) when done
+            if (++stage == S) {
+              stage = 0;
+              phase ^= 1u;
+            }
+          }
+          if (!ok) break;
+          if (num_kb > 0) {
+            umma_commit<PAIR>(&tfull_bar[acc]);  // accumulator complete (both CTAs)
+          } else {                               // K == 0: nothing to wait for
+            mbar_arrive(&tfull_bar[acc]);
+            if (PAIR) mbar_arrive_cluster(mapa_shared(smem_u32(&tfull_bar[acc]), 1));
+          }
         }
       }
       // Every MMA this thread issued must finish before TMEM is released.
@@ -675,6 +790,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const int q = warp & 3;  // TMEM lanes [32q, 32q+32) are reachable from this warp
     uint8_t* slots = sEpi + (warp - 2) * 2 * kEpiSlotBytes;  // unused unless G::kTmaStore
     int slab = 0;
+    uint32_t use0 = 0, use1 = 0;  // WIDE: tiles whose accumulator half 0 / 1 this warp drained
     for (int local = 0;; ++local) {
       int tile;
       if (dyn) {
@@ -686,30 +802,62 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         tile = static_tile(local);
       }
       if (tile < 0) break;
-      const int acc = WIDE ? 0 : local & 1;
-      const uint32_t acc_phase = WIDE ? local & 1 : (local >> 1) & 1;
       int mb, col0, halves;
       decode(tile, mb, col0, halves);
-      const int nb = col0 / BN;  // 256-column tile index (every epilogue but WIDE dH)
-      const bool ok = mbar_wait(&tfull_bar[acc], acc_phase, abort_flag, p.err, kErrWaitEpilogue);
-      if (!__all_sync(0xffffffffu, ok)) break;
-      tc_fence_after();
       const int row = mb * G::kTileM + static_cast<int>(rank) * BM + q * 32 + lane;
-      const uint32_t taddr =
-          tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN);
       const int row0 = row - lane;  // first row of this warp
-      if (EPI == EPI_LSE) epi_lse(p, taddr, row, M, nb);
-      if (EPI == EPI_LSE_KEEP) epi_lse_keep(p, &tmC, taddr, row, row0, M, nb, slots, slab, lane);
-      if (EPI == EPI_GRAD) epi_grad_tma(p, &tmC, taddr, row, row0, M, nb, slots, slab, lane);
-      if (EPI == EPI_DH) epi_dh(p, taddr, row, M, col0, halves * BN);
-      if (EPI == EPI_DW) epi_dw_tma(p, &tmC, taddr, row0, nb, num_kb == 0, slots, slab, lane);
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) {
-        if (PAIR)
-          mbar_arrive_cluster(mapa_shared(smem_u32(&tempty_bar[acc]), 0));  // leader's barrier
-        else
-          mbar_arrive(&tempty_bar[acc]);
+      const uint32_t lanes = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
+      // hands accumulator (half) a back to the MMA issuer
+      auto release = [&](int a) {
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+          if (PAIR)
+            mbar_arrive_cluster(mapa_shared(smem_u32(&tempty_bar[a]), 0));  // leader's barrier
+          else
+            mbar_arrive(&tempty_bar[a]);
+        }
+      };
+      if constexpr (WIDE) {
+        // each half as soon as it is complete; a half that starts past the
+        // last column has no output (no partials, G or dH columns)
+        bool stop = false;
+        for (int h = 0; h < halves; ++h) {
+          const uint32_t par = (h == 0 ? use0 : use1) & 1u;
+          const bool ok = mbar_wait(&tfull_bar[h], par, abort_flag, p.err, kErrWaitEpilogue);
+          if (!__all_sync(0xffffffffu, ok)) {
+            stop = true;
+            break;
+          }
+          tc_fence_after();
+          const int c = col0 + h * BN;
+          const uint32_t taddr = lanes + static_cast<uint32_t>(h * BN);
+          if (c < p.n) {  // warp-uniform
+            if (EPI == EPI_LSE) epi_lse(p, taddr, row, M, c / BN);
+            if (EPI == EPI_GRAD) epi_grad_tma(p, &tmC, taddr, row, row0, M, c / BN, slots, slab, lane);
+            if (EPI == EPI_DH) epi_dh(p, taddr, row, M, c, BN);
+          }
+          release(h);
+          if (h == 0)
+            ++use0;
+          else
+            ++use1;
+        }
+        if (stop) break;
+      } else {
+        const int acc = local & 1;
+        const uint32_t acc_phase = (local >> 1) & 1;
+        const int nb = col0 / BN;
+        const bool ok = mbar_wait(&tfull_bar[acc], acc_phase, abort_flag, p.err, kErrWaitEpilogue);
+        if (!__all_sync(0xffffffffu, ok)) break;
+        tc_fence_after();
+        const uint32_t taddr = lanes + static_cast<uint32_t>(acc * BN);
+        if (EPI == EPI_LSE) epi_lse(p, taddr, row, M, nb);
+        if (EPI == EPI_GRAD) epi_grad_tma(p, &tmC, taddr, row, row0, M, nb, slots, slab, lane);
+        if (EPI == EPI_LSE_KEEP) epi_lse_keep(p, &tmC, taddr, row, row0, M, nb, slots, slab, lane);
+        if (EPI == EPI_DH) epi_dh(p, taddr, row, M, col0, BN);
+        if (EPI == EPI_DW) epi_dw_tma(p, &tmC, taddr, row0, nb, num_kb == 0, slots, slab, lane);
+        release(acc);
       }
     }
     if (G::kTmaStore) {
@@ -836,6 +984,10 @@ cudaError_t launch_gemm(int epi, bool a_mn, bool b_mn, bool pair, const CUtensor
                         cudaStream_t s, bool wide) {
   if (wide && pair && epi == EPI_DH && !a_mn && b_mn)
     return launch_one<EPI_DH, false, true, true, true>(ta, tb, tc, args, grid, s);
+  if (wide && pair && epi == EPI_LSE && !a_mn && !b_mn)
+    return launch_one<EPI_LSE, false, false, true, true>(ta, tb, tc, args, grid, s);
+  if (wide && pair && epi == EPI_GRAD && !a_mn && !b_mn)
+    return launch_one<EPI_GRAD, false, false, true, true>(ta, tb, tc, args, grid, s);
 #define SPO_GEMM_CASE(E, AM, BMN)                                                        \
   if (epi == E && a_mn == AM && b_mn == BMN)                                             \
     return pair ? launch_one<E, AM, BMN, true>(ta, tb, tc, args, grid, s)                \

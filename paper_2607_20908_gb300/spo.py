@@ -675,6 +675,7 @@ SPO_TUNE_DEFAULTS = 13
 SPO_TUNE_KSYNC_FWD, SPO_TUNE_KSYNC_GRAD, SPO_TUNE_KSYNC_DH, SPO_TUNE_KSYNC_DW = 14, 15, 16, 17
 SPO_TUNE_KSYNC_EPOCH = 18
 SPO_TUNE_DH_WIDE = 19
+SPO_TUNE_LOGITS_WIDE = 20
 
 
 def spo_set_tuning(key: int, value: int):

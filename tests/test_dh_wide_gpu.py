@@ -90,3 +90,29 @@ def test_wide_dh_default_threshold(spo):
         assert torch.equal(got, want), V
     with pytest.raises(spo.SpoError):
         spo.spo_set_tuning(spo.SPO_TUNE_DH_WIDE, 3)
+
+
+@pytest.mark.parametrize("T,d,V", [
+    (2048, 1024, 40960),   # 8 x 40 wide tiles: whole tiles, then the last round's halves
+    (600, 320, 4200),      # the vocabulary ends inside a wide tile's first half
+    (1000, 512, 5000),     # ... inside its second half
+])
+def test_logits_wide_tiles_give_the_same_bits(spo, T, d, V):
+    """The forward (logsumexp partials per 256-column vocabulary tile) and the
+    recompute (G) with 256 x 512 tiles (SPO_TUNE_LOGITS_WIDE): logp, entropy,
+    lse, dH and dW are the same bits as with 256 x 256 tiles."""
+    H, W, tgt, gv = _inputs(T, d, V, seed=T + V)
+    out = {}
+    try:
+        for wide in (0, 3):
+            spo.spo_set_tuning(spo.SPO_TUNE_LOGITS_WIDE, wide)
+            logp, ent, lse = spo.spo_logprobs_fwd(H, W, tgt)
+            dH, dW = spo.spo_policy_loss_bwd(H, W, tgt, lse, gv)
+            torch.cuda.synchronize()
+            out[wide] = (logp, ent, lse, dH, dW)
+    finally:
+        spo.spo_set_tuning(spo.SPO_TUNE_DEFAULTS, 0)
+    assert torch.isfinite(out[0][0]).all()
+    for k, (a, b) in enumerate(zip(out[0], out[3])):
+        assert torch.equal(a, b), ("logp", "entropy", "lse", "dH", "dW")[k]
+    assert spo.spo_device_error() == 0
