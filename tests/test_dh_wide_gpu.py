@@ -116,3 +116,26 @@ def test_logits_wide_tiles_give_the_same_bits(spo, T, d, V):
     for k, (a, b) in enumerate(zip(out[0], out[3])):
         assert torch.equal(a, b), ("logp", "entropy", "lse", "dH", "dW")[k]
     assert spo.spo_device_error() == 0
+
+
+def test_wide_tiles_on_the_static_schedule(spo):
+    """Every GEMM on the static round robin (no tile counter) with all three
+    wide-tile GEMMs forced: the same bits as 256 x 256 tiles everywhere on the
+    dynamic schedule."""
+    H, W, tgt, gv = _inputs(1000, 768, 6000, seed=99)
+    try:
+        spo.spo_set_tuning(spo.SPO_TUNE_DH_WIDE, 0)
+        spo.spo_set_tuning(spo.SPO_TUNE_LOGITS_WIDE, 0)
+        _, _, lse0 = spo.spo_logprobs_fwd(H, W, tgt)
+        want = spo.spo_policy_loss_bwd(H, W, tgt, lse0, gv)
+        spo.spo_set_tuning(spo.SPO_TUNE_DYNAMIC_MASK, 0)
+        spo.spo_set_tuning(spo.SPO_TUNE_DH_WIDE, 2)
+        spo.spo_set_tuning(spo.SPO_TUNE_LOGITS_WIDE, 3)
+        _, _, lse1 = spo.spo_logprobs_fwd(H, W, tgt)
+        got = spo.spo_policy_loss_bwd(H, W, tgt, lse1, gv)
+        torch.cuda.synchronize()
+    finally:
+        spo.spo_set_tuning(spo.SPO_TUNE_DEFAULTS, 0)
+    assert torch.equal(lse1, lse0)
+    assert torch.equal(got[0], want[0]) and torch.equal(got[1], want[1])
+    assert spo.spo_device_error() == 0
