@@ -92,7 +92,7 @@ SAMPLE_SEQS, SAMPLE_TOKENS = 8, 8   # CPU sample: one group of 8 rollouts, first
 # x 151936 / 8192 rows, the mean of its two passes).  The logits GEMMs' traffic is proportional to
 # the tokens (checked against full-size captures: 6.88 and 13.57 GB); dH's grows faster than its
 # waves (its CTA pairs drift further apart over more waves), so its figure is a lower estimate.
-TRAFFIC = {"sources_sha256_16": "be78931200864388",
+TRAFFIC = {"sources_sha256_16": "34fcd1bc1917c195",
            "bytes": {"logits_lse_fwd": 6.695e9, "logits_grad_recompute": 16.44e9,
                      "gemm_dH": 27.33e9, "gemm_dW": 16.97e9},
            "derivation": "reduced-case captures scaled by tokens (T = 8192 -> 16384) or vocabulary "

@@ -10,7 +10,10 @@
 // 32 KB per CTA in pair mode, 6 when the epilogue stages its TMA stores, 4 of
 // 48 KB alone), warp 1 issues tcgen05.mma from one thread into one of two TMEM
 // accumulators (2 x 256 columns), and warps 2-5 drain the other accumulator
-// through the epilogue, so MMA and epilogue overlap.  Tiles are taken in a
+// through the epilogue, so MMA and epilogue overlap.  Wide tiles (dH and the
+// recompute, pair mode) are 256 x 512: two N = 256 MMAs per k-step fill both
+// accumulators from a ring of 4 stages of 48 KB, and the two halves are
+// drained one after the other while MMAs fill the other half.  Tiles are taken in a
 // grouped raster order, statically or from an atomic counter whose values the
 // leader's producer publishes to both CTAs through a shared-memory ring.
 // Operands may be K-major (rows of K contiguous) or MN-major (rows of M or N
