@@ -677,11 +677,13 @@ SPO_API spo_status spo_policy_loss_fwd_noalloc(const float* logp, const float* o
  *     epilogue no longer overlapping the next tile's MMAs costs nothing),
  *     2 = always.  A wave reads G's row slabs half as often.  Results are
  *     bit-identical either way.
- *   SPO_TUNE_LOGITS_WIDE (default 2): the logits GEMMs with 256 x 512 tiles,
- *     bit 0 the forward (logits + logsumexp), bit 1 the backward's recompute
- *     (G); pair mode only.  The two accumulator halves are drained one after
- *     the other while MMAs fill the other half.  Results are bit-identical
- *     either way.
+ *   SPO_TUNE_LOGITS_WIDE (default 6): the logits GEMMs with 256 x 512 tiles,
+ *     bit 0 the forward (logits + logsumexp) in every call, bit 1 the
+ *     backward's recompute (G), bit 2 the forward inside spo_grpo_step (where
+ *     it shares the power budget with the backward; alone, at full clock, the
+ *     256 x 256 tile is faster); pair mode only.  The two accumulator halves
+ *     are drained one after the other while MMAs fill the other half.
+ *     Results are bit-identical either way.
  *   SPO_TUNE_DEFAULTS (value ignored): every setting back to its default.
  * Results do not depend on any setting beyond fp32 summation order. */
 typedef enum spo_tune_key {

@@ -206,7 +206,8 @@ int g_tune_ksync_epoch = spo::kDefaultKsyncEpoch;
 // dH with 256 x 512 tiles per CTA pair (pair mode only): 0 never, 1 for
 // reductions of at least spo::kDhWideMinK vocabulary rows, 2 always.
 int g_tune_dh_wide = spo::kDefaultDhWide;
-// The logits GEMMs with 256 x 512 tiles: bit 0 the forward, bit 1 the recompute.
+// The logits GEMMs with 256 x 512 tiles: bit 0 the forward in every call, bit 1
+// the recompute, bit 2 the forward inside spo_grpo_step.
 int g_tune_logits_wide = spo::kDefaultLogitsWide;
 
 // ------------------------------------------------------------ tracing
@@ -279,9 +280,11 @@ enum TraceKind : int {
 // Launches GEMM epilogue `epi`.  Its schedule, tile counter and trace kind are
 // those of the product it computes (0 logits, 1 recompute, 2 dH, 3 dW): the
 // kept-exponential forward is the logits product.
+// in_step: the launch belongs to spo_grpo_step (the forward then takes wide
+// tiles under bit 2 of the logits setting).
 spo_status traced_gemm(int epi, bool a_mn, bool b_mn, const CUtensorMap& ta, const CUtensorMap& tb,
                        const CUtensorMap& tc, const spo::GemmArgs& args_in, int grid, cudaStream_t s,
-                       int* counters) {
+                       int* counters, bool in_step = false) {
   const int kind = epi == spo::EPI_LSE_KEEP ? spo::EPI_LSE : epi;
   if (kind < 0 || kind > 3) return fail(SPO_ERR_INVALID_ARG, "GEMM kind %d", epi);
   spo::GemmArgs args = args_in;
@@ -302,7 +305,7 @@ spo_status traced_gemm(int epi, bool a_mn, bool b_mn, const CUtensorMap& ta, con
   }
   const bool wide = (kind == spo::EPI_DH &&
                      (g_tune_dh_wide == 2 || (g_tune_dh_wide == 1 && args.k_static >= spo::kDhWideMinK))) ||
-                    (epi == spo::EPI_LSE && (g_tune_logits_wide & 1)) ||
+                    (epi == spo::EPI_LSE && ((g_tune_logits_wide & 1) || (in_step && (g_tune_logits_wide & 4)))) ||
                     (epi == spo::EPI_GRAD && (g_tune_logits_wide & 2));
   return traced(kind, s, "gemm launch", [&] {
     return spo::launch_gemm(epi, a_mn, b_mn, g_tune_pair != 0, ta, tb, tc, args, grid, s, wide);
@@ -339,7 +342,7 @@ uint32_t b_box_rows() { return static_cast<uint32_t>(spo::gemm_b_box_rows(g_tune
 spo_status logprobs_impl(const void* H, const void* W, const int32_t* tgt, const uint8_t* mask,
                          int64_t T, int64_t d, int64_t V, int64_t v_offset, float inv_temp,
                          float* logp, float* entropy, float* lse, float* rec, void* ws,
-                         cudaStream_t s, void* keep = nullptr) {
+                         cudaStream_t s, void* keep = nullptr, bool in_step = false) {
   spo_status st;
   DevInfo di;
   if ((st = device_info(&di)) != SPO_OK) return st;
@@ -377,7 +380,7 @@ spo_status logprobs_impl(const void* H, const void* W, const int32_t* tgt, const
                      w.counters);
   } else {
     st = traced_gemm(spo::EPI_LSE, false, false, ta, tb, ta, a, grid_for(di, w.T_pad, V), s,
-                     w.counters);
+                     w.counters, in_step);
   }
   if (st != SPO_OK) return st;
   // a3: split-vocab combine, scattered back to token positions (skipped tokens read 0)
@@ -1201,7 +1204,7 @@ SPO_API spo_status spo_grpo_step(const spo_grpo_batch* b, const spo_grpo_params*
   if (st != SPO_OK) return st;
   // a2 + a3 over the loss tokens (the forward's region of the workspace)
   if ((st = logprobs_impl(b->H, b->W, b->tgt, lm, b->T, b->d, b->V, 0, q->inv_temp, logp,
-                          o->entropy, lse, nullptr, ws, s)) != SPO_OK)
+                          o->entropy, lse, nullptr, ws, s, nullptr, true)) != SPO_OK)
     return st;
   // a4 + a5.  At a step's few hundred sequences the per-group scan of the
   // advantages runs inside the loss launch (its first phase, with the group
@@ -1324,7 +1327,7 @@ SPO_API spo_status spo_set_tuning(int key, int64_t value) {
       g_tune_dh_wide = static_cast<int>(value);
       return ok();
     case SPO_TUNE_LOGITS_WIDE:
-      if (value < 0 || value > 3) return fail(SPO_ERR_INVALID_ARG, "logits wide must be in [0, 3]");
+      if (value < 0 || value > 7) return fail(SPO_ERR_INVALID_ARG, "logits wide must be in [0, 7]");
       g_tune_logits_wide = static_cast<int>(value);
       return ok();
     case SPO_TUNE_DEFAULTS:

@@ -74,7 +74,7 @@ constexpr unsigned long long kKsyncMaxWaitNs = 20000ull;  // 20 us
 // Wide tiles: k-blocks at each end of a tile whose two accumulator halves are
 // issued one after the other, so each half's drain overlaps MMAs (fewer than
 // the four stages of a wide ring, which hold them meanwhile).
-constexpr int kWideOverlap = 2;
+constexpr int kWideOverlap = 3;
 
 __device__ __forceinline__ void ksync_wait(unsigned long long* kstate, long long prog, int window) {
   const unsigned long long t0 = globaltimer();

@@ -42,13 +42,14 @@ constexpr int kDefaultKsyncEpoch = 16;
 // negligible at K = 151936 (1.5 ms of MMA per tile), a few % at K = 8192.
 constexpr int kDefaultDhWide = 1;
 constexpr int kDhWideMinK = 32768;
-// The logits GEMMs with 256 x 512 tiles: bit 0 the forward, bit 1 the
-// recompute.  At K = d = 5120 a wide tile's epilogue overlaps the MMAs only
-// through the split drain of its two halves; the forward's exp2-heavy
-// epilogue outlasts that (2.5 % slower alone at full clock), the recompute's
-// does not, and under the power cap the recompute's wide tiles leave more of
-// the budget to the kernels around them.
-constexpr int kDefaultLogitsWide = 2;
+// The logits GEMMs with 256 x 512 tiles: bit 0 the forward in every call, bit
+// 1 the recompute, bit 2 the forward inside spo_grpo_step.  At K = d = 5120 a
+// wide tile's epilogue overlaps the MMAs only through the split drain of its
+// two halves.  The forward's epilogue outlasts that (a few % slower alone at
+// full clock, where a forward-only call runs), the recompute's does not; in
+// the power-capped step both wide tiles leave more of the budget to the
+// kernels around them.
+constexpr int kDefaultLogitsWide = 6;
 
 // What the epilogue does with a finished 128 x 256 fp32 accumulator tile.
 enum EpiKind : int {

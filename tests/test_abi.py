@@ -232,11 +232,11 @@ def test_tuning_keys_host_validation(lib):
     """spo_set_tuning checks each value on the host (no device involved)."""
     from paper_2607_20908_gb300 import spo
     ok = [(spo.SPO_TUNE_DH_WIDE, 0), (spo.SPO_TUNE_DH_WIDE, 1), (spo.SPO_TUNE_DH_WIDE, 2),
-          (spo.SPO_TUNE_LOGITS_WIDE, 0), (spo.SPO_TUNE_LOGITS_WIDE, 3),
+          (spo.SPO_TUNE_LOGITS_WIDE, 0), (spo.SPO_TUNE_LOGITS_WIDE, 7),
           (spo.SPO_TUNE_PAIR_MMA, 0), (spo.SPO_TUNE_GROUP_M_DH, 8), (spo.SPO_TUNE_KSYNC_DH, 64),
           (spo.SPO_TUNE_DW_SPLIT_ROWS, 4096)]
     bad = [(spo.SPO_TUNE_DH_WIDE, 3), (spo.SPO_TUNE_DH_WIDE, -1), (spo.SPO_TUNE_PAIR_MMA, 2),
-           (spo.SPO_TUNE_LOGITS_WIDE, 4),
+           (spo.SPO_TUNE_LOGITS_WIDE, 8),
            (spo.SPO_TUNE_GROUP_M_DH, 0), (spo.SPO_TUNE_DW_SPLIT_ROWS, 100),
            (spo.SPO_TUNE_KSYNC_EPOCH, 0), (99, 0)]
     try:

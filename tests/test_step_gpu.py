@@ -248,6 +248,31 @@ def test_k_progress_throttle_changes_no_bit(spo):
     assert spo.spo_device_error() == 0
 
 
+@pytest.mark.parametrize("shape", [dict(d=512, V=8192, T_per_seq=64),
+                                   dict(d=320, V=5000, T_per_seq=125, n_groups=2, rollouts=4)])
+def test_step_forward_wide_tiles_change_no_bit(spo, shape):
+    """Inside the one-call step the forward GEMM takes 256 x 512 tiles (bit 2 of
+    SPO_TUNE_LOGITS_WIDE, on by default): the step's outputs are the same bits
+    as with 256 x 256 tiles for both logits GEMMs, and as the separate calls
+    (whose forward keeps 256 x 256 tiles)."""
+    case = inputs.tiny_case(seed=1064, **shape)
+    o = P.run_oracle(case)
+    b = _dev(case, o["old"], o["ref"])
+    try:
+        spo.spo_set_tuning(spo.SPO_TUNE_LOGITS_WIDE, 0)
+        want = _fused(spo, case, b)
+        spo.spo_set_tuning(spo.SPO_TUNE_LOGITS_WIDE, 6)
+        got = _fused(spo, case, b)
+        sep = _separate(spo, case, b)
+        torch.cuda.synchronize()
+    finally:
+        spo.spo_set_tuning(spo.SPO_TUNE_DEFAULTS, 0)
+    for k in ("logp", "entropy", "lse", "loss", "g", "dH", "dW"):
+        assert torch.equal(got[k], want[k]), k
+        assert torch.equal(sep[k], want[k]), k
+    assert spo.spo_device_error() == 0
+
+
 def test_step_ragged_workload_two_chunks_equals_separate_calls(spo):
     """The ragged multi-turn workload (65536 packed tokens, ~40% masked, about
     39k loss tokens): the backward runs in two chunks of the forward's
