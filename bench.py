@@ -92,12 +92,13 @@ SAMPLE_SEQS, SAMPLE_TOKENS = 8, 8   # CPU sample: one group of 8 rollouts, first
 # x 151936 / 8192 rows, the mean of its two passes).  The logits GEMMs' traffic is proportional to
 # the tokens (checked against full-size captures: 6.88 and 13.57 GB); dH's grows faster than its
 # waves (its CTA pairs drift further apart over more waves), so its figure is a lower estimate.
-TRAFFIC = {"sources_sha256_16": "34fcd1bc1917c195",
-           "bytes": {"logits_lse_fwd": 6.695e9, "logits_grad_recompute": 16.44e9,
-                     "gemm_dH": 27.33e9, "gemm_dW": 16.97e9},
-           "derivation": "reduced-case captures scaled by tokens (T = 8192 -> 16384) or vocabulary "
-                         "rows (V = 8192 -> 151936); dH a lower estimate (23-35 GB over eight "
-                         "captures of the same kernel)"}
+TRAFFIC = {"sources_sha256_16": "a941936797edddb8",
+           "bytes": {"logits_lse_fwd": 8.889e9, "logits_grad_recompute": 16.62e9,
+                     "gemm_dH": 29.00e9, "gemm_dW": 17.03e9},
+           "derivation": "reduced-case captures, every GEMM in the tile form the one-call step "
+                         "uses, scaled by tokens (T = 8192 -> 16384) or vocabulary rows "
+                         "(V = 8192 -> 151936); dH a lower estimate (23-35 GB over nine captures "
+                         "of the same kernel)"}
 KERNEL_SOURCES = ["paper_2607_20908_gb300/csrc/gemm.cu", "paper_2607_20908_gb300/csrc/tc.cuh",
                   "paper_2607_20908_gb300/csrc/gemm.h"]
 
